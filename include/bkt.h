@@ -1,0 +1,190 @@
+/*
+ * bkt.h -- C ABI of the GB300-native bucketed LSTM-CTC training step.
+ *
+ * Method: "Accelerating Recurrent Neural Network Training using Sequence
+ * Bucketing and Multi-GPU Data Parallelization" (arXiv 1708.05604).
+ *   - bkt_plan_buckets: Section III.A (eq. 1-2, the length histogram f and
+ *     procedure DYNAMICBUCKETING), Section III.B step 3 (reshuffle every
+ *     epoch) and Section IV.A (shorter buckets are fed first).
+ *   - bkt_lstm_ctc_step: the training step of Section IV (an LSTM, ref. [1],
+ *     trained with the CTC cost, ref. [15]) over one length-bucketed
+ *     mini-batch, forward + back-propagation through time, on one GPU.
+ *   - bkt_sgd_update: the parameter update.  (The paper's update rule is
+ *     ADADELTA, Section III.B step 4; this step uses plain SGD.)
+ *
+ * Conventions
+ *   - Every entry point returns an int status (BKT_OK = 0).  On failure
+ *     bkt_last_error() returns a message for the calling thread.
+ *   - "host" pointers are ordinary CPU memory; "device" pointers are CUDA
+ *     global memory of the device current when the ctx was created.  The
+ *     caller owns every buffer it passes; the library owns what it creates
+ *     (plans, contexts) and frees it in the matching *_free / *_destroy.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy stream).
+ *     Device work is enqueued asynchronously on it; device-side errors are
+ *     reported by bkt_ctx_sync_status().
+ *   - No entry point falls back to the CPU.  Without a usable GPU the calls
+ *     that need one return BKT_ECUDA.
+ */
+#ifndef BKT_H
+#define BKT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define BKT_OK 0
+#define BKT_EINVAL 1   /* bad argument: sizes, NULL pointers, Q > max length */
+#define BKT_ENOMEM 2   /* host or device allocation failed */
+#define BKT_ECUDA 3    /* a CUDA runtime call failed (message has the name) */
+#define BKT_EDEVICE 4  /* a device-side input check failed (label >= classes or == blank) */
+
+#define BKT_GEMM_FP32 0 /* all contractions in fp32 (SIMT FMA) */
+#define BKT_GEMM_BF16 1 /* token-axis contractions: bf16 operands, fp32 accumulation */
+
+/* ------------------------------------------------------------------ */
+/* Bucketing planner (host only; no GPU needed).                       */
+
+typedef struct bkt_plan bkt_plan; /* opaque, library-owned */
+
+typedef struct bkt_plan_view {
+  int32_t n_buckets;            /* Q */
+  const int32_t *bounds;        /* [Q] inclusive upper length of each bucket, ascending; bounds[Q-1] = max length */
+  int64_t dp_cost;              /* optimal value of eq. 2: sum over sequences of their bucket's bound */
+  int64_t n_seqs;               /* n */
+  const int32_t *order;         /* [n] sequence ids (0..n-1) in emission order */
+  int32_t n_batches;
+  const int32_t *batch_off;     /* [n_batches+1] batch k is order[batch_off[k] .. batch_off[k+1]) */
+  const int32_t *batch_bucket;  /* [n_batches] bucket index of each batch, non-decreasing */
+  int64_t padded_timesteps;     /* sum over batches of |batch| * max length in the batch */
+  int64_t unpadded_timesteps;   /* sum of all lengths */
+} bkt_plan_view;
+
+/* Plans one epoch (Section III.A, procedure DYNAMICBUCKETING, plus Section
+ * III.B step 3 and Section IV.A).
+ *   lengths  host int32 [n], every entry >= 1.
+ *   n_buckets Q >= 1 and Q <= max(lengths); batch >= 1.
+ * Steps: histogram f[l] of the lengths (l = 0..max); the dynamic program
+ * dp[q][i] = min_j dp[q-1][j] + i * (f[j+1] + ... + f[i]) with the j loop
+ * descending and a strict "<" (ties keep the largest j); walk back from
+ * i = max length.  Sequence s goes to the first bucket q with
+ * lengths[s] <= bounds[q]; each bucket lists its sequences in ascending id,
+ * then one SplitMix64 stream with state seed + (epoch+1)*0x9E3779B97F4A7C15
+ * shuffles the buckets in ascending order (Fisher-Yates, k = m-1 down to 1,
+ * j = next() mod (k+1)).  Buckets are cut into consecutive batches of
+ * `batch` (the last one of a bucket may be smaller) and emitted shortest
+ * bucket first.  Empty buckets emit no batch.
+ * On success *out receives a plan to be released with bkt_plan_free.     */
+int bkt_plan_buckets(const int32_t *lengths, int64_t n, int32_t n_buckets,
+                     int32_t batch, uint64_t seed, uint64_t epoch,
+                     bkt_plan **out);
+
+/* Fills *view with pointers into the plan (valid until bkt_plan_free). */
+int bkt_plan_get(const bkt_plan *plan, bkt_plan_view *view);
+
+void bkt_plan_free(bkt_plan *plan);
+
+/* ------------------------------------------------------------------ */
+/* Model and parameters.                                               */
+
+typedef struct bkt_model_cfg {
+  int32_t n_layers;       /* >= 1 stacked LSTM layers */
+  int32_t bidirectional;  /* 0 or 1; layer l+1 reads [h_forward, h_reverse] */
+  int32_t in_dim;         /* features per time step (4 for pen samples) */
+  int32_t hidden;         /* H, units per direction */
+  int32_t n_classes;      /* C, output classes including the blank */
+  int32_t blank;          /* blank class index, 0 <= blank < C */
+  int32_t gemm_precision; /* BKT_GEMM_FP32 or BKT_GEMM_BF16 */
+} bkt_model_cfg;
+
+/* Number of fp32 parameters.  Flat layout, every block row-major:
+ *   for layer l, for direction d (0 forward, 1 reverse):
+ *     W_ih [4H x D_l], W_hh [4H x H], b [4H]   (gate row blocks i, f, g, o)
+ *   then W_out [C x dirs*H], b_out [C];   D_0 = in_dim, D_l = dirs*H.
+ * Returns 0 for an invalid cfg.                                          */
+int64_t bkt_param_count(const bkt_model_cfg *cfg);
+
+/* ------------------------------------------------------------------ */
+/* Step context: device workspace for batches up to the given sizes.   */
+
+typedef struct bkt_ctx bkt_ctx; /* opaque, library-owned */
+
+/* Allocates the workspace on the current device.
+ *   max_tokens     upper bound on the sum of lengths in one batch
+ *   max_batch      upper bound on sequences per batch
+ *   max_label_len  upper bound on one sequence's label length U          */
+int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens,
+                   int32_t max_batch, int32_t max_label_len, bkt_ctx **out);
+
+void bkt_ctx_destroy(bkt_ctx *ctx);
+
+/* One mini-batch.  Sequence i has lengths[i] >= 1 feature rows starting at
+ * row x_offsets[i] of x, and label_lengths[i] >= 0 labels starting at
+ * labels[label_offsets[i]].  The batch may be any subset of a resident
+ * dataset, in any order.                                                 */
+typedef struct bkt_batch {
+  int32_t n_seq;
+  const int32_t *lengths;       /* host [n_seq] */
+  const int64_t *x_offsets;     /* host [n_seq], in rows of in_dim floats */
+  const int32_t *label_lengths; /* host [n_seq] */
+  const int64_t *label_offsets; /* host [n_seq] */
+  const float *x;               /* device, fp32 rows [*, in_dim] */
+  const int32_t *labels;        /* device, int32 in 1..C-1 (never the blank) */
+} bkt_batch;
+
+/* The training step on one mini-batch (Section IV): packs the batch
+ * time-major sorted by length (the active batch shrinks as sequences end;
+ * no padded time step is computed), runs the stacked LSTM forward, the
+ * output layer + log-softmax, CTC (log-space forward/backward variables),
+ * the softmax gradient, and back-propagation through time.
+ *   params  device fp32 [bkt_param_count]
+ *   grads   device fp32 [bkt_param_count], overwritten with
+ *           d(sum_i loss_i)/d(params)
+ *   loss    device fp32 [n_seq]: loss[i] = -ln p(labels_i | x_i) of batch
+ *           entry i; +inf when the sequence admits no alignment
+ *           (lengths[i] < label_lengths[i] + repeated neighbours), which
+ *           then adds nothing to grads.
+ * Host-side argument checks return BKT_EINVAL before anything is enqueued.
+ * Enqueued on `stream`; the call returns before the GPU finishes.        */
+int bkt_lstm_ctc_step(bkt_ctx *ctx, const bkt_batch *batch,
+                      const float *params, float *grads, float *loss,
+                      void *stream);
+
+/* params[i] -= lr * grads[i] for i < n (device fp32 pointers; 16-byte
+ * vectors when both are 16-byte aligned), enqueued on `stream`.          */
+int bkt_sgd_update(float *params, const float *grads, int64_t n, float lr,
+                   void *stream);
+
+/* Waits for the work this ctx enqueued, then returns BKT_OK or the first
+ * device-side error (BKT_EDEVICE) raised since the previous call, and
+ * clears it.                                                             */
+int bkt_ctx_sync_status(bkt_ctx *ctx);
+
+/* ------------------------------------------------------------------ */
+/* Per-kernel timing with CUDA events on the launching stream.         */
+
+typedef struct bkt_kernel_time {
+  const char *name;  /* static string */
+  int64_t launches;
+  double total_ms;
+} bkt_kernel_time;
+
+/* enable != 0: record an event pair around every kernel this ctx launches
+ * from now on; 0: stop.  Counters start from zero on enable.             */
+int bkt_ctx_set_timing(bkt_ctx *ctx, int32_t enable);
+
+/* Synchronises, folds the recorded events into per-kernel totals and
+ * copies up to `cap` entries to out; *n_out = number of kernels seen.    */
+int bkt_ctx_kernel_times(bkt_ctx *ctx, bkt_kernel_time *out, int32_t cap,
+                         int32_t *n_out);
+
+/* Message for the last failed call on this thread ("" if none). */
+const char *bkt_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BKT_H */

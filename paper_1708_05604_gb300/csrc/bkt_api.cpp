@@ -1,0 +1,787 @@
+// bkt_api.cpp -- host side of libbkt: the bucketing planner (Section III.A of
+// arXiv 1708.05604), the step context and the step engine that enqueues the
+// CUDA kernels of one training step (Section IV).  Entry points are declared,
+// with their contracts, in include/bkt.h.
+#include "../../include/bkt.h"
+
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "bkt_internal.h"
+
+namespace {
+
+thread_local std::string g_err;
+
+int set_err(int code, const char *fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_err = buf;
+  return code;
+}
+
+int cuda_err(const char *what, cudaError_t e) {
+  return set_err(BKT_ECUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+// ---------------------------------------------------------------------------
+// Planner.
+constexpr int64_t kDpInf = int64_t(1) << 62;
+
+uint64_t splitmix64_next(uint64_t &state) {
+  state += 0x9E3779B97F4A7C15ULL;
+  uint64_t z = state;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+  return z ^ (z >> 31);
+}
+
+}  // namespace
+
+struct bkt_plan {
+  std::vector<int32_t> bounds, order, batch_off, batch_bucket;
+  int64_t dp_cost = 0, padded = 0, unpadded = 0;
+};
+
+extern "C" int bkt_plan_buckets(const int32_t *lengths, int64_t n, int32_t Q, int32_t batch,
+                                uint64_t seed, uint64_t epoch, bkt_plan **out) {
+  if (!out) return set_err(BKT_EINVAL, "bkt_plan_buckets: out is NULL");
+  *out = nullptr;
+  if (!lengths || n < 1) return set_err(BKT_EINVAL, "bkt_plan_buckets: no lengths");
+  if (Q < 1 || batch < 1) return set_err(BKT_EINVAL, "bkt_plan_buckets: n_buckets and batch must be >= 1");
+  if (n > INT32_MAX - 1) return set_err(BKT_EINVAL, "bkt_plan_buckets: too many sequences");
+  int32_t lmax = 0;
+  int64_t total = 0;
+  for (int64_t i = 0; i < n; ++i) {
+    if (lengths[i] < 1) return set_err(BKT_EINVAL, "bkt_plan_buckets: lengths[%lld] = %d < 1", (long long)i, lengths[i]);
+    lmax = std::max(lmax, lengths[i]);
+    total += lengths[i];
+  }
+  if (Q > lmax) return set_err(BKT_EINVAL, "bkt_plan_buckets: %d buckets but the longest sequence has length %d", Q, lmax);
+
+  bkt_plan *p = new (std::nothrow) bkt_plan;
+  if (!p) return set_err(BKT_ENOMEM, "bkt_plan_buckets: out of host memory");
+  try {
+    // Histogram f[l] and its prefix sums F[i] = f[0] + ... + f[i]; the
+    // charge of a group (j, i] with upper bound i is i * (F[i] - F[j]).
+    const int32_t nf = lmax + 1;
+    std::vector<int64_t> F(nf, 0);
+    for (int64_t i = 0; i < n; ++i) F[lengths[i]] += 1;
+    for (int32_t l = 1; l < nf; ++l) F[l] += F[l - 1];
+    // dp rows q-1 and q, back-pointers for every q.
+    std::vector<int64_t> prev_row(nf, kDpInf), row(nf, kDpInf);
+    std::vector<int32_t> back((size_t)(Q + 1) * nf, -1);
+    prev_row[0] = 0;
+    for (int32_t q = 1; q <= Q; ++q) {
+      std::fill(row.begin(), row.end(), kDpInf);
+      int32_t *bq = back.data() + (size_t)q * nf;
+      // dp[q-1][j] is finite only for j >= q-1.
+      for (int32_t i = q; i < nf; ++i) {
+        const int64_t Fi = F[i];
+        int64_t best = kDpInf;
+        int32_t arg = -1;
+        for (int32_t j = i - 1; j >= q - 1; --j) {
+          const int64_t v = (int64_t)i * (Fi - F[j]) + prev_row[j];
+          if (v < best) {  // strict: ties keep the larger j
+            best = v;
+            arg = j;
+          }
+        }
+        row[i] = best;
+        bq[i] = arg;
+      }
+      std::swap(prev_row, row);
+    }
+    if (prev_row[lmax] >= kDpInf) {
+      delete p;
+      return set_err(BKT_EINVAL, "bkt_plan_buckets: infeasible bucket count");
+    }
+    p->dp_cost = prev_row[lmax];
+    p->bounds.assign(Q, 0);
+    for (int32_t q = Q, cur = lmax; q >= 1; --q) {
+      p->bounds[q - 1] = cur;
+      cur = back[(size_t)q * nf + cur];
+    }
+    // Bucket of every length value, then counting sort by bucket.
+    std::vector<int32_t> bucket_of_len(nf, 0);
+    for (int32_t q = 0, l = 1; l < nf; ++l) {
+      while (l > p->bounds[q]) ++q;
+      bucket_of_len[l] = q;
+    }
+    std::vector<int64_t> start(Q + 1, 0);
+    for (int64_t i = 0; i < n; ++i) start[bucket_of_len[lengths[i]] + 1] += 1;
+    for (int32_t q = 0; q < Q; ++q) start[q + 1] += start[q];
+    p->order.resize(n);
+    {
+      std::vector<int64_t> fill(start.begin(), start.end() - 1);
+      for (int64_t i = 0; i < n; ++i) p->order[fill[bucket_of_len[lengths[i]]]++] = (int32_t)i;
+    }
+    uint64_t state = seed + (epoch + 1ULL) * 0x9E3779B97F4A7C15ULL;
+    for (int32_t q = 0; q < Q; ++q) {
+      int32_t *lst = p->order.data() + start[q];
+      const int64_t m = start[q + 1] - start[q];
+      for (int64_t k = m - 1; k >= 1; --k) {
+        const int64_t j = (int64_t)(splitmix64_next(state) % (uint64_t)(k + 1));
+        std::swap(lst[k], lst[j]);
+      }
+    }
+    for (int32_t q = 0; q < Q; ++q) {
+      for (int64_t s = start[q]; s < start[q + 1]; s += batch) {
+        const int64_t e = std::min<int64_t>(s + batch, start[q + 1]);
+        int32_t mx = 0;
+        for (int64_t r = s; r < e; ++r) mx = std::max(mx, lengths[p->order[r]]);
+        p->batch_off.push_back((int32_t)s);
+        p->batch_bucket.push_back(q);
+        p->padded += (e - s) * (int64_t)mx;
+      }
+    }
+    p->batch_off.push_back((int32_t)n);
+    p->unpadded = total;
+  } catch (const std::bad_alloc &) {
+    delete p;
+    return set_err(BKT_ENOMEM, "bkt_plan_buckets: out of host memory");
+  }
+  *out = p;
+  return BKT_OK;
+}
+
+extern "C" int bkt_plan_get(const bkt_plan *p, bkt_plan_view *v) {
+  if (!p || !v) return set_err(BKT_EINVAL, "bkt_plan_get: NULL argument");
+  v->n_buckets = (int32_t)p->bounds.size();
+  v->bounds = p->bounds.data();
+  v->dp_cost = p->dp_cost;
+  v->n_seqs = (int64_t)p->order.size();
+  v->order = p->order.data();
+  v->n_batches = (int32_t)p->batch_bucket.size();
+  v->batch_off = p->batch_off.data();
+  v->batch_bucket = p->batch_bucket.data();
+  v->padded_timesteps = p->padded;
+  v->unpadded_timesteps = p->unpadded;
+  return BKT_OK;
+}
+
+extern "C" void bkt_plan_free(bkt_plan *p) { delete p; }
+
+extern "C" const char *bkt_last_error(void) { return g_err.c_str(); }
+
+// ---------------------------------------------------------------------------
+// Parameters.
+namespace {
+
+bool cfg_ok(const bkt_model_cfg *c) {
+  return c && c->n_layers >= 1 && c->n_layers <= 64 && (c->bidirectional == 0 || c->bidirectional == 1) &&
+         c->in_dim >= 1 && c->in_dim <= 16 && c->hidden >= 1 && c->hidden <= 2048 &&
+         c->n_classes >= 2 && c->n_classes <= 1024 && c->blank >= 0 && c->blank < c->n_classes &&
+         (c->gemm_precision == BKT_GEMM_FP32 || c->gemm_precision == BKT_GEMM_BF16);
+}
+
+struct Layout {
+  int dirs, H, C, L, D0;
+  std::vector<int64_t> w_ih;  // [L*dirs] offset of W_ih of (layer, dir)
+  int64_t w_out, b_out, total;
+  int D(int l) const { return l == 0 ? D0 : dirs * H; }
+  int64_t w_hh(int l, int d) const { return w_ih[l * dirs + d] + (int64_t)4 * H * D(l); }
+  int64_t bias(int l, int d) const { return w_hh(l, d) + (int64_t)4 * H * H; }
+  int64_t stride(int l) const { return (int64_t)4 * H * (D(l) + H + 1); }
+};
+
+Layout make_layout(const bkt_model_cfg *c) {
+  Layout lo;
+  lo.dirs = c->bidirectional ? 2 : 1;
+  lo.H = c->hidden;
+  lo.C = c->n_classes;
+  lo.L = c->n_layers;
+  lo.D0 = c->in_dim;
+  int64_t off = 0;
+  for (int l = 0; l < lo.L; ++l)
+    for (int d = 0; d < lo.dirs; ++d) {
+      lo.w_ih.push_back(off);
+      off += lo.stride(l);
+    }
+  lo.w_out = off;
+  off += (int64_t)lo.C * lo.dirs * lo.H;
+  lo.b_out = off;
+  off += lo.C;
+  lo.total = off;
+  return lo;
+}
+
+}  // namespace
+
+extern "C" int64_t bkt_param_count(const bkt_model_cfg *cfg) {
+  if (!cfg_ok(cfg)) return 0;
+  return make_layout(cfg).total;
+}
+
+// ---------------------------------------------------------------------------
+// Context.
+namespace {
+
+struct EventTimer : bkt::KernelTimer {
+  struct Rec {
+    const char *name;
+    cudaEvent_t a, b;
+  };
+  struct Total {
+    const char *name;
+    int64_t launches;
+    double ms;
+  };
+  std::vector<Rec> pending;
+  std::vector<cudaEvent_t> pool;
+  std::vector<Total> totals;  // first-seen order; names are static strings
+  bool on = false;
+  cudaEvent_t get() {
+    if (!pool.empty()) {
+      cudaEvent_t e = pool.back();
+      pool.pop_back();
+      return e;
+    }
+    cudaEvent_t e = nullptr;
+    cudaEventCreate(&e);
+    return e;
+  }
+  void begin(const char *name, cudaStream_t s) override {
+    if (!on) return;
+    if (pending.size() >= 32768) fold();
+    Rec r{name, get(), get()};
+    cudaEventRecord(r.a, s);
+    pending.push_back(r);
+  }
+  void end(cudaStream_t s) override {
+    if (!on || pending.empty()) return;
+    cudaEventRecord(pending.back().b, s);
+  }
+  void fold() {
+    for (auto &r : pending) {
+      float ms = 0.f;
+      cudaEventSynchronize(r.b);
+      cudaEventElapsedTime(&ms, r.a, r.b);
+      Total *t = nullptr;
+      for (auto &x : totals)
+        if (std::strcmp(x.name, r.name) == 0) t = &x;
+      if (!t) {
+        totals.push_back(Total{r.name, 0, 0.0});
+        t = &totals.back();
+      }
+      t->launches += 1;
+      t->ms += ms;
+      pool.push_back(r.a);
+      pool.push_back(r.b);
+    }
+    pending.clear();
+  }
+  ~EventTimer() override {
+    for (auto &r : pending) {
+      cudaEventDestroy(r.a);
+      cudaEventDestroy(r.b);
+    }
+    for (auto e : pool) cudaEventDestroy(e);
+  }
+};
+
+constexpr int kStageSlots = 4;
+
+}  // namespace
+
+struct bkt_ctx {
+  bkt_model_cfg cfg;
+  Layout lo;
+  int64_t max_tokens;
+  int32_t max_batch, max_label_len, S_cap;
+  int device = 0, sm_count = 0;
+  std::vector<void *> allocs;
+  // device workspace
+  float *X = nullptr;                  // packed input [NT x in_dim]
+  std::vector<float *> Y;              // per layer [NT x dirs*H]
+  std::vector<float *> Z, Cst;         // per layer*dirs [NT x 4H], [NT x H]
+  float *logit = nullptr;              // [NT x C]
+  float *alpha = nullptr, *beta = nullptr;  // [NT x S_cap]
+  float *dY = nullptr;                 // [NT x dirs*H]
+  float *part = nullptr;               // split-K partial sums
+  size_t part_floats = 0;
+  int32_t *tok_t = nullptr, *tok_r = nullptr, *row_ok = nullptr, *status = nullptr;
+  int32_t *prev_tok[2] = {nullptr, nullptr};  // previous token of each token per direction, -1 at the start
+  void *idx_dev = nullptr;
+  size_t idx_bytes = 0;
+  // pinned staging ring for the per-step index block
+  void *stage = nullptr;
+  cudaEvent_t stage_ev[kStageSlots] = {};
+  bool stage_used[kStageSlots] = {};
+  int stage_next = 0;
+  cudaStream_t last_stream = nullptr;
+  EventTimer timer;
+  std::vector<bkt::RecGeom> geom;  // per layer
+
+  ~bkt_ctx() {
+    for (int i = 0; i < kStageSlots; ++i)
+      if (stage_ev[i]) cudaEventDestroy(stage_ev[i]);
+    if (stage) cudaFreeHost(stage);
+    for (void *p : allocs) cudaFree(p);
+  }
+  template <typename T>
+  cudaError_t alloc(T **p, size_t count) {
+    void *q = nullptr;
+    cudaError_t e = cudaMalloc(&q, std::max<size_t>(count, 1) * sizeof(T));
+    if (e == cudaSuccess) {
+      allocs.push_back(q);
+      *p = (T *)q;
+    }
+    return e;
+  }
+};
+
+namespace {
+
+// Layout of the per-step index block (same in staging and on the device).
+struct IdxLayout {
+  size_t row_len, row_lab_len, row_orig, row_xoff, row_lab_off, row_ctc_off, tok_off, bytes;
+};
+IdxLayout idx_layout(int32_t b, int64_t T) {
+  IdxLayout L;
+  size_t o = 0;
+  auto take = [&](size_t n) {
+    size_t r = o;
+    o += (n + 15) & ~size_t(15);
+    return r;
+  };
+  L.row_len = take(4 * (size_t)b);
+  L.row_lab_len = take(4 * (size_t)b);
+  L.row_orig = take(4 * (size_t)b);
+  L.row_xoff = take(8 * (size_t)b);
+  L.row_lab_off = take(8 * (size_t)b);
+  L.row_ctc_off = take(8 * (size_t)b);
+  L.tok_off = take(4 * (size_t)(T + 1));
+  L.bytes = o;
+  return L;
+}
+
+}  // namespace
+
+extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int32_t max_batch,
+                              int32_t max_label_len, bkt_ctx **out) {
+  if (!out) return set_err(BKT_EINVAL, "bkt_ctx_create: out is NULL");
+  *out = nullptr;
+  if (!cfg_ok(cfg)) return set_err(BKT_EINVAL, "bkt_ctx_create: invalid model cfg");
+  if (max_tokens < 1 || max_tokens > (int64_t)INT32_MAX / 4 || max_batch < 1 || max_batch > 4096 ||
+      max_label_len < 0 || max_label_len > 4096)
+    return set_err(BKT_EINVAL, "bkt_ctx_create: capacity out of range");
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_err("cudaGetDevice", e);
+  bkt_ctx *c = new (std::nothrow) bkt_ctx;
+  if (!c) return set_err(BKT_ENOMEM, "bkt_ctx_create: out of host memory");
+  c->cfg = *cfg;
+  c->lo = make_layout(cfg);
+  c->max_tokens = max_tokens;
+  c->max_batch = max_batch;
+  c->max_label_len = max_label_len;
+  c->S_cap = 2 * max_label_len + 1;
+  c->device = dev;
+  e = cudaDeviceGetAttribute(&c->sm_count, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) {
+    delete c;
+    return cuda_err("cudaDeviceGetAttribute", e);
+  }
+  const Layout &lo = c->lo;
+  const size_t NT = (size_t)max_tokens, DH = (size_t)lo.dirs * lo.H, H = lo.H;
+#define BKT_ALLOC(ptr, n)                                                                       \
+  do {                                                                                          \
+    const size_t bytes_ = (size_t)(n) * sizeof(*(ptr));                                         \
+    e = c->alloc(&(ptr), (n));                                                                  \
+    if (e != cudaSuccess) {                                                                     \
+      delete c;                                                                                 \
+      return set_err(BKT_ENOMEM, "bkt_ctx_create: cudaMalloc of %zu bytes failed: %s", bytes_, \
+                     cudaGetErrorName(e));                                                      \
+    }                                                                                           \
+  } while (0)
+  BKT_ALLOC(c->X, NT * cfg->in_dim);
+  c->Y.resize(lo.L);
+  c->Z.resize((size_t)lo.L * lo.dirs);
+  c->Cst.resize((size_t)lo.L * lo.dirs);
+  for (int l = 0; l < lo.L; ++l) {
+    BKT_ALLOC(c->Y[l], NT * DH);
+    for (int d = 0; d < lo.dirs; ++d) {
+      BKT_ALLOC(c->Z[l * lo.dirs + d], NT * 4 * H);
+      BKT_ALLOC(c->Cst[l * lo.dirs + d], NT * H);
+    }
+  }
+  BKT_ALLOC(c->logit, NT * lo.C);
+  BKT_ALLOC(c->alpha, NT * (size_t)c->S_cap);
+  BKT_ALLOC(c->beta, NT * (size_t)c->S_cap);
+  BKT_ALLOC(c->dY, NT * DH);
+  // split-K partials: at most 64 splits of the largest weight block (and
+  // of the bias columns), see the step engine.
+  size_t maxMN = std::max<size_t>((size_t)lo.C * DH, 4 * H * std::max<size_t>(DH, (size_t)cfg->in_dim));
+  maxMN = std::max(maxMN, 4 * H * H);
+  c->part_floats = 64 * maxMN;
+  BKT_ALLOC(c->part, c->part_floats);
+  BKT_ALLOC(c->tok_t, NT);
+  BKT_ALLOC(c->tok_r, NT);
+  BKT_ALLOC(c->prev_tok[0], NT);
+  BKT_ALLOC(c->prev_tok[1], NT);
+  BKT_ALLOC(c->row_ok, (size_t)max_batch);
+  BKT_ALLOC(c->status, 1);
+  IdxLayout il = idx_layout(max_batch, max_tokens);
+  c->idx_bytes = il.bytes;
+  {
+    char *p = nullptr;
+    BKT_ALLOC(p, il.bytes);
+    c->idx_dev = p;
+  }
+#undef BKT_ALLOC
+  e = cudaMemset(c->status, 0, sizeof(int32_t));
+  if (e != cudaSuccess) {
+    delete c;
+    return cuda_err("cudaMemset", e);
+  }
+  e = cudaMallocHost(&c->stage, il.bytes * kStageSlots);
+  if (e != cudaSuccess) {
+    delete c;
+    return set_err(BKT_ENOMEM, "bkt_ctx_create: cudaMallocHost failed: %s", cudaGetErrorName(e));
+  }
+  for (int i = 0; i < kStageSlots; ++i) {
+    e = cudaEventCreateWithFlags(&c->stage_ev[i], cudaEventDisableTiming);
+    if (e != cudaSuccess) {
+      delete c;
+      return cuda_err("cudaEventCreate", e);
+    }
+  }
+  for (int l = 0; l < lo.L; ++l)
+    c->geom.push_back(bkt::plan_recurrent(lo.H, max_batch, lo.dirs, c->sm_count));
+  *out = c;
+  return BKT_OK;
+}
+
+extern "C" void bkt_ctx_destroy(bkt_ctx *c) {
+  if (!c) return;
+  cudaSetDevice(c->device);
+  cudaDeviceSynchronize();
+  delete c;
+}
+
+extern "C" int bkt_ctx_set_timing(bkt_ctx *c, int32_t enable) {
+  if (!c) return set_err(BKT_EINVAL, "bkt_ctx_set_timing: NULL ctx");
+  c->timer.fold();
+  c->timer.totals.clear();
+  c->timer.on = enable != 0;
+  return BKT_OK;
+}
+
+extern "C" int bkt_ctx_kernel_times(bkt_ctx *c, bkt_kernel_time *out, int32_t cap, int32_t *n_out) {
+  if (!c || !n_out) return set_err(BKT_EINVAL, "bkt_ctx_kernel_times: NULL argument");
+  c->timer.fold();
+  int32_t n = 0;
+  for (const auto &t : c->timer.totals) {
+    if (out && n < cap) {
+      out[n].name = t.name;
+      out[n].launches = t.launches;
+      out[n].total_ms = t.ms;
+    }
+    ++n;
+  }
+  *n_out = n;
+  return BKT_OK;
+}
+
+extern "C" int bkt_ctx_sync_status(bkt_ctx *c) {
+  if (!c) return set_err(BKT_EINVAL, "bkt_ctx_sync_status: NULL ctx");
+  cudaError_t e = cudaSetDevice(c->device);
+  if (e != cudaSuccess) return cuda_err("cudaSetDevice", e);
+  e = cudaStreamSynchronize(c->last_stream);
+  if (e != cudaSuccess) return cuda_err("cudaStreamSynchronize", e);
+  int32_t st = 0;
+  e = cudaMemcpy(&st, c->status, sizeof st, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_err("cudaMemcpy(status)", e);
+  if (st != 0) {
+    cudaMemset(c->status, 0, sizeof st);
+    return set_err(BKT_EDEVICE, "device check failed: a label is out of range or equals the blank (flags 0x%x)", st);
+  }
+  return BKT_OK;
+}
+
+extern "C" int bkt_sgd_update(float *params, const float *grads, int64_t n, float lr, void *stream) {
+  if (n < 0 || (n > 0 && (!params || !grads))) return set_err(BKT_EINVAL, "bkt_sgd_update: bad arguments");
+  if (n == 0) return BKT_OK;
+  cudaError_t e = bkt::launch_sgd(params, grads, n, lr, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_err("sgd kernel launch", e);
+  return BKT_OK;
+}
+
+// ---------------------------------------------------------------------------
+// The step.
+namespace {
+
+struct Launch {
+  bkt_ctx *c;
+  cudaStream_t s;
+  const char *failed = nullptr;
+  cudaError_t err = cudaSuccess;
+  template <typename F>
+  bool run(const char *name, F &&f) {
+    if (failed) return false;
+    c->timer.begin(name, s);
+    cudaError_t e = f();
+    c->timer.end(s);
+    if (e != cudaSuccess) {
+      failed = name;
+      err = e;
+      return false;
+    }
+    return true;
+  }
+};
+
+// Number of token splits for a reduction over n_tok rows into an M x N block.
+int choose_splits(int M, int N, int n_tok, int sm_count, size_t part_cap) {
+  const int tiles = ((M + 63) / 64) * ((N + 63) / 64);
+  int s = std::max(1, (2 * sm_count + tiles - 1) / tiles);
+  s = std::min(s, std::max(1, n_tok / 256));
+  s = std::min(s, 64);
+  while (s > 1 && (size_t)s * M * N > part_cap) --s;
+  return s;
+}
+
+}  // namespace
+
+extern "C" int bkt_lstm_ctc_step(bkt_ctx *c, const bkt_batch *bt, const float *params, float *grads,
+                                 float *loss, void *stream) {
+  if (!c || !bt || !params || !grads || !loss) return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: NULL argument");
+  const int32_t b = bt->n_seq;
+  if (b < 1 || b > c->max_batch)
+    return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: n_seq %d outside 1..%d", b, c->max_batch);
+  if (!bt->lengths || !bt->x_offsets || !bt->label_lengths || !bt->label_offsets || !bt->x || !bt->labels)
+    return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: NULL batch array");
+  int64_t n_tok = 0;
+  int32_t S_max = 1;
+  for (int32_t i = 0; i < b; ++i) {
+    if (bt->lengths[i] < 1) return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: lengths[%d] = %d < 1", i, bt->lengths[i]);
+    if (bt->label_lengths[i] < 0 || bt->label_lengths[i] > c->max_label_len)
+      return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: label_lengths[%d] = %d outside 0..%d", i,
+                     bt->label_lengths[i], c->max_label_len);
+    if (bt->x_offsets[i] < 0 || bt->label_offsets[i] < 0)
+      return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: negative offset for sequence %d", i);
+    n_tok += bt->lengths[i];
+    S_max = std::max(S_max, 2 * bt->label_lengths[i] + 1);
+  }
+  if (n_tok > c->max_tokens)
+    return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: %lld tokens exceed the ctx capacity %lld", (long long)n_tok,
+                   (long long)c->max_tokens);
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e = cudaSetDevice(c->device);
+  if (e != cudaSuccess) return cuda_err("cudaSetDevice", e);
+
+  // ---- a4 (host part): stable sort by length, longest first; time offsets.
+  std::vector<int32_t> perm(b);
+  for (int32_t i = 0; i < b; ++i) perm[i] = i;
+  std::stable_sort(perm.begin(), perm.end(),
+                   [&](int32_t x, int32_t y) { return bt->lengths[x] > bt->lengths[y]; });
+  const int32_t T = bt->lengths[perm[0]];
+  IdxLayout il = idx_layout(b, T);
+  const int slot = c->stage_next;
+  c->stage_next = (slot + 1) % kStageSlots;
+  if (c->stage_used[slot]) {
+    e = cudaEventSynchronize(c->stage_ev[slot]);
+    if (e != cudaSuccess) return cuda_err("cudaEventSynchronize(stage)", e);
+  }
+  char *st = (char *)c->stage + (size_t)slot * c->idx_bytes;
+  int32_t *row_len = (int32_t *)(st + il.row_len), *row_lab_len = (int32_t *)(st + il.row_lab_len),
+          *row_orig = (int32_t *)(st + il.row_orig), *tok_off = (int32_t *)(st + il.tok_off);
+  int64_t *row_xoff = (int64_t *)(st + il.row_xoff), *row_lab_off = (int64_t *)(st + il.row_lab_off),
+          *row_ctc_off = (int64_t *)(st + il.row_ctc_off);
+  int64_t ctc_off = 0;
+  for (int32_t r = 0; r < b; ++r) {
+    const int32_t i = perm[r];
+    row_len[r] = bt->lengths[i];
+    row_lab_len[r] = bt->label_lengths[i];
+    row_orig[r] = i;
+    row_xoff[r] = bt->x_offsets[i];
+    row_lab_off[r] = bt->label_offsets[i];
+    row_ctc_off[r] = ctc_off;
+    ctc_off += (int64_t)bt->lengths[i] * (2 * bt->label_lengths[i] + 1);
+  }
+  {
+    int32_t active = b, acc = 0;
+    for (int32_t t = 0; t < T; ++t) {
+      while (active > 0 && row_len[active - 1] <= t) --active;
+      tok_off[t] = acc;
+      acc += active;
+    }
+    tok_off[T] = acc;
+  }
+  e = cudaMemcpyAsync(c->idx_dev, st, il.bytes, cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return cuda_err("cudaMemcpyAsync(index block)", e);
+  e = cudaEventRecord(c->stage_ev[slot], s);
+  if (e != cudaSuccess) return cuda_err("cudaEventRecord(stage)", e);
+  c->stage_used[slot] = true;
+  c->last_stream = s;
+
+  bkt::DevIdx ix;
+  char *dv = (char *)c->idx_dev;
+  ix.b = b;
+  ix.T = T;
+  ix.n_tok = (int32_t)n_tok;
+  ix.S_max = S_max;
+  ix.row_len = (const int32_t *)(dv + il.row_len);
+  ix.row_lab_len = (const int32_t *)(dv + il.row_lab_len);
+  ix.row_orig = (const int32_t *)(dv + il.row_orig);
+  ix.row_xoff = (const int64_t *)(dv + il.row_xoff);
+  ix.row_lab_off = (const int64_t *)(dv + il.row_lab_off);
+  ix.row_ctc_off = (const int64_t *)(dv + il.row_ctc_off);
+  ix.tok_off = (const int32_t *)(dv + il.tok_off);
+  ix.tok_t = c->tok_t;
+  ix.tok_r = c->tok_r;
+
+  const Layout &lo = c->lo;
+  const int H = lo.H, dirs = lo.dirs, DH = dirs * H, C = lo.C, NT = (int)n_tok;
+  Launch L{c, s};
+
+  // ---- a4: packed time-major input
+  L.run("layout_gather", [&] { return bkt::launch_layout(ix, bt->x, lo.D0, c->X, c->tok_t, c->tok_r, c->prev_tok, s); });
+
+  // ---- forward, layer by layer
+  for (int l = 0; l < lo.L; ++l) {
+    float *Zl[2] = {c->Z[l * dirs], dirs > 1 ? c->Z[l * dirs + 1] : nullptr};
+    if (l == 0) {
+      // a5, narrow input: both directions in one launch
+      L.run("proj_narrow", [&] {
+        return bkt::launch_proj_narrow(c->X, NT, lo.D0, params, lo.w_ih[0], lo.stride(0), H, dirs, Zl, s);
+      });
+    } else {
+      for (int d = 0; d < dirs; ++d) {
+        bkt::GemmArgs g{};
+        g.M = NT;
+        g.N = 4 * H;
+        g.K = DH;
+        g.A = c->Y[l - 1];
+        g.lda = DH;
+        g.B = params + lo.w_ih[l * dirs + d];
+        g.ldb = DH;
+        g.C = Zl[d];
+        g.ldc = 4 * H;
+        g.bias = params + lo.bias(l, d);
+        g.splits = 1;
+        L.run("gemm_proj", [&] { return bkt::launch_gemm_f32(false, true, g, s); });
+      }
+    }
+    bkt::RecArgs ra{};
+    ra.ix = ix;
+    ra.H = H;
+    ra.dirs = dirs;
+    for (int d = 0; d < dirs; ++d) {
+      ra.Z[d] = Zl[d];
+      ra.Cst[d] = c->Cst[l * dirs + d];
+      ra.Whh[d] = params + lo.w_hh(l, d);
+    }
+    ra.Y = c->Y[l];
+    L.run("lstm_fwd", [&] { return bkt::launch_lstm_fwd(ra, c->geom[l], s); });
+  }
+
+  // ---- a7: output layer and log-softmax
+  float *Ytop = c->Y[lo.L - 1];
+  L.run("out_logsoftmax", [&] {
+    return bkt::launch_out_logsoftmax(Ytop, NT, DH, params + lo.w_out, params + lo.b_out, C, c->logit, s);
+  });
+  // ---- a8, a9: CTC
+  L.run("ctc_tables", [&] {
+    return bkt::launch_ctc_tables(ix, c->logit, C, c->cfg.blank, bt->labels, c->alpha, c->beta, loss, c->row_ok,
+                                  c->status, s);
+  });
+  L.run("ctc_grad", [&] {
+    return bkt::launch_ctc_grad(ix, c->logit, C, c->cfg.blank, bt->labels, c->alpha, c->beta, c->row_ok, s);
+  });
+
+  // ---- a10: output layer backward
+  auto reduce_tokens = [&](const char *name, const float *A, int64_t lda, int M, const float *B, int64_t ldb,
+                           const int32_t *gather, int N, float *out) {
+    bkt::GemmArgs g{};
+    g.M = M;
+    g.N = N;
+    g.K = NT;
+    g.A = A;
+    g.lda = lda;
+    g.B = B;
+    g.ldb = ldb;
+    g.gather = gather;
+    g.P = c->part;
+    g.splits = choose_splits(M, N, NT, c->sm_count, c->part_floats);
+    L.run(name, [&] { return bkt::launch_gemm_f32(true, false, g, s); });
+    L.run("splitk_reduce", [&] { return bkt::launch_splitk_reduce(c->part, g.splits, (int64_t)M * N, out, s); });
+  };
+  auto bias_grad = [&](const float *A, int64_t lda, int M, float *out) {
+    int splits = std::min(64, std::max(1, std::min(2 * c->sm_count / std::max(1, (M + 255) / 256), NT / 64)));
+    while (splits > 1 && (size_t)splits * M > c->part_floats) --splits;
+    L.run("colsum", [&] { return bkt::launch_colsum_partial(A, lda, NT, M, c->part, splits, s); });
+    L.run("splitk_reduce", [&] { return bkt::launch_splitk_reduce(c->part, splits, M, out, s); });
+  };
+  reduce_tokens("gemm_dw_out", c->logit, C, C, Ytop, DH, nullptr, DH, grads + lo.w_out);
+  bias_grad(c->logit, C, C, grads + lo.b_out);
+  {
+    bkt::GemmArgs g{};
+    g.M = NT;
+    g.N = DH;
+    g.K = C;
+    g.A = c->logit;
+    g.lda = C;
+    g.B = params + lo.w_out;
+    g.ldb = DH;
+    g.C = c->dY;
+    g.ldc = DH;
+    g.splits = 1;
+    L.run("gemm_dy_out", [&] { return bkt::launch_gemm_f32(false, false, g, s); });
+  }
+
+  // ---- a11, a12: BPTT and weight gradients, top layer first
+  for (int l = lo.L - 1; l >= 0; --l) {
+    bkt::RecArgs ra{};
+    ra.ix = ix;
+    ra.H = H;
+    ra.dirs = dirs;
+    for (int d = 0; d < dirs; ++d) {
+      ra.Z[d] = c->Z[l * dirs + d];
+      ra.Cst[d] = c->Cst[l * dirs + d];
+      ra.Whh[d] = params + lo.w_hh(l, d);
+    }
+    ra.Y = c->Y[l];
+    ra.dY = c->dY;
+    L.run("lstm_bwd", [&] { return bkt::launch_lstm_bwd(ra, c->geom[l], s); });
+    const int D = lo.D(l);
+    const float *Xl = (l == 0) ? c->X : c->Y[l - 1];
+    for (int d = 0; d < dirs; ++d) {
+      const float *dZ = c->Z[l * dirs + d];
+      const int64_t wi = lo.w_ih[l * dirs + d];
+      reduce_tokens("gemm_dw_ih", dZ, 4 * H, 4 * H, Xl, D, nullptr, D, grads + wi);
+      // h_{t-1} of token (t, r): the row's previous token in its direction
+      reduce_tokens("gemm_dw_hh", dZ, 4 * H, 4 * H, c->Y[l] + d * H, DH, c->prev_tok[d], H,
+                    grads + lo.w_hh(l, d));
+      bias_grad(dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
+    }
+    if (l > 0) {
+      for (int d = 0; d < dirs; ++d) {
+        bkt::GemmArgs g{};
+        g.M = NT;
+        g.N = DH;
+        g.K = 4 * H;
+        g.A = c->Z[l * dirs + d];
+        g.lda = 4 * H;
+        g.B = params + lo.w_ih[l * dirs + d];
+        g.ldb = DH;
+        g.C = c->dY;
+        g.ldc = DH;
+        g.accumulate = d > 0;
+        g.splits = 1;
+        L.run("gemm_dx", [&] { return bkt::launch_gemm_f32(false, false, g, s); });
+      }
+    }
+  }
+  if (L.failed) return cuda_err(L.failed, L.err);
+  return BKT_OK;
+}

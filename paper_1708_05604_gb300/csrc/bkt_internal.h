@@ -1,0 +1,125 @@
+// bkt_internal.h -- declarations shared by the host step engine and the CUDA
+// kernels of libbkt.  Not part of the public ABI (see include/bkt.h).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace bkt {
+
+// Device-side view of one packed mini-batch.  Rows are the batch's sequences
+// sorted by length, longest first (stable), so the sequences still running at
+// time t are rows 0 .. batch_size(t)-1 and token (t, r) sits at
+// tok_off[t] + r of the time-major packed arrays.
+struct DevIdx {
+  int32_t b;       // sequences in the batch
+  int32_t T;       // longest length
+  int32_t n_tok;   // sum of lengths
+  int32_t S_max;   // largest 2U+1 in the batch
+  const int32_t *row_len;      // [b]
+  const int32_t *row_lab_len;  // [b]
+  const int32_t *row_orig;     // [b] position of the row in the caller's batch
+  const int64_t *row_xoff;     // [b] first feature row in the caller's x
+  const int64_t *row_lab_off;  // [b] first label in the caller's labels
+  const int64_t *row_ctc_off;  // [b] offset of the row's [L x S] CTC tables
+  const int32_t *tok_off;      // [T+1]
+  const int32_t *tok_t;        // [n_tok] time index of each packed token
+  const int32_t *tok_r;        // [n_tok] row of each packed token
+};
+
+// Records per-kernel CUDA events when timing is on (owned by the ctx).
+struct KernelTimer {
+  virtual ~KernelTimer() {}
+  virtual void begin(const char *name, cudaStream_t s) = 0;
+  virtual void end(cudaStream_t s) = 0;
+};
+
+// Every launcher below enqueues on `s` and returns the launch status.
+
+// a4: fills tok_t / tok_r, the previous-step token of every token for each
+// direction (prev_tok[0]: (t-1, r); prev_tok[1]: (t+1, r); -1 where the
+// direction starts), and gathers the caller's feature rows into the packed
+// time-major X [n_tok x in_dim].
+cudaError_t launch_layout(const DevIdx &ix, const float *x, int in_dim, float *X,
+                          int32_t *tok_t, int32_t *tok_r, int32_t *const *prev_tok,
+                          cudaStream_t s);
+
+// a5 for a narrow input (in_dim <= 16): Z_d[tok][n] = b_d[n] + W_d[n] . X[tok]
+// for both directions; W_d = params + w_off + d * w_stride, b_d follows W_hh.
+cudaError_t launch_proj_narrow(const float *X, int n_tok, int in_dim, const float *params,
+                               int64_t w_off, int64_t w_stride, int H, int dirs,
+                               float *const *Z, cudaStream_t s);
+
+// Generic fp32 GEMM: C[m][n] (+)= sum_k opA(m,k) opB(k,n) (+ bias[n]).
+//   opA(m,k) = a_t ? A[k*lda+m] : A[m*lda+k]
+//   opB(k,n) = b_t ? B[n*ldb+k] : B[row(k)*ldb+n], row(k) = gather ? gather[k] : k,
+//              a negative gather entry reads zeros.
+//   splits > 1: partial sums go to P[z][m*N+n] (C, bias, accumulate unused).
+struct GemmArgs {
+  int M, N, K;
+  const float *A; int64_t lda;
+  const float *B; int64_t ldb;
+  const int32_t *gather;
+  float *C; int64_t ldc;
+  const float *bias;
+  int accumulate;
+  float *P; int splits;
+};
+cudaError_t launch_gemm_f32(bool a_t, bool b_t, const GemmArgs &g, cudaStream_t s);
+
+// out[i] = sum_z P[z*n + i] for i < n (fixed summation order).
+cudaError_t launch_splitk_reduce(const float *P, int splits, int64_t n, float *out,
+                                 cudaStream_t s);
+
+// P[z][m] = sum over rows k of split z of A[k*lda + m], m < M.
+cudaError_t launch_colsum_partial(const float *A, int64_t lda, int K, int M, float *P,
+                                  int splits, cudaStream_t s);
+
+// a7: logp[tok][c] = log-softmax_c(b[c] + W[c] . Y[tok]).
+cudaError_t launch_out_logsoftmax(const float *Y, int n_tok, int DH, const float *W,
+                                  const float *bias, int C, float *logp, cudaStream_t s);
+
+// a8: log-space CTC forward (alpha) and backward (beta-hat) tables, one CTA
+// per (row, direction); writes the per-sequence loss and the row's flag.
+cudaError_t launch_ctc_tables(const DevIdx &ix, const float *logp, int C, int blank,
+                              const int32_t *labels, float *alpha, float *beta,
+                              float *loss, int32_t *row_ok, int32_t *status,
+                              cudaStream_t s);
+
+// a9: dlogit = softmax - posterior, written over logp in place.
+cudaError_t launch_ctc_grad(const DevIdx &ix, float *logp_dlogit, int C, int blank,
+                            const int32_t *labels, const float *alpha, const float *beta,
+                            const int32_t *row_ok, cudaStream_t s);
+
+// Cluster geometry of the recurrent kernels for one layer.
+struct RecGeom {
+  int cs;        // CTAs per cluster (hidden units split cs ways)
+  int bc;        // batch rows per cluster
+  int ks;        // threads sharing one (row, unit) pair along k (power of 2 <= 8)
+  int threads;   // threads per CTA
+  int w_smem;    // 1: the CTA's W_hh slice lives in shared memory
+  size_t smem_fwd, smem_bwd;
+};
+RecGeom plan_recurrent(int H, int b, int dirs, int sm_count);
+
+// a6: persistent recurrent forward for both directions of one layer.
+//   Z[d]  [n_tok x 4H] pre-activations in, activated gates (i,f,g,o) out
+//   Cst[d] [n_tok x H] cell states; Y [n_tok x dirs*H] hidden outputs
+//   Whh[d] = recurrent weights [4H x H] of direction d
+struct RecArgs {
+  DevIdx ix;
+  int H, dirs;
+  float *Z[2];
+  float *Cst[2];
+  const float *Whh[2];
+  float *Y;            // forward output / backward: h source for nothing
+  const float *dY;     // backward: d loss / d Y of this layer [n_tok x dirs*H]
+};
+cudaError_t launch_lstm_fwd(const RecArgs &a, const RecGeom &g, cudaStream_t s);
+// a11: BPTT for both directions; Z[d] holds the gates on entry and dz on exit.
+cudaError_t launch_lstm_bwd(const RecArgs &a, const RecGeom &g, cudaStream_t s);
+
+// a13
+cudaError_t launch_sgd(float *p, const float *g, int64_t n, float lr, cudaStream_t s);
+
+}  // namespace bkt

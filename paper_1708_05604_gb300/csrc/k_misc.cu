@@ -1,0 +1,164 @@
+// k_misc.cu -- the bandwidth-bound kernels of the step: the packed-layout
+// gather (a4), the narrow input projection (a5 for in_dim <= 16), split-K
+// and column-sum reductions used by the weight gradients (a10, a12), and the
+// SGD update (a13).
+#include "bkt_internal.h"
+
+namespace bkt {
+
+// ---------------------------------------------------------------------------
+// a4.  One CTA per time step t; thread r < batch_size(t) owns token
+// (t, r) = tok_off[t] + r.  The caller's rows are read where they lie
+// (x + (row_xoff[r] + t) * in_dim), so the batch can be any subset of a
+// resident dataset.
+__global__ void layout_kernel(DevIdx ix, const float *__restrict__ x, int in_dim,
+                              float *__restrict__ X, int32_t *__restrict__ tok_t,
+                              int32_t *__restrict__ tok_r, int32_t *__restrict__ prev_f,
+                              int32_t *__restrict__ prev_b) {
+  const int t = blockIdx.x;
+  const int base = ix.tok_off[t];
+  const int nb = ix.tok_off[t + 1] - base;
+  for (int r = threadIdx.x; r < nb; r += blockDim.x) {
+    const int tok = base + r;
+    tok_t[tok] = t;
+    tok_r[tok] = r;
+    prev_f[tok] = t > 0 ? ix.tok_off[t - 1] + r : -1;
+    prev_b[tok] = (t + 1 < ix.row_len[r]) ? ix.tok_off[t + 1] + r : -1;
+    const float *src = x + (ix.row_xoff[r] + t) * (int64_t)in_dim;
+    float *dst = X + (int64_t)tok * in_dim;
+    if (in_dim == 4 && ((reinterpret_cast<uintptr_t>(src) & 15) == 0)) {
+      *reinterpret_cast<float4 *>(dst) = __ldg(reinterpret_cast<const float4 *>(src));
+    } else {
+      for (int k = 0; k < in_dim; ++k) dst[k] = __ldg(src + k);
+    }
+  }
+}
+
+cudaError_t launch_layout(const DevIdx &ix, const float *x, int in_dim, float *X, int32_t *tok_t,
+                          int32_t *tok_r, int32_t *const *prev_tok, cudaStream_t s) {
+  int threads = ((ix.b + 31) / 32) * 32;
+  if (threads > 1024) threads = 1024;
+  layout_kernel<<<ix.T, threads, 0, s>>>(ix, x, in_dim, X, tok_t, tok_r, prev_tok[0], prev_tok[1]);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// a5 with a narrow input.  Thread n of a CTA owns output column n of one
+// direction: W row n (in_dim values) and b[n] stay in registers while the CTA
+// walks a chunk of tokens; each token row of X is read once per CTA
+// (broadcast) and the [tok x 4H] output is written coalesced along n.
+constexpr int kProjTok = 64;
+
+template <int D>
+__global__ void __launch_bounds__(128) proj_narrow_kernel(const float *__restrict__ X, int n_tok,
+                                                         const float *__restrict__ params, int64_t w_off,
+                                                         int64_t w_stride, int H, float *Z0, float *Z1) {
+  const int d = blockIdx.z;
+  const int n = blockIdx.x * 128 + threadIdx.x;
+  const int G = 4 * H;
+  if (n >= G) return;
+  const float *W = params + w_off + d * w_stride;
+  const float *bias = W + (int64_t)G * D + (int64_t)G * H;
+  float w[D];
+#pragma unroll
+  for (int k = 0; k < D; ++k) w[k] = W[(int64_t)n * D + k];
+  const float bn = bias[n];
+  float *Z = d == 0 ? Z0 : Z1;
+  const int t0 = blockIdx.y * kProjTok;
+  const int t1 = min(n_tok, t0 + kProjTok);
+  for (int tok = t0; tok < t1; ++tok) {
+    float z = bn;
+#pragma unroll
+    for (int k = 0; k < D; ++k) z = fmaf(w[k], __ldg(X + (int64_t)tok * D + k), z);
+    Z[(int64_t)tok * G + n] = z;
+  }
+}
+
+cudaError_t launch_proj_narrow(const float *X, int n_tok, int in_dim, const float *params, int64_t w_off,
+                               int64_t w_stride, int H, int dirs, float *const *Z, cudaStream_t s) {
+  dim3 grid((4 * H + 127) / 128, (n_tok + kProjTok - 1) / kProjTok, dirs);
+  float *Z1 = dirs > 1 ? Z[1] : Z[0];
+  switch (in_dim) {
+#define BKT_CASE(D) \
+  case D:           \
+    proj_narrow_kernel<D><<<grid, 128, 0, s>>>(X, n_tok, params, w_off, w_stride, H, Z[0], Z1); \
+    break;
+    BKT_CASE(1) BKT_CASE(2) BKT_CASE(3) BKT_CASE(4) BKT_CASE(5) BKT_CASE(6) BKT_CASE(7) BKT_CASE(8)
+    BKT_CASE(9) BKT_CASE(10) BKT_CASE(11) BKT_CASE(12) BKT_CASE(13) BKT_CASE(14) BKT_CASE(15) BKT_CASE(16)
+#undef BKT_CASE
+    default:
+      return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// Split-K reduction: out[i] = P[0][i] + P[1][i] + ... in split order.
+__global__ void splitk_reduce_kernel(const float *__restrict__ P, int splits, int64_t n, float *__restrict__ out) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    float acc = 0.f;
+    for (int z = 0; z < splits; ++z) acc += P[(int64_t)z * n + i];
+    out[i] = acc;
+  }
+}
+
+cudaError_t launch_splitk_reduce(const float *P, int splits, int64_t n, float *out, cudaStream_t s) {
+  int64_t blocks = (n + 255) / 256;
+  if (blocks > 4096) blocks = 4096;
+  if (blocks < 1) blocks = 1;
+  splitk_reduce_kernel<<<(int)blocks, 256, 0, s>>>(P, splits, n, out);
+  return cudaGetLastError();
+}
+
+// Column sums over a token range: P[z][m] = sum_{k in split z} A[k*lda + m].
+__global__ void colsum_partial_kernel(const float *__restrict__ A, int64_t lda, int K, int M, float *__restrict__ P,
+                                      int splits) {
+  const int m = blockIdx.x * blockDim.x + threadIdx.x;
+  const int z = blockIdx.y;
+  if (m >= M) return;
+  const int chunk = (K + splits - 1) / splits;
+  const int k0 = z * chunk, k1 = min(K, k0 + chunk);
+  float acc = 0.f;
+  for (int k = k0; k < k1; ++k) acc += A[(int64_t)k * lda + m];
+  P[(int64_t)z * M + m] = acc;
+}
+
+cudaError_t launch_colsum_partial(const float *A, int64_t lda, int K, int M, float *P, int splits, cudaStream_t s) {
+  dim3 grid((M + 255) / 256, splits);
+  colsum_partial_kernel<<<grid, 256, 0, s>>>(A, lda, K, M, P, splits);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// a13: theta <- theta - lr * g, 16-byte vectors over the aligned body.
+__global__ void sgd_kernel(float *__restrict__ p, const float *__restrict__ g, int64_t n, float lr, int vec) {
+  const int64_t n4 = vec ? n / 4 : 0;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int64_t i0 = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  float4 *p4 = reinterpret_cast<float4 *>(p);
+  const float4 *g4 = reinterpret_cast<const float4 *>(g);
+  for (int64_t i = i0; i < n4; i += stride) {
+    float4 a = p4[i];
+    const float4 b = g4[i];
+    a.x = fmaf(-lr, b.x, a.x);
+    a.y = fmaf(-lr, b.y, a.y);
+    a.z = fmaf(-lr, b.z, a.z);
+    a.w = fmaf(-lr, b.w, a.w);
+    p4[i] = a;
+  }
+  for (int64_t i = n4 * 4 + i0; i < n; i += stride) p[i] = fmaf(-lr, g[i], p[i]);
+}
+
+cudaError_t launch_sgd(float *p, const float *g, int64_t n, float lr, cudaStream_t s) {
+  const int vec = ((reinterpret_cast<uintptr_t>(p) | reinterpret_cast<uintptr_t>(g)) & 15) == 0;
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  int64_t blocks = (n / 4 + 255) / 256;
+  if (blocks > 4LL * sms) blocks = 4LL * sms;
+  if (blocks < 1) blocks = 1;
+  sgd_kernel<<<(int)blocks, 256, 0, s>>>(p, g, n, lr, vec);
+  return cudaGetLastError();
+}
+
+}  // namespace bkt

@@ -1,0 +1,224 @@
+"""GPU parity: the CUDA training step (through the C ABI) against the fp64
+oracle, element by element per parameter block, on seeded synthetic inputs.
+Sizes let the oracle finish in seconds while spanning several tiles, clusters
+and ragged tails; the last tests use full-size batches of the workloads and
+check sampled per-sequence losses plus properties that hold at any size."""
+import math
+
+import numpy as np
+import pytest
+
+from paper_1708_05604_gb300 import binding, synth
+
+from gpu_util import BF16_TOL, FP32_TOL, compare, gpu_step, oracle_step
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built(cuda_device):
+    from paper_1708_05604_gb300 import build
+    build.build()
+    binding.lib()
+
+
+def tol_for(cfg):
+    return BF16_TOL if cfg.get("gemm_bf16") else FP32_TOL
+
+
+def make_case(wname, n, max_len, seed=0):
+    w = synth.WORKLOADS[wname]
+    ds = synth.make_workload(w, seed=seed, n_seqs=n, max_len=max_len)
+    cfg = w.model_cfg()
+    rng = np.random.default_rng(seed + 100)
+    params = synth.draw_params(rng, binding.param_count(cfg))
+    return cfg, ds, params
+
+
+# (workload, sequences, length cap): oracle-sized versions of every workload
+SMALL = [
+    ("lstm1_uni_h32", 16, None),
+    ("lstm1_bi_h128", 9, 260),
+    ("lstm3_bi_h256_bf16", 3, 70),
+    ("lstm2_uni_h512", 3, 90),
+    ("lstm3_bi_h256_bf16_bimodal", 3, 60),
+]
+
+
+@pytest.mark.parametrize("wname,n,max_len", SMALL)
+def test_step_parity_small(wname, n, max_len):
+    cfg, ds, params = make_case(wname, n, max_len)
+    lg, gg = gpu_step(cfg, ds, params)
+    lo, go = oracle_step(cfg, ds, params)
+    compare(cfg, lg, gg, lo, go, tol_for(cfg))
+
+
+def tiny_cfg(layers, bi, H, C=7):
+    return {"n_layers": layers, "bidirectional": bi, "in_dim": 4, "hidden": H, "n_classes": C,
+            "blank": 0}
+
+
+@pytest.mark.parametrize("layers,bi,H", [(1, True, 5), (2, True, 6), (2, False, 12), (3, True, 8)])
+def test_step_parity_odd_shapes(layers, bi, H):
+    """Hidden sizes that are not multiples of 4 or of the cluster size."""
+    cfg = tiny_cfg(layers, bi, H)
+    rng = np.random.default_rng(layers * 7 + H)
+    ds = synth.make_dataset([11, 1, 7, 30, 7, 2, 19], 3, rng, n_classes=cfg["n_classes"])
+    params = rng.uniform(-0.4, 0.4, size=binding.param_count(cfg)).astype(np.float32)
+    lg, gg = gpu_step(cfg, ds, params)
+    lo, go = oracle_step(cfg, ds, params)
+    compare(cfg, lg, gg, lo, go, FP32_TOL)
+
+
+def test_edge_cases_one_step():
+    """Length-1 sequence, empty label, repeated labels, no alignment, equal lengths."""
+    cfg = synth.WORKLOADS["lstm1_bi_h128"].model_cfg()
+    rng = np.random.default_rng(3)
+    ds = synth.make_dataset([1, 40, 40, 40, 25, 9, 6], 3, rng)
+    lab = ds.labels.copy()
+    U = ds.label_lengths.copy()
+    # seq 1: no labels at all
+    U[1] = 0
+    # seq 2: every label the same (needs blanks between repeats)
+    # seq 5: 3 labels that all repeat -> needs 5 steps; length 9 fits
+    # seq 6: length 6 with 4 identical labels -> needs 7 steps: no alignment
+    U[6] = 4
+    labels = []
+    for i in range(ds.n):
+        if i == 2:
+            labels.append(np.full(U[i], 17, np.int32))
+        elif i == 5:
+            labels.append(np.array([4, 4, 4], np.int32)[:U[i]])
+        elif i == 6:
+            labels.append(np.full(4, 9, np.int32))
+        else:
+            labels.append(rng.integers(1, 81, size=U[i]).astype(np.int32))
+    labels = np.concatenate(labels)
+    off = np.zeros(ds.n + 1, np.int64)
+    np.cumsum(U, out=off[1:])
+    ds = synth.Dataset(ds.lengths, ds.x, ds.x_off, U.astype(np.int32), labels, off)
+    params = synth.draw_params(rng, binding.param_count(cfg))
+    lg, gg = gpu_step(cfg, ds, params)
+    lo, go = oracle_step(cfg, ds, params)
+    assert math.isinf(lo[6]) and math.isinf(lg[6]) and lg[6] > 0
+    compare(cfg, lg, gg, lo, go, FP32_TOL)
+
+
+def test_single_sequence_and_permutation_invariance():
+    """A sequence's loss does not depend on its batch-mates or batch order
+    (the packed layout adds no padding to the arithmetic)."""
+    cfg, ds, params = make_case("lstm1_bi_h128", 12, 200, seed=5)
+    lg, gg = gpu_step(cfg, ds, params)
+    perm = np.array([7, 3, 11, 0, 5, 9, 1, 2, 10, 4, 8, 6])
+    lp, gp = gpu_step(cfg, ds, params, seq_ids=perm)
+    np.testing.assert_allclose(lp, lg[perm], rtol=2e-6)
+    for i in (0, 4, 11):
+        l1, g1 = gpu_step(cfg, ds, params, seq_ids=[i])
+        assert abs(l1[0] - lg[i]) <= 2e-6 * abs(lg[i])
+    # the batch gradient is the sum of two halves' gradients
+    la, ga = gpu_step(cfg, ds, params, seq_ids=np.arange(6))
+    lb, gb = gpu_step(cfg, ds, params, seq_ids=np.arange(6, 12))
+    assert np.linalg.norm(ga + gb - gg) <= 1e-5 * np.linalg.norm(gg)
+
+
+def test_step_is_deterministic():
+    cfg, ds, params = make_case("lstm1_bi_h128", 10, 150, seed=2)
+    l1, g1 = gpu_step(cfg, ds, params)
+    l2, g2 = gpu_step(cfg, ds, params)
+    assert np.array_equal(l1, l2) and np.array_equal(g1, g2)
+
+
+def test_sgd_update():
+    """p - lr * g with one fp32 rounding: within one ulp of the operands'
+    magnitude of the exact value (lr as the fp32 the kernel receives)."""
+    import torch
+    rng = np.random.default_rng(0)
+
+    def check(p, g, lr, got):
+        lr32 = np.float64(np.float32(lr))
+        exact = p.astype(np.float64) - lr32 * g.astype(np.float64)
+        scale = np.abs(p.astype(np.float64)) + np.abs(lr32 * g.astype(np.float64))
+        assert np.all(np.abs(got.astype(np.float64) - exact) <= 2.0 ** -23 * scale + 1e-30)
+
+    for n in (1, 5, 7409, 100003):
+        p = rng.standard_normal(n).astype(np.float32)
+        g = rng.standard_normal(n).astype(np.float32)
+        tp, tg = torch.from_numpy(p).cuda(), torch.from_numpy(g).cuda()
+        binding.sgd_update(tp, tg, 1e-3)
+        torch.cuda.synchronize()
+        check(p, g, 1e-3, tp.cpu().numpy())
+    # unaligned views take the scalar path
+    tp = torch.from_numpy(p).cuda()
+    tg = torch.from_numpy(g).cuda()
+    binding.sgd_update(tp[1:], tg[1:], 0.5)
+    torch.cuda.synchronize()
+    check(p[1:], g[1:], 0.5, tp[1:].cpu().numpy())
+
+
+def test_argument_errors():
+    import torch
+    cfg, ds, params = make_case("lstm1_uni_h32", 4, 50)
+    ctx = binding.Ctx(cfg, max_tokens=100, max_batch=2, max_label_len=4)
+    dd = binding.DeviceDataset(ds)
+    p = torch.from_numpy(params).cuda()
+    g = torch.zeros_like(p)
+    loss = torch.zeros(4, device="cuda")
+    with pytest.raises(binding.BktError) as e:
+        ctx.step(dd, [0, 1, 2], p, g, loss)       # more sequences than max_batch
+    assert e.value.rc == binding.BKT_EINVAL
+    small = binding.Ctx(cfg, max_tokens=10, max_batch=2, max_label_len=40)
+    with pytest.raises(binding.BktError):
+        small.step(dd, [0, 1], p, g, loss)        # more tokens than the ctx holds
+    short = binding.Ctx(cfg, max_tokens=1000, max_batch=4, max_label_len=0)
+    with pytest.raises(binding.BktError):
+        short.step(dd, [0, 1], p, g, loss)        # labels longer than max_label_len
+    # a label equal to the blank is caught on the device
+    bad = synth.Dataset(ds.lengths, ds.x, ds.x_off, ds.label_lengths, ds.labels.copy(), ds.lab_off)
+    bad.labels[0] = 0
+    ctx2 = binding.Ctx(cfg, max_tokens=int(ds.lengths.sum()), max_batch=4,
+                       max_label_len=int(ds.label_lengths.max()))
+    ctx2.step(binding.DeviceDataset(bad), [0, 1, 2, 3], p, g, loss)
+    with pytest.raises(binding.BktError) as e:
+        ctx2.sync_status()
+    assert e.value.rc == binding.BKT_EDEVICE
+    ctx2.sync_status()  # cleared
+
+
+# ---------------------------------------------------------------------------
+# Full-size batches, launched as the benchmark launches them.
+
+def full_batch(wname, Q, which="longest", seed=0):
+    w = synth.WORKLOADS[wname]
+    ds = synth.make_workload(w, seed=seed)
+    plan = binding.plan_buckets(ds.lengths, Q, w.batch, seed=seed, epoch=0)
+    batches = [plan["order"][plan["batch_off"][k]:plan["batch_off"][k + 1]]
+               for k in range(plan["n_batches"])]
+    if which == "longest":
+        ids = max(batches, key=lambda b: int(ds.lengths[b].max()))
+    else:
+        ids = batches[0]
+    return w, ds, ids
+
+
+@pytest.mark.parametrize("wname,Q", [("lstm1_bi_h128", 4), ("lstm1_bi_h128", 1),
+                                     ("lstm1_uni_h32", 2), ("lstm2_uni_h512", 4),
+                                     ("lstm3_bi_h256_bf16", 16)])
+def test_full_size_batch_sampled(wname, Q):
+    w, ds, ids = full_batch(wname, Q)
+    cfg = w.model_cfg()
+    params = synth.draw_params(np.random.default_rng(1), binding.param_count(cfg))
+    dd = binding.DeviceDataset(ds)
+    lg, gg = gpu_step(cfg, ds, params, seq_ids=ids, dd=dd)
+    assert np.all(np.isfinite(gg))
+    # sampled outputs: the oracle's loss of a few sequences, one at a time
+    # (the shortest ones, so the oracle stays within seconds)
+    order = np.argsort(ds.lengths[ids])
+    n_sample = 1 if cfg["hidden"] >= 512 else 2
+    for pos in order[:n_sample]:
+        lo, _ = oracle_step(cfg, ds, params, seq_ids=[ids[pos]])
+        assert abs(lg[pos] - lo[0]) <= tol_for(cfg) * abs(lo[0]), (pos, lg[pos], lo[0])
+    # linearity over sequences: grad(batch) = grad(first half) + grad(second half)
+    h = ids.size // 2
+    _, ga = gpu_step(cfg, ds, params, seq_ids=ids[:h], dd=dd)
+    _, gb = gpu_step(cfg, ds, params, seq_ids=ids[h:], dd=dd)
+    assert np.linalg.norm(ga + gb - gg) <= 1e-4 * np.linalg.norm(gg)

@@ -1,0 +1,94 @@
+"""Host-side checks of libbkt that need no GPU: the library loads and exports
+every entry point include/bkt.h declares, the planner matches the oracle
+bit for bit, and the parameter layout and argument checks hold."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_1708_05604_gb300 import binding, synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_1708_05604_gb300 import build
+    build.build()
+    return binding.lib()
+
+
+def header_functions():
+    names = set()
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            txt = open(os.path.join(ROOT, "include", fn)).read()
+            txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+            names |= set(re.findall(r"\b(bkt_\w+)\s*\(", txt))
+    return sorted(names)
+
+
+def test_exports_every_declared_symbol(lib):
+    names = header_functions()
+    assert len(names) >= 12
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in include/ but not exported"
+    assert set(binding.EXPORTS) == set(names)
+
+
+PLAN_CASES = [(w, Q) for w in synth.WORKLOAD_ORDER for Q in synth.WORKLOADS[w].bucket_counts]
+
+
+@pytest.mark.parametrize("wname,Q", PLAN_CASES)
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_planner_bit_exact_vs_oracle(lib, wname, Q, seed):
+    w = synth.WORKLOADS[wname]
+    rng = np.random.default_rng(seed)
+    L = synth.draw_lengths(rng, w.n_seqs, w.length_dist)
+    for epoch in (0, 3):
+        a = binding.plan_buckets(L, Q, w.batch, seed=seed, epoch=epoch)
+        b = oracle.plan(L, Q, w.batch, seed=seed, epoch=epoch)
+        for k in ("bounds", "order", "batch_off", "batch_bucket"):
+            assert np.array_equal(a[k], b[k]), (k, wname, Q, seed, epoch)
+        assert a["dp_cost"] == b["dp_cost"]
+        assert a["n_batches"] == b["n_batches"]
+        assert a["padded_timesteps"] == b["padded_timesteps"]
+        assert a["unpadded_timesteps"] == int(L.sum())
+
+
+@pytest.mark.parametrize("seed", range(30))
+def test_planner_small_random_vs_oracle(lib, seed):
+    rng = np.random.default_rng(500 + seed)
+    lmax = int(rng.integers(1, 40))
+    n = int(rng.integers(1, 60))
+    L = rng.integers(1, lmax + 1, size=n).astype(np.int32)
+    for Q in range(1, min(int(L.max()), 8) + 1):
+        B = int(rng.integers(1, 9))
+        a = binding.plan_buckets(L, Q, B, seed=seed, epoch=seed % 3)
+        b = oracle.plan(L, Q, B, seed=seed, epoch=seed % 3)
+        for k in ("bounds", "order", "batch_off", "batch_bucket"):
+            assert np.array_equal(a[k], b[k]), (k, L.tolist(), Q, B)
+        assert a["dp_cost"] == b["dp_cost"]
+
+
+def test_planner_rejects_bad_input(lib):
+    with pytest.raises(binding.BktError) as e:
+        binding.plan_buckets([3, 0, 2], 1, 2, 0)
+    assert e.value.rc == binding.BKT_EINVAL
+    with pytest.raises(binding.BktError):
+        binding.plan_buckets([3, 1, 2], 4, 2, 0)   # Q > max length
+    with pytest.raises(binding.BktError):
+        binding.plan_buckets([3, 1, 2], 1, 0, 0)   # batch 0
+    assert "buckets" in lib.bkt_last_error().decode()
+
+
+def test_param_count_matches_oracle_layout(lib):
+    for w in synth.WORKLOADS.values():
+        cfg = w.model_cfg()
+        assert binding.param_count(cfg) == oracle.param_count(
+            cfg["n_layers"], cfg["bidirectional"], cfg["in_dim"], cfg["hidden"], cfg["n_classes"])
+    bad = dict(synth.WORKLOADS["lstm1_uni_h32"].model_cfg(), blank=81)
+    assert binding.param_count(bad) == 0
