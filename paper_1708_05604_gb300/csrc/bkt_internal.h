@@ -91,8 +91,11 @@ cudaError_t launch_ctc_grad(const DevIdx &ix, float *logp_dlogit, int C, int bla
                             const int32_t *labels, const float *alpha, const float *beta,
                             const int32_t *row_ok, cudaStream_t s);
 
-// Cluster geometry of the recurrent kernels for one layer.
+// Geometry of the recurrent kernels for one layer.
+//   mode 1: one CTA per bc rows holds all of W_hh (H in {32, 64, 128});
+//   mode 0: a cluster of cs CTAs per bc rows splits the hidden units.
 struct RecGeom {
+  int mode;
   int cs;        // CTAs per cluster (hidden units split cs ways)
   int bc;        // batch rows per cluster
   int ks;        // threads sharing one (row, unit) pair along k (power of 2 <= 8)
@@ -118,6 +121,11 @@ struct RecArgs {
 cudaError_t launch_lstm_fwd(const RecArgs &a, const RecGeom &g, cudaStream_t s);
 // a11: BPTT for both directions; Z[d] holds the gates on entry and dz on exit.
 cudaError_t launch_lstm_bwd(const RecArgs &a, const RecGeom &g, cudaStream_t s);
+
+// Single-CTA recurrent kernels (k_lstm_cta.cu).
+bool cta_supported(int H);
+int cta_rows_per_block(int H, int b, int dirs, int sm_count);
+cudaError_t launch_lstm_cta(const RecArgs &a, int bc, bool bwd, cudaStream_t s);
 
 // a13
 cudaError_t launch_sgd(float *p, const float *g, int64_t n, float lr, cudaStream_t s);

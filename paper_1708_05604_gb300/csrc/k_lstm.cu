@@ -331,6 +331,15 @@ RecGeom plan_recurrent(int H, int b, int dirs, int sm_count) {
   const int Tcap = kTokSmemCap - 1;
   const size_t lim = 220 * 1024;
   RecGeom g{};
+  if (cta_supported(H)) {
+    g.mode = 1;
+    g.cs = 1;
+    g.bc = cta_rows_per_block(H, b, dirs, sm_count);
+    g.ks = 1;
+    g.threads = 4 * H;
+    g.w_smem = 1;
+    return g;
+  }
   int cs = 16;
   while (cs > 1 && (H % cs != 0 || H / cs < 8)) cs >>= 1;
   for (;; cs >>= 1) {
@@ -395,12 +404,14 @@ cudaError_t launch_rec(K kernel, const RecArgs &a, const RecGeom &g, bool bwd, c
 }  // namespace
 
 cudaError_t launch_lstm_fwd(const RecArgs &a, const RecGeom &g, cudaStream_t s) {
+  if (g.mode == 1) return launch_lstm_cta(a, g.bc, false, s);
   if (a.H % g.cs != 0) return cudaErrorInvalidValue;
   if (!g.w_smem && (a.H % 4) != 0) return cudaErrorInvalidValue;
   return g.w_smem ? launch_rec(lstm_fwd_kernel<true>, a, g, false, s) : launch_rec(lstm_fwd_kernel<false>, a, g, false, s);
 }
 
 cudaError_t launch_lstm_bwd(const RecArgs &a, const RecGeom &g, cudaStream_t s) {
+  if (g.mode == 1) return launch_lstm_cta(a, g.bc, true, s);
   if (a.H % g.cs != 0) return cudaErrorInvalidValue;
   if (!g.w_smem && (a.H % 4) != 0) return cudaErrorInvalidValue;
   return g.w_smem ? launch_rec(lstm_bwd_kernel<true>, a, g, true, s) : launch_rec(lstm_bwd_kernel<false>, a, g, true, s);
