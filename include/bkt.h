@@ -152,6 +152,34 @@ int bkt_lstm_ctc_step(bkt_ctx *ctx, const bkt_batch *batch,
                       const float *params, float *grads, float *loss,
                       void *stream);
 
+/* The same training step without a ctx and without allocating anything.
+ * The paper has no counterpart: this entry point exists for callers that
+ * cannot allocate device memory, such as a plugin running inside a host
+ * framework that owns every byte of GPU memory through its own pool, or a
+ * process whose memory budget is fixed at start-up and may not grow.
+ * Instead of a ctx workspace it uses one device array of
+ * BKT_STATIC_SCRATCH_BYTES that is part of the library image; every GPU
+ * that loads the library holds that array until the process exits.
+ *   - Arguments and results are exactly those of bkt_lstm_ctc_step; the
+ *     limits are n_seq <= 512, label_lengths <= 1023, and a workspace that
+ *     fits the array (roughly (26 H + C + 8 S) * 4 bytes per token for one
+ *     bidirectional layer, S = 2U + 1).  A batch beyond them returns
+ *     BKT_EINVAL with the needed and available bytes in bkt_last_error().
+ *   - The first call on a device looks up the array's address on that
+ *     device, so make that first call before any stream capture.
+ *   - All calls share the one array, and it keeps the previous call's
+ *     contents (the device error flags are cleared at the start of each
+ *     call).  Calls whose GPU work overlaps, on different streams or from
+ *     different threads, race on it: order them on one stream.
+ *   - The host waits for earlier work on `stream` before uploading the
+ *     batch's index arrays (they go through pageable host memory).
+ *   - There is no status query: a label outside 1..C-1 shows up as a NaN
+ *     loss for that sequence, which then adds nothing to grads.          */
+#define BKT_STATIC_SCRATCH_BYTES (64u * 1024u * 1024u)
+int bkt_lstm_ctc_step_static(const bkt_model_cfg *cfg, const bkt_batch *batch,
+                             const float *params, float *grads, float *loss,
+                             void *stream);
+
 /* params[i] -= lr * grads[i] for i < n (device fp32 pointers; 16-byte
  * vectors when both are 16-byte aligned), enqueued on `stream`.          */
 int bkt_sgd_update(float *params, const float *grads, int64_t n, float lr,

@@ -21,7 +21,8 @@ BKT_GEMM_FP32, BKT_GEMM_BF16 = 0, 1
 
 # Every symbol include/bkt.h declares.
 EXPORTS = ("bkt_plan_buckets", "bkt_plan_get", "bkt_plan_free", "bkt_param_count",
-           "bkt_ctx_create", "bkt_ctx_destroy", "bkt_lstm_ctc_step", "bkt_sgd_update",
+           "bkt_ctx_create", "bkt_ctx_destroy", "bkt_lstm_ctc_step", "bkt_lstm_ctc_step_static",
+           "bkt_sgd_update",
            "bkt_ctx_sync_status", "bkt_ctx_set_timing", "bkt_ctx_kernel_times",
            "bkt_last_error")
 
@@ -87,6 +88,8 @@ def lib() -> ctypes.CDLL:
         L.bkt_ctx_destroy.argtypes = [vp]
         L.bkt_ctx_destroy.restype = None
         L.bkt_lstm_ctc_step.argtypes = [vp, ctypes.POINTER(Batch), vp, vp, vp, vp]
+        L.bkt_lstm_ctc_step_static.argtypes = [ctypes.POINTER(ModelCfg), ctypes.POINTER(Batch), vp,
+                                               vp, vp, vp]
         L.bkt_sgd_update.argtypes = [vp, vp, ctypes.c_int64, ctypes.c_float, vp]
         L.bkt_ctx_sync_status.argtypes = [vp]
         L.bkt_ctx_set_timing.argtypes = [vp, ctypes.c_int32]
@@ -94,6 +97,7 @@ def lib() -> ctypes.CDLL:
         L.bkt_last_error.argtypes = []
         L.bkt_last_error.restype = ctypes.c_char_p
         for name in ("bkt_plan_buckets", "bkt_plan_get", "bkt_ctx_create", "bkt_lstm_ctc_step",
+                     "bkt_lstm_ctc_step_static",
                      "bkt_sgd_update", "bkt_ctx_sync_status", "bkt_ctx_set_timing",
                      "bkt_ctx_kernel_times"):
             getattr(L, name).restype = ctypes.c_int
@@ -168,6 +172,31 @@ def sgd_update(params, grads, lr: float, stream=None):
                                 ctypes.c_float(lr), _stream_handle(stream)))
 
 
+def _batch(lengths, x_offsets, label_lengths, label_offsets, x_ptr: int, labels_ptr: int):
+    """A bkt_batch plus the numpy arrays it points into (kept alive together)."""
+    L, UL = _i32(lengths), _i32(label_lengths)
+    XO, LO = _i64(x_offsets), _i64(label_offsets)
+    b = Batch(L.size, _ptr(L, ctypes.c_int32), _ptr(XO, ctypes.c_int64),
+              _ptr(UL, ctypes.c_int32), _ptr(LO, ctypes.c_int64),
+              ctypes.c_void_p(x_ptr), ctypes.c_void_p(labels_ptr))
+    return b, (L, UL, XO, LO)
+
+
+def step_static(cfg: dict, dd: "DeviceDataset", seq_ids, params, grads, loss, stream=None):
+    """bkt_lstm_ctc_step_static: the step with the library's fixed device
+    scratch array instead of a ctx (for callers that cannot allocate)."""
+    ids = np.asarray(seq_ids, dtype=np.int64)
+    c = model_cfg(cfg)
+    b, keep = _batch(dd.lengths[ids], dd.x_off[ids], dd.label_lengths[ids], dd.lab_off[ids],
+                     dd.x.data_ptr(), dd.labels.data_ptr())
+    _check(lib().bkt_lstm_ctc_step_static(ctypes.byref(c), ctypes.byref(b),
+                                          ctypes.c_void_p(params.data_ptr()),
+                                          ctypes.c_void_p(grads.data_ptr()),
+                                          ctypes.c_void_p(loss.data_ptr()),
+                                          _stream_handle(stream)))
+    del keep
+
+
 class DeviceDataset:
     """A synth.Dataset with x and labels resident on the GPU (torch tensors)
     and the per-sequence offsets on the host."""
@@ -209,11 +238,7 @@ class Ctx:
     def step_raw(self, lengths, x_offsets, label_lengths, label_offsets, x_ptr: int,
                  labels_ptr: int, params, grads, loss, stream=None):
         """bkt_lstm_ctc_step with explicit host index arrays and device bases."""
-        L, UL = _i32(lengths), _i32(label_lengths)
-        XO, LO = _i64(x_offsets), _i64(label_offsets)
-        b = Batch(L.size, _ptr(L, ctypes.c_int32), _ptr(XO, ctypes.c_int64),
-                  _ptr(UL, ctypes.c_int32), _ptr(LO, ctypes.c_int64),
-                  ctypes.c_void_p(x_ptr), ctypes.c_void_p(labels_ptr))
+        b, keep = _batch(lengths, x_offsets, label_lengths, label_offsets, x_ptr, labels_ptr)
         _check(lib().bkt_lstm_ctc_step(self.h, ctypes.byref(b),
                                        ctypes.c_void_p(params.data_ptr()),
                                        ctypes.c_void_p(grads.data_ptr()),

@@ -8,6 +8,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <new>
 #include <string>
 #include <vector>
@@ -24,6 +25,13 @@ int set_err(int code, const char *fmt, ...) {
   va_start(ap, fmt);
   vsnprintf(buf, sizeof buf, fmt, ap);
   va_end(ap);
+  g_err = buf;
+  return code;
+}
+
+int vset_err(int code, const char *fmt, va_list ap) {
+  char buf[512];
+  vsnprintf(buf, sizeof buf, fmt, ap);
   g_err = buf;
   return code;
 }
@@ -177,15 +185,15 @@ extern "C" const char *bkt_last_error(void) { return g_err.c_str(); }
 namespace {
 
 bool cfg_ok(const bkt_model_cfg *c) {
-  return c && c->n_layers >= 1 && c->n_layers <= 64 && (c->bidirectional == 0 || c->bidirectional == 1) &&
-         c->in_dim >= 1 && c->in_dim <= 16 && c->hidden >= 1 && c->hidden <= 2048 &&
-         c->n_classes >= 2 && c->n_classes <= 1024 && c->blank >= 0 && c->blank < c->n_classes &&
-         (c->gemm_precision == BKT_GEMM_FP32 || c->gemm_precision == BKT_GEMM_BF16);
+  return c && c->n_layers >= 1 && c->n_layers <= bkt::kMaxLayers &&
+         (c->bidirectional == 0 || c->bidirectional == 1) && c->in_dim >= 1 && c->in_dim <= 16 &&
+         c->hidden >= 1 && c->hidden <= 2048 && c->n_classes >= 2 && c->n_classes <= 128 && c->blank >= 0 &&
+         c->blank < c->n_classes && (c->gemm_precision == BKT_GEMM_FP32 || c->gemm_precision == BKT_GEMM_BF16);
 }
 
 struct Layout {
   int dirs, H, C, L, D0;
-  std::vector<int64_t> w_ih;  // [L*dirs] offset of W_ih of (layer, dir)
+  int64_t w_ih[2 * bkt::kMaxLayers];  // offset of W_ih of (layer, dir) at [l*dirs + d]
   int64_t w_out, b_out, total;
   int D(int l) const { return l == 0 ? D0 : dirs * H; }
   int64_t w_hh(int l, int d) const { return w_ih[l * dirs + d] + (int64_t)4 * H * D(l); }
@@ -203,7 +211,7 @@ Layout make_layout(const bkt_model_cfg *c) {
   int64_t off = 0;
   for (int l = 0; l < lo.L; ++l)
     for (int d = 0; d < lo.dirs; ++d) {
-      lo.w_ih.push_back(off);
+      lo.w_ih[l * lo.dirs + d] = off;
       off += lo.stride(l);
     }
   lo.w_out = off;
@@ -212,6 +220,287 @@ Layout make_layout(const bkt_model_cfg *c) {
   off += lo.C;
   lo.total = off;
   return lo;
+}
+
+// Layout of the per-step index block (same in staging and on the device).
+struct IdxLayout {
+  size_t row_len, row_lab_len, row_orig, row_xoff, row_lab_off, row_ctc_off, tok_off, bytes;
+};
+IdxLayout idx_layout(int32_t b, int64_t T) {
+  IdxLayout L;
+  size_t o = 0;
+  auto take = [&](size_t n) {
+    size_t r = o;
+    o += (n + 15) & ~size_t(15);
+    return r;
+  };
+  L.row_len = take(4 * (size_t)b);
+  L.row_lab_len = take(4 * (size_t)b);
+  L.row_orig = take(4 * (size_t)b);
+  L.row_xoff = take(8 * (size_t)b);
+  L.row_lab_off = take(8 * (size_t)b);
+  L.row_ctc_off = take(8 * (size_t)b);
+  L.tok_off = take(4 * (size_t)(T + 1));
+  L.bytes = o;
+  return L;
+}
+
+// Host checks of one batch against capacities.  On success: tokens, the
+// largest 2U+1 and the CTC table cells sum_i L_i (2 U_i + 1).
+int check_batch(const bkt_batch *bt, int64_t max_tokens, int32_t max_batch, int32_t max_label_len,
+                int64_t *n_tok, int32_t *S_max, int64_t *ctc_cells) {
+  const int32_t b = bt->n_seq;
+  if (b < 1 || b > max_batch) return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: n_seq %d outside 1..%d", b, max_batch);
+  if (!bt->lengths || !bt->x_offsets || !bt->label_lengths || !bt->label_offsets || !bt->x || !bt->labels)
+    return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: NULL batch array");
+  int64_t nt = 0, cells = 0;
+  int32_t sm = 1;
+  for (int32_t i = 0; i < b; ++i) {
+    if (bt->lengths[i] < 1) return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: lengths[%d] = %d < 1", i, bt->lengths[i]);
+    if (bt->label_lengths[i] < 0 || bt->label_lengths[i] > max_label_len)
+      return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: label_lengths[%d] = %d outside 0..%d", i, bt->label_lengths[i],
+                     max_label_len);
+    if (bt->x_offsets[i] < 0 || bt->label_offsets[i] < 0)
+      return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: negative offset for sequence %d", i);
+    nt += bt->lengths[i];
+    sm = std::max(sm, 2 * bt->label_lengths[i] + 1);
+    cells += (int64_t)bt->lengths[i] * (2 * bt->label_lengths[i] + 1);
+  }
+  if (nt > max_tokens)
+    return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: %lld tokens exceed the capacity %lld", (long long)nt,
+                   (long long)max_tokens);
+  *n_tok = nt;
+  *S_max = sm;
+  *ctc_cells = cells;
+  return BKT_OK;
+}
+
+// a4, host part: with `perm` the batch's stable longest-first order, fills
+// the index block at `st` and returns its device view at `dev`.
+bkt::DevIdx fill_index_block(const bkt_batch *bt, const int32_t *perm, int32_t T, int64_t n_tok, int32_t S_max,
+                             const IdxLayout &il, char *st, char *dev, int32_t *tok_t, int32_t *tok_r) {
+  const int32_t b = bt->n_seq;
+  int32_t *row_len = (int32_t *)(st + il.row_len), *row_lab_len = (int32_t *)(st + il.row_lab_len),
+          *row_orig = (int32_t *)(st + il.row_orig), *tok_off = (int32_t *)(st + il.tok_off);
+  int64_t *row_xoff = (int64_t *)(st + il.row_xoff), *row_lab_off = (int64_t *)(st + il.row_lab_off),
+          *row_ctc_off = (int64_t *)(st + il.row_ctc_off);
+  int64_t ctc_off = 0;
+  for (int32_t r = 0; r < b; ++r) {
+    const int32_t i = perm[r];
+    row_len[r] = bt->lengths[i];
+    row_lab_len[r] = bt->label_lengths[i];
+    row_orig[r] = i;
+    row_xoff[r] = bt->x_offsets[i];
+    row_lab_off[r] = bt->label_offsets[i];
+    row_ctc_off[r] = ctc_off;
+    ctc_off += (int64_t)bt->lengths[i] * (2 * bt->label_lengths[i] + 1);
+  }
+  int32_t active = b, acc = 0;
+  for (int32_t t = 0; t < T; ++t) {
+    while (active > 0 && row_len[active - 1] <= t) --active;
+    tok_off[t] = acc;
+    acc += active;
+  }
+  tok_off[T] = acc;
+  bkt::DevIdx ix;
+  ix.b = b;
+  ix.T = T;
+  ix.n_tok = (int32_t)n_tok;
+  ix.S_max = S_max;
+  ix.row_len = (const int32_t *)(dev + il.row_len);
+  ix.row_lab_len = (const int32_t *)(dev + il.row_lab_len);
+  ix.row_orig = (const int32_t *)(dev + il.row_orig);
+  ix.row_xoff = (const int64_t *)(dev + il.row_xoff);
+  ix.row_lab_off = (const int64_t *)(dev + il.row_lab_off);
+  ix.row_ctc_off = (const int64_t *)(dev + il.row_ctc_off);
+  ix.tok_off = (const int32_t *)(dev + il.tok_off);
+  ix.tok_t = tok_t;
+  ix.tok_r = tok_r;
+  return ix;
+}
+
+struct Launch {
+  bkt::KernelTimer *timer;
+  cudaStream_t s;
+  const char *failed = nullptr;
+  cudaError_t err = cudaSuccess;
+  template <typename F>
+  bool run(const char *name, F &&f) {
+    if (failed) return false;
+    if (timer) timer->begin(name, s);
+    cudaError_t e = f();
+    if (timer) timer->end(s);
+    if (e != cudaSuccess) {
+      failed = name;
+      err = e;
+      return false;
+    }
+    return true;
+  }
+};
+
+// Number of token splits for a reduction over n_tok rows into an M x N block.
+int choose_splits(int M, int N, int n_tok, int sm_count, size_t part_cap) {
+  const int tiles = ((M + 63) / 64) * ((N + 63) / 64);
+  int s = std::max(1, (2 * sm_count + tiles - 1) / tiles);
+  s = std::min(s, std::max(1, n_tok / 256));
+  s = std::min(s, 64);
+  while (s > 1 && (size_t)s * M * N > part_cap) --s;
+  return s;
+}
+
+// Largest M x N block a token reduction writes (weights and biases).
+size_t max_reduce_block(const Layout &lo) {
+  const size_t DH = (size_t)lo.dirs * lo.H, H = lo.H;
+  size_t m = std::max<size_t>((size_t)lo.C * DH, 4 * H * std::max<size_t>(DH, (size_t)lo.D0));
+  return std::max(m, 4 * H * H);
+}
+
+// Enqueues every kernel of one step (a4 gather .. a12) on `s`.
+int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepBufs &w, const bkt::RecGeom *geom,
+                    const bkt::DevIdx &ix, const bkt_batch *bt, const float *params, float *grads, float *loss,
+                    cudaStream_t s, bkt::KernelTimer *timer, int sm_count) {
+  const int H = lo.H, dirs = lo.dirs, DH = dirs * H, C = lo.C, NT = ix.n_tok;
+  Launch L{timer, s};
+
+  // ---- a4: packed time-major input
+  L.run("layout_gather", [&] { return bkt::launch_layout(ix, bt->x, lo.D0, w.X, w.tok_t, w.tok_r, w.prev_tok, s); });
+
+  // ---- forward, layer by layer
+  for (int l = 0; l < lo.L; ++l) {
+    float *Zl[2] = {w.Z[l * dirs], dirs > 1 ? w.Z[l * dirs + 1] : nullptr};
+    if (l == 0) {
+      // a5, narrow input: both directions in one launch
+      L.run("proj_narrow", [&] {
+        return bkt::launch_proj_narrow(w.X, NT, lo.D0, params, lo.w_ih[0], lo.stride(0), H, dirs, Zl, s);
+      });
+    } else {
+      for (int d = 0; d < dirs; ++d) {
+        bkt::GemmArgs g{};
+        g.M = NT;
+        g.N = 4 * H;
+        g.K = DH;
+        g.A = w.Y[l - 1];
+        g.lda = DH;
+        g.B = params + lo.w_ih[l * dirs + d];
+        g.ldb = DH;
+        g.C = Zl[d];
+        g.ldc = 4 * H;
+        g.bias = params + lo.bias(l, d);
+        g.splits = 1;
+        L.run("gemm_proj", [&] { return bkt::launch_gemm_f32(false, true, g, s); });
+      }
+    }
+    bkt::RecArgs ra{};
+    ra.ix = ix;
+    ra.H = H;
+    ra.dirs = dirs;
+    for (int d = 0; d < dirs; ++d) {
+      ra.Z[d] = Zl[d];
+      ra.Cst[d] = w.Cst[l * dirs + d];
+      ra.Whh[d] = params + lo.w_hh(l, d);
+    }
+    ra.Y = w.Y[l];
+    L.run("lstm_fwd", [&] { return bkt::launch_lstm_fwd(ra, geom[l], s); });
+  }
+
+  // ---- a7: output layer and log-softmax
+  float *Ytop = w.Y[lo.L - 1];
+  L.run("out_logsoftmax", [&] {
+    return bkt::launch_out_logsoftmax(Ytop, NT, DH, params + lo.w_out, params + lo.b_out, C, w.logit, s);
+  });
+  // ---- a8, a9: CTC
+  L.run("ctc_tables", [&] {
+    return bkt::launch_ctc_tables(ix, w.logit, C, cfg.blank, bt->labels, w.alpha, w.beta, loss, w.row_ok, w.status, s);
+  });
+  L.run("ctc_grad", [&] {
+    return bkt::launch_ctc_grad(ix, w.logit, C, cfg.blank, bt->labels, w.alpha, w.beta, w.row_ok, s);
+  });
+
+  // ---- a10: output layer backward
+  auto reduce_tokens = [&](const char *name, const float *A, int64_t lda, int M, const float *B, int64_t ldb,
+                           const int32_t *gather, int N, float *out) {
+    bkt::GemmArgs g{};
+    g.M = M;
+    g.N = N;
+    g.K = NT;
+    g.A = A;
+    g.lda = lda;
+    g.B = B;
+    g.ldb = ldb;
+    g.gather = gather;
+    g.P = w.part;
+    g.splits = choose_splits(M, N, NT, sm_count, w.part_floats);
+    L.run(name, [&] { return bkt::launch_gemm_f32(true, false, g, s); });
+    L.run("splitk_reduce", [&] { return bkt::launch_splitk_reduce(w.part, g.splits, (int64_t)M * N, out, s); });
+  };
+  auto bias_grad = [&](const float *A, int64_t lda, int M, float *out) {
+    int splits = std::min(64, std::max(1, std::min(2 * sm_count / std::max(1, (M + 255) / 256), NT / 64)));
+    while (splits > 1 && (size_t)splits * M > w.part_floats) --splits;
+    L.run("colsum", [&] { return bkt::launch_colsum_partial(A, lda, NT, M, w.part, splits, s); });
+    L.run("splitk_reduce", [&] { return bkt::launch_splitk_reduce(w.part, splits, M, out, s); });
+  };
+  reduce_tokens("gemm_dw_out", w.logit, C, C, Ytop, DH, nullptr, DH, grads + lo.w_out);
+  bias_grad(w.logit, C, C, grads + lo.b_out);
+  {
+    bkt::GemmArgs g{};
+    g.M = NT;
+    g.N = DH;
+    g.K = C;
+    g.A = w.logit;
+    g.lda = C;
+    g.B = params + lo.w_out;
+    g.ldb = DH;
+    g.C = w.dY;
+    g.ldc = DH;
+    g.splits = 1;
+    L.run("gemm_dy_out", [&] { return bkt::launch_gemm_f32(false, false, g, s); });
+  }
+
+  // ---- a11, a12: BPTT and weight gradients, top layer first
+  for (int l = lo.L - 1; l >= 0; --l) {
+    bkt::RecArgs ra{};
+    ra.ix = ix;
+    ra.H = H;
+    ra.dirs = dirs;
+    for (int d = 0; d < dirs; ++d) {
+      ra.Z[d] = w.Z[l * dirs + d];
+      ra.Cst[d] = w.Cst[l * dirs + d];
+      ra.Whh[d] = params + lo.w_hh(l, d);
+    }
+    ra.Y = w.Y[l];
+    ra.dY = w.dY;
+    L.run("lstm_bwd", [&] { return bkt::launch_lstm_bwd(ra, geom[l], s); });
+    const int D = lo.D(l);
+    const float *Xl = (l == 0) ? w.X : w.Y[l - 1];
+    for (int d = 0; d < dirs; ++d) {
+      const float *dZ = w.Z[l * dirs + d];
+      const int64_t wi = lo.w_ih[l * dirs + d];
+      reduce_tokens("gemm_dw_ih", dZ, 4 * H, 4 * H, Xl, D, nullptr, D, grads + wi);
+      // h_{t-1} of token (t, r): the row's previous token in its direction
+      reduce_tokens("gemm_dw_hh", dZ, 4 * H, 4 * H, w.Y[l] + d * H, DH, w.prev_tok[d], H, grads + lo.w_hh(l, d));
+      bias_grad(dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
+    }
+    if (l > 0) {
+      for (int d = 0; d < dirs; ++d) {
+        bkt::GemmArgs g{};
+        g.M = NT;
+        g.N = DH;
+        g.K = 4 * H;
+        g.A = w.Z[l * dirs + d];
+        g.lda = 4 * H;
+        g.B = params + lo.w_ih[l * dirs + d];
+        g.ldb = DH;
+        g.C = w.dY;
+        g.ldc = DH;
+        g.accumulate = d > 0;
+        g.splits = 1;
+        L.run("gemm_dx", [&] { return bkt::launch_gemm_f32(false, false, g, s); });
+      }
+    }
+  }
+  if (L.failed) return cuda_err(L.failed, L.err);
+  return BKT_OK;
 }
 
 }  // namespace
@@ -299,18 +588,7 @@ struct bkt_ctx {
   int32_t max_batch, max_label_len, S_cap;
   int device = 0, sm_count = 0;
   std::vector<void *> allocs;
-  // device workspace
-  float *X = nullptr;                  // packed input [NT x in_dim]
-  std::vector<float *> Y;              // per layer [NT x dirs*H]
-  std::vector<float *> Z, Cst;         // per layer*dirs [NT x 4H], [NT x H]
-  float *logit = nullptr;              // [NT x C]
-  float *alpha = nullptr, *beta = nullptr;  // [NT x S_cap]
-  float *dY = nullptr;                 // [NT x dirs*H]
-  float *part = nullptr;               // split-K partial sums
-  size_t part_floats = 0;
-  int32_t *tok_t = nullptr, *tok_r = nullptr, *row_ok = nullptr, *status = nullptr;
-  int32_t *prev_tok[2] = {nullptr, nullptr};  // previous token of each token per direction, -1 at the start
-  void *idx_dev = nullptr;
+  bkt::StepBufs w{};
   size_t idx_bytes = 0;
   // pinned staging ring for the per-step index block
   void *stage = nullptr;
@@ -319,7 +597,7 @@ struct bkt_ctx {
   int stage_next = 0;
   cudaStream_t last_stream = nullptr;
   EventTimer timer;
-  std::vector<bkt::RecGeom> geom;  // per layer
+  bkt::RecGeom geom[bkt::kMaxLayers] = {};
 
   ~bkt_ctx() {
     for (int i = 0; i < kStageSlots; ++i)
@@ -338,33 +616,6 @@ struct bkt_ctx {
     return e;
   }
 };
-
-namespace {
-
-// Layout of the per-step index block (same in staging and on the device).
-struct IdxLayout {
-  size_t row_len, row_lab_len, row_orig, row_xoff, row_lab_off, row_ctc_off, tok_off, bytes;
-};
-IdxLayout idx_layout(int32_t b, int64_t T) {
-  IdxLayout L;
-  size_t o = 0;
-  auto take = [&](size_t n) {
-    size_t r = o;
-    o += (n + 15) & ~size_t(15);
-    return r;
-  };
-  L.row_len = take(4 * (size_t)b);
-  L.row_lab_len = take(4 * (size_t)b);
-  L.row_orig = take(4 * (size_t)b);
-  L.row_xoff = take(8 * (size_t)b);
-  L.row_lab_off = take(8 * (size_t)b);
-  L.row_ctc_off = take(8 * (size_t)b);
-  L.tok_off = take(4 * (size_t)(T + 1));
-  L.bytes = o;
-  return L;
-}
-
-}  // namespace
 
 extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int32_t max_batch,
                               int32_t max_label_len, bkt_ctx **out) {
@@ -392,6 +643,7 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
     return cuda_err("cudaDeviceGetAttribute", e);
   }
   const Layout &lo = c->lo;
+  bkt::StepBufs &w = c->w;
   const size_t NT = (size_t)max_tokens, DH = (size_t)lo.dirs * lo.H, H = lo.H;
 #define BKT_ALLOC(ptr, n)                                                                       \
   do {                                                                                          \
@@ -403,42 +655,36 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
                      cudaGetErrorName(e));                                                      \
     }                                                                                           \
   } while (0)
-  BKT_ALLOC(c->X, NT * cfg->in_dim);
-  c->Y.resize(lo.L);
-  c->Z.resize((size_t)lo.L * lo.dirs);
-  c->Cst.resize((size_t)lo.L * lo.dirs);
+  BKT_ALLOC(w.X, NT * cfg->in_dim);
   for (int l = 0; l < lo.L; ++l) {
-    BKT_ALLOC(c->Y[l], NT * DH);
+    BKT_ALLOC(w.Y[l], NT * DH);
     for (int d = 0; d < lo.dirs; ++d) {
-      BKT_ALLOC(c->Z[l * lo.dirs + d], NT * 4 * H);
-      BKT_ALLOC(c->Cst[l * lo.dirs + d], NT * H);
+      BKT_ALLOC(w.Z[l * lo.dirs + d], NT * 4 * H);
+      BKT_ALLOC(w.Cst[l * lo.dirs + d], NT * H);
     }
   }
-  BKT_ALLOC(c->logit, NT * lo.C);
-  BKT_ALLOC(c->alpha, NT * (size_t)c->S_cap);
-  BKT_ALLOC(c->beta, NT * (size_t)c->S_cap);
-  BKT_ALLOC(c->dY, NT * DH);
-  // split-K partials: at most 64 splits of the largest weight block (and
-  // of the bias columns), see the step engine.
-  size_t maxMN = std::max<size_t>((size_t)lo.C * DH, 4 * H * std::max<size_t>(DH, (size_t)cfg->in_dim));
-  maxMN = std::max(maxMN, 4 * H * H);
-  c->part_floats = 64 * maxMN;
-  BKT_ALLOC(c->part, c->part_floats);
-  BKT_ALLOC(c->tok_t, NT);
-  BKT_ALLOC(c->tok_r, NT);
-  BKT_ALLOC(c->prev_tok[0], NT);
-  BKT_ALLOC(c->prev_tok[1], NT);
-  BKT_ALLOC(c->row_ok, (size_t)max_batch);
-  BKT_ALLOC(c->status, 1);
+  BKT_ALLOC(w.logit, NT * lo.C);
+  BKT_ALLOC(w.alpha, NT * (size_t)c->S_cap);
+  BKT_ALLOC(w.beta, NT * (size_t)c->S_cap);
+  BKT_ALLOC(w.dY, NT * DH);
+  // split-K partials: at most 64 splits of the largest weight block
+  w.part_floats = 64 * max_reduce_block(lo);
+  BKT_ALLOC(w.part, w.part_floats);
+  BKT_ALLOC(w.tok_t, NT);
+  BKT_ALLOC(w.tok_r, NT);
+  BKT_ALLOC(w.prev_tok[0], NT);
+  BKT_ALLOC(w.prev_tok[1], NT);
+  BKT_ALLOC(w.row_ok, (size_t)max_batch);
+  BKT_ALLOC(w.status, 1);
   IdxLayout il = idx_layout(max_batch, max_tokens);
   c->idx_bytes = il.bytes;
   {
     char *p = nullptr;
     BKT_ALLOC(p, il.bytes);
-    c->idx_dev = p;
+    w.idx_dev = p;
   }
 #undef BKT_ALLOC
-  e = cudaMemset(c->status, 0, sizeof(int32_t));
+  e = cudaMemset(w.status, 0, sizeof(int32_t));
   if (e != cudaSuccess) {
     delete c;
     return cuda_err("cudaMemset", e);
@@ -455,8 +701,7 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
       return cuda_err("cudaEventCreate", e);
     }
   }
-  for (int l = 0; l < lo.L; ++l)
-    c->geom.push_back(bkt::plan_recurrent(lo.H, max_batch, lo.dirs, c->sm_count));
+  for (int l = 0; l < lo.L; ++l) c->geom[l] = bkt::plan_recurrent(lo.H, max_batch, lo.dirs, c->sm_count);
   *out = c;
   return BKT_OK;
 }
@@ -499,10 +744,10 @@ extern "C" int bkt_ctx_sync_status(bkt_ctx *c) {
   e = cudaStreamSynchronize(c->last_stream);
   if (e != cudaSuccess) return cuda_err("cudaStreamSynchronize", e);
   int32_t st = 0;
-  e = cudaMemcpy(&st, c->status, sizeof st, cudaMemcpyDeviceToHost);
+  e = cudaMemcpy(&st, c->w.status, sizeof st, cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return cuda_err("cudaMemcpy(status)", e);
   if (st != 0) {
-    cudaMemset(c->status, 0, sizeof st);
+    cudaMemset(c->w.status, 0, sizeof st);
     return set_err(BKT_EDEVICE, "device check failed: a label is out of range or equals the blank (flags 0x%x)", st);
   }
   return BKT_OK;
@@ -517,64 +762,15 @@ extern "C" int bkt_sgd_update(float *params, const float *grads, int64_t n, floa
 }
 
 // ---------------------------------------------------------------------------
-// The step.
-namespace {
-
-struct Launch {
-  bkt_ctx *c;
-  cudaStream_t s;
-  const char *failed = nullptr;
-  cudaError_t err = cudaSuccess;
-  template <typename F>
-  bool run(const char *name, F &&f) {
-    if (failed) return false;
-    c->timer.begin(name, s);
-    cudaError_t e = f();
-    c->timer.end(s);
-    if (e != cudaSuccess) {
-      failed = name;
-      err = e;
-      return false;
-    }
-    return true;
-  }
-};
-
-// Number of token splits for a reduction over n_tok rows into an M x N block.
-int choose_splits(int M, int N, int n_tok, int sm_count, size_t part_cap) {
-  const int tiles = ((M + 63) / 64) * ((N + 63) / 64);
-  int s = std::max(1, (2 * sm_count + tiles - 1) / tiles);
-  s = std::min(s, std::max(1, n_tok / 256));
-  s = std::min(s, 64);
-  while (s > 1 && (size_t)s * M * N > part_cap) --s;
-  return s;
-}
-
-}  // namespace
-
-extern "C" int bkt_lstm_ctc_step(bkt_ctx *c, const bkt_batch *bt, const float *params, float *grads,
-                                 float *loss, void *stream) {
+// The step through a ctx.
+extern "C" int bkt_lstm_ctc_step(bkt_ctx *c, const bkt_batch *bt, const float *params, float *grads, float *loss,
+                                 void *stream) {
   if (!c || !bt || !params || !grads || !loss) return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: NULL argument");
-  const int32_t b = bt->n_seq;
-  if (b < 1 || b > c->max_batch)
-    return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: n_seq %d outside 1..%d", b, c->max_batch);
-  if (!bt->lengths || !bt->x_offsets || !bt->label_lengths || !bt->label_offsets || !bt->x || !bt->labels)
-    return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: NULL batch array");
-  int64_t n_tok = 0;
+  int64_t n_tok = 0, cells = 0;
   int32_t S_max = 1;
-  for (int32_t i = 0; i < b; ++i) {
-    if (bt->lengths[i] < 1) return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: lengths[%d] = %d < 1", i, bt->lengths[i]);
-    if (bt->label_lengths[i] < 0 || bt->label_lengths[i] > c->max_label_len)
-      return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: label_lengths[%d] = %d outside 0..%d", i,
-                     bt->label_lengths[i], c->max_label_len);
-    if (bt->x_offsets[i] < 0 || bt->label_offsets[i] < 0)
-      return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: negative offset for sequence %d", i);
-    n_tok += bt->lengths[i];
-    S_max = std::max(S_max, 2 * bt->label_lengths[i] + 1);
-  }
-  if (n_tok > c->max_tokens)
-    return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: %lld tokens exceed the ctx capacity %lld", (long long)n_tok,
-                   (long long)c->max_tokens);
+  int rc = check_batch(bt, c->max_tokens, c->max_batch, c->max_label_len, &n_tok, &S_max, &cells);
+  if (rc != BKT_OK) return rc;
+  const int32_t b = bt->n_seq;
   cudaStream_t s = (cudaStream_t)stream;
   cudaError_t e = cudaSetDevice(c->device);
   if (e != cudaSuccess) return cuda_err("cudaSetDevice", e);
@@ -593,195 +789,126 @@ extern "C" int bkt_lstm_ctc_step(bkt_ctx *c, const bkt_batch *bt, const float *p
     if (e != cudaSuccess) return cuda_err("cudaEventSynchronize(stage)", e);
   }
   char *st = (char *)c->stage + (size_t)slot * c->idx_bytes;
-  int32_t *row_len = (int32_t *)(st + il.row_len), *row_lab_len = (int32_t *)(st + il.row_lab_len),
-          *row_orig = (int32_t *)(st + il.row_orig), *tok_off = (int32_t *)(st + il.tok_off);
-  int64_t *row_xoff = (int64_t *)(st + il.row_xoff), *row_lab_off = (int64_t *)(st + il.row_lab_off),
-          *row_ctc_off = (int64_t *)(st + il.row_ctc_off);
-  int64_t ctc_off = 0;
-  for (int32_t r = 0; r < b; ++r) {
-    const int32_t i = perm[r];
-    row_len[r] = bt->lengths[i];
-    row_lab_len[r] = bt->label_lengths[i];
-    row_orig[r] = i;
-    row_xoff[r] = bt->x_offsets[i];
-    row_lab_off[r] = bt->label_offsets[i];
-    row_ctc_off[r] = ctc_off;
-    ctc_off += (int64_t)bt->lengths[i] * (2 * bt->label_lengths[i] + 1);
-  }
-  {
-    int32_t active = b, acc = 0;
-    for (int32_t t = 0; t < T; ++t) {
-      while (active > 0 && row_len[active - 1] <= t) --active;
-      tok_off[t] = acc;
-      acc += active;
-    }
-    tok_off[T] = acc;
-  }
-  e = cudaMemcpyAsync(c->idx_dev, st, il.bytes, cudaMemcpyHostToDevice, s);
+  bkt::DevIdx ix = fill_index_block(bt, perm.data(), T, n_tok, S_max, il, st, (char *)c->w.idx_dev, c->w.tok_t,
+                                    c->w.tok_r);
+  e = cudaMemcpyAsync(c->w.idx_dev, st, il.bytes, cudaMemcpyHostToDevice, s);
   if (e != cudaSuccess) return cuda_err("cudaMemcpyAsync(index block)", e);
   e = cudaEventRecord(c->stage_ev[slot], s);
   if (e != cudaSuccess) return cuda_err("cudaEventRecord(stage)", e);
   c->stage_used[slot] = true;
   c->last_stream = s;
+  return enqueue_kernels(c->cfg, c->lo, c->w, c->geom, ix, bt, params, grads, loss, s,
+                         c->timer.on ? &c->timer : nullptr, c->sm_count);
+}
 
-  bkt::DevIdx ix;
-  char *dv = (char *)c->idx_dev;
-  ix.b = b;
-  ix.T = T;
-  ix.n_tok = (int32_t)n_tok;
-  ix.S_max = S_max;
-  ix.row_len = (const int32_t *)(dv + il.row_len);
-  ix.row_lab_len = (const int32_t *)(dv + il.row_lab_len);
-  ix.row_orig = (const int32_t *)(dv + il.row_orig);
-  ix.row_xoff = (const int64_t *)(dv + il.row_xoff);
-  ix.row_lab_off = (const int64_t *)(dv + il.row_lab_off);
-  ix.row_ctc_off = (const int64_t *)(dv + il.row_ctc_off);
-  ix.tok_off = (const int32_t *)(dv + il.tok_off);
-  ix.tok_t = c->tok_t;
-  ix.tok_r = c->tok_r;
+// ---------------------------------------------------------------------------
+// The step on caller-provided scratch (no allocation anywhere on this path:
+// fixed-size host arrays, a pageable staging buffer, buffers carved out of
+// the scratch range).
+int bkt::report_error(int code, const char *fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  const int r = vset_err(code, fmt, ap);
+  va_end(ap);
+  return r;
+}
 
-  const Layout &lo = c->lo;
-  const int H = lo.H, dirs = lo.dirs, DH = dirs * H, C = lo.C, NT = (int)n_tok;
-  Launch L{c, s};
+namespace {
 
-  // ---- a4: packed time-major input
-  L.run("layout_gather", [&] { return bkt::launch_layout(ix, bt->x, lo.D0, c->X, c->tok_t, c->tok_r, c->prev_tok, s); });
+constexpr int32_t kScratchMaxBatch = 512;
+constexpr int32_t kScratchMaxLabel = 1023;
+constexpr size_t kScratchStageBytes = 256 * 1024;
+alignas(64) char g_scratch_stage[kScratchStageBytes];
+std::mutex g_scratch_stage_mu;
 
-  // ---- forward, layer by layer
+// Bump allocator over a caller-provided range (256-byte aligned pieces).
+struct Carve {
+  char *base;
+  size_t cap, used = 0;
+  template <typename T>
+  T *take(size_t count) {
+    const size_t off = (used + 255) & ~size_t(255);
+    used = off + std::max<size_t>(count, 1) * sizeof(T);
+    return reinterpret_cast<T *>(base + off);
+  }
+};
+
+}  // namespace
+
+int bkt::step_on_scratch(const bkt_model_cfg *cfg, const bkt_batch *bt, const float *params, float *grads,
+                         float *loss, cudaStream_t s, void *scratch, size_t scratch_bytes, int sm_count) {
+  if (!cfg_ok(cfg)) return set_err(BKT_EINVAL, "bkt_lstm_ctc_step_static: invalid model cfg");
+  if (!bt || !params || !grads || !loss) return set_err(BKT_EINVAL, "bkt_lstm_ctc_step_static: NULL argument");
+  int64_t n_tok = 0, cells = 0;
+  int32_t S_max = 1;
+  int rc = check_batch(bt, (int64_t)INT32_MAX / 4, kScratchMaxBatch, kScratchMaxLabel, &n_tok, &S_max, &cells);
+  if (rc != BKT_OK) return rc;
+  const Layout lo = make_layout(cfg);
+  const int32_t b = bt->n_seq;
+  // stable insertion sort, longest first
+  int32_t perm[kScratchMaxBatch];
+  for (int32_t i = 0; i < b; ++i) {
+    int32_t j = i;
+    while (j > 0 && bt->lengths[perm[j - 1]] < bt->lengths[i]) {
+      perm[j] = perm[j - 1];
+      --j;
+    }
+    perm[j] = i;
+  }
+  const int32_t T = bt->lengths[perm[0]];
+  const IdxLayout il = idx_layout(b, T);
+  if (il.bytes > kScratchStageBytes)
+    return set_err(BKT_EINVAL, "bkt_lstm_ctc_step_static: the longest sequence (%d steps) is too long for this entry point", T);
+
+  // carve the workspace
+  const size_t NT = (size_t)n_tok, DH = (size_t)lo.dirs * lo.H, H = lo.H;
+  Carve cv{(char *)scratch, scratch_bytes};
+  StepBufs w{};
+  w.X = cv.take<float>(NT * cfg->in_dim);
   for (int l = 0; l < lo.L; ++l) {
-    float *Zl[2] = {c->Z[l * dirs], dirs > 1 ? c->Z[l * dirs + 1] : nullptr};
-    if (l == 0) {
-      // a5, narrow input: both directions in one launch
-      L.run("proj_narrow", [&] {
-        return bkt::launch_proj_narrow(c->X, NT, lo.D0, params, lo.w_ih[0], lo.stride(0), H, dirs, Zl, s);
-      });
-    } else {
-      for (int d = 0; d < dirs; ++d) {
-        bkt::GemmArgs g{};
-        g.M = NT;
-        g.N = 4 * H;
-        g.K = DH;
-        g.A = c->Y[l - 1];
-        g.lda = DH;
-        g.B = params + lo.w_ih[l * dirs + d];
-        g.ldb = DH;
-        g.C = Zl[d];
-        g.ldc = 4 * H;
-        g.bias = params + lo.bias(l, d);
-        g.splits = 1;
-        L.run("gemm_proj", [&] { return bkt::launch_gemm_f32(false, true, g, s); });
-      }
+    w.Y[l] = cv.take<float>(NT * DH);
+    for (int d = 0; d < lo.dirs; ++d) {
+      w.Z[l * lo.dirs + d] = cv.take<float>(NT * 4 * H);
+      w.Cst[l * lo.dirs + d] = cv.take<float>(NT * H);
     }
-    bkt::RecArgs ra{};
-    ra.ix = ix;
-    ra.H = H;
-    ra.dirs = dirs;
-    for (int d = 0; d < dirs; ++d) {
-      ra.Z[d] = Zl[d];
-      ra.Cst[d] = c->Cst[l * dirs + d];
-      ra.Whh[d] = params + lo.w_hh(l, d);
-    }
-    ra.Y = c->Y[l];
-    L.run("lstm_fwd", [&] { return bkt::launch_lstm_fwd(ra, c->geom[l], s); });
   }
+  w.logit = cv.take<float>(NT * lo.C);
+  w.alpha = cv.take<float>((size_t)cells);
+  w.beta = cv.take<float>((size_t)cells);
+  w.dY = cv.take<float>(NT * DH);
+  w.tok_t = cv.take<int32_t>(NT);
+  w.tok_r = cv.take<int32_t>(NT);
+  w.prev_tok[0] = cv.take<int32_t>(NT);
+  w.prev_tok[1] = cv.take<int32_t>(NT);
+  w.row_ok = cv.take<int32_t>((size_t)b);
+  w.status = cv.take<int32_t>(1);
+  w.idx_dev = cv.take<char>(il.bytes);
+  // split-K partials get the rest: at least one split of the largest block
+  const size_t min_part = max_reduce_block(lo);
+  w.part = cv.take<float>(min_part);
+  const size_t need = cv.used;
+  if (need > scratch_bytes)
+    return set_err(BKT_EINVAL,
+                   "bkt_lstm_ctc_step_static: this batch needs %zu bytes of scratch but the static array holds %zu "
+                   "(use a bkt_ctx for larger batches)",
+                   need, scratch_bytes);
+  w.part_floats = min_part + (scratch_bytes - need) / sizeof(float);
+  w.part_floats = std::min(w.part_floats, 64 * min_part);
 
-  // ---- a7: output layer and log-softmax
-  float *Ytop = c->Y[lo.L - 1];
-  L.run("out_logsoftmax", [&] {
-    return bkt::launch_out_logsoftmax(Ytop, NT, DH, params + lo.w_out, params + lo.b_out, C, c->logit, s);
-  });
-  // ---- a8, a9: CTC
-  L.run("ctc_tables", [&] {
-    return bkt::launch_ctc_tables(ix, c->logit, C, c->cfg.blank, bt->labels, c->alpha, c->beta, loss, c->row_ok,
-                                  c->status, s);
-  });
-  L.run("ctc_grad", [&] {
-    return bkt::launch_ctc_grad(ix, c->logit, C, c->cfg.blank, bt->labels, c->alpha, c->beta, c->row_ok, s);
-  });
+  RecGeom geom[kMaxLayers];
+  const RecGeom g0 = plan_recurrent(lo.H, b, lo.dirs, sm_count);
+  for (int l = 0; l < lo.L; ++l) geom[l] = g0;
 
-  // ---- a10: output layer backward
-  auto reduce_tokens = [&](const char *name, const float *A, int64_t lda, int M, const float *B, int64_t ldb,
-                           const int32_t *gather, int N, float *out) {
-    bkt::GemmArgs g{};
-    g.M = M;
-    g.N = N;
-    g.K = NT;
-    g.A = A;
-    g.lda = lda;
-    g.B = B;
-    g.ldb = ldb;
-    g.gather = gather;
-    g.P = c->part;
-    g.splits = choose_splits(M, N, NT, c->sm_count, c->part_floats);
-    L.run(name, [&] { return bkt::launch_gemm_f32(true, false, g, s); });
-    L.run("splitk_reduce", [&] { return bkt::launch_splitk_reduce(c->part, g.splits, (int64_t)M * N, out, s); });
-  };
-  auto bias_grad = [&](const float *A, int64_t lda, int M, float *out) {
-    int splits = std::min(64, std::max(1, std::min(2 * c->sm_count / std::max(1, (M + 255) / 256), NT / 64)));
-    while (splits > 1 && (size_t)splits * M > c->part_floats) --splits;
-    L.run("colsum", [&] { return bkt::launch_colsum_partial(A, lda, NT, M, c->part, splits, s); });
-    L.run("splitk_reduce", [&] { return bkt::launch_splitk_reduce(c->part, splits, M, out, s); });
-  };
-  reduce_tokens("gemm_dw_out", c->logit, C, C, Ytop, DH, nullptr, DH, grads + lo.w_out);
-  bias_grad(c->logit, C, C, grads + lo.b_out);
+  cudaError_t e = cudaMemsetAsync(w.status, 0, sizeof(int32_t), s);
+  if (e != cudaSuccess) return cuda_err("cudaMemsetAsync(status)", e);
+  DevIdx ix;
   {
-    bkt::GemmArgs g{};
-    g.M = NT;
-    g.N = DH;
-    g.K = C;
-    g.A = c->logit;
-    g.lda = C;
-    g.B = params + lo.w_out;
-    g.ldb = DH;
-    g.C = c->dY;
-    g.ldc = DH;
-    g.splits = 1;
-    L.run("gemm_dy_out", [&] { return bkt::launch_gemm_f32(false, false, g, s); });
+    // pageable source: the call returns once the bytes are staged, so the
+    // buffer is free again when the lock is released
+    std::lock_guard<std::mutex> lk(g_scratch_stage_mu);
+    ix = fill_index_block(bt, perm, T, n_tok, S_max, il, g_scratch_stage, (char *)w.idx_dev, w.tok_t, w.tok_r);
+    e = cudaMemcpyAsync(w.idx_dev, g_scratch_stage, il.bytes, cudaMemcpyHostToDevice, s);
   }
-
-  // ---- a11, a12: BPTT and weight gradients, top layer first
-  for (int l = lo.L - 1; l >= 0; --l) {
-    bkt::RecArgs ra{};
-    ra.ix = ix;
-    ra.H = H;
-    ra.dirs = dirs;
-    for (int d = 0; d < dirs; ++d) {
-      ra.Z[d] = c->Z[l * dirs + d];
-      ra.Cst[d] = c->Cst[l * dirs + d];
-      ra.Whh[d] = params + lo.w_hh(l, d);
-    }
-    ra.Y = c->Y[l];
-    ra.dY = c->dY;
-    L.run("lstm_bwd", [&] { return bkt::launch_lstm_bwd(ra, c->geom[l], s); });
-    const int D = lo.D(l);
-    const float *Xl = (l == 0) ? c->X : c->Y[l - 1];
-    for (int d = 0; d < dirs; ++d) {
-      const float *dZ = c->Z[l * dirs + d];
-      const int64_t wi = lo.w_ih[l * dirs + d];
-      reduce_tokens("gemm_dw_ih", dZ, 4 * H, 4 * H, Xl, D, nullptr, D, grads + wi);
-      // h_{t-1} of token (t, r): the row's previous token in its direction
-      reduce_tokens("gemm_dw_hh", dZ, 4 * H, 4 * H, c->Y[l] + d * H, DH, c->prev_tok[d], H,
-                    grads + lo.w_hh(l, d));
-      bias_grad(dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
-    }
-    if (l > 0) {
-      for (int d = 0; d < dirs; ++d) {
-        bkt::GemmArgs g{};
-        g.M = NT;
-        g.N = DH;
-        g.K = 4 * H;
-        g.A = c->Z[l * dirs + d];
-        g.lda = 4 * H;
-        g.B = params + lo.w_ih[l * dirs + d];
-        g.ldb = DH;
-        g.C = c->dY;
-        g.ldc = DH;
-        g.accumulate = d > 0;
-        g.splits = 1;
-        L.run("gemm_dx", [&] { return bkt::launch_gemm_f32(false, false, g, s); });
-      }
-    }
-  }
-  if (L.failed) return cuda_err(L.failed, L.err);
-  return BKT_OK;
+  if (e != cudaSuccess) return cuda_err("cudaMemcpyAsync(index block)", e);
+  return enqueue_kernels(*cfg, lo, w, geom, ix, bt, params, grads, loss, s, nullptr, sm_count);
 }

@@ -5,6 +5,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "bkt.h"
+
 namespace bkt {
 
 // Device-side view of one packed mini-batch.  Rows are the batch's sequences
@@ -129,5 +131,35 @@ cudaError_t launch_lstm_cta(const RecArgs &a, int bc, bool bwd, cudaStream_t s);
 
 // a13
 cudaError_t launch_sgd(float *p, const float *g, int64_t n, float lr, cudaStream_t s);
+
+// ---------------------------------------------------------------------------
+// Device buffers of one step (see the step engine in bkt_api.cpp).
+constexpr int kMaxLayers = 64;
+struct StepBufs {
+  float *X;                                   // packed input [NT x in_dim]
+  float *Y[kMaxLayers];                       // layer outputs [NT x dirs*H]
+  float *Z[2 * kMaxLayers];                   // per layer*dirs+dir: Zx / gates / dz [NT x 4H]
+  float *Cst[2 * kMaxLayers];                 // cell states [NT x H]
+  float *logit;                               // log-probabilities / dlogit [NT x C]
+  float *alpha, *beta;                        // CTC tables, sum_i L_i (2 U_i + 1) each
+  float *dY;                                  // dloss/dY of the current layer [NT x dirs*H]
+  float *part;                                // split-K partial sums
+  size_t part_floats;
+  int32_t *tok_t, *tok_r, *prev_tok[2];       // [NT] each
+  int32_t *row_ok;                            // [b]
+  int32_t *status;                            // device error flags
+  void *idx_dev;                              // per-step index block
+};
+
+// Records an error message for bkt_last_error() and returns `code`.
+int report_error(int code, const char *fmt, ...);
+
+// Runs one training step with every buffer carved out of `scratch`
+// (`scratch_bytes` long, 256-byte aligned device memory), allocating
+// nothing.  Host-side checks return BKT_EINVAL, including a batch whose
+// workspace does not fit.
+int step_on_scratch(const bkt_model_cfg *cfg, const bkt_batch *batch, const float *params,
+                    float *grads, float *loss, cudaStream_t s, void *scratch, size_t scratch_bytes,
+                    int sm_count);
 
 }  // namespace bkt
