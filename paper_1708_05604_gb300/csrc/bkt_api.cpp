@@ -339,21 +339,12 @@ struct Launch {
   }
 };
 
-// Number of token splits for a reduction over n_tok rows into an M x N block.
-int choose_splits(int M, int N, int n_tok, int sm_count, size_t part_cap) {
-  const int tiles = ((M + 63) / 64) * ((N + 63) / 64);
-  int s = std::max(1, (2 * sm_count + tiles - 1) / tiles);
-  s = std::min(s, std::max(1, n_tok / 256));
-  s = std::min(s, 64);
-  while (s > 1 && (size_t)s * M * N > part_cap) --s;
-  return s;
-}
-
-// Largest M x N block a token reduction writes (weights and biases).
+// Largest M x N block a token reduction writes: [W_out | b_out] or
+// [W_ih | W_hh | b] of one layer and direction.
 size_t max_reduce_block(const Layout &lo) {
   const size_t DH = (size_t)lo.dirs * lo.H, H = lo.H;
-  size_t m = std::max<size_t>((size_t)lo.C * DH, 4 * H * std::max<size_t>(DH, (size_t)lo.D0));
-  return std::max(m, 4 * H * H);
+  const size_t Dm = std::max<size_t>(DH, (size_t)lo.D0);
+  return std::max<size_t>((size_t)lo.C * (DH + 1), 4 * H * (Dm + H + 1));
 }
 
 // Enqueues every kernel of one step (a4 gather .. a12) on `s`.
@@ -418,30 +409,28 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
   });
 
   // ---- a10: output layer backward
-  auto reduce_tokens = [&](const char *name, const float *A, int64_t lda, int M, const float *B, int64_t ldb,
-                           const int32_t *gather, int N, float *out) {
-    bkt::GemmArgs g{};
+  // [dW_out | db_out] = dlogit^T [Y | 1]
+  auto wgrad = [&](const float *A, int64_t lda, int M, const float *B1, int64_t ldb1, int D1, const float *B2,
+                   int64_t ldb2, const int32_t *gather2, int D2, float *o1, float *o2, float *o3) {
+    bkt::WgradArgs g{};
     g.M = M;
-    g.N = N;
+    g.N = D1 + D2 + 1;
     g.K = NT;
     g.A = A;
     g.lda = lda;
-    g.B = B;
-    g.ldb = ldb;
-    g.gather = gather;
+    g.D1 = D1;
+    g.B1 = B1;
+    g.ldb1 = ldb1;
+    g.D2 = D2;
+    g.B2 = B2;
+    g.ldb2 = ldb2;
+    g.gather2 = gather2;
+    g.ones = 1;
     g.P = w.part;
-    g.splits = choose_splits(M, N, NT, sm_count, w.part_floats);
-    L.run(name, [&] { return bkt::launch_gemm_f32(true, false, g, s); });
-    L.run("splitk_reduce", [&] { return bkt::launch_splitk_reduce(w.part, g.splits, (int64_t)M * N, out, s); });
+    g.splits = bkt::wgrad_splits(g.M, g.N, NT, sm_count, w.part_floats);
+    L.run("wgrad", [&] { return bkt::launch_wgrad(g, o1, o2, o3, s); });
   };
-  auto bias_grad = [&](const float *A, int64_t lda, int M, float *out) {
-    int splits = std::min(64, std::max(1, std::min(2 * sm_count / std::max(1, (M + 255) / 256), NT / 64)));
-    while (splits > 1 && (size_t)splits * M > w.part_floats) --splits;
-    L.run("colsum", [&] { return bkt::launch_colsum_partial(A, lda, NT, M, w.part, splits, s); });
-    L.run("splitk_reduce", [&] { return bkt::launch_splitk_reduce(w.part, splits, M, out, s); });
-  };
-  reduce_tokens("gemm_dw_out", w.logit, C, C, Ytop, DH, nullptr, DH, grads + lo.w_out);
-  bias_grad(w.logit, C, C, grads + lo.b_out);
+  wgrad(w.logit, C, C, Ytop, DH, DH, nullptr, 0, nullptr, 0, grads + lo.w_out, nullptr, grads + lo.b_out);
   {
     bkt::GemmArgs g{};
     g.M = NT;
@@ -474,12 +463,10 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     const int D = lo.D(l);
     const float *Xl = (l == 0) ? w.X : w.Y[l - 1];
     for (int d = 0; d < dirs; ++d) {
-      const float *dZ = w.Z[l * dirs + d];
-      const int64_t wi = lo.w_ih[l * dirs + d];
-      reduce_tokens("gemm_dw_ih", dZ, 4 * H, 4 * H, Xl, D, nullptr, D, grads + wi);
-      // h_{t-1} of token (t, r): the row's previous token in its direction
-      reduce_tokens("gemm_dw_hh", dZ, 4 * H, 4 * H, w.Y[l] + d * H, DH, w.prev_tok[d], H, grads + lo.w_hh(l, d));
-      bias_grad(dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
+      // [dW_ih | dW_hh | db] = dZ^T [X_l | h_{t-1} | 1]; h_{t-1} of token
+      // (t, r) is the row's previous token in its direction (zeros at the start)
+      wgrad(w.Z[l * dirs + d], 4 * H, 4 * H, Xl, D, D, w.Y[l] + d * H, DH, w.prev_tok[d], H,
+            grads + lo.w_ih[l * dirs + d], grads + lo.w_hh(l, d), grads + lo.bias(l, d));
     }
     if (l > 0) {
       for (int d = 0; d < dirs; ++d) {

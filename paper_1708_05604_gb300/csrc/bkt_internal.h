@@ -69,13 +69,21 @@ struct GemmArgs {
 };
 cudaError_t launch_gemm_f32(bool a_t, bool b_t, const GemmArgs &g, cudaStream_t s);
 
-// out[i] = sum_z P[z*n + i] for i < n (fixed summation order).
-cudaError_t launch_splitk_reduce(const float *P, int splits, int64_t n, float *out,
-                                 cudaStream_t s);
-
-// P[z][m] = sum over rows k of split z of A[k*lda + m], m < M.
-cudaError_t launch_colsum_partial(const float *A, int64_t lda, int K, int M, float *P,
-                                  int splits, cudaStream_t s);
+// Fused weight-gradient contraction over tokens (k_wgrad.cu):
+//   G[m][n] = sum_k A[k*lda + m] * Bv[k][n],  Bv[k] = [B1[k] (D1) | B2[gather2[k]] (D2) | 1 (ones)]
+// split over `splits` token ranges into P, then reduced in order and
+// scattered: column n < D1 -> out1[m*D1+n], n < D1+D2 -> out2[m*D2+n-D1],
+// the ones column -> out3[m].
+struct WgradArgs {
+  int M, N, K;
+  const float *A; int64_t lda;
+  int D1; const float *B1; int64_t ldb1;
+  int D2; const float *B2; int64_t ldb2; const int32_t *gather2;
+  int ones;
+  float *P; int splits;
+};
+int wgrad_splits(int M, int N, int K, int sm_count, size_t part_floats);
+cudaError_t launch_wgrad(const WgradArgs &g, float *out1, float *out2, float *out3, cudaStream_t s);
 
 // a7: logp[tok][c] = log-softmax_c(b[c] + W[c] . Y[tok]).
 cudaError_t launch_out_logsoftmax(const float *Y, int n_tok, int DH, const float *W,

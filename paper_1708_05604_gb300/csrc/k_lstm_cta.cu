@@ -5,18 +5,21 @@
 // direction over each sequence's own length), but one CTA holds the whole
 // 4H x H fp32 W_hh of its direction, so a time step needs no inter-SM
 // exchange at all: two CTA barriers per step are the only synchronisation.
-// For H = 128 the matrix is 256 KB, more than shared memory: each thread keeps
-// RK of its H weights in registers and the remaining H - RK in shared memory
-// (laid out so a warp reads 512 consecutive bytes).
+// For H = 128 the matrix is 256 KB, more than shared memory.  2H threads each
+// own two rows (or, in BPTT, two column segments), keep RK weights of each in
+// registers (192 registers for H = 128) and the rest in shared memory (laid
+// out so a warp reads 512 consecutive bytes).  Each h value read from shared
+// memory feeds both rows, so a step moves half the shared-memory bytes of a
+// one-row-per-thread layout, which was bound by shared-memory bandwidth.
 //
-// Forward, 4H threads, thread t owns gate row t:
-//   phase A (all threads): z_t = Zx[t] + W_hh[t,:] . h_{s-1}   (h broadcast
-//            from shared memory), activation of row t (tanh for the g block,
+// Forward, 2H threads, thread t owns gate rows t (i or f) and t + 2H (g or o):
+//   phase A (all threads): z_r = Zx[r] + W_hh[r,:] . h_{s-1}   (h broadcast
+//            from shared memory), activation of row r (tanh for the g block,
 //            sigmoid otherwise), written to shared memory and, in place over
 //            Zx, to global memory;
 //   phase B (threads t < H = unit t): c = f c + i g, h = o tanh(c).
-// BPTT, 4H threads, thread t = (q, k) owns the column segment
-// W_hh[q*H .. q*H+H-1, k]:
+// BPTT, 2H threads, thread t = (q, kc) owns the column segments
+// W_hh[q*H .. q*H+H-1, k] for k = kc and kc + H/2 of gate block q:
 //   phase B (threads t < H = unit t): dh = dY + sum_q part[q][t]; dc, dz of
 //            the four gates (written in place over the gates);
 //   phase A (all threads): part[q][k] = sum_i W_hh[q*H+i, k] dz[q*H+i].
@@ -38,34 +41,39 @@ __device__ __forceinline__ float sigm(float x) { return 1.f / (1.f + expf(-x)); 
 }  // namespace
 
 template <int H, int RK, int BC>
-__global__ void __launch_bounds__(4 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
-  constexpr int G = 4 * H, SK = H - RK, H4 = H / 4;
+__global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
+  constexpr int G = 4 * H, NTH = 2 * H, SK = H - RK, H4 = H / 4;
   extern __shared__ __align__(16) float sm[];
-  float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [SK/4][G]
-  float *hs = sm + SK * G;                       // [2][BC][H]
+  float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [SK/4][2][NTH]
+  float *hs = sm + 2 * SK * NTH;                 // [2][BC][H]
   float *zs = hs + 2 * BC * H;                   // [BC][G]
   const int T = a.ix.T;
   const bool toff_sm = T + 1 <= kTokCap;
   int *toff_s = reinterpret_cast<int *>(zs + BC * G);
   const int *toff = toff_sm ? toff_s : a.ix.tok_off;
   const int t = threadIdx.x;
-  const int q = t / H;
+  const bool lo_half = t < H;  // rows t (i or f) and t + 2H (g or o)
   const int n_groups = (a.ix.b + BC - 1) / BC;
   const int d = blockIdx.x / n_groups, grp = blockIdx.x % n_groups;
   const int r0 = grp * BC;
   const int DH = a.dirs * H;
 
-  const float *Wrow = a.Whh[d] + (size_t)t * H;
-  float wr[RK > 0 ? RK : 1];
+  const float *W0 = a.Whh[d] + (size_t)t * H;
+  const float *W1 = a.Whh[d] + (size_t)(t + NTH) * H;
+  float w0[RK], w1[RK];
 #pragma unroll
-  for (int i = 0; i < RK; ++i) wr[i] = __ldg(Wrow + i);
-  for (int i4 = 0; i4 < SK / 4; ++i4) {
-    const float *w = Wrow + RK + 4 * i4;
-    Ws4[i4 * G + t] = make_float4(__ldg(w), __ldg(w + 1), __ldg(w + 2), __ldg(w + 3));
+  for (int i = 0; i < RK; ++i) {
+    w0[i] = __ldg(W0 + i);
+    w1[i] = __ldg(W1 + i);
   }
-  for (int i = t; i < 2 * BC * H; i += G) hs[i] = 0.f;
+  for (int i4 = 0; i4 < SK / 4; ++i4) {
+    const float *u = W0 + RK + 4 * i4, *v = W1 + RK + 4 * i4;
+    Ws4[(2 * i4) * NTH + t] = make_float4(__ldg(u), __ldg(u + 1), __ldg(u + 2), __ldg(u + 3));
+    Ws4[(2 * i4 + 1) * NTH + t] = make_float4(__ldg(v), __ldg(v + 1), __ldg(v + 2), __ldg(v + 3));
+  }
+  for (int i = t; i < 2 * BC * H; i += NTH) hs[i] = 0.f;
   if (toff_sm)
-    for (int i = t; i <= T; i += G) toff_s[i] = a.ix.tok_off[i];
+    for (int i = t; i <= T; i += NTH) toff_s[i] = a.ix.tok_off[i];
   int len[BC];
 #pragma unroll
   for (int b = 0; b < BC; ++b) len[b] = (r0 + b < a.ix.b) ? a.ix.row_len[r0 + b] : 0;
@@ -79,66 +87,81 @@ __global__ void __launch_bounds__(4 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
     const int tt = d == 0 ? s : len[b] - 1 - s;
     return toff[tt] + r0 + b;
   };
-  float zn[BC], cst[BC];
+  float zn0[BC], zn1[BC], cst[BC];
   int tokn[BC];
 #pragma unroll
   for (int b = 0; b < BC; ++b) {
     cst[b] = 0.f;
     tokn[b] = 0;
-    zn[b] = 0.f;
+    zn0[b] = zn1[b] = 0.f;
     if (len[b] > 0) {
       tokn[b] = tok_at(b, 0);
-      zn[b] = Z[(size_t)tokn[b] * G + t];
+      zn0[b] = Z[(size_t)tokn[b] * G + t];
+      zn1[b] = Z[(size_t)tokn[b] * G + NTH + t];
     }
   }
   for (int s = 0; s < Tg; ++s) {
     const int p = s & 1;
-    float zc[BC];
+    float zc0[BC], zc1[BC];
     int tc[BC];
 #pragma unroll
     for (int b = 0; b < BC; ++b) {
-      zc[b] = zn[b];
+      zc0[b] = zn0[b];
+      zc1[b] = zn1[b];
       tc[b] = tokn[b];
       if (s + 1 < len[b]) {
         tokn[b] = tok_at(b, s + 1);
-        zn[b] = Z[(size_t)tokn[b] * G + t];
+        zn0[b] = Z[(size_t)tokn[b] * G + t];
+        zn1[b] = Z[(size_t)tokn[b] * G + NTH + t];
       }
     }
-    // phase A
-    float acc[BC];
+    // phase A: two rows per thread, two accumulators per row
+    float a0[BC], a1[BC], e0[BC], e1[BC];
 #pragma unroll
-    for (int b = 0; b < BC; ++b) acc[b] = 0.f;
+    for (int b = 0; b < BC; ++b) a0[b] = a1[b] = e0[b] = e1[b] = 0.f;
     const float4 *h4 = reinterpret_cast<const float4 *>(hs + p * BC * H);
 #pragma unroll
     for (int i4 = 0; i4 < RK / 4; ++i4) {
 #pragma unroll
       for (int b = 0; b < BC; ++b) {
         const float4 hv = h4[b * H4 + i4];
-        float x = fmaf(wr[4 * i4], hv.x, acc[b]);
-        x = fmaf(wr[4 * i4 + 1], hv.y, x);
-        x = fmaf(wr[4 * i4 + 2], hv.z, x);
-        acc[b] = fmaf(wr[4 * i4 + 3], hv.w, x);
+        a0[b] = fmaf(w0[4 * i4], hv.x, a0[b]);
+        a1[b] = fmaf(w1[4 * i4], hv.x, a1[b]);
+        e0[b] = fmaf(w0[4 * i4 + 1], hv.y, e0[b]);
+        e1[b] = fmaf(w1[4 * i4 + 1], hv.y, e1[b]);
+        a0[b] = fmaf(w0[4 * i4 + 2], hv.z, a0[b]);
+        a1[b] = fmaf(w1[4 * i4 + 2], hv.z, a1[b]);
+        e0[b] = fmaf(w0[4 * i4 + 3], hv.w, e0[b]);
+        e1[b] = fmaf(w1[4 * i4 + 3], hv.w, e1[b]);
       }
     }
-#pragma unroll 8
+#pragma unroll
     for (int i4 = 0; i4 < SK / 4; ++i4) {
-      const float4 w = Ws4[i4 * G + t];
+      const float4 u = Ws4[(2 * i4) * NTH + t];
+      const float4 v = Ws4[(2 * i4 + 1) * NTH + t];
 #pragma unroll
       for (int b = 0; b < BC; ++b) {
         const float4 hv = h4[b * H4 + RK / 4 + i4];
-        float x = fmaf(w.x, hv.x, acc[b]);
-        x = fmaf(w.y, hv.y, x);
-        x = fmaf(w.z, hv.z, x);
-        acc[b] = fmaf(w.w, hv.w, x);
+        a0[b] = fmaf(u.x, hv.x, a0[b]);
+        a1[b] = fmaf(v.x, hv.x, a1[b]);
+        e0[b] = fmaf(u.y, hv.y, e0[b]);
+        e1[b] = fmaf(v.y, hv.y, e1[b]);
+        a0[b] = fmaf(u.z, hv.z, a0[b]);
+        a1[b] = fmaf(v.z, hv.z, a1[b]);
+        e0[b] = fmaf(u.w, hv.w, e0[b]);
+        e1[b] = fmaf(v.w, hv.w, e1[b]);
       }
     }
 #pragma unroll
     for (int b = 0; b < BC; ++b) {
       if (s < len[b]) {
-        const float z = acc[b] + zc[b];
-        const float v = (q == 2) ? tanhf(z) : sigm(z);
-        zs[b * G + t] = v;
-        Z[(size_t)tc[b] * G + t] = v;
+        const float v0 = sigm(a0[b] + e0[b] + zc0[b]);                       // i or f
+        const float z1 = a1[b] + e1[b] + zc1[b];
+        const float v1 = lo_half ? tanhf(z1) : sigm(z1);                      // g or o
+        zs[b * G + t] = v0;
+        zs[b * G + NTH + t] = v1;
+        Z[(size_t)tc[b] * G + t] = v0;
+        Z[(size_t)tc[b] * G + NTH + t] = v1;
       }
     }
     __syncthreads();
@@ -162,33 +185,39 @@ __global__ void __launch_bounds__(4 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
 }
 
 template <int H, int RK, int BC>
-__global__ void __launch_bounds__(4 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
-  constexpr int G = 4 * H, SK = H - RK;
+__global__ void __launch_bounds__(2 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
+  constexpr int G = 4 * H, NTH = 2 * H, SK = H - RK;
   extern __shared__ __align__(16) float sm[];
-  float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [SK/4][G], W[q*H+RK+4*i4 .. +3][k]
-  float *dzs = sm + SK * G;                      // [BC][G]
+  float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [SK/4][2][NTH]: W[q*H+RK+4*i4 .. +3][k], k = kc, kc+H/2
+  float *dzs = sm + 2 * SK * NTH;                // [BC][G]
   float *red = dzs + BC * G;                     // [BC][G] partials, index q*H + k
   const int T = a.ix.T;
   const bool toff_sm = T + 1 <= kTokCap;
   int *toff_s = reinterpret_cast<int *>(red + BC * G);
   const int *toff = toff_sm ? toff_s : a.ix.tok_off;
   const int t = threadIdx.x;
-  const int q = t / H, k = t % H;
+  constexpr int H2 = H / 2;
+  const int q = t / H2, kc = t % H2;  // columns kc and kc + H/2 of gate block q
   const int n_groups = (a.ix.b + BC - 1) / BC;
   const int d = blockIdx.x / n_groups, grp = blockIdx.x % n_groups;
   const int r0 = grp * BC;
   const int DH = a.dirs * H;
 
-  const float *Wcol = a.Whh[d] + (size_t)q * H * H + k;  // W[q*H + i][k] = Wcol[i*H]
-  float wc[RK > 0 ? RK : 1];
+  const float *C0 = a.Whh[d] + (size_t)q * H * H + kc;       // W[q*H + i][kc] = C0[i*H]
+  const float *C1 = a.Whh[d] + (size_t)q * H * H + kc + H2;  // W[q*H + i][kc + H/2]
+  float w0[RK], w1[RK];
 #pragma unroll
-  for (int i = 0; i < RK; ++i) wc[i] = __ldg(Wcol + (size_t)i * H);
+  for (int i = 0; i < RK; ++i) {
+    w0[i] = __ldg(C0 + (size_t)i * H);
+    w1[i] = __ldg(C1 + (size_t)i * H);
+  }
   for (int i4 = 0; i4 < SK / 4; ++i4) {
-    const float *w = Wcol + (size_t)(RK + 4 * i4) * H;
-    Ws4[i4 * G + t] = make_float4(__ldg(w), __ldg(w + H), __ldg(w + 2 * H), __ldg(w + 3 * H));
+    const float *u = C0 + (size_t)(RK + 4 * i4) * H, *v = C1 + (size_t)(RK + 4 * i4) * H;
+    Ws4[(2 * i4) * NTH + t] = make_float4(__ldg(u), __ldg(u + H), __ldg(u + 2 * H), __ldg(u + 3 * H));
+    Ws4[(2 * i4 + 1) * NTH + t] = make_float4(__ldg(v), __ldg(v + H), __ldg(v + 2 * H), __ldg(v + 3 * H));
   }
   if (toff_sm)
-    for (int i = t; i <= T; i += G) toff_s[i] = a.ix.tok_off[i];
+    for (int i = t; i <= T; i += NTH) toff_s[i] = a.ix.tok_off[i];
   int len[BC];
 #pragma unroll
   for (int b = 0; b < BC; ++b) len[b] = (r0 + b < a.ix.b) ? a.ix.row_len[r0 + b] : 0;
@@ -231,7 +260,7 @@ __global__ void __launch_bounds__(4 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
         if (s < len[b]) {
           float dh_rec = 0.f;
           if (s + 1 < len[b])
-            dh_rec = red[b * G + t] + red[b * G + H + t] + red[b * G + 2 * H + t] + red[b * G + 3 * H + t];
+            dh_rec = (red[b * G + t] + red[b * G + H + t]) + (red[b * G + 2 * H + t] + red[b * G + 3 * H + t]);
           const float ig = gn[b][0], fg = gn[b][1], gg = gn[b][2], og = gn[b][3];
           const float ct = cn[b], cp = cpn[b];
           const float dh = dyn[b] + dh_rec;
@@ -257,30 +286,40 @@ __global__ void __launch_bounds__(4 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
       }
     }
     __syncthreads();
-    // phase A
+    // phase A: two columns of one gate block per thread (one dz read feeds
+    // both), two accumulators each
 #pragma unroll
     for (int b = 0; b < BC; ++b) {
       if (s < len[b]) {
-        const float4 *dz4 = reinterpret_cast<const float4 *>(dzs + b * G + q * H);
-        float acc = 0.f;
+        const float4 *d0 = reinterpret_cast<const float4 *>(dzs + b * G + q * H);
+        float a0 = 0.f, a1 = 0.f, e0 = 0.f, e1 = 0.f;
 #pragma unroll
         for (int i4 = 0; i4 < RK / 4; ++i4) {
-          const float4 v = dz4[i4];
-          float x = fmaf(wc[4 * i4], v.x, acc);
-          x = fmaf(wc[4 * i4 + 1], v.y, x);
-          x = fmaf(wc[4 * i4 + 2], v.z, x);
-          acc = fmaf(wc[4 * i4 + 3], v.w, x);
+          const float4 x = d0[i4];
+          a0 = fmaf(w0[4 * i4], x.x, a0);
+          a1 = fmaf(w1[4 * i4], x.x, a1);
+          e0 = fmaf(w0[4 * i4 + 1], x.y, e0);
+          e1 = fmaf(w1[4 * i4 + 1], x.y, e1);
+          a0 = fmaf(w0[4 * i4 + 2], x.z, a0);
+          a1 = fmaf(w1[4 * i4 + 2], x.z, a1);
+          e0 = fmaf(w0[4 * i4 + 3], x.w, e0);
+          e1 = fmaf(w1[4 * i4 + 3], x.w, e1);
         }
-#pragma unroll 8
+#pragma unroll
         for (int i4 = 0; i4 < SK / 4; ++i4) {
-          const float4 w = Ws4[i4 * G + t];
-          const float4 v = dz4[RK / 4 + i4];
-          float x = fmaf(w.x, v.x, acc);
-          x = fmaf(w.y, v.y, x);
-          x = fmaf(w.z, v.z, x);
-          acc = fmaf(w.w, v.w, x);
+          const float4 u = Ws4[(2 * i4) * NTH + t], v = Ws4[(2 * i4 + 1) * NTH + t];
+          const float4 x = d0[RK / 4 + i4];
+          a0 = fmaf(u.x, x.x, a0);
+          a1 = fmaf(v.x, x.x, a1);
+          e0 = fmaf(u.y, x.y, e0);
+          e1 = fmaf(v.y, x.y, e1);
+          a0 = fmaf(u.z, x.z, a0);
+          a1 = fmaf(v.z, x.z, a1);
+          e0 = fmaf(u.w, x.w, e0);
+          e1 = fmaf(v.w, x.w, e1);
         }
-        red[b * G + q * H + k] = acc;
+        red[b * G + q * H + kc] = a0 + e0;
+        red[b * G + q * H + kc + H2] = a1 + e1;
       }
     }
     __syncthreads();
@@ -292,7 +331,7 @@ namespace {
 
 size_t cta_smem_bytes(bool bwd, int H, int RK, int BC, int T) {
   const size_t f = bwd ? (size_t)(H - RK) * 4 * H + 2 * (size_t)BC * 4 * H
-                       : (size_t)(H - RK) * 4 * H + 2 * (size_t)BC * H + (size_t)BC * 4 * H;
+                       : (size_t)(H - RK) * 4 * H + 2 * (size_t)BC * H + (size_t)BC * 4 * H;  // W: 2 rows x (H-RK) x 2H threads
   const size_t i = (T + 1 <= kTokCap) ? (size_t)(T + 1) : 0;
   return (f + i) * 4 + 16;
 }
@@ -305,21 +344,21 @@ cudaError_t launch_cta(const RecArgs &a, bool bwd, cudaStream_t s) {
     cudaError_t e = cudaFuncSetAttribute(lstm_bwd_cta_kernel<H, RK, BC>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    lstm_bwd_cta_kernel<H, RK, BC><<<ng * a.dirs, 4 * H, smem, s>>>(a);
+    lstm_bwd_cta_kernel<H, RK, BC><<<ng * a.dirs, 2 * H, smem, s>>>(a);
   } else {
     cudaError_t e = cudaFuncSetAttribute(lstm_fwd_cta_kernel<H, RK, BC>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    lstm_fwd_cta_kernel<H, RK, BC><<<ng * a.dirs, 4 * H, smem, s>>>(a);
+    lstm_fwd_cta_kernel<H, RK, BC><<<ng * a.dirs, 2 * H, smem, s>>>(a);
   }
   return cudaGetLastError();
 }
 
-template <int H, int RK>
+template <int H, int RK1, int RK2>
 cudaError_t launch_cta_bc(const RecArgs &a, int bc, bool bwd, cudaStream_t s) {
   switch (bc) {
-    case 1: return launch_cta<H, RK, 1>(a, bwd, s);
-    case 2: return launch_cta<H, RK, 2>(a, bwd, s);
+    case 1: return launch_cta<H, RK1, 1>(a, bwd, s);
+    case 2: return launch_cta<H, RK2, 2>(a, bwd, s);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -335,9 +374,9 @@ int cta_rows_per_block(int H, int b, int dirs, int sm_count) {
 
 cudaError_t launch_lstm_cta(const RecArgs &a, int bc, bool bwd, cudaStream_t s) {
   switch (a.H) {
-    case 32: return launch_cta_bc<32, 32>(a, bc, bwd, s);
-    case 64: return launch_cta_bc<64, 64>(a, bc, bwd, s);
-    case 128: return launch_cta_bc<128, 64>(a, bc, bwd, s);
+    case 32: return launch_cta_bc<32, 32, 32>(a, bc, bwd, s);
+    case 64: return launch_cta_bc<64, 64, 48>(a, bc, bwd, s);
+    case 128: return launch_cta_bc<128, 96, 64>(a, bc, bwd, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -1,7 +1,6 @@
 // k_misc.cu -- the bandwidth-bound kernels of the step: the packed-layout
-// gather (a4), the narrow input projection (a5 for in_dim <= 16), split-K
-// and column-sum reductions used by the weight gradients (a10, a12), and the
-// SGD update (a13).
+// gather (a4), the narrow input projection (a5 for in_dim <= 16) and the SGD
+// update (a13).
 #include "bkt_internal.h"
 
 namespace bkt {
@@ -89,43 +88,6 @@ cudaError_t launch_proj_narrow(const float *X, int n_tok, int in_dim, const floa
     default:
       return cudaErrorInvalidValue;
   }
-  return cudaGetLastError();
-}
-
-// ---------------------------------------------------------------------------
-// Split-K reduction: out[i] = P[0][i] + P[1][i] + ... in split order.
-__global__ void splitk_reduce_kernel(const float *__restrict__ P, int splits, int64_t n, float *__restrict__ out) {
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-    float acc = 0.f;
-    for (int z = 0; z < splits; ++z) acc += P[(int64_t)z * n + i];
-    out[i] = acc;
-  }
-}
-
-cudaError_t launch_splitk_reduce(const float *P, int splits, int64_t n, float *out, cudaStream_t s) {
-  int64_t blocks = (n + 255) / 256;
-  if (blocks > 4096) blocks = 4096;
-  if (blocks < 1) blocks = 1;
-  splitk_reduce_kernel<<<(int)blocks, 256, 0, s>>>(P, splits, n, out);
-  return cudaGetLastError();
-}
-
-// Column sums over a token range: P[z][m] = sum_{k in split z} A[k*lda + m].
-__global__ void colsum_partial_kernel(const float *__restrict__ A, int64_t lda, int K, int M, float *__restrict__ P,
-                                      int splits) {
-  const int m = blockIdx.x * blockDim.x + threadIdx.x;
-  const int z = blockIdx.y;
-  if (m >= M) return;
-  const int chunk = (K + splits - 1) / splits;
-  const int k0 = z * chunk, k1 = min(K, k0 + chunk);
-  float acc = 0.f;
-  for (int k = k0; k < k1; ++k) acc += A[(int64_t)k * lda + m];
-  P[(int64_t)z * M + m] = acc;
-}
-
-cudaError_t launch_colsum_partial(const float *A, int64_t lda, int K, int M, float *P, int splits, cudaStream_t s) {
-  dim3 grid((M + 255) / 256, splits);
-  colsum_partial_kernel<<<grid, 256, 0, s>>>(A, lda, K, M, P, splits);
   return cudaGetLastError();
 }
 
