@@ -352,6 +352,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
                     const bkt::DevIdx &ix, const bkt_batch *bt, const float *params, float *grads, float *loss,
                     cudaStream_t s, bkt::KernelTimer *timer, int sm_count) {
   const int H = lo.H, dirs = lo.dirs, DH = dirs * H, C = lo.C, NT = ix.n_tok;
+  const bool bf16 = cfg.gemm_precision == BKT_GEMM_BF16;
   Launch L{timer, s};
 
   // ---- a4: packed time-major input
@@ -365,6 +366,27 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
       L.run("proj_narrow", [&] {
         return bkt::launch_proj_narrow(w.X, NT, lo.D0, params, lo.w_ih[0], lo.stride(0), H, dirs, Zl, s);
       });
+    } else if (bf16) {
+      // a5 on the tensor cores: Zx = bf16(Y_{l-1}) bf16(W_ih)^T + b, fp32 accumulation
+      L.run("cast_bf16", [&] { return bkt::launch_cast_bf16(w.Y[l - 1], DH, NT, DH, w.Yb, DH, s); });
+      for (int d = 0; d < dirs; ++d) {
+        L.run("cast_bf16", [&] {
+          return bkt::launch_cast_bf16(params + lo.w_ih[l * dirs + d], DH, 4 * H, DH, w.Wb, DH, s);
+        });
+        bkt::TcGemmArgs g{};
+        g.M = NT;
+        g.N = 4 * H;
+        g.K = DH;
+        g.A = w.Yb;
+        g.lda = DH;
+        g.B = w.Wb;
+        g.ldb = DH;
+        g.D = Zl[d];
+        g.ldd = 4 * H;
+        g.bias = params + lo.bias(l, d);
+        g.err = w.status;
+        L.run("gemm_tc", [&] { return bkt::launch_gemm_bf16_tc(g, s); });
+      }
     } else {
       for (int d = 0; d < dirs; ++d) {
         bkt::GemmArgs g{};
@@ -462,13 +484,74 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     L.run("lstm_bwd", [&] { return bkt::launch_lstm_bwd(ra, geom[l], s); });
     const int D = lo.D(l);
     const float *Xl = (l == 0) ? w.X : w.Y[l - 1];
-    for (int d = 0; d < dirs; ++d) {
-      // [dW_ih | dW_hh | db] = dZ^T [X_l | h_{t-1} | 1]; h_{t-1} of token
-      // (t, r) is the row's previous token in its direction (zeros at the start)
-      wgrad(w.Z[l * dirs + d], 4 * H, 4 * H, Xl, D, D, w.Y[l] + d * H, DH, w.prev_tok[d], H,
-            grads + lo.w_ih[l * dirs + d], grads + lo.w_hh(l, d), grads + lo.bias(l, d));
+    if (bf16) {
+      const int NTp = (NT + 7) & ~7;
+      auto tc_reduce = [&](const void *B, int N, float *out) {
+        bkt::TcGemmArgs g{};
+        g.M = 4 * H;
+        g.N = N;
+        g.K = NT;
+        g.A = w.dZT;
+        g.lda = NTp;
+        g.B = B;
+        g.ldb = NTp;
+        g.P = w.part;
+        g.splits = bkt::tc_splits(g.M, g.N, NT, sm_count, w.part_floats);
+        g.err = w.status;
+        L.run("gemm_tc", [&] { return bkt::launch_gemm_bf16_tc(g, s); });
+        L.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, g.splits, g.M, g.N, out, s); });
+      };
+      for (int d = 0; d < dirs; ++d) {
+        const float *dZ = w.Z[l * dirs + d];
+        // dW_hh = dz^T h_{t-1} on the tensor cores (both operands transposed to bf16)
+        L.run("transpose_bf16", [&] { return bkt::launch_transpose_bf16(dZ, 4 * H, nullptr, NT, 4 * H, w.dZT, NTp, s); });
+        L.run("transpose_bf16", [&] {
+          return bkt::launch_transpose_bf16(w.Y[l] + d * H, DH, w.prev_tok[d], NT, H, w.BT, NTp, s);
+        });
+        tc_reduce(w.BT, H, grads + lo.w_hh(l, d));
+        if (l == 0) {
+          // narrow input: [dW_ih | db] = dz^T [X | 1] in fp32
+          wgrad(dZ, 4 * H, 4 * H, Xl, D, D, nullptr, 0, nullptr, 0, grads + lo.w_ih[l * dirs + d], nullptr,
+                grads + lo.bias(l, d));
+        } else {
+          L.run("transpose_bf16", [&] { return bkt::launch_transpose_bf16(Xl, D, nullptr, NT, D, w.BT, NTp, s); });
+          tc_reduce(w.BT, D, grads + lo.w_ih[l * dirs + d]);
+          int splits = std::min(64, std::max(1, std::min(2 * sm_count / ((4 * H + 255) / 256), NT / 64)));
+          while (splits > 1 && (size_t)splits * 4 * H > w.part_floats) --splits;
+          L.run("colsum", [&] { return bkt::launch_colsum(dZ, 4 * H, NT, 4 * H, w.part, splits, s); });
+          L.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, splits, 1, 4 * H, grads + lo.bias(l, d), s); });
+        }
+      }
+    } else {
+      for (int d = 0; d < dirs; ++d) {
+        // [dW_ih | dW_hh | db] = dZ^T [X_l | h_{t-1} | 1]; h_{t-1} of token
+        // (t, r) is the row's previous token in its direction (zeros at the start)
+        wgrad(w.Z[l * dirs + d], 4 * H, 4 * H, Xl, D, D, w.Y[l] + d * H, DH, w.prev_tok[d], H,
+              grads + lo.w_ih[l * dirs + d], grads + lo.w_hh(l, d), grads + lo.bias(l, d));
+      }
     }
-    if (l > 0) {
+    if (l > 0 && bf16) {
+      // dX = dz W_ih on the tensor cores, both directions accumulated into dY
+      for (int d = 0; d < dirs; ++d) {
+        L.run("cast_bf16", [&] { return bkt::launch_cast_bf16(w.Z[l * dirs + d], 4 * H, NT, 4 * H, w.dZb, 4 * H, s); });
+        L.run("transpose_bf16", [&] {
+          return bkt::launch_transpose_bf16(params + lo.w_ih[l * dirs + d], DH, nullptr, 4 * H, DH, w.WTb, 4 * H, s);
+        });
+        bkt::TcGemmArgs g{};
+        g.M = NT;
+        g.N = DH;
+        g.K = 4 * H;
+        g.A = w.dZb;
+        g.lda = 4 * H;
+        g.B = w.WTb;
+        g.ldb = 4 * H;
+        g.D = w.dY;
+        g.ldd = DH;
+        g.accumulate = d > 0;
+        g.err = w.status;
+        L.run("gemm_tc", [&] { return bkt::launch_gemm_bf16_tc(g, s); });
+      }
+    } else if (l > 0) {
       for (int d = 0; d < dirs; ++d) {
         bkt::GemmArgs g{};
         g.M = NT;
@@ -663,6 +746,22 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
   BKT_ALLOC(w.prev_tok[1], NT);
   BKT_ALLOC(w.row_ok, (size_t)max_batch);
   BKT_ALLOC(w.status, 1);
+  if (cfg->gemm_precision == BKT_GEMM_BF16) {
+    const size_t NTp = (NT + 7) & ~size_t(7);
+    uint16_t *p = nullptr;
+    BKT_ALLOC(p, NT * DH);
+    w.Yb = p;
+    BKT_ALLOC(p, NT * 4 * H);
+    w.dZb = p;
+    BKT_ALLOC(p, 4 * H * NTp);
+    w.dZT = p;
+    BKT_ALLOC(p, DH * NTp);
+    w.BT = p;
+    BKT_ALLOC(p, 4 * H * DH);
+    w.Wb = p;
+    BKT_ALLOC(p, DH * 4 * H);
+    w.WTb = p;
+  }
   IdxLayout il = idx_layout(max_batch, max_tokens);
   c->idx_bytes = il.bytes;
   {
@@ -735,7 +834,9 @@ extern "C" int bkt_ctx_sync_status(bkt_ctx *c) {
   if (e != cudaSuccess) return cuda_err("cudaMemcpy(status)", e);
   if (st != 0) {
     cudaMemset(c->w.status, 0, sizeof st);
-    return set_err(BKT_EDEVICE, "device check failed: a label is out of range or equals the blank (flags 0x%x)", st);
+    return set_err(BKT_EDEVICE, "device check failed (flags 0x%x):%s%s", st,
+                   (st & 1) ? " a label is out of range or equals the blank;" : "",
+                   (st & 2) ? " a tensor-core pipeline wait timed out;" : "");
   }
   return BKT_OK;
 }
@@ -870,6 +971,15 @@ int bkt::step_on_scratch(const bkt_model_cfg *cfg, const bkt_batch *bt, const fl
   w.row_ok = cv.take<int32_t>((size_t)b);
   w.status = cv.take<int32_t>(1);
   w.idx_dev = cv.take<char>(il.bytes);
+  if (cfg->gemm_precision == BKT_GEMM_BF16) {
+    const size_t NTp = (NT + 7) & ~size_t(7);
+    w.Yb = cv.take<uint16_t>(NT * DH);
+    w.dZb = cv.take<uint16_t>(NT * 4 * H);
+    w.dZT = cv.take<uint16_t>(4 * H * NTp);
+    w.BT = cv.take<uint16_t>(DH * NTp);
+    w.Wb = cv.take<uint16_t>(4 * H * DH);
+    w.WTb = cv.take<uint16_t>(DH * 4 * H);
+  }
   // split-K partials get the rest: at least one split of the largest block
   const size_t min_part = max_reduce_block(lo);
   w.part = cv.take<float>(min_part);

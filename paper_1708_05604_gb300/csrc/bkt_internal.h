@@ -84,6 +84,34 @@ struct WgradArgs {
 };
 int wgrad_splits(int M, int N, int K, int sm_count, size_t part_floats);
 cudaError_t launch_wgrad(const WgradArgs &g, float *out1, float *out2, float *out3, cudaStream_t s);
+// out[m*N + n] = sum_z P[z][m][n] (fixed order).
+cudaError_t launch_splitk_sum(const float *P, int splits, int M, int N, float *out, cudaStream_t s);
+
+// Operand preparation for the bf16 GEMMs (k_convert.cu).
+cudaError_t launch_cast_bf16(const float *src, int64_t lds, int R, int C, void *dst, int64_t ldd, cudaStream_t s);
+// dst[c][r] = bf16(src[src_row ? src_row[r] : r][c]), zeros where src_row[r] < 0.
+cudaError_t launch_transpose_bf16(const float *src, int64_t lds, const int32_t *src_row, int R, int C, void *dst,
+                                  int64_t ldd, cudaStream_t s);
+cudaError_t launch_colsum(const float *A, int64_t lda, int R, int M, float *P, int splits, cudaStream_t s);
+
+// bf16 tensor-core GEMM (k_gemm_tc.cu):
+//   D[m][n] (+)= sum_k A[m][k] B[n][k] (+ bias[n]); A, B bf16 with K contiguous
+//   (lda, ldb multiples of 8 elements, 16-byte aligned bases); D fp32 row-major.
+//   P != null: split the k range over `splits` and write partial tiles
+//   P[z][m][n] instead (D, bias, accumulate unused).  err: device flag word
+//   (bit 1 set if a pipeline wait timed out).
+struct TcGemmArgs {
+  int M, N, K;
+  const void *A; int64_t lda;
+  const void *B; int64_t ldb;
+  float *D; int64_t ldd;
+  const float *bias;
+  int accumulate;
+  float *P; int splits;
+  int32_t *err;
+};
+int tc_splits(int M, int N, int K, int sm_count, size_t part_floats);
+cudaError_t launch_gemm_bf16_tc(const TcGemmArgs &g, cudaStream_t s);
 
 // a7: logp[tok][c] = log-softmax_c(b[c] + W[c] . Y[tok]).
 cudaError_t launch_out_logsoftmax(const float *Y, int n_tok, int DH, const float *W,
@@ -157,6 +185,13 @@ struct StepBufs {
   int32_t *row_ok;                            // [b]
   int32_t *status;                            // device error flags
   void *idx_dev;                              // per-step index block
+  // bf16 GEMM path only (null otherwise)
+  void *Yb;                                   // [NT x dirs*H] bf16 layer input of a projection
+  void *dZb;                                  // [NT x 4H] bf16 dz (input-gradient GEMM)
+  void *dZT;                                  // [4H x NTp] bf16 dz transposed (weight gradients)
+  void *BT;                                   // [max(dirs*H, H) x NTp] bf16 transposed X or h_{t-1}
+  void *Wb;                                   // [4H x dirs*H] bf16 W_ih of one layer and direction
+  void *WTb;                                  // [dirs*H x 4H] bf16 W_ih transposed
 };
 
 // Records an error message for bkt_last_error() and returns `code`.

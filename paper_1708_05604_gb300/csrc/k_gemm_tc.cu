@@ -1,0 +1,297 @@
+// k_gemm_tc.cu -- bf16 GEMM on the 5th-generation tensor cores for the
+// contractions of the bf16 path (input projection of layers > 1, weight
+// gradients, input gradients):
+//   D[m][n] (+)= sum_k A[m][k] * B[n][k]  (+ bias[n]),   fp32 accumulation
+// A [M x K] and B [N x K] are bf16 with K contiguous (row-major); D is fp32.
+//
+// One CTA computes a 128 x 256 tile.  Warp 0 (one lane) streams 64-wide k
+// slabs of A and B into shared memory with TMA (128-byte swizzle) through a
+// 4-stage mbarrier ring; warp 1 (one lane) issues tcgen05.mma (M=128, N=256,
+// K=16 per instruction) into a 256-column TMEM accumulator and releases each
+// stage with tcgen05.commit; after the last slab all four warps read the
+// accumulator back with tcgen05.ld (warp w owns TMEM lanes 32w..32w+31, i.e.
+// tile rows) and write fp32 to global memory.  The token range can be split
+// over gridDim.z, each split writing its own partial tile.  Every mbarrier
+// wait is bounded: on expiry the CTA records an error flag, still waits for
+// its issued MMAs through the final commit, frees TMEM and exits.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <mutex>
+
+#include "bkt_internal.h"
+
+namespace bkt {
+
+namespace {
+
+constexpr int TBM = 128, TBN = 256, TBK = 64, TSTAGES = 4;
+constexpr uint32_t kAStage = TBM * TBK * 2;  // 16 KB
+constexpr uint32_t kBStage = TBN * TBK * 2;  // 32 KB
+constexpr uint32_t kTxBytes = kAStage + kBStage;
+constexpr size_t kTcSmem = 1024 + (size_t)TSTAGES * (kAStage + kBStage) + 256;
+constexpr uint32_t kWaitPolls = 1u << 22;
+// kind::f16 instruction descriptor: D fp32 (bit 4), A and B bf16 (bits 7, 10),
+// both K-major (bits 15, 16 clear), N >> 3 at bit 17, M >> 4 at bit 24.
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(TBN >> 3) << 17) |
+                            ((uint32_t)(TBM >> 4) << 24);
+
+__device__ __forceinline__ uint32_t su32(const void *p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t a, uint32_t n) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(a), "r"(n) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t a, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(a), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t a) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(a) : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(a), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait for the phase with the given parity; false on expiry.
+__device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity) {
+  for (uint32_t i = 0; i < kWaitPolls; ++i)
+    if (mbar_try(a, parity)) return true;
+  return false;
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y, uint32_t mbar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(mbar)
+      : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_commit(uint32_t mbar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(mbar) : "memory");
+}
+__device__ __forceinline__ void tc_mma(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+// Shared-memory matrix descriptor of a K-major tile written by TMA with the
+// 128-byte swizzle: rows of 128 B, 8-row groups 1024 B apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1 << 16;            // leading byte offset (not used by swizzled K-major)
+  d |= (uint64_t)(1024 >> 4) << 32;  // stride byte offset
+  d |= (uint64_t)1 << 46;            // descriptor version
+  d |= (uint64_t)2 << 61;            // 128-byte swizzle
+  return d;
+}
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr)
+      : "memory");
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+}  // namespace
+
+__global__ void __launch_bounds__(128, 1)
+    gemm_bf16_tc_kernel(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb, TcGemmArgs g) {
+  extern __shared__ uint8_t tc_smem_raw[];
+  uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(tc_smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t *sA = base;
+  uint8_t *sB = base + TSTAGES * kAStage;
+  uint64_t *bars = reinterpret_cast<uint64_t *>(sB + TSTAGES * kBStage);  // full[S], empty[S], done
+  uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 2 * TSTAGES + 1);
+  int *abort_s = reinterpret_cast<int *>(tslot + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m0 = blockIdx.x * TBM, n0 = blockIdx.y * TBN;
+  const int splits = g.P ? g.splits : 1;
+  const int nkb = (g.K + TBK - 1) / TBK;
+  const int chunk = (nkb + splits - 1) / splits;
+  const int kb0 = blockIdx.z * chunk;
+  const int nk = max(0, min(nkb, kb0 + chunk) - kb0);
+  const uint32_t full0 = su32(bars), empty0 = su32(bars + TSTAGES), done = su32(bars + 2 * TSTAGES);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < TSTAGES; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    mbar_init(done, 1);
+    *abort_s = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tslot)), "r"(TBN)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tslot;
+
+  if (warp == 0) {
+    if (lane == 0) {  // TMA producer
+      for (int i = 0; i < nk; ++i) {
+        const int s = i % TSTAGES;
+        if (i >= TSTAGES && !mbar_wait(empty0 + 8 * s, ((i / TSTAGES) - 1) & 1)) {
+          *abort_s = 1;
+          break;
+        }
+        mbar_expect_tx(full0 + 8 * s, kTxBytes);
+        const int kx = (kb0 + i) * TBK;
+        tma_load_2d(su32(sA + s * kAStage), &ta, kx, m0, full0 + 8 * s);
+        tma_load_2d(su32(sB + s * kBStage), &tb, kx, n0, full0 + 8 * s);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {  // MMA issuer
+      int issued = 0;
+      for (int i = 0; i < nk; ++i) {
+        const int s = i % TSTAGES;
+        if (!mbar_wait(full0 + 8 * s, (i / TSTAGES) & 1)) {
+          *abort_s = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a0 = su32(sA + s * kAStage), b0 = su32(sB + s * kBStage);
+#pragma unroll
+        for (int kk = 0; kk < TBK / 16; ++kk)
+          tc_mma(tmem, sw128_desc(a0 + kk * 32), sw128_desc(b0 + kk * 32), kIdesc, (i > 0 || kk > 0) ? 1u : 0u);
+        tc_commit(empty0 + 8 * s);
+        ++issued;
+      }
+      // the final commit tracks every MMA issued above
+      if (issued > 0) tc_commit(done);
+      else mbar_arrive(done);
+    }
+    __syncwarp();
+  }
+
+  // epilogue: TMEM -> registers -> global
+  const bool ready = mbar_wait(done, 0);
+  if (!ready) *abort_s = 1;
+  tc_fence_after();
+  const int row = warp * 32 + lane;
+  const int m = m0 + row;
+  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+  const bool write = ready && m < g.M;
+  float *out;
+  int64_t ld;
+  if (g.P) {
+    out = g.P + (int64_t)blockIdx.z * g.M * g.N + (int64_t)m * g.N;
+    ld = g.N;
+  } else {
+    out = g.D + (int64_t)m * g.ldd;
+    ld = g.ldd;
+  }
+  const bool vec = ((ld & 3) == 0) && ((reinterpret_cast<uintptr_t>(g.P ? g.P : g.D) & 15) == 0);
+#pragma unroll 1
+  for (int c0 = 0; c0 < TBN; c0 += 32) {
+    uint32_t v[32];
+    __syncwarp();
+    tmem_ld32(trow + c0, v);
+    if (!write) continue;
+    const int nb = n0 + c0;
+    if (nb >= g.N) continue;
+    float x[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) x[j] = nk > 0 ? __uint_as_float(v[j]) : 0.f;
+    if (!g.P) {
+      if (g.bias)
+#pragma unroll
+        for (int j = 0; j < 32; ++j) x[j] += (nb + j < g.N) ? g.bias[nb + j] : 0.f;
+      if (g.accumulate)
+#pragma unroll
+        for (int j = 0; j < 32; ++j) x[j] += (nb + j < g.N) ? out[nb + j] : 0.f;
+    }
+    if (vec && nb + 32 <= g.N) {
+#pragma unroll
+      for (int j = 0; j < 32; j += 4)
+        *reinterpret_cast<float4 *>(out + nb + j) = make_float4(x[j], x[j + 1], x[j + 2], x[j + 3]);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (nb + j < g.N) out[nb + j] = x[j];
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TBN) : "memory");
+  if (threadIdx.x == 0 && *abort_s && g.err) atomicOr(g.err, 2);
+}
+
+// ---------------------------------------------------------------------------
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2-D bf16 map over a row-major [rows x inner] matrix with row stride `ld`
+// elements; boxes of 64 (inner) x box_rows with the 128-byte swizzle.
+bool make_map(CUtensorMap *map, const void *base, uint64_t inner, uint64_t rows, int64_t ld, uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {inner, rows};
+  cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
+  cuuint32_t box[2] = {(cuuint32_t)TBK, box_rows};
+  cuuint32_t es[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+int tc_splits(int M, int N, int K, int sm_count, size_t part_floats) {
+  const int tiles = ((M + TBM - 1) / TBM) * ((N + TBN - 1) / TBN);
+  const int nkb = (K + TBK - 1) / TBK;
+  int s = std::max(1, sm_count / std::max(1, tiles));
+  s = std::min(s, std::max(1, nkb / 4));  // at least 4 k slabs per split
+  s = std::min(s, 64);
+  while (s > 1 && (size_t)s * M * N > part_floats) --s;
+  return s;
+}
+
+cudaError_t launch_gemm_bf16_tc(const TcGemmArgs &g, cudaStream_t s) {
+  if (g.M <= 0 || g.N <= 0) return cudaSuccess;
+  if (g.K <= 0 || (g.lda & 7) || (g.ldb & 7) || (reinterpret_cast<uintptr_t>(g.A) & 15) ||
+      (reinterpret_cast<uintptr_t>(g.B) & 15) || (g.P && g.splits < 1) || (!g.P && !g.D))
+    return cudaErrorInvalidValue;
+  CUtensorMap ta, tb;
+  if (!make_map(&ta, g.A, (uint64_t)g.K, (uint64_t)g.M, g.lda, TBM)) return cudaErrorInvalidValue;
+  if (!make_map(&tb, g.B, (uint64_t)g.K, (uint64_t)g.N, g.ldb, TBN)) return cudaErrorInvalidValue;
+  cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kTcSmem);
+  if (e != cudaSuccess) return e;
+  dim3 grid((g.M + TBM - 1) / TBM, (g.N + TBN - 1) / TBN, g.P ? g.splits : 1);
+  if (grid.y > 65535u || grid.z > 65535u) return cudaErrorInvalidConfiguration;
+  gemm_bf16_tc_kernel<<<grid, 128, kTcSmem, s>>>(ta, tb, g);
+  return cudaGetLastError();
+}
+
+}  // namespace bkt

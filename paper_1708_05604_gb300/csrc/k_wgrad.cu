@@ -168,4 +168,12 @@ cudaError_t launch_wgrad(const WgradArgs &g, float *out1, float *out2, float *ou
   return cudaGetLastError();
 }
 
+cudaError_t launch_splitk_sum(const float *P, int splits, int M, int N, float *out, cudaStream_t s) {
+  const int64_t total = (int64_t)M * N;
+  if (total <= 0) return cudaSuccess;
+  int blocks = (int)std::min<int64_t>(4096, (total + 255) / 256);
+  wgrad_reduce_kernel<<<blocks, 256, 0, s>>>(P, splits, M, N, N, 0, out, nullptr, nullptr);
+  return cudaGetLastError();
+}
+
 }  // namespace bkt

@@ -222,3 +222,21 @@ def test_full_size_batch_sampled(wname, Q):
     _, ga = gpu_step(cfg, ds, params, seq_ids=ids[:h], dd=dd)
     _, gb = gpu_step(cfg, ds, params, seq_ids=ids[h:], dd=dd)
     assert np.linalg.norm(ga + gb - gg) <= 1e-4 * np.linalg.norm(gg)
+
+
+def test_bf16_workload_runs_on_tensor_cores():
+    """The bf16 workloads route their contractions through the tcgen05 GEMM
+    (and stay within the bf16 tolerance while differing from fp32 rounding)."""
+    import torch
+    cfg, ds, params = make_case("lstm3_bi_h256_bf16", 4, 80, seed=3)
+    ctx = binding.Ctx(cfg, int(ds.lengths.sum()), ds.n, int(ds.label_lengths.max()))
+    ctx.set_timing(True)
+    lg, gg = gpu_step(cfg, ds, params, ctx=ctx)
+    names = {n: c for n, c, _ in ctx.kernel_times()}
+    assert names.get("gemm_tc", 0) >= 2 * 2 + 2 * 3 * 2, names   # projections, dX, weight grads
+    lo, go = oracle_step(cfg, ds, params)
+    worst = compare(cfg, lg, gg, lo, go, BF16_TOL)
+    assert worst > 1e-6   # bf16 operands really are in play
+    fcfg = dict(cfg, gemm_bf16=False)
+    lf, gf = gpu_step(fcfg, ds, params)
+    compare(fcfg, lf, gf, lo, go, FP32_TOL)
