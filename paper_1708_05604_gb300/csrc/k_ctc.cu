@@ -114,16 +114,20 @@ cudaError_t launch_out_logsoftmax(const float *Y, int n_tok, int DH, const float
 // the next step.  Emissions are prefetched 8 steps ahead into registers.
 namespace {
 
+// The recursion's serial chain runs T steps; the hardware exp2/log2
+// approximations keep each step short.  Their error (a few ulp on arguments
+// in (-inf, 0] and on sums in [1, 3]) is re-anchored every step by the
+// running-maximum shift, so it does not grow with T.
 __device__ __forceinline__ float lse3(float a, float b, float c) {
   const float m = fmaxf(a, fmaxf(b, c));
   if (m == -CUDART_INF_F) return -CUDART_INF_F;
-  return m + logf(expf(a - m) + expf(b - m) + expf(c - m));
+  return m + __logf(__expf(a - m) + __expf(b - m) + __expf(c - m));
 }
 
 __device__ __forceinline__ float lse2(float a, float b) {
   const float m = fmaxf(a, b);
   if (m == -CUDART_INF_F) return -CUDART_INF_F;
-  return m + logf(expf(a - m) + expf(b - m));
+  return m + __logf(__expf(a - m) + __expf(b - m));
 }
 
 constexpr int kPre = 8;  // emission prefetch depth (steps)

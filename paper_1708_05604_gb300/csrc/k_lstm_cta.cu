@@ -1,31 +1,38 @@
-// k_lstm_cta.cu -- single-CTA persistent recurrent kernels for H <= 128
-// (a6 forward, a11 BPTT).
+// k_lstm_cta.cu -- single-CTA persistent recurrent kernels for H in {32, 64,
+// 128} (a6 forward, a11 BPTT).
 //
 // Same recurrence as the cluster kernels (gates i, f, g, o; the reverse
 // direction over each sequence's own length), but one CTA holds the whole
 // 4H x H fp32 W_hh of its direction, so a time step needs no inter-SM
-// exchange at all: two CTA barriers per step are the only synchronisation.
-// For H = 128 the matrix is 256 KB, more than shared memory.  2H threads each
-// own two rows (or, in BPTT, two column segments), keep RK weights of each in
-// registers (192 registers for H = 128) and the rest in shared memory (laid
-// out so a warp reads 512 consecutive bytes).  Each h value read from shared
-// memory feeds both rows, so a step moves half the shared-memory bytes of a
-// one-row-per-thread layout, which was bound by shared-memory bandwidth.
+// exchange at all.
 //
-// Forward, 2H threads, thread t owns gate rows t (i or f) and t + 2H (g or o):
-//   phase A (all threads): z_r = Zx[r] + W_hh[r,:] . h_{s-1}   (h broadcast
-//            from shared memory), activation of row r (tanh for the g block,
-//            sigmoid otherwise), written to shared memory and, in place over
-//            Zx, to global memory;
-//   phase B (threads t < H = unit t): c = f c + i g, h = o tanh(c).
-// BPTT, 2H threads, thread t = (q, kc) owns the column segments
-// W_hh[q*H .. q*H+H-1, k] for k = kc and kc + H/2 of gate block q:
-//   phase B (threads t < H = unit t): dh = dY + sum_q part[q][t]; dc, dz of
-//            the four gates (written in place over the gates);
-//   phase A (all threads): part[q][k] = sum_i W_hh[q*H+i, k] dz[q*H+i].
+// Register tiling.  2H threads; lane l of warp w belongs to row group
+// rg = 4w + l/8 and k slice ks = l % 8.  Row group rg is the 16 gate rows of
+// units u0..u0+3 (u0 = 4 rg), ordered [i, f, g, o] per unit; k slice ks is the
+// KPT = H/8 columns ks*KPT .. ks*KPT+KPT-1.  Each thread keeps its 16 x KPT
+// tile of W_hh for the whole sequence: RKK columns in registers (192 weights
+// at H = 128) and the rest in shared memory.  A thread reads only the KPT
+// values of h (forward) or the 16 values of dz (backward) that its tile
+// needs, so the shared-memory bytes per step stay small; a shared-memory
+// broadcast of all of h to every thread would cost 1 KB of load bandwidth
+// per thread per step.
+//
+// Forward step: 16 partial dot products per thread over its k slice; an
+// 8-lane shuffle reduce-scatter leaves lane ks with rows 2ks, 2ks+1 of the
+// group, i.e. (i, f) or (g, o) of unit u0 + ks/2; activations; the two lanes
+// of a unit swap their pair and both update c = f c + i g, h = o tanh(c);
+// h goes to the other half of a double buffer; one CTA barrier.
+// BPTT step: (B) lanes 2j, 2j+1 form dh = dY + sum of the per-warp partials
+// of W_hh^T dz for unit j, and dz of its four gates (written in place over the
+// gates); barrier; (A) each thread multiplies its tile by the 16 dz values of
+// its rows, a shuffle reduce-scatter over the warp's four row groups sums the
+// tile products per column, and each warp stores its column partials;
+// barrier.
 // A CTA owns BC consecutive rows of the length-sorted batch (BC = 1 when the
-// batch fits the GPU) and stops after its longest row.  Per-step global loads
-// are issued one step ahead.
+// batch fits the GPU) and stops after its longest row.  Each thread keeps the
+// global inputs of the next kPF steps in flight with asynchronous copies into
+// a small shared-memory ring (global-memory latency under load is about one
+// time step).
 #include <algorithm>
 
 #include "bkt_internal.h"
@@ -35,43 +42,103 @@ namespace bkt {
 namespace {
 
 constexpr int kTokCap = 8192;  // time offsets staged in shared memory up to this T
+constexpr int kPF = 4;         // steps of per-step global inputs kept in flight
+constexpr int kRing = kPF + 1; // ring slots: a copy never lands in the slot read this step
 
 __device__ __forceinline__ float sigm(float x) { return 1.f / (1.f + expf(-x)); }
 
+// Per-thread asynchronous copies (global -> shared) for the step inputs:
+// one commit group per step, so waiting for all but the newest kPF-1 groups
+// makes the oldest step's values visible to the issuing thread.
+__device__ __forceinline__ void cp_async4(float *dst, const float *src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
+               "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_wait_all_but_newest() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(kPF - 1) : "memory");
+}
+
+// Reduce-scatter over the 8 lanes of a k-slice group (lane bits 0..2): on
+// return, lane l holds the group sums of positions 2(l%8) and 2(l%8)+1.
+__device__ __forceinline__ void reduce_scatter8(const float (&v)[16], int lane, float &o0, float &o1) {
+  const bool b2 = (lane >> 2) & 1, b1 = (lane >> 1) & 1, b0 = lane & 1;
+  float r8[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float send = b2 ? v[i] : v[i + 8], keep = b2 ? v[i + 8] : v[i];
+    r8[i] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+  }
+  float r4[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float send = b1 ? r8[i] : r8[i + 4], keep = b1 ? r8[i + 4] : r8[i];
+    r4[i] = keep + __shfl_xor_sync(0xffffffffu, send, 2);
+  }
+  const float s0 = b0 ? r4[0] : r4[2], k0 = b0 ? r4[2] : r4[0];
+  const float s1 = b0 ? r4[1] : r4[3], k1 = b0 ? r4[3] : r4[1];
+  o0 = k0 + __shfl_xor_sync(0xffffffffu, s0, 1);
+  o1 = k1 + __shfl_xor_sync(0xffffffffu, s1, 1);
+}
+
+// Reduce-scatter of KPT column sums over the warp's four row groups (lane
+// bits 3, 4): on return, lane holds the sums of columns
+// rgl*(KPT/4) .. rgl*(KPT/4) + KPT/4 - 1 of its slice (rgl = lane / 8).
+template <int KPT>
+__device__ __forceinline__ void reduce_groups(const float (&v)[KPT], int lane, float (&out)[KPT / 4]) {
+  const bool b4 = (lane >> 4) & 1, b3 = (lane >> 3) & 1;
+  float r[KPT / 2];
+#pragma unroll
+  for (int i = 0; i < KPT / 2; ++i) {
+    const float send = b4 ? v[i] : v[i + KPT / 2], keep = b4 ? v[i + KPT / 2] : v[i];
+    r[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
+  }
+#pragma unroll
+  for (int i = 0; i < KPT / 4; ++i) {
+    const float send = b3 ? r[i] : r[i + KPT / 4], keep = b3 ? r[i + KPT / 4] : r[i];
+    out[i] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+  }
+}
+
 }  // namespace
 
-template <int H, int RK, int BC>
+template <int H, int RKK, int BC>
 __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
-  constexpr int G = 4 * H, NTH = 2 * H, SK = H - RK, H4 = H / 4;
+  constexpr int G = 4 * H, NTH = 2 * H, KPT = H / 8, SKK = KPT - RKK, HS = KPT + 4;
+  static_assert(SKK % 4 == 0 && RKK % 4 == 0, "k split in float4 steps");
   extern __shared__ __align__(16) float sm[];
-  float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [SK/4][2][NTH]
-  float *hs = sm + 2 * SK * NTH;                 // [2][BC][H]
-  float *zs = hs + 2 * BC * H;                   // [BC][G]
+  float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [SKK/4][16][NTH]
+  float *hs = sm + SKK * 16 * NTH;               // [2][BC][8 slices][HS]
+  float *zr = hs + 2 * BC * 8 * HS;              // [BC][kRing][NTH][2] Zx of upcoming steps
   const int T = a.ix.T;
   const bool toff_sm = T + 1 <= kTokCap;
-  int *toff_s = reinterpret_cast<int *>(zs + BC * G);
+  int *toff_s = reinterpret_cast<int *>(zr + BC * kRing * NTH * 2);
   const int *toff = toff_sm ? toff_s : a.ix.tok_off;
-  const int t = threadIdx.x;
-  const bool lo_half = t < H;  // rows t (i or f) and t + 2H (g or o)
+  const int t = threadIdx.x, lane = t & 31;
+  const int ks = lane & 7, rg = (t >> 5) * 4 + (lane >> 3);
+  const int u0 = 4 * rg, kb = ks * KPT;
+  const int unit = u0 + (ks >> 1), pair = ks & 1;  // after the reduce-scatter
+  const int q0 = 2 * pair;                         // this lane's gates q0, q0 + 1
   const int n_groups = (a.ix.b + BC - 1) / BC;
   const int d = blockIdx.x / n_groups, grp = blockIdx.x % n_groups;
   const int r0 = grp * BC;
   const int DH = a.dirs * H;
+  const float *__restrict__ Whh = a.Whh[d];
 
-  const float *W0 = a.Whh[d] + (size_t)t * H;
-  const float *W1 = a.Whh[d] + (size_t)(t + NTH) * H;
-  float w0[RK], w1[RK];
+  float w[16][RKK > 0 ? RKK : 1];
 #pragma unroll
-  for (int i = 0; i < RK; ++i) {
-    w0[i] = __ldg(W0 + i);
-    w1[i] = __ldg(W1 + i);
+  for (int ri = 0; ri < 16; ++ri) {
+    const float *row = Whh + (size_t)((ri & 3) * H + u0 + (ri >> 2)) * H + kb;
+#pragma unroll
+    for (int kk = 0; kk < RKK; ++kk) w[ri][kk] = __ldg(row + kk);
+#pragma unroll
+    for (int k4 = 0; k4 < SKK / 4; ++k4) {
+      const float *p = row + RKK + 4 * k4;
+      Ws4[(k4 * 16 + ri) * NTH + t] = make_float4(__ldg(p), __ldg(p + 1), __ldg(p + 2), __ldg(p + 3));
+    }
   }
-  for (int i4 = 0; i4 < SK / 4; ++i4) {
-    const float *u = W0 + RK + 4 * i4, *v = W1 + RK + 4 * i4;
-    Ws4[(2 * i4) * NTH + t] = make_float4(__ldg(u), __ldg(u + 1), __ldg(u + 2), __ldg(u + 3));
-    Ws4[(2 * i4 + 1) * NTH + t] = make_float4(__ldg(v), __ldg(v + 1), __ldg(v + 2), __ldg(v + 3));
-  }
-  for (int i = t; i < 2 * BC * H; i += NTH) hs[i] = 0.f;
+  for (int i = t; i < 2 * BC * 8 * HS; i += NTH) hs[i] = 0.f;
   if (toff_sm)
     for (int i = t; i <= T; i += NTH) toff_s[i] = a.ix.tok_off[i];
   int len[BC];
@@ -83,138 +150,123 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
   float *__restrict__ Z = a.Z[d];
   float *__restrict__ Cs = a.Cst[d];
   float *__restrict__ Y = a.Y;
+  const int zo0 = q0 * H + unit, zo1 = zo0 + H;  // offsets of this lane's gates in a Z row
+  const int hslot = (unit / KPT) * HS + unit % KPT;
   auto tok_at = [&](int b, int s) {
     const int tt = d == 0 ? s : len[b] - 1 - s;
     return toff[tt] + r0 + b;
   };
-  float zn0[BC], zn1[BC], cst[BC];
-  int tokn[BC];
-#pragma unroll
-  for (int b = 0; b < BC; ++b) {
-    cst[b] = 0.f;
-    tokn[b] = 0;
-    zn0[b] = zn1[b] = 0.f;
-    if (len[b] > 0) {
-      tokn[b] = tok_at(b, 0);
-      zn0[b] = Z[(size_t)tokn[b] * G + t];
-      zn1[b] = Z[(size_t)tokn[b] * G + NTH + t];
+  float cst[BC];
+  auto issue = [&](int b, int s) {  // Zx of step s of row b into its ring slot
+    if (s < len[b]) {
+      const int tk = tok_at(b, s);
+      float *slot = zr + (((size_t)b * kRing + s % kRing) * NTH + t) * 2;
+      cp_async4(slot, Z + (size_t)tk * G + zo0);
+      cp_async4(slot + 1, Z + (size_t)tk * G + zo1);
     }
+  };
+#pragma unroll
+  for (int b = 0; b < BC; ++b) cst[b] = 0.f;
+  for (int j = 0; j < kPF; ++j) {
+#pragma unroll
+    for (int b = 0; b < BC; ++b) issue(b, j);
+    cp_commit();
   }
   for (int s = 0; s < Tg; ++s) {
     const int p = s & 1;
-    float zc0[BC], zc1[BC];
-    int tc[BC];
+    cp_wait_all_but_newest();
 #pragma unroll
     for (int b = 0; b < BC; ++b) {
-      zc0[b] = zn0[b];
-      zc1[b] = zn1[b];
-      tc[b] = tokn[b];
-      if (s + 1 < len[b]) {
-        tokn[b] = tok_at(b, s + 1);
-        zn0[b] = Z[(size_t)tokn[b] * G + t];
-        zn1[b] = Z[(size_t)tokn[b] * G + NTH + t];
-      }
-    }
-    // phase A: two rows per thread, two accumulators per row
-    float a0[BC], a1[BC], e0[BC], e1[BC];
+      if (s >= len[b]) continue;  // uniform over the CTA
+      const float *slot = zr + (((size_t)b * kRing + s % kRing) * NTH + t) * 2;
+      const float zc0 = slot[0], zc1 = slot[1];
+      const int tc = tok_at(b, s);
+      issue(b, s + kPF);
+      const float *hv = hs + (p * BC + b) * 8 * HS + ks * HS;
+      float acc[16];
 #pragma unroll
-    for (int b = 0; b < BC; ++b) a0[b] = a1[b] = e0[b] = e1[b] = 0.f;
-    const float4 *h4 = reinterpret_cast<const float4 *>(hs + p * BC * H);
+      for (int ri = 0; ri < 16; ++ri) acc[ri] = 0.f;
 #pragma unroll
-    for (int i4 = 0; i4 < RK / 4; ++i4) {
+      for (int k4 = 0; k4 < RKK / 4; ++k4) {
+        const float4 h4 = *reinterpret_cast<const float4 *>(hv + 4 * k4);
 #pragma unroll
-      for (int b = 0; b < BC; ++b) {
-        const float4 hv = h4[b * H4 + i4];
-        a0[b] = fmaf(w0[4 * i4], hv.x, a0[b]);
-        a1[b] = fmaf(w1[4 * i4], hv.x, a1[b]);
-        e0[b] = fmaf(w0[4 * i4 + 1], hv.y, e0[b]);
-        e1[b] = fmaf(w1[4 * i4 + 1], hv.y, e1[b]);
-        a0[b] = fmaf(w0[4 * i4 + 2], hv.z, a0[b]);
-        a1[b] = fmaf(w1[4 * i4 + 2], hv.z, a1[b]);
-        e0[b] = fmaf(w0[4 * i4 + 3], hv.w, e0[b]);
-        e1[b] = fmaf(w1[4 * i4 + 3], hv.w, e1[b]);
-      }
-    }
-#pragma unroll
-    for (int i4 = 0; i4 < SK / 4; ++i4) {
-      const float4 u = Ws4[(2 * i4) * NTH + t];
-      const float4 v = Ws4[(2 * i4 + 1) * NTH + t];
-#pragma unroll
-      for (int b = 0; b < BC; ++b) {
-        const float4 hv = h4[b * H4 + RK / 4 + i4];
-        a0[b] = fmaf(u.x, hv.x, a0[b]);
-        a1[b] = fmaf(v.x, hv.x, a1[b]);
-        e0[b] = fmaf(u.y, hv.y, e0[b]);
-        e1[b] = fmaf(v.y, hv.y, e1[b]);
-        a0[b] = fmaf(u.z, hv.z, a0[b]);
-        a1[b] = fmaf(v.z, hv.z, a1[b]);
-        e0[b] = fmaf(u.w, hv.w, e0[b]);
-        e1[b] = fmaf(v.w, hv.w, e1[b]);
-      }
-    }
-#pragma unroll
-    for (int b = 0; b < BC; ++b) {
-      if (s < len[b]) {
-        const float v0 = sigm(a0[b] + e0[b] + zc0[b]);                       // i or f
-        const float z1 = a1[b] + e1[b] + zc1[b];
-        const float v1 = lo_half ? tanhf(z1) : sigm(z1);                      // g or o
-        zs[b * G + t] = v0;
-        zs[b * G + NTH + t] = v1;
-        Z[(size_t)tc[b] * G + t] = v0;
-        Z[(size_t)tc[b] * G + NTH + t] = v1;
-      }
-    }
-    __syncthreads();
-    // phase B
-    if (t < H) {
-#pragma unroll
-      for (int b = 0; b < BC; ++b) {
-        if (s < len[b]) {
-          const float ig = zs[b * G + t], fg = zs[b * G + H + t], gg = zs[b * G + 2 * H + t],
-                      og = zs[b * G + 3 * H + t];
-          cst[b] = fmaf(fg, cst[b], ig * gg);
-          const float h = og * tanhf(cst[b]);
-          hs[(p ^ 1) * BC * H + b * H + t] = h;
-          Cs[(size_t)tc[b] * H + t] = cst[b];
-          Y[(size_t)tc[b] * DH + d * H + t] = h;
+        for (int ri = 0; ri < 16; ++ri) {
+          float x = fmaf(w[ri][4 * k4], h4.x, acc[ri]);
+          x = fmaf(w[ri][4 * k4 + 1], h4.y, x);
+          x = fmaf(w[ri][4 * k4 + 2], h4.z, x);
+          acc[ri] = fmaf(w[ri][4 * k4 + 3], h4.w, x);
         }
       }
+#pragma unroll
+      for (int k4 = 0; k4 < SKK / 4; ++k4) {
+        const float4 h4 = *reinterpret_cast<const float4 *>(hv + RKK + 4 * k4);
+#pragma unroll
+        for (int ri = 0; ri < 16; ++ri) {
+          const float4 wv = Ws4[(k4 * 16 + ri) * NTH + t];
+          float x = fmaf(wv.x, h4.x, acc[ri]);
+          x = fmaf(wv.y, h4.y, x);
+          x = fmaf(wv.z, h4.z, x);
+          acc[ri] = fmaf(wv.w, h4.w, x);
+        }
+      }
+      float v0, v1;
+      reduce_scatter8(acc, lane, v0, v1);
+      // lane pair 0 holds (i, f), pair 1 holds (g, o) of `unit`
+      const float a0 = pair ? tanhf(v0 + zc0) : sigm(v0 + zc0);
+      const float a1 = sigm(v1 + zc1);
+      Z[(size_t)tc * G + zo0] = a0;
+      Z[(size_t)tc * G + zo1] = a1;
+      const float x0 = __shfl_xor_sync(0xffffffffu, a0, 1), x1 = __shfl_xor_sync(0xffffffffu, a1, 1);
+      const float ig = pair ? x0 : a0, fg = pair ? x1 : a1, gg = pair ? a0 : x0, og = pair ? a1 : x1;
+      cst[b] = fmaf(fg, cst[b], ig * gg);
+      const float h = og * tanhf(cst[b]);
+      if (pair == 0) {
+        hs[((p ^ 1) * BC + b) * 8 * HS + hslot] = h;
+      } else {
+        Cs[(size_t)tc * H + unit] = cst[b];
+        Y[(size_t)tc * DH + d * H + unit] = h;
+      }
     }
+    cp_commit();
     __syncthreads();
   }
+  asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
-template <int H, int RK, int BC>
+template <int H, int RKK, int BC>
 __global__ void __launch_bounds__(2 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
-  constexpr int G = 4 * H, NTH = 2 * H, SK = H - RK;
+  constexpr int G = 4 * H, NTH = 2 * H, KPT = H / 8, SKK = KPT - RKK, NW = NTH / 32;
+  static_assert(SKK % 4 == 0 && RKK % 4 == 0 && KPT % 4 == 0, "k split in float4 steps");
   extern __shared__ __align__(16) float sm[];
-  float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [SK/4][2][NTH]: W[q*H+RK+4*i4 .. +3][k], k = kc, kc+H/2
-  float *dzs = sm + 2 * SK * NTH;                // [BC][G]
-  float *red = dzs + BC * G;                     // [BC][G] partials, index q*H + k
+  float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [SKK/4][16][NTH]
+  float *dzs = sm + SKK * 16 * NTH;              // [BC][H][4] unit-major dz
+  float *red = dzs + BC * G;                     // [BC][NW][H] per-warp column partials
+  float *ring = red + BC * NW * H;               // [BC][kRing][NTH][8] inputs of upcoming steps
   const int T = a.ix.T;
   const bool toff_sm = T + 1 <= kTokCap;
-  int *toff_s = reinterpret_cast<int *>(red + BC * G);
+  int *toff_s = reinterpret_cast<int *>(ring + BC * kRing * NTH * 8);
   const int *toff = toff_sm ? toff_s : a.ix.tok_off;
-  const int t = threadIdx.x;
-  constexpr int H2 = H / 2;
-  const int q = t / H2, kc = t % H2;  // columns kc and kc + H/2 of gate block q
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  const int ks = lane & 7, rgl = lane >> 3, rg = warp * 4 + rgl;
+  const int u0 = 4 * rg, kb = ks * KPT;
+  const int unit = t >> 1, pair = t & 1;  // phase B: lanes 2j, 2j+1 serve unit j
   const int n_groups = (a.ix.b + BC - 1) / BC;
   const int d = blockIdx.x / n_groups, grp = blockIdx.x % n_groups;
   const int r0 = grp * BC;
   const int DH = a.dirs * H;
+  const float *__restrict__ Whh = a.Whh[d];
 
-  const float *C0 = a.Whh[d] + (size_t)q * H * H + kc;       // W[q*H + i][kc] = C0[i*H]
-  const float *C1 = a.Whh[d] + (size_t)q * H * H + kc + H2;  // W[q*H + i][kc + H/2]
-  float w0[RK], w1[RK];
+  float w[16][RKK > 0 ? RKK : 1];
 #pragma unroll
-  for (int i = 0; i < RK; ++i) {
-    w0[i] = __ldg(C0 + (size_t)i * H);
-    w1[i] = __ldg(C1 + (size_t)i * H);
-  }
-  for (int i4 = 0; i4 < SK / 4; ++i4) {
-    const float *u = C0 + (size_t)(RK + 4 * i4) * H, *v = C1 + (size_t)(RK + 4 * i4) * H;
-    Ws4[(2 * i4) * NTH + t] = make_float4(__ldg(u), __ldg(u + H), __ldg(u + 2 * H), __ldg(u + 3 * H));
-    Ws4[(2 * i4 + 1) * NTH + t] = make_float4(__ldg(v), __ldg(v + H), __ldg(v + 2 * H), __ldg(v + 3 * H));
+  for (int ri = 0; ri < 16; ++ri) {
+    const float *row = Whh + (size_t)((ri & 3) * H + u0 + (ri >> 2)) * H + kb;
+#pragma unroll
+    for (int kk = 0; kk < RKK; ++kk) w[ri][kk] = __ldg(row + kk);
+#pragma unroll
+    for (int k4 = 0; k4 < SKK / 4; ++k4) {
+      const float *p = row + RKK + 4 * k4;
+      Ws4[(k4 * 16 + ri) * NTH + t] = make_float4(__ldg(p), __ldg(p + 1), __ldg(p + 2), __ldg(p + 3));
+    }
   }
   if (toff_sm)
     for (int i = t; i <= T; i += NTH) toff_s[i] = a.ix.tok_off[i];
@@ -231,129 +283,141 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
     const int tt = d == 0 ? s : len[b] - 1 - s;
     return toff[tt] + r0 + b;
   };
-  // unit t's prefetched inputs (threads t < H)
-  float gn[BC][4], cn[BC], cpn[BC], dyn[BC], dc[BC];
-  int tokn[BC];
-  auto prefetch = [&](int b, int s) {
-    const int tk = tok_at(b, s);
-    tokn[b] = tk;
+  // phase B inputs of `unit` (gates, c_t, c_{t-1}, dY), kPF steps ahead
+  float dc[BC];
+  auto issue = [&](int b, int s) {
+    if (s >= 0 && s < len[b]) {
+      const int tk = tok_at(b, s);
+      float *slot = ring + (((size_t)b * kRing + s % kRing) * NTH + t) * 8;
 #pragma unroll
-    for (int g = 0; g < 4; ++g) gn[b][g] = Z[(size_t)tk * G + g * H + t];
-    cn[b] = Cs[(size_t)tk * H + t];
-    cpn[b] = s > 0 ? Cs[(size_t)tok_at(b, s - 1) * H + t] : 0.f;
-    dyn[b] = dY[(size_t)tk * DH + d * H + t];
+      for (int g = 0; g < 4; ++g) cp_async4(slot + g, Z + (size_t)tk * G + g * H + unit);
+      cp_async4(slot + 4, Cs + (size_t)tk * H + unit);
+      if (s > 0) cp_async4(slot + 5, Cs + (size_t)tok_at(b, s - 1) * H + unit);
+      else slot[5] = 0.f;
+      cp_async4(slot + 6, dY + (size_t)tk * DH + d * H + unit);
+    }
   };
 #pragma unroll
-  for (int b = 0; b < BC; ++b) {
-    dc[b] = 0.f;
-    tokn[b] = 0;
-    cn[b] = cpn[b] = dyn[b] = 0.f;
+  for (int b = 0; b < BC; ++b) dc[b] = 0.f;
+  for (int j = 0; j < kPF; ++j) {
 #pragma unroll
-    for (int g = 0; g < 4; ++g) gn[b][g] = 0.f;
-    if (t < H && Tg - 1 < len[b]) prefetch(b, Tg - 1);
+    for (int b = 0; b < BC; ++b) issue(b, Tg - 1 - j);
+    cp_commit();
   }
   for (int s = Tg - 1; s >= 0; --s) {
-    // phase B
-    if (t < H) {
-#pragma unroll
-      for (int b = 0; b < BC; ++b) {
-        if (s < len[b]) {
-          float dh_rec = 0.f;
-          if (s + 1 < len[b])
-            dh_rec = (red[b * G + t] + red[b * G + H + t]) + (red[b * G + 2 * H + t] + red[b * G + 3 * H + t]);
-          const float ig = gn[b][0], fg = gn[b][1], gg = gn[b][2], og = gn[b][3];
-          const float ct = cn[b], cp = cpn[b];
-          const float dh = dyn[b] + dh_rec;
-          const int tk = tokn[b];
-          if (s - 1 >= 0 && s - 1 < len[b]) prefetch(b, s - 1);
-          const float tch = tanhf(ct);
-          float dcv = fmaf(dh * og, 1.f - tch * tch, dc[b]);
-          const float dzi = dcv * gg * ig * (1.f - ig);
-          const float dzf = dcv * cp * fg * (1.f - fg);
-          const float dzg = dcv * ig * (1.f - gg * gg);
-          const float dzo = dh * tch * og * (1.f - og);
-          dc[b] = dcv * fg;
-          dzs[b * G + t] = dzi;
-          dzs[b * G + H + t] = dzf;
-          dzs[b * G + 2 * H + t] = dzg;
-          dzs[b * G + 3 * H + t] = dzo;
-          float *zr = Z + (size_t)tk * G + t;
-          zr[0] = dzi;
-          zr[H] = dzf;
-          zr[2 * H] = dzg;
-          zr[3 * H] = dzo;
-        }
-      }
-    }
-    __syncthreads();
-    // phase A: two columns of one gate block per thread (one dz read feeds
-    // both), two accumulators each
+    cp_wait_all_but_newest();
+    // phase B: dz of unit j from dh = dY + recurrent part
 #pragma unroll
     for (int b = 0; b < BC; ++b) {
-      if (s < len[b]) {
-        const float4 *d0 = reinterpret_cast<const float4 *>(dzs + b * G + q * H);
-        float a0 = 0.f, a1 = 0.f, e0 = 0.f, e1 = 0.f;
+      if (s >= len[b]) continue;  // uniform over the CTA
+      float dh_rec = 0.f;
+      if (s + 1 < len[b]) {
+        const float *rp = red + (size_t)b * NW * H + unit;
 #pragma unroll
-        for (int i4 = 0; i4 < RK / 4; ++i4) {
-          const float4 x = d0[i4];
-          a0 = fmaf(w0[4 * i4], x.x, a0);
-          a1 = fmaf(w1[4 * i4], x.x, a1);
-          e0 = fmaf(w0[4 * i4 + 1], x.y, e0);
-          e1 = fmaf(w1[4 * i4 + 1], x.y, e1);
-          a0 = fmaf(w0[4 * i4 + 2], x.z, a0);
-          a1 = fmaf(w1[4 * i4 + 2], x.z, a1);
-          e0 = fmaf(w0[4 * i4 + 3], x.w, e0);
-          e1 = fmaf(w1[4 * i4 + 3], x.w, e1);
-        }
-#pragma unroll
-        for (int i4 = 0; i4 < SK / 4; ++i4) {
-          const float4 u = Ws4[(2 * i4) * NTH + t], v = Ws4[(2 * i4 + 1) * NTH + t];
-          const float4 x = d0[RK / 4 + i4];
-          a0 = fmaf(u.x, x.x, a0);
-          a1 = fmaf(v.x, x.x, a1);
-          e0 = fmaf(u.y, x.y, e0);
-          e1 = fmaf(v.y, x.y, e1);
-          a0 = fmaf(u.z, x.z, a0);
-          a1 = fmaf(v.z, x.z, a1);
-          e0 = fmaf(u.w, x.w, e0);
-          e1 = fmaf(v.w, x.w, e1);
-        }
-        red[b * G + q * H + kc] = a0 + e0;
-        red[b * G + q * H + kc + H2] = a1 + e1;
+        for (int wi = 0; wi < NW; ++wi) dh_rec += rp[wi * H];
       }
+      const float *slot = ring + (((size_t)b * kRing + s % kRing) * NTH + t) * 8;
+      const float ig = slot[0], fg = slot[1], gg = slot[2], og = slot[3];
+      const float ct = slot[4], cp = slot[5];
+      const float dh = slot[6] + dh_rec;
+      const int tk = tok_at(b, s);
+      issue(b, s - kPF);
+      const float tch = tanhf(ct);
+      const float dcv = fmaf(dh * og, 1.f - tch * tch, dc[b]);
+      const float dzi = dcv * gg * ig * (1.f - ig);
+      const float dzf = dcv * cp * fg * (1.f - fg);
+      const float dzg = dcv * ig * (1.f - gg * gg);
+      const float dzo = dh * tch * og * (1.f - og);
+      dc[b] = dcv * fg;
+      const float z0 = pair ? dzg : dzi, z1 = pair ? dzo : dzf;
+      *reinterpret_cast<float2 *>(dzs + ((size_t)b * H + unit) * 4 + 2 * pair) = make_float2(z0, z1);
+      Z[(size_t)tk * G + (2 * pair) * H + unit] = z0;
+      Z[(size_t)tk * G + (2 * pair + 1) * H + unit] = z1;
+    }
+    cp_commit();
+    __syncthreads();
+    // phase A: column partials of W_hh^T dz over this warp's 16 x 4 rows
+#pragma unroll
+    for (int b = 0; b < BC; ++b) {
+      if (s >= len[b]) continue;
+      const float4 *dz4 = reinterpret_cast<const float4 *>(dzs + ((size_t)b * H + u0) * 4);
+      float dz[16];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float4 v = dz4[u];
+        dz[4 * u] = v.x;
+        dz[4 * u + 1] = v.y;
+        dz[4 * u + 2] = v.z;
+        dz[4 * u + 3] = v.w;
+      }
+      float part[KPT];
+#pragma unroll
+      for (int kk = 0; kk < RKK; ++kk) {
+        float x = 0.f;
+#pragma unroll
+        for (int ri = 0; ri < 16; ++ri) x = fmaf(w[ri][kk], dz[ri], x);
+        part[kk] = x;
+      }
+#pragma unroll
+      for (int k4 = 0; k4 < SKK / 4; ++k4) {
+        float x0 = 0.f, x1 = 0.f, x2 = 0.f, x3 = 0.f;
+#pragma unroll
+        for (int ri = 0; ri < 16; ++ri) {
+          const float4 wv = Ws4[(k4 * 16 + ri) * NTH + t];
+          x0 = fmaf(wv.x, dz[ri], x0);
+          x1 = fmaf(wv.y, dz[ri], x1);
+          x2 = fmaf(wv.z, dz[ri], x2);
+          x3 = fmaf(wv.w, dz[ri], x3);
+        }
+        part[RKK + 4 * k4] = x0;
+        part[RKK + 4 * k4 + 1] = x1;
+        part[RKK + 4 * k4 + 2] = x2;
+        part[RKK + 4 * k4 + 3] = x3;
+      }
+      float out[KPT / 4];
+      reduce_groups<KPT>(part, lane, out);
+      // lane (rgl, ks) now holds columns kb + rgl*(KPT/4) .. + KPT/4 - 1
+      float *dst = red + ((size_t)b * NW + warp) * H + kb + rgl * (KPT / 4);
+#pragma unroll
+      for (int i = 0; i < KPT / 4; ++i) dst[i] = out[i];
     }
     __syncthreads();
   }
+  asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
 // ---------------------------------------------------------------------------
 namespace {
 
-size_t cta_smem_bytes(bool bwd, int H, int RK, int BC, int T) {
-  const size_t f = bwd ? (size_t)(H - RK) * 4 * H + 2 * (size_t)BC * 4 * H
-                       : (size_t)(H - RK) * 4 * H + 2 * (size_t)BC * H + (size_t)BC * 4 * H;  // W: 2 rows x (H-RK) x 2H threads
+size_t cta_smem_bytes(bool bwd, int H, int RKK, int BC, int T) {
+  const int KPT = H / 8, SKK = KPT - RKK, NTH = 2 * H;
+  const size_t wf = (size_t)SKK * 16 * NTH;
+  const size_t f = bwd ? wf + (size_t)BC * 4 * H + (size_t)BC * (NTH / 32) * H + (size_t)BC * kRing * NTH * 8
+                       : wf + (size_t)2 * BC * 8 * (KPT + 4) + (size_t)BC * kRing * NTH * 2;
   const size_t i = (T + 1 <= kTokCap) ? (size_t)(T + 1) : 0;
   return (f + i) * 4 + 16;
 }
 
-template <int H, int RK, int BC>
+template <int H, int RKK, int BC>
 cudaError_t launch_cta(const RecArgs &a, bool bwd, cudaStream_t s) {
-  const size_t smem = cta_smem_bytes(bwd, H, RK, BC, a.ix.T);
+  const size_t smem = cta_smem_bytes(bwd, H, RKK, BC, a.ix.T);
   const int ng = (a.ix.b + BC - 1) / BC;
   if (bwd) {
-    cudaError_t e = cudaFuncSetAttribute(lstm_bwd_cta_kernel<H, RK, BC>,
+    cudaError_t e = cudaFuncSetAttribute(lstm_bwd_cta_kernel<H, RKK, BC>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    lstm_bwd_cta_kernel<H, RK, BC><<<ng * a.dirs, 2 * H, smem, s>>>(a);
+    lstm_bwd_cta_kernel<H, RKK, BC><<<ng * a.dirs, 2 * H, smem, s>>>(a);
   } else {
-    cudaError_t e = cudaFuncSetAttribute(lstm_fwd_cta_kernel<H, RK, BC>,
+    cudaError_t e = cudaFuncSetAttribute(lstm_fwd_cta_kernel<H, RKK, BC>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    lstm_fwd_cta_kernel<H, RK, BC><<<ng * a.dirs, 2 * H, smem, s>>>(a);
+    lstm_fwd_cta_kernel<H, RKK, BC><<<ng * a.dirs, 2 * H, smem, s>>>(a);
   }
   return cudaGetLastError();
 }
 
+// Columns of the k slice held in registers (RKK of KPT = H/8) for one and two
+// batch rows per CTA.
 template <int H, int RK1, int RK2>
 cudaError_t launch_cta_bc(const RecArgs &a, int bc, bool bwd, cudaStream_t s) {
   switch (bc) {
@@ -374,9 +438,9 @@ int cta_rows_per_block(int H, int b, int dirs, int sm_count) {
 
 cudaError_t launch_lstm_cta(const RecArgs &a, int bc, bool bwd, cudaStream_t s) {
   switch (a.H) {
-    case 32: return launch_cta_bc<32, 32, 32>(a, bc, bwd, s);
-    case 64: return launch_cta_bc<64, 64, 48>(a, bc, bwd, s);
-    case 128: return launch_cta_bc<128, 96, 64>(a, bc, bwd, s);
+    case 32: return launch_cta_bc<32, 4, 4>(a, bc, bwd, s);
+    case 64: return launch_cta_bc<64, 8, 4>(a, bc, bwd, s);
+    case 128: return launch_cta_bc<128, 12, 8>(a, bc, bwd, s);
     default: return cudaErrorInvalidValue;
   }
 }
