@@ -452,7 +452,38 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     g.splits = bkt::wgrad_splits(g.M, g.N, NT, sm_count, w.part_floats);
     L.run("wgrad", [&] { return bkt::launch_wgrad(g, o1, o2, o3, s); });
   };
-  wgrad(w.logit, C, C, Ytop, DH, DH, nullptr, 0, nullptr, 0, grads + lo.w_out, nullptr, grads + lo.b_out);
+  // fp32 contractions over tokens on the tensor cores (3xTF32): the
+  // token-major operands are transposed and split into hi + lo parts first
+  const int NTq = (NT + 7) & ~7;
+  auto split_A = [&](const float *A, int64_t lda, int M) {
+    L.run("transpose_split", [&] { return bkt::launch_transpose_split(A, lda, nullptr, NT, M, w.AT, w.ATl, NTq, s); });
+  };
+  auto tf32_reduce = [&](int M, const float *B, int64_t ldb, const int32_t *gather, int N, float *out) {
+    L.run("transpose_split", [&] { return bkt::launch_transpose_split(B, ldb, gather, NT, N, w.BTf, w.BTl, NTq, s); });
+    bkt::TcGemmArgs g{};
+    g.M = M;
+    g.N = N;
+    g.K = NT;
+    g.A = w.AT;
+    g.lda = NTq;
+    g.B = w.BTf;
+    g.ldb = NTq;
+    g.P = w.part;
+    g.splits = bkt::tf32x3_splits(M, N, NT, sm_count, w.part_floats);
+    g.err = w.status;
+    L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.ATl, w.BTl, s); });
+    L.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, g.splits, M, N, out, s); });
+  };
+  auto bias_sum = [&](const float *A, int64_t lda, int M, float *out) {
+    int splits = std::min(64, std::max(1, std::min(2 * sm_count / ((M + 255) / 256), NT / 64)));
+    while (splits > 1 && (size_t)splits * M > w.part_floats) --splits;
+    L.run("colsum", [&] { return bkt::launch_colsum(A, lda, NT, M, w.part, splits, s); });
+    L.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, splits, 1, M, out, s); });
+  };
+  // [dW_out | db_out] = dlogit^T [Y | 1]
+  split_A(w.logit, C, C);
+  tf32_reduce(C, Ytop, DH, nullptr, DH, grads + lo.w_out);
+  bias_sum(w.logit, C, C, grads + lo.b_out);
   {
     bkt::GemmArgs g{};
     g.M = NT;
@@ -524,10 +555,19 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
       }
     } else {
       for (int d = 0; d < dirs; ++d) {
-        // [dW_ih | dW_hh | db] = dZ^T [X_l | h_{t-1} | 1]; h_{t-1} of token
-        // (t, r) is the row's previous token in its direction (zeros at the start)
-        wgrad(w.Z[l * dirs + d], 4 * H, 4 * H, Xl, D, D, w.Y[l] + d * H, DH, w.prev_tok[d], H,
-              grads + lo.w_ih[l * dirs + d], grads + lo.w_hh(l, d), grads + lo.bias(l, d));
+        // dW_hh = dz^T h_{t-1}; h_{t-1} of token (t, r) is the row's previous
+        // token in its direction (zeros at the start)
+        const float *dZ = w.Z[l * dirs + d];
+        split_A(dZ, 4 * H, 4 * H);
+        tf32_reduce(4 * H, w.Y[l] + d * H, DH, w.prev_tok[d], H, grads + lo.w_hh(l, d));
+        if (l == 0) {
+          // narrow input: [dW_ih | db] = dz^T [X | 1] on the FMA pipe
+          wgrad(dZ, 4 * H, 4 * H, Xl, D, D, nullptr, 0, nullptr, 0, grads + lo.w_ih[l * dirs + d], nullptr,
+                grads + lo.bias(l, d));
+        } else {
+          tf32_reduce(4 * H, Xl, D, nullptr, D, grads + lo.w_ih[l * dirs + d]);
+          bias_sum(dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
+        }
       }
     }
     if (l > 0 && bf16) {
@@ -746,6 +786,13 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
   BKT_ALLOC(w.prev_tok[1], NT);
   BKT_ALLOC(w.row_ok, (size_t)max_batch);
   BKT_ALLOC(w.status, 1);
+  {
+    const size_t NTq = (NT + 7) & ~size_t(7), MA = std::max<size_t>(4 * H, (size_t)lo.C);
+    BKT_ALLOC(w.AT, MA * NTq);
+    BKT_ALLOC(w.ATl, MA * NTq);
+    BKT_ALLOC(w.BTf, DH * NTq);
+    BKT_ALLOC(w.BTl, DH * NTq);
+  }
   if (cfg->gemm_precision == BKT_GEMM_BF16) {
     const size_t NTp = (NT + 7) & ~size_t(7);
     uint16_t *p = nullptr;
@@ -971,6 +1018,13 @@ int bkt::step_on_scratch(const bkt_model_cfg *cfg, const bkt_batch *bt, const fl
   w.row_ok = cv.take<int32_t>((size_t)b);
   w.status = cv.take<int32_t>(1);
   w.idx_dev = cv.take<char>(il.bytes);
+  {
+    const size_t NTq = (NT + 7) & ~size_t(7), MA = std::max<size_t>(4 * H, (size_t)lo.C);
+    w.AT = cv.take<float>(MA * NTq);
+    w.ATl = cv.take<float>(MA * NTq);
+    w.BTf = cv.take<float>(DH * NTq);
+    w.BTl = cv.take<float>(DH * NTq);
+  }
   if (cfg->gemm_precision == BKT_GEMM_BF16) {
     const size_t NTp = (NT + 7) & ~size_t(7);
     w.Yb = cv.take<uint16_t>(NT * DH);

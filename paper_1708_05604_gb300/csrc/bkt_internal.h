@@ -93,6 +93,10 @@ cudaError_t launch_cast_bf16(const float *src, int64_t lds, int R, int C, void *
 cudaError_t launch_transpose_bf16(const float *src, int64_t lds, const int32_t *src_row, int R, int C, void *dst,
                                   int64_t ldd, cudaStream_t s);
 cudaError_t launch_colsum(const float *A, int64_t lda, int R, int M, float *P, int splits, cudaStream_t s);
+// hi[c][r] + lo[c][r] = src[src_row ? src_row[r] : r][c] to 2^-22 relative,
+// hi and lo both tf32 values (zeros where src_row[r] < 0).
+cudaError_t launch_transpose_split(const float *src, int64_t lds, const int32_t *src_row, int R, int C, float *hi,
+                                   float *lo, int64_t ldd, cudaStream_t s);
 
 // bf16 tensor-core GEMM (k_gemm_tc.cu):
 //   D[m][n] (+)= sum_k A[m][k] B[n][k] (+ bias[n]); A, B bf16 with K contiguous
@@ -112,6 +116,11 @@ struct TcGemmArgs {
 };
 int tc_splits(int M, int N, int K, int sm_count, size_t part_floats);
 cudaError_t launch_gemm_bf16_tc(const TcGemmArgs &g, cudaStream_t s);
+// fp32 GEMM on the tensor cores with split precision (3xTF32): A = A (hi) +
+// A_lo, B = B (hi) + B_lo, all fp32 row-major with K contiguous (lda, ldb
+// multiples of 4, 16-byte aligned); D (or partials) as for the bf16 GEMM.
+int tf32x3_splits(int M, int N, int K, int sm_count, size_t part_floats);
+cudaError_t launch_gemm_tf32x3_tc(const TcGemmArgs &g, const void *A_lo, const void *B_lo, cudaStream_t s);
 
 // a7: logp[tok][c] = log-softmax_c(b[c] + W[c] . Y[tok]).
 cudaError_t launch_out_logsoftmax(const float *Y, int n_tok, int DH, const float *W,
@@ -185,6 +194,9 @@ struct StepBufs {
   int32_t *row_ok;                            // [b]
   int32_t *status;                            // device error flags
   void *idx_dev;                              // per-step index block
+  // split-precision (3xTF32) operands of the fp32 contractions over tokens
+  float *AT, *ATl;                            // [max(4H, C) x NTq] transposed dz / dlogit, hi and lo
+  float *BTf, *BTl;                           // [dirs*H x NTq] transposed X, h_{t-1} or Y, hi and lo
   // bf16 GEMM path only (null otherwise)
   void *Yb;                                   // [NT x dirs*H] bf16 layer input of a projection
   void *dZb;                                  // [NT x 4H] bf16 dz (input-gradient GEMM)

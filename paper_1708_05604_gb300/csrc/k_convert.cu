@@ -74,6 +74,49 @@ cudaError_t launch_transpose_bf16(const float *src, int64_t lds, const int32_t *
   return cudaGetLastError();
 }
 
+// fp32 [R x C] -> two fp32 [C x R] arrays hi, lo, each a tf32 value (11
+// significant bits) with |x - hi - lo| <= 2^-22 |x|, for the split-precision
+// tensor-core GEMM; optional row gather as above.
+__global__ void transpose_split_kernel(const float *__restrict__ src, int64_t lds, const int32_t *__restrict__ src_row,
+                                       int R, int C, float *__restrict__ hi, float *__restrict__ lo, int64_t ldd) {
+  __shared__ float tile[32][33];
+  const int r0 = blockIdx.x * 32, c0 = blockIdx.y * 32;
+  const int tx = threadIdx.x, ty = threadIdx.y;  // 32 x 8
+#pragma unroll
+  for (int i = 0; i < 32; i += 8) {
+    const int r = r0 + ty + i, c = c0 + tx;
+    float v = 0.f;
+    if (r < R && c < C) {
+      const int sr = src_row ? src_row[r] : r;
+      if (sr >= 0) v = src[(int64_t)sr * lds + c];
+    }
+    tile[ty + i][tx] = v;
+  }
+  __syncthreads();
+#pragma unroll
+  for (int i = 0; i < 32; i += 8) {
+    const int c = c0 + ty + i, r = r0 + tx;
+    if (c < C && r < R) {
+      // both parts rounded to the nearest tf32 value (11 significant bits),
+      // so the tensor core uses them exactly: |x - hi - lo| <= 2^-22 |x|
+      const float x = tile[tx][ty + i];
+      const float h = __uint_as_float((__float_as_uint(x) + 0x1000u) & 0xFFFFE000u);
+      const float l = __uint_as_float((__float_as_uint(x - h) + 0x1000u) & 0xFFFFE000u);
+      hi[(int64_t)c * ldd + r] = h;
+      lo[(int64_t)c * ldd + r] = l;
+    }
+  }
+}
+
+cudaError_t launch_transpose_split(const float *src, int64_t lds, const int32_t *src_row, int R, int C, float *hi,
+                                   float *lo, int64_t ldd, cudaStream_t s) {
+  if (R <= 0 || C <= 0) return cudaSuccess;
+  dim3 grid((R + 31) / 32, (C + 31) / 32);
+  if (grid.y > 65535u) return cudaErrorInvalidConfiguration;
+  transpose_split_kernel<<<grid, dim3(32, 8), 0, s>>>(src, lds, src_row, R, C, hi, lo, ldd);
+  return cudaGetLastError();
+}
+
 __global__ void colsum_kernel(const float *__restrict__ A, int64_t lda, int R, int M, float *__restrict__ P,
                               int splits) {
   const int m = blockIdx.x * blockDim.x + threadIdx.x;

@@ -105,6 +105,26 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// 3xTF32 variant: fp32 operands split as a = hi + lo (hi = a with the low 13
+// mantissa bits cleared, exactly representable in tf32); the tile product is
+// A_hi B_hi + A_hi B_lo + A_lo B_hi with fp32 accumulation, which leaves a
+// relative error near 2^-20 per product.  128 x 128 tiles, 32-wide k slabs
+// (128 bytes of fp32 per row), 3 stages of {A_hi, A_lo, B_hi, B_lo}.
+constexpr int FBM = 128, FBN = 128, FBK = 32, FSTAGES = 3;
+constexpr uint32_t kFTile = FBM * FBK * 4;  // 16 KB
+constexpr uint32_t kFStage = 4 * kFTile;
+constexpr size_t kFSmem = 1024 + (size_t)FSTAGES * kFStage + 256;
+// kind::tf32 descriptor: D fp32 (bit 4), A and B tf32 (format 2 at bits 7, 10)
+constexpr uint32_t kIdescTf32 = (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(FBN >> 3) << 17) |
+                                ((uint32_t)(FBM >> 4) << 24);
+
+__device__ __forceinline__ void tc_mma_tf32(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n}\n" ::"r"(d),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+
 }  // namespace
 
 __global__ void __launch_bounds__(128, 1)
@@ -236,6 +256,139 @@ __global__ void __launch_bounds__(128, 1)
   if (threadIdx.x == 0 && *abort_s && g.err) atomicOr(g.err, 2);
 }
 
+__global__ void __launch_bounds__(128, 1)
+    gemm_tf32x3_tc_kernel(const __grid_constant__ CUtensorMap tah, const __grid_constant__ CUtensorMap tal,
+                          const __grid_constant__ CUtensorMap tbh, const __grid_constant__ CUtensorMap tbl,
+                          TcGemmArgs g) {
+  extern __shared__ uint8_t tc_smem_raw[];
+  uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(tc_smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t *bars = reinterpret_cast<uint64_t *>(base + FSTAGES * kFStage);  // full[S], empty[S], done
+  uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 2 * FSTAGES + 1);
+  int *abort_s = reinterpret_cast<int *>(tslot + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m0 = blockIdx.x * FBM, n0 = blockIdx.y * FBN;
+  const int splits = g.P ? g.splits : 1;
+  const int nkb = (g.K + FBK - 1) / FBK;
+  const int chunk = (nkb + splits - 1) / splits;
+  const int kb0 = blockIdx.z * chunk;
+  const int nk = max(0, min(nkb, kb0 + chunk) - kb0);
+  const uint32_t full0 = su32(bars), empty0 = su32(bars + FSTAGES), done = su32(bars + 2 * FSTAGES);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < FSTAGES; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    mbar_init(done, 1);
+    *abort_s = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tslot)), "r"(FBN)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tslot;
+
+  if (warp == 0) {
+    if (lane == 0) {  // TMA producer
+      for (int i = 0; i < nk; ++i) {
+        const int s = i % FSTAGES;
+        if (i >= FSTAGES && !mbar_wait(empty0 + 8 * s, ((i / FSTAGES) - 1) & 1)) {
+          *abort_s = 1;
+          break;
+        }
+        uint8_t *st = base + s * kFStage;
+        mbar_expect_tx(full0 + 8 * s, kFStage);
+        const int kx = (kb0 + i) * FBK;
+        tma_load_2d(su32(st), &tah, kx, m0, full0 + 8 * s);
+        tma_load_2d(su32(st + kFTile), &tal, kx, m0, full0 + 8 * s);
+        tma_load_2d(su32(st + 2 * kFTile), &tbh, kx, n0, full0 + 8 * s);
+        tma_load_2d(su32(st + 3 * kFTile), &tbl, kx, n0, full0 + 8 * s);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {  // MMA issuer
+      int issued = 0;
+      for (int i = 0; i < nk; ++i) {
+        const int s = i % FSTAGES;
+        if (!mbar_wait(full0 + 8 * s, (i / FSTAGES) & 1)) {
+          *abort_s = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t ah = su32(base + s * kFStage), al = ah + kFTile, bh = ah + 2 * kFTile, bl = ah + 3 * kFTile;
+#pragma unroll
+        for (int kk = 0; kk < FBK / 8; ++kk) {
+          const uint32_t o = kk * 32;
+          tc_mma_tf32(tmem, sw128_desc(ah + o), sw128_desc(bh + o), kIdescTf32, (i > 0 || kk > 0) ? 1u : 0u);
+          tc_mma_tf32(tmem, sw128_desc(ah + o), sw128_desc(bl + o), kIdescTf32, 1u);
+          tc_mma_tf32(tmem, sw128_desc(al + o), sw128_desc(bh + o), kIdescTf32, 1u);
+        }
+        tc_commit(empty0 + 8 * s);
+        ++issued;
+      }
+      if (issued > 0) tc_commit(done);
+      else mbar_arrive(done);
+    }
+    __syncwarp();
+  }
+
+  const bool ready = mbar_wait(done, 0);
+  if (!ready) *abort_s = 1;
+  tc_fence_after();
+  const int m = m0 + warp * 32 + lane;
+  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+  const bool write = ready && m < g.M;
+  float *out;
+  int64_t ld;
+  if (g.P) {
+    out = g.P + (int64_t)blockIdx.z * g.M * g.N + (int64_t)m * g.N;
+    ld = g.N;
+  } else {
+    out = g.D + (int64_t)m * g.ldd;
+    ld = g.ldd;
+  }
+  const bool vec = ((ld & 3) == 0) && ((reinterpret_cast<uintptr_t>(g.P ? g.P : g.D) & 15) == 0);
+#pragma unroll 1
+  for (int c0 = 0; c0 < FBN; c0 += 32) {
+    uint32_t v[32];
+    __syncwarp();
+    tmem_ld32(trow + c0, v);
+    if (!write) continue;
+    const int nb = n0 + c0;
+    if (nb >= g.N) continue;
+    float x[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) x[j] = nk > 0 ? __uint_as_float(v[j]) : 0.f;
+    if (!g.P) {
+      if (g.bias)
+#pragma unroll
+        for (int j = 0; j < 32; ++j) x[j] += (nb + j < g.N) ? g.bias[nb + j] : 0.f;
+      if (g.accumulate)
+#pragma unroll
+        for (int j = 0; j < 32; ++j) x[j] += (nb + j < g.N) ? out[nb + j] : 0.f;
+    }
+    if (vec && nb + 32 <= g.N) {
+#pragma unroll
+      for (int j = 0; j < 32; j += 4)
+        *reinterpret_cast<float4 *>(out + nb + j) = make_float4(x[j], x[j + 1], x[j + 2], x[j + 3]);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (nb + j < g.N) out[nb + j] = x[j];
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(FBN) : "memory");
+  if (threadIdx.x == 0 && *abort_s && g.err) atomicOr(g.err, 2);
+}
+
 // ---------------------------------------------------------------------------
 namespace {
 
@@ -252,17 +405,20 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-// 2-D bf16 map over a row-major [rows x inner] matrix with row stride `ld`
-// elements; boxes of 64 (inner) x box_rows with the 128-byte swizzle.
-bool make_map(CUtensorMap *map, const void *base, uint64_t inner, uint64_t rows, int64_t ld, uint32_t box_rows) {
+// 2-D map over a row-major [rows x inner] matrix with row stride `ld`
+// elements; boxes of 128 bytes (inner) x box_rows with the 128-byte swizzle.
+bool make_map(CUtensorMap *map, const void *base, uint64_t inner, uint64_t rows, int64_t ld, uint32_t box_rows,
+              bool fp32 = false) {
   auto fn = encode_fn();
   if (!fn) return false;
+  const int esz = fp32 ? 4 : 2;
   cuuint64_t dims[2] = {inner, rows};
-  cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
-  cuuint32_t box[2] = {(cuuint32_t)TBK, box_rows};
+  cuuint64_t strides[1] = {(cuuint64_t)ld * esz};
+  cuuint32_t box[2] = {(cuuint32_t)(128 / esz), box_rows};
   cuuint32_t es[2] = {1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+  return fn(map, fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+            const_cast<void *>(base), dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -291,6 +447,39 @@ cudaError_t launch_gemm_bf16_tc(const TcGemmArgs &g, cudaStream_t s) {
   dim3 grid((g.M + TBM - 1) / TBM, (g.N + TBN - 1) / TBN, g.P ? g.splits : 1);
   if (grid.y > 65535u || grid.z > 65535u) return cudaErrorInvalidConfiguration;
   gemm_bf16_tc_kernel<<<grid, 128, kTcSmem, s>>>(ta, tb, g);
+  return cudaGetLastError();
+}
+
+int tf32x3_splits(int M, int N, int K, int sm_count, size_t part_floats) {
+  const int tiles = ((M + FBM - 1) / FBM) * ((N + FBN - 1) / FBN);
+  const int nkb = (K + FBK - 1) / FBK;
+  int s = std::max(1, sm_count / std::max(1, tiles));
+  s = std::min(s, std::max(1, nkb / 4));
+  // at most 4096 tokens per accumulator: keeps fp32 accumulation chains short
+  s = std::max(s, (K + 4095) / 4096);
+  s = std::min(s, 64);
+  while (s > 1 && (size_t)s * M * N > part_floats) --s;
+  return s;
+}
+
+cudaError_t launch_gemm_tf32x3_tc(const TcGemmArgs &g, const void *A_lo, const void *B_lo, cudaStream_t s) {
+  if (g.M <= 0 || g.N <= 0) return cudaSuccess;
+  if (g.K <= 0 || (g.lda & 3) || (g.ldb & 3) || ((reinterpret_cast<uintptr_t>(g.A) | reinterpret_cast<uintptr_t>(g.B) |
+                                                   reinterpret_cast<uintptr_t>(A_lo) | reinterpret_cast<uintptr_t>(B_lo)) &
+                                                  15) ||
+      (g.P && g.splits < 1) || (!g.P && !g.D))
+    return cudaErrorInvalidValue;
+  CUtensorMap tah, tal, tbh, tbl;
+  if (!make_map(&tah, g.A, (uint64_t)g.K, (uint64_t)g.M, g.lda, FBM, true) ||
+      !make_map(&tal, A_lo, (uint64_t)g.K, (uint64_t)g.M, g.lda, FBM, true) ||
+      !make_map(&tbh, g.B, (uint64_t)g.K, (uint64_t)g.N, g.ldb, FBN, true) ||
+      !make_map(&tbl, B_lo, (uint64_t)g.K, (uint64_t)g.N, g.ldb, FBN, true))
+    return cudaErrorInvalidValue;
+  cudaError_t e = cudaFuncSetAttribute(gemm_tf32x3_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFSmem);
+  if (e != cudaSuccess) return e;
+  dim3 grid((g.M + FBM - 1) / FBM, (g.N + FBN - 1) / FBN, g.P ? g.splits : 1);
+  if (grid.y > 65535u || grid.z > 65535u) return cudaErrorInvalidConfiguration;
+  gemm_tf32x3_tc_kernel<<<grid, 128, kFSmem, s>>>(tah, tal, tbh, tbl, g);
   return cudaGetLastError();
 }
 
