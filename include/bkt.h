@@ -162,8 +162,8 @@ int bkt_lstm_ctc_step(bkt_ctx *ctx, const bkt_batch *batch,
  * that loads the library holds that array until the process exits.
  *   - Arguments and results are exactly those of bkt_lstm_ctc_step; the
  *     limits are n_seq <= 512, label_lengths <= 1023, and a workspace that
- *     fits the array (about (14 H + C + 2 S + 8) * 4 bytes per token for one
- *     bidirectional layer, S = 2U + 1: some 8,000 tokens at H = 128).  A batch beyond them returns
+ *     fits the array (about (26 H + C + 2 S + 8) * 4 bytes per token for one
+ *     bidirectional layer, S = 2U + 1: some 4,500 tokens at H = 128).  A batch beyond them returns
  *     BKT_EINVAL with the needed and available bytes in bkt_last_error().
  *   - The first call on a device looks up the array's address on that
  *     device, so make that first call before any stream capture.
