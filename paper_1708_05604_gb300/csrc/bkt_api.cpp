@@ -418,10 +418,29 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
   }
 
   // ---- a7: output layer and log-softmax
+  // logits = Y W_out^T + b_out on the tensor cores (3xTF32; both operands are
+  // already K-contiguous, so they are split without transposing), then a
+  // log-softmax pass in place
   float *Ytop = w.Y[lo.L - 1];
-  L.run("out_logsoftmax", [&] {
-    return bkt::launch_out_logsoftmax(Ytop, NT, DH, params + lo.w_out, params + lo.b_out, C, w.logit, s);
-  });
+  const int DHp = (DH + 3) & ~3;  // split rows padded to 16 bytes for TMA
+  L.run("split_rows", [&] { return bkt::launch_split_rows(Ytop, DH, NT, DH, w.BTf, w.BTl, DHp, s); });
+  L.run("split_rows", [&] { return bkt::launch_split_rows(params + lo.w_out, DH, C, DH, w.Wh, w.Wl, DHp, s); });
+  {
+    bkt::TcGemmArgs g{};
+    g.M = NT;
+    g.N = C;
+    g.K = DH;
+    g.A = w.BTf;
+    g.lda = DHp;
+    g.B = w.Wh;
+    g.ldb = DHp;
+    g.D = w.logit;
+    g.ldd = C;
+    g.bias = params + lo.b_out;
+    g.err = w.status;
+    L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.BTl, w.Wl, s); });
+  }
+  L.run("log_softmax", [&] { return bkt::launch_log_softmax_rows(w.logit, C, NT, C, s); });
   // ---- a8, a9: CTC
   L.run("ctc_tables", [&] {
     return bkt::launch_ctc_tables(ix, w.logit, C, cfg.blank, bt->labels, w.alpha, w.beta, loss, w.row_ok, w.status, s);
@@ -431,27 +450,6 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
   });
 
   // ---- a10: output layer backward
-  // [dW_out | db_out] = dlogit^T [Y | 1]
-  auto wgrad = [&](const float *A, int64_t lda, int M, const float *B1, int64_t ldb1, int D1, const float *B2,
-                   int64_t ldb2, const int32_t *gather2, int D2, float *o1, float *o2, float *o3) {
-    bkt::WgradArgs g{};
-    g.M = M;
-    g.N = D1 + D2 + 1;
-    g.K = NT;
-    g.A = A;
-    g.lda = lda;
-    g.D1 = D1;
-    g.B1 = B1;
-    g.ldb1 = ldb1;
-    g.D2 = D2;
-    g.B2 = B2;
-    g.ldb2 = ldb2;
-    g.gather2 = gather2;
-    g.ones = 1;
-    g.P = w.part;
-    g.splits = bkt::wgrad_splits(g.M, g.N, NT, sm_count, w.part_floats);
-    L.run("wgrad", [&] { return bkt::launch_wgrad(g, o1, o2, o3, s); });
-  };
   // fp32 contractions over tokens on the tensor cores (3xTF32): the
   // token-major operands are transposed and split into hi + lo parts first
   const int NTq = (NT + 7) & ~7;
@@ -480,23 +478,36 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     L.run("colsum", [&] { return bkt::launch_colsum(A, lda, NT, M, w.part, splits, s); });
     L.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, splits, 1, M, out, s); });
   };
+  // [dW_ih | db] of the first layer: dz^T [X | 1] with X of in_dim columns
+  auto narrow = [&](const float *dZ, const float *X, int D, float *ow, float *ob) {
+    L.run("narrow_wgrad", [&] {
+      return bkt::launch_narrow_wgrad(dZ, 4 * H, 4 * H, X, D, NT, w.part, w.part_floats, sm_count, ow, ob, s);
+    });
+  };
   // [dW_out | db_out] = dlogit^T [Y | 1]
   split_A(w.logit, C, C);
   tf32_reduce(C, Ytop, DH, nullptr, DH, grads + lo.w_out);
   bias_sum(w.logit, C, C, grads + lo.b_out);
   {
-    bkt::GemmArgs g{};
+    // dY = dlogit W_out on the tensor cores: dlogit split with its rows padded
+    // to a multiple of 4 floats (TMA strides), W_out split transposed
+    const int Cp = (C + 3) & ~3;
+    L.run("split_rows", [&] { return bkt::launch_split_rows(w.logit, C, NT, C, w.Lh, w.Ll, Cp, s); });
+    L.run("transpose_split", [&] {
+      return bkt::launch_transpose_split(params + lo.w_out, DH, nullptr, C, DH, w.Wh, w.Wl, Cp, s);
+    });
+    bkt::TcGemmArgs g{};
     g.M = NT;
     g.N = DH;
     g.K = C;
-    g.A = w.logit;
-    g.lda = C;
-    g.B = params + lo.w_out;
-    g.ldb = DH;
-    g.C = w.dY;
-    g.ldc = DH;
-    g.splits = 1;
-    L.run("gemm_dy_out", [&] { return bkt::launch_gemm_f32(false, false, g, s); });
+    g.A = w.Lh;
+    g.lda = Cp;
+    g.B = w.Wh;
+    g.ldb = Cp;
+    g.D = w.dY;
+    g.ldd = DH;
+    g.err = w.status;
+    L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.Ll, w.Wl, s); });
   }
 
   // ---- a11, a12: BPTT and weight gradients, top layer first
@@ -542,8 +553,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         tc_reduce(w.BT, H, grads + lo.w_hh(l, d));
         if (l == 0) {
           // narrow input: [dW_ih | db] = dz^T [X | 1] in fp32
-          wgrad(dZ, 4 * H, 4 * H, Xl, D, D, nullptr, 0, nullptr, 0, grads + lo.w_ih[l * dirs + d], nullptr,
-                grads + lo.bias(l, d));
+          narrow(dZ, Xl, D, grads + lo.w_ih[l * dirs + d], grads + lo.bias(l, d));
         } else {
           L.run("transpose_bf16", [&] { return bkt::launch_transpose_bf16(Xl, D, nullptr, NT, D, w.BT, NTp, s); });
           tc_reduce(w.BT, D, grads + lo.w_ih[l * dirs + d]);
@@ -562,8 +572,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         tf32_reduce(4 * H, w.Y[l] + d * H, DH, w.prev_tok[d], H, grads + lo.w_hh(l, d));
         if (l == 0) {
           // narrow input: [dW_ih | db] = dz^T [X | 1] on the FMA pipe
-          wgrad(dZ, 4 * H, 4 * H, Xl, D, D, nullptr, 0, nullptr, 0, grads + lo.w_ih[l * dirs + d], nullptr,
-                grads + lo.bias(l, d));
+          narrow(dZ, Xl, D, grads + lo.w_ih[l * dirs + d], grads + lo.bias(l, d));
         } else {
           tf32_reduce(4 * H, Xl, D, nullptr, D, grads + lo.w_ih[l * dirs + d]);
           bias_sum(dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
@@ -790,8 +799,13 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
     const size_t NTq = (NT + 7) & ~size_t(7), MA = std::max<size_t>(4 * H, (size_t)lo.C);
     BKT_ALLOC(w.AT, MA * NTq);
     BKT_ALLOC(w.ATl, MA * NTq);
-    BKT_ALLOC(w.BTf, DH * NTq);
-    BKT_ALLOC(w.BTl, DH * NTq);
+    const size_t DHp = (DH + 3) & ~size_t(3), Cp = ((size_t)lo.C + 3) & ~size_t(3);
+    BKT_ALLOC(w.BTf, DHp * NTq);
+    BKT_ALLOC(w.BTl, DHp * NTq);
+    BKT_ALLOC(w.Lh, NT * Cp);
+    BKT_ALLOC(w.Ll, NT * Cp);
+    BKT_ALLOC(w.Wh, Cp * DHp);
+    BKT_ALLOC(w.Wl, Cp * DHp);
   }
   if (cfg->gemm_precision == BKT_GEMM_BF16) {
     const size_t NTp = (NT + 7) & ~size_t(7);
@@ -1022,8 +1036,13 @@ int bkt::step_on_scratch(const bkt_model_cfg *cfg, const bkt_batch *bt, const fl
     const size_t NTq = (NT + 7) & ~size_t(7), MA = std::max<size_t>(4 * H, (size_t)lo.C);
     w.AT = cv.take<float>(MA * NTq);
     w.ATl = cv.take<float>(MA * NTq);
-    w.BTf = cv.take<float>(DH * NTq);
-    w.BTl = cv.take<float>(DH * NTq);
+    const size_t DHp = (DH + 3) & ~size_t(3), Cp = ((size_t)lo.C + 3) & ~size_t(3);
+    w.BTf = cv.take<float>(DHp * NTq);
+    w.BTl = cv.take<float>(DHp * NTq);
+    w.Lh = cv.take<float>(NT * Cp);
+    w.Ll = cv.take<float>(NT * Cp);
+    w.Wh = cv.take<float>(Cp * DHp);
+    w.Wl = cv.take<float>(Cp * DHp);
   }
   if (cfg->gemm_precision == BKT_GEMM_BF16) {
     const size_t NTp = (NT + 7) & ~size_t(7);

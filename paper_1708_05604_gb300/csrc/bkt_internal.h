@@ -69,21 +69,10 @@ struct GemmArgs {
 };
 cudaError_t launch_gemm_f32(bool a_t, bool b_t, const GemmArgs &g, cudaStream_t s);
 
-// Fused weight-gradient contraction over tokens (k_wgrad.cu):
-//   G[m][n] = sum_k A[k*lda + m] * Bv[k][n],  Bv[k] = [B1[k] (D1) | B2[gather2[k]] (D2) | 1 (ones)]
-// split over `splits` token ranges into P, then reduced in order and
-// scattered: column n < D1 -> out1[m*D1+n], n < D1+D2 -> out2[m*D2+n-D1],
-// the ones column -> out3[m].
-struct WgradArgs {
-  int M, N, K;
-  const float *A; int64_t lda;
-  int D1; const float *B1; int64_t ldb1;
-  int D2; const float *B2; int64_t ldb2; const int32_t *gather2;
-  int ones;
-  float *P; int splits;
-};
-int wgrad_splits(int M, int N, int K, int sm_count, size_t part_floats);
-cudaError_t launch_wgrad(const WgradArgs &g, float *out1, float *out2, float *out3, cudaStream_t s);
+// [out_w | out_b][m] = sum over the K token rows of A[k][m] [X[k] | 1] for an
+// input X of D <= 16 columns (out_w row-major [M x D]); fixed summation order.
+cudaError_t launch_narrow_wgrad(const float *A, int64_t lda, int M, const float *X, int D, int K, float *P,
+                                size_t part_floats, int sm_count, float *out_w, float *out_b, cudaStream_t s);
 // out[m*N + n] = sum_z P[z][m][n] (fixed order).
 cudaError_t launch_splitk_sum(const float *P, int splits, int M, int N, float *out, cudaStream_t s);
 
@@ -97,6 +86,11 @@ cudaError_t launch_colsum(const float *A, int64_t lda, int R, int M, float *P, i
 // hi and lo both tf32 values (zeros where src_row[r] < 0).
 cudaError_t launch_transpose_split(const float *src, int64_t lds, const int32_t *src_row, int R, int C, float *hi,
                                    float *lo, int64_t ldd, cudaStream_t s);
+// The same split without transposing (row-major, destination stride ldd).
+cudaError_t launch_split_rows(const float *src, int64_t lds, int R, int C, float *hi, float *lo, int64_t ldd,
+                              cudaStream_t s);
+// x[r][:C] <- log-softmax(x[r][:C]) in place (C <= 128).
+cudaError_t launch_log_softmax_rows(float *x, int64_t ld, int R, int C, cudaStream_t s);
 
 // bf16 tensor-core GEMM (k_gemm_tc.cu):
 //   D[m][n] (+)= sum_k A[m][k] B[n][k] (+ bias[n]); A, B bf16 with K contiguous
@@ -197,6 +191,8 @@ struct StepBufs {
   // split-precision (3xTF32) operands of the fp32 contractions over tokens
   float *AT, *ATl;                            // [max(4H, C) x NTq] transposed dz / dlogit, hi and lo
   float *BTf, *BTl;                           // [dirs*H x NTq] transposed X, h_{t-1} or Y, hi and lo
+  float *Lh, *Ll;                             // [NT x Cp] dlogit split, rows padded to Cp = C rounded to 4
+  float *Wh, *Wl;                             // [Cp x dirs*H] W_out split (or its transpose)
   // bf16 GEMM path only (null otherwise)
   void *Yb;                                   // [NT x dirs*H] bf16 layer input of a projection
   void *dZb;                                  // [NT x 4H] bf16 dz (input-gradient GEMM)

@@ -117,6 +117,63 @@ cudaError_t launch_transpose_split(const float *src, int64_t lds, const int32_t 
   return cudaGetLastError();
 }
 
+// fp32 [R x C] (stride lds) -> hi, lo [R x C] (stride ldd >= C) as in the
+// transposing split; padding columns C..ldd-1 are left untouched.
+__global__ void split_rows_kernel(const float *__restrict__ src, int64_t lds, int R, int C, float *__restrict__ hi,
+                                  float *__restrict__ lo, int64_t ldd) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < (int64_t)R * C;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int r = (int)(i / C), c = (int)(i % C);
+    const float x = src[(int64_t)r * lds + c];
+    const float h = __uint_as_float((__float_as_uint(x) + 0x1000u) & 0xFFFFE000u);
+    const float l = __uint_as_float((__float_as_uint(x - h) + 0x1000u) & 0xFFFFE000u);
+    hi[(int64_t)r * ldd + c] = h;
+    lo[(int64_t)r * ldd + c] = l;
+  }
+}
+
+cudaError_t launch_split_rows(const float *src, int64_t lds, int R, int C, float *hi, float *lo, int64_t ldd,
+                              cudaStream_t s) {
+  if (R <= 0 || C <= 0) return cudaSuccess;
+  const int blocks = (int)std::min<int64_t>(8192, ((int64_t)R * C + 255) / 256);
+  split_rows_kernel<<<blocks, 256, 0, s>>>(src, lds, R, C, hi, lo, ldd);
+  return cudaGetLastError();
+}
+
+// In-place log-softmax over the C columns of each row, one warp per row.
+__global__ void log_softmax_rows_kernel(float *__restrict__ x, int64_t ld, int R, int C) {
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (r >= R) return;
+  float *row = x + (int64_t)r * ld;
+  float v[4];
+  float mx = -INFINITY;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int c = lane + 32 * j;
+    v[j] = c < C ? row[c] : -INFINITY;
+    mx = fmaxf(mx, v[j]);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  float se = 0.f;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) se += (lane + 32 * j < C) ? expf(v[j] - mx) : 0.f;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
+  const float lz = mx + logf(se);
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+    if (lane + 32 * j < C) row[lane + 32 * j] = v[j] - lz;
+}
+
+cudaError_t launch_log_softmax_rows(float *x, int64_t ld, int R, int C, cudaStream_t s) {
+  if (R <= 0) return cudaSuccess;
+  if (C > 128) return cudaErrorInvalidValue;
+  log_softmax_rows_kernel<<<(R + 7) / 8, 256, 0, s>>>(x, ld, R, C);
+  return cudaGetLastError();
+}
+
 __global__ void colsum_kernel(const float *__restrict__ A, int64_t lda, int R, int M, float *__restrict__ P,
                               int splits) {
   const int m = blockIdx.x * blockDim.x + threadIdx.x;

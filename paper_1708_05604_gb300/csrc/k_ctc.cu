@@ -5,9 +5,10 @@
 // thousands of steps fp32 log-probabilities reach magnitudes of 1e3-1e4,
 // where an fp32 ulp is ~1e-3 and the posterior exp(alpha + beta - ln p)
 // would lose three digits.  So each table row is kept relative to a running
-// offset: after step t the row is shifted by its maximum m_t, the shifts are
-// summed in double for ln p, and the stored rows hold alpha_t - M_t with
-// values near 0.  The posterior normalises per time step,
+// offset: every few steps the row is shifted by its maximum, the shifts are
+// summed in double for ln p, and the stored rows hold alpha_t minus the
+// offset, values of magnitude tens at most.  The posterior normalises per
+// time step,
 //   gamma_t(s) = exp(a_t(s) + b_t(s) - lse_s'(a_t(s') + b_t(s'))),
 // which is exactly alpha beta / p because sum_s alpha_t(s) beta_t(s) = p at
 // every t, and is independent of the offsets.
@@ -110,8 +111,9 @@ cudaError_t launch_out_logsoftmax(const float *Y, int n_tok, int DH, const float
 // where bh_t(s) = beta_t(s) + lp_t(l'_s) (beta with the emission at t).
 // Both start from the two admissible end positions.  Each step keeps one
 // CTA barrier: step t reads row t-1 from one shared buffer and writes row t
-// into the other, plus one max per warp; the row maximum is folded in on
-// the next step.  Emissions are prefetched 8 steps ahead into registers.
+// into the other.  Every 8 steps the row maximum is reduced (one max per
+// warp) and folded in on the next step.  Emissions are prefetched 8 steps
+// ahead into registers.
 namespace {
 
 // The recursion's serial chain runs T steps; the hardware exp2/log2
@@ -229,9 +231,14 @@ __global__ void __launch_bounds__(512) ctc_tables_kernel(DevIdx ix, const float 
       if (step >= L) break;
       const float *cur = p ? buf1 : buf0;
       float *nxt = p ? buf0 : buf1;
-      const float *wm = wmax + p * 32;
-      float mprev = wm[0];
-      for (int i = 1; i < nw; ++i) mprev = fmaxf(mprev, wm[i]);
+      // the row is re-anchored to its maximum every kPre steps; in between a
+      // row can rise by at most ln 3 per step, so values stay small
+      float mprev = 0.f;
+      if (u == 0) {
+        const float *wm = wmax + p * 32;
+        mprev = wm[0];
+        for (int i = 1; i < nw; ++i) mprev = fmaxf(mprev, wm[i]);
+      }
       const int tprev = fwd ? step - 1 : L - step;
       float lm = -CUDART_INF_F;
 #pragma unroll
@@ -249,9 +256,11 @@ __global__ void __launch_bounds__(512) ctc_tables_kernel(DevIdx ix, const float 
         em[j][u] = (step + kPre < L) ? emis(step + kPre, j) : 0.f;
       }
       M += (double)mprev;
+      if (u == kPre - 1 || step == L - 1) {  // uniform over the CTA
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) lm = fmaxf(lm, __shfl_xor_sync(0xffffffffu, lm, o));
-      if (lane == 0) wmax[(p ^ 1) * 32 + wid] = lm;
+        for (int o = 16; o > 0; o >>= 1) lm = fmaxf(lm, __shfl_xor_sync(0xffffffffu, lm, o));
+        if (lane == 0) wmax[(p ^ 1) * 32 + wid] = lm;
+      }
       p ^= 1;
       __syncthreads();
     }
