@@ -414,6 +414,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
       ra.Whh[d] = params + lo.w_hh(l, d);
     }
     ra.Y = w.Y[l];
+    ra.status = w.status;
     L.run("lstm_fwd", [&] { return bkt::launch_lstm_fwd(ra, geom[l], s); });
   }
 
@@ -522,6 +523,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
       ra.Whh[d] = params + lo.w_hh(l, d);
     }
     ra.Y = w.Y[l];
+    ra.status = w.status;
     ra.dY = w.dY;
     L.run("lstm_bwd", [&] { return bkt::launch_lstm_bwd(ra, geom[l], s); });
     const int D = lo.D(l);
@@ -895,9 +897,10 @@ extern "C" int bkt_ctx_sync_status(bkt_ctx *c) {
   if (e != cudaSuccess) return cuda_err("cudaMemcpy(status)", e);
   if (st != 0) {
     cudaMemset(c->w.status, 0, sizeof st);
-    return set_err(BKT_EDEVICE, "device check failed (flags 0x%x):%s%s", st,
+    return set_err(BKT_EDEVICE, "device check failed (flags 0x%x):%s%s%s", st,
                    (st & 1) ? " a label is out of range or equals the blank;" : "",
-                   (st & 2) ? " a tensor-core pipeline wait timed out;" : "");
+                   (st & 2) ? " a tensor-core pipeline wait timed out;" : "",
+                   (st & 4) ? " a recurrent cluster exchange wait timed out;" : "");
   }
   return BKT_OK;
 }

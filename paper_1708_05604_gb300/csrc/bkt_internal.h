@@ -134,7 +134,8 @@ cudaError_t launch_ctc_grad(const DevIdx &ix, float *logp_dlogit, int C, int bla
 
 // Geometry of the recurrent kernels for one layer.
 //   mode 1: one CTA per bc rows holds all of W_hh (H in {32, 64, 128});
-//   mode 0: a cluster of cs CTAs per bc rows splits the hidden units.
+//   mode 2: register-tiled cluster of cs CTAs per bc rows (H in {256, 512});
+//   mode 0: a cluster of cs CTAs per bc rows splits the hidden units (any H).
 struct RecGeom {
   int mode;
   int cs;        // CTAs per cluster (hidden units split cs ways)
@@ -158,10 +159,18 @@ struct RecArgs {
   const float *Whh[2];
   float *Y;            // forward output / backward: h source for nothing
   const float *dY;     // backward: d loss / d Y of this layer [n_tok x dirs*H]
+  int32_t *status;     // device error flags (bit 4: a cluster exchange wait timed out)
 };
 cudaError_t launch_lstm_fwd(const RecArgs &a, const RecGeom &g, cudaStream_t s);
 // a11: BPTT for both directions; Z[d] holds the gates on entry and dz on exit.
 cudaError_t launch_lstm_bwd(const RecArgs &a, const RecGeom &g, cudaStream_t s);
+
+// Register-tiled cluster kernels for H = 256 and 512 (k_lstm_cl.cu):
+// CTAs per cluster for H (0: not handled there), batch rows per cluster for a
+// batch of b rows (0: the configuration cannot launch), launch.
+int cl_cluster_size(int H);
+int plan_cl_rows(int H, int b, int dirs);
+cudaError_t launch_lstm_cl(const RecArgs &a, int bc, bool bwd, cudaStream_t s);
 
 // Single-CTA recurrent kernels (k_lstm_cta.cu).
 bool cta_supported(int H);

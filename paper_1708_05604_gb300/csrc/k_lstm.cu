@@ -340,6 +340,18 @@ RecGeom plan_recurrent(int H, int b, int dirs, int sm_count) {
     g.w_smem = 1;
     return g;
   }
+  if (cl_cluster_size(H) > 0) {
+    const int bc = plan_cl_rows(H, b, dirs);
+    if (bc > 0) {
+      g.mode = 2;
+      g.cs = cl_cluster_size(H);
+      g.bc = bc;
+      g.ks = 1;
+      g.threads = 256;
+      g.w_smem = 1;
+      return g;
+    }
+  }
   int cs = 16;
   while (cs > 1 && (H % cs != 0 || H / cs < 8)) cs >>= 1;
   for (;; cs >>= 1) {
@@ -405,6 +417,7 @@ cudaError_t launch_rec(K kernel, const RecArgs &a, const RecGeom &g, bool bwd, c
 
 cudaError_t launch_lstm_fwd(const RecArgs &a, const RecGeom &g, cudaStream_t s) {
   if (g.mode == 1) return launch_lstm_cta(a, g.bc, false, s);
+  if (g.mode == 2) return launch_lstm_cl(a, g.bc, false, s);
   if (a.H % g.cs != 0) return cudaErrorInvalidValue;
   if (!g.w_smem && (a.H % 4) != 0) return cudaErrorInvalidValue;
   return g.w_smem ? launch_rec(lstm_fwd_kernel<true>, a, g, false, s) : launch_rec(lstm_fwd_kernel<false>, a, g, false, s);
@@ -412,6 +425,7 @@ cudaError_t launch_lstm_fwd(const RecArgs &a, const RecGeom &g, cudaStream_t s) 
 
 cudaError_t launch_lstm_bwd(const RecArgs &a, const RecGeom &g, cudaStream_t s) {
   if (g.mode == 1) return launch_lstm_cta(a, g.bc, true, s);
+  if (g.mode == 2) return launch_lstm_cl(a, g.bc, true, s);
   if (a.H % g.cs != 0) return cudaErrorInvalidValue;
   if (!g.w_smem && (a.H % 4) != 0) return cudaErrorInvalidValue;
   return g.w_smem ? launch_rec(lstm_bwd_kernel<true>, a, g, true, s) : launch_rec(lstm_bwd_kernel<false>, a, g, true, s);
