@@ -388,20 +388,27 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         L.run("gemm_tc", [&] { return bkt::launch_gemm_bf16_tc(g, s); });
       }
     } else {
+      // a5 in fp32 on the tensor cores (3xTF32): Zx = Y_{l-1} W_ih^T + b; both
+      // operands are K-contiguous, split into hi + lo rows padded to 16 bytes
+      const int DHq = (DH + 3) & ~3;
+      L.run("split_rows", [&] { return bkt::launch_split_rows(w.Y[l - 1], DH, NT, DH, w.AT, w.ATl, DHq, s); });
       for (int d = 0; d < dirs; ++d) {
-        bkt::GemmArgs g{};
+        L.run("split_rows", [&] {
+          return bkt::launch_split_rows(params + lo.w_ih[l * dirs + d], DH, 4 * H, DH, w.Wh, w.Wl, DHq, s);
+        });
+        bkt::TcGemmArgs g{};
         g.M = NT;
         g.N = 4 * H;
         g.K = DH;
-        g.A = w.Y[l - 1];
-        g.lda = DH;
-        g.B = params + lo.w_ih[l * dirs + d];
-        g.ldb = DH;
-        g.C = Zl[d];
-        g.ldc = 4 * H;
+        g.A = w.AT;
+        g.lda = DHq;
+        g.B = w.Wh;
+        g.ldb = DHq;
+        g.D = Zl[d];
+        g.ldd = 4 * H;
         g.bias = params + lo.bias(l, d);
-        g.splits = 1;
-        L.run("gemm_proj", [&] { return bkt::launch_gemm_f32(false, true, g, s); });
+        g.err = w.status;
+        L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.ATl, w.Wl, s); });
       }
     }
     bkt::RecArgs ra{};
@@ -603,20 +610,29 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         L.run("gemm_tc", [&] { return bkt::launch_gemm_bf16_tc(g, s); });
       }
     } else if (l > 0) {
+      // dX = dz W_ih in fp32 on the tensor cores (3xTF32): dz rows are
+      // K-contiguous already, W_ih is transposed while it is split
       for (int d = 0; d < dirs; ++d) {
-        bkt::GemmArgs g{};
+        L.run("split_rows", [&] {
+          return bkt::launch_split_rows(w.Z[l * dirs + d], 4 * H, NT, 4 * H, w.AT, w.ATl, 4 * H, s);
+        });
+        L.run("transpose_split", [&] {
+          return bkt::launch_transpose_split(params + lo.w_ih[l * dirs + d], DH, nullptr, 4 * H, DH, w.Wh, w.Wl,
+                                             4 * H, s);
+        });
+        bkt::TcGemmArgs g{};
         g.M = NT;
         g.N = DH;
         g.K = 4 * H;
-        g.A = w.Z[l * dirs + d];
+        g.A = w.AT;
         g.lda = 4 * H;
-        g.B = params + lo.w_ih[l * dirs + d];
-        g.ldb = DH;
-        g.C = w.dY;
-        g.ldc = DH;
+        g.B = w.Wh;
+        g.ldb = 4 * H;
+        g.D = w.dY;
+        g.ldd = DH;
         g.accumulate = d > 0;
-        g.splits = 1;
-        L.run("gemm_dx", [&] { return bkt::launch_gemm_f32(false, false, g, s); });
+        g.err = w.status;
+        L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.ATl, w.Wl, s); });
       }
     }
   }
@@ -806,8 +822,10 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
     BKT_ALLOC(w.BTl, DHp * NTq);
     BKT_ALLOC(w.Lh, NT * Cp);
     BKT_ALLOC(w.Ll, NT * Cp);
-    BKT_ALLOC(w.Wh, Cp * DHp);
-    BKT_ALLOC(w.Wl, Cp * DHp);
+    // W_out split; for fp32 stacks also W_ih (and its transpose) of a layer > 0
+    const size_t WW = std::max(Cp * DHp, (lo.L > 1 && cfg->gemm_precision != BKT_GEMM_BF16) ? 4 * (size_t)H * DHp : 0);
+    BKT_ALLOC(w.Wh, WW);
+    BKT_ALLOC(w.Wl, WW);
   }
   if (cfg->gemm_precision == BKT_GEMM_BF16) {
     const size_t NTp = (NT + 7) & ~size_t(7);
@@ -1044,8 +1062,9 @@ int bkt::step_on_scratch(const bkt_model_cfg *cfg, const bkt_batch *bt, const fl
     w.BTl = cv.take<float>(DHp * NTq);
     w.Lh = cv.take<float>(NT * Cp);
     w.Ll = cv.take<float>(NT * Cp);
-    w.Wh = cv.take<float>(Cp * DHp);
-    w.Wl = cv.take<float>(Cp * DHp);
+    const size_t WW = std::max(Cp * DHp, (lo.L > 1 && cfg->gemm_precision != BKT_GEMM_BF16) ? 4 * (size_t)H * DHp : 0);
+    w.Wh = cv.take<float>(WW);
+    w.Wl = cv.take<float>(WW);
   }
   if (cfg->gemm_precision == BKT_GEMM_BF16) {
     const size_t NTp = (NT + 7) & ~size_t(7);

@@ -52,23 +52,6 @@ cudaError_t launch_proj_narrow(const float *X, int n_tok, int in_dim, const floa
                                int64_t w_off, int64_t w_stride, int H, int dirs,
                                float *const *Z, cudaStream_t s);
 
-// Generic fp32 GEMM: C[m][n] (+)= sum_k opA(m,k) opB(k,n) (+ bias[n]).
-//   opA(m,k) = a_t ? A[k*lda+m] : A[m*lda+k]
-//   opB(k,n) = b_t ? B[n*ldb+k] : B[row(k)*ldb+n], row(k) = gather ? gather[k] : k,
-//              a negative gather entry reads zeros.
-//   splits > 1: partial sums go to P[z][m*N+n] (C, bias, accumulate unused).
-struct GemmArgs {
-  int M, N, K;
-  const float *A; int64_t lda;
-  const float *B; int64_t ldb;
-  const int32_t *gather;
-  float *C; int64_t ldc;
-  const float *bias;
-  int accumulate;
-  float *P; int splits;
-};
-cudaError_t launch_gemm_f32(bool a_t, bool b_t, const GemmArgs &g, cudaStream_t s);
-
 // [out_w | out_b][m] = sum over the K token rows of A[k][m] [X[k] | 1] for an
 // input X of D <= 16 columns (out_w row-major [M x D]); fixed summation order.
 cudaError_t launch_narrow_wgrad(const float *A, int64_t lda, int M, const float *X, int D, int K, float *P,
@@ -115,10 +98,6 @@ cudaError_t launch_gemm_bf16_tc(const TcGemmArgs &g, cudaStream_t s);
 // multiples of 4, 16-byte aligned); D (or partials) as for the bf16 GEMM.
 int tf32x3_splits(int M, int N, int K, int sm_count, size_t part_floats);
 cudaError_t launch_gemm_tf32x3_tc(const TcGemmArgs &g, const void *A_lo, const void *B_lo, cudaStream_t s);
-
-// a7: logp[tok][c] = log-softmax_c(b[c] + W[c] . Y[tok]).
-cudaError_t launch_out_logsoftmax(const float *Y, int n_tok, int DH, const float *W,
-                                  const float *bias, int C, float *logp, cudaStream_t s);
 
 // a8: log-space CTC forward (alpha) and backward (beta-hat) tables, one CTA
 // per (row, direction); writes the per-sequence loss and the row's flag.

@@ -1,5 +1,5 @@
-// k_ctc.cu -- output layer + log-softmax (a7), the CTC forward/backward
-// tables (a8) and the softmax gradient (a9).
+// k_ctc.cu -- the CTC forward/backward tables (a8) and the softmax
+// gradient (a9).
 //
 // CTC follows Graves et al. 2006 (the paper's ref. [15]) in log space.  Over
 // thousands of steps fp32 log-probabilities reach magnitudes of 1e3-1e4,
@@ -18,87 +18,7 @@
 
 namespace bkt {
 
-// ---------------------------------------------------------------------------
-// a7.  A CTA owns 32 tokens; warp w owns tokens 4w..4w+3 and lane l owns
-// classes l, l+32, l+64, l+96.  Y and W_out arrive in 32-deep k slabs through
-// shared memory.  The log-softmax is a warp reduction per token.
-constexpr int kOutTok = 32, kOutK = 32, kMaxClasses = 128;
-
-__global__ void __launch_bounds__(256) out_logsoftmax_kernel(const float *__restrict__ Y, int n_tok, int DH,
-                                                             const float *__restrict__ W,
-                                                             const float *__restrict__ bias, int C,
-                                                             float *__restrict__ logp) {
-  __shared__ float Ys[kOutK][kOutTok + 1];
-  __shared__ float Ws[kOutK][kMaxClasses];
-  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
-  const int t0 = blockIdx.x * kOutTok;
-  float acc[4][4];
-#pragma unroll
-  for (int i = 0; i < 4; ++i)
-#pragma unroll
-    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
-  for (int k0 = 0; k0 < DH; k0 += kOutK) {
-    for (int e = tid; e < kOutTok * kOutK; e += 256) {
-      const int tt = e / kOutK, kk = e % kOutK;
-      const int tok = t0 + tt, k = k0 + kk;
-      Ys[kk][tt] = (tok < n_tok && k < DH) ? Y[(int64_t)tok * DH + k] : 0.f;
-    }
-    for (int e = tid; e < kMaxClasses * kOutK; e += 256) {
-      const int c = e / kOutK, kk = e % kOutK;
-      const int k = k0 + kk;
-      Ws[kk][c] = (c < C && k < DH) ? W[(int64_t)c * DH + k] : 0.f;
-    }
-    __syncthreads();
-#pragma unroll 8
-    for (int kk = 0; kk < kOutK; ++kk) {
-      float wv[4], yv[4];
-#pragma unroll
-      for (int j = 0; j < 4; ++j) wv[j] = Ws[kk][lane + 32 * j];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) yv[i] = Ys[kk][w * 4 + i];
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(yv[i], wv[j], acc[i][j]);
-    }
-    __syncthreads();
-  }
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int tok = t0 + w * 4 + i;
-    float v[4];
-    float mx = -CUDART_INF_F;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int c = lane + 32 * j;
-      v[j] = (c < C) ? acc[i][j] + bias[c] : -CUDART_INF_F;
-      mx = fmaxf(mx, v[j]);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    float se = 0.f;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) se += (lane + 32 * j < C) ? expf(v[j] - mx) : 0.f;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
-    const float lz = mx + logf(se);
-    if (tok < n_tok) {
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int c = lane + 32 * j;
-        if (c < C) logp[(int64_t)tok * C + c] = v[j] - lz;
-      }
-    }
-  }
-}
-
-cudaError_t launch_out_logsoftmax(const float *Y, int n_tok, int DH, const float *W, const float *bias, int C,
-                                  float *logp, cudaStream_t s) {
-  if (C > kMaxClasses) return cudaErrorInvalidValue;
-  const int blocks = (n_tok + kOutTok - 1) / kOutTok;
-  out_logsoftmax_kernel<<<blocks, 256, 0, s>>>(Y, n_tok, DH, W, bias, C, logp);
-  return cudaGetLastError();
-}
+constexpr int kMaxClasses = 128;
 
 // ---------------------------------------------------------------------------
 // a8.  One CTA per (row, direction).  Thread i owns extended-label positions

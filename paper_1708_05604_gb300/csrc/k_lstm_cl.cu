@@ -48,7 +48,11 @@ constexpr int kClTokCap = 8192;  // time offsets staged in shared memory up to t
 constexpr int kClPolls = 1 << 22;
 constexpr int32_t kErrExchange = 4;
 
-__device__ __forceinline__ float sigm_cl(float x) { return 1.f / (1.f + expf(-x)); }
+// Gate nonlinearities from the exponential intrinsic: sigma(x) = 1 / (1 + e^-x)
+// and tanh(x) = 1 - 2 / (1 + e^2x) (absolute error a few 1e-8; both saturate
+// correctly when the exponential overflows to +inf or underflows to 0).
+__device__ __forceinline__ float sigm_cl(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
+__device__ __forceinline__ float tanh_cl(float x) { return 1.f - __fdividef(2.f, 1.f + __expf(2.f * x)); }
 
 __device__ __forceinline__ uint32_t smem_addr(const void *p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -94,6 +98,14 @@ __device__ __forceinline__ void st_async4(uint32_t raddr, float4 v, uint32_t rmb
                : "memory");
 }
 
+// Per-thread asynchronous 4-byte copy global -> shared (the next step's
+// inputs are requested a whole step before they are read).
+__device__ __forceinline__ void cp_async4_cl(float *dst, const float *src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_addr(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_commit_cl() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_wait_all_cl() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
 // Reduce-scatter of N values over the KS lanes that differ in lane bits
 // 0 .. log2(KS)-1: on return v[0 .. N/KS - 1] of lane l holds the sums of
 // positions (l % KS) * N/KS .. (l % KS + 1) * N/KS - 1.
@@ -117,39 +129,48 @@ __device__ __forceinline__ void reduce_scatter_lanes(float (&v)[N], int lane) {
   }
 }
 
-template <int H, int CS, int BC>
+template <int H, int CS, int BC, int NH>
 struct ClGeom {
   static constexpr int Hc = H / CS;          // hidden units per CTA
   static constexpr int KS = H / 64;          // 64-column slices (forward)
   static constexpr int R = 4 * Hc;           // gate rows per CTA
   static constexpr int RSL = R / 64;         // 64-row slices (BPTT)
+  static constexpr int BH = BC / NH;         // rows per half
   static constexpr int HPAD = H + 4 * KS;    // h row: 4 floats of padding after each slice
-  static constexpr int DZS = R * BC + 4 * RSL;  // dz buffer: [R][BC], 4 floats after each 64 rows
-  static constexpr uint32_t kXBytes = BC * H * 4;  // bytes a CTA receives per step
+  static constexpr int DZS = R * BH + 4 * RSL;  // dz buffer of a half: [R][BH], 4 floats after each 64 rows
+  static constexpr uint32_t kXBytes = BH * H * 4;  // bytes a CTA receives per half and step
   static_assert(Hc * KS == kClThreads && (H / 4) * RSL == kClThreads, "256 threads per CTA");
-  static_assert(Hc % 4 == 0 && BC % 4 == 0, "float4 exchange");
-  static size_t fwd_floats() { return (size_t)8 * 4 * kClThreads * 4 + 2 * BC * HPAD + 2 * BC * Hc; }
-  static size_t bwd_floats() { return (size_t)32 * kClThreads * 4 + 2 * DZS + (size_t)2 * CS * BC * Hc; }
+  static_assert(Hc % 4 == 0 && BH % 4 == 0 && BC == BH * NH, "float4 exchange");
+  static constexpr int PPT = (Hc * BH + kClThreads - 1) / kClThreads;  // BPTT pairs per thread and half
+  static size_t fwd_floats() {
+    return (size_t)8 * 4 * kClThreads * 4 + 2 * NH * BH * (HPAD + Hc);
+  }
+  static size_t bwd_floats() {
+    return (size_t)32 * kClThreads * 4 + 2 * NH * (DZS + (size_t)CS * BH * Hc) + (size_t)2 * NH * kClThreads * PPT * 8;
+  }
 };
 
-size_t cl_tail_bytes(int T) { return 16 + (T + 1 <= kClTokCap ? (size_t)(T + 1) * 4 : 0); }
+size_t cl_tail_bytes(int NH, int T) { return 16 * NH + (T + 1 <= kClTokCap ? (size_t)(T + 1) * 4 : 0); }
 
 }  // namespace
 
-template <int H, int CS, int BC>
+// Rows of a cluster are processed as NH halves of BH rows, one after the
+// other within a step, each with its own receive buffers and mbarriers, so
+// the exchange of one half overlaps the arithmetic of the other.
+template <int H, int CS, int BC, int NH>
 __global__ void __launch_bounds__(kClThreads, 1) lstm_fwd_cl_kernel(RecArgs a) {
-  using Gm = ClGeom<H, CS, BC>;
-  constexpr int Hc = Gm::Hc, KS = Gm::KS, HPAD = Gm::HPAD, G = 4 * H, NTH = kClThreads;
-  constexpr int NV = 4 * BC, NPL = NV / KS;  // partial sums per thread, per lane after the reduction
+  using Gm = ClGeom<H, CS, BC, NH>;
+  constexpr int Hc = Gm::Hc, KS = Gm::KS, HPAD = Gm::HPAD, BH = Gm::BH, G = 4 * H, NTH = kClThreads;
+  constexpr int NV = 4 * BH, NPL = NV / KS;  // partial sums per thread, per lane after the reduction
   static_assert(NPL == 2 || NPL % 4 == 0, "a lane finishes whole units or one gate pair");
-  constexpr int RPL = NPL >= 4 ? NPL / 4 : 1;  // batch rows finished per lane
-  constexpr int SEND4 = BC * Hc / 4;           // float4 sent to each CTA per step
+  constexpr int RPL = NPL >= 4 ? NPL / 4 : 1;  // rows of a half finished per lane
+  constexpr int SEND4 = BH * Hc / 4;           // float4 sent to each CTA per half and step
   extern __shared__ __align__(16) float sm[];
   float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [8][4][NTH] columns 32..63 of each slice
-  float *hb = sm + 8 * 4 * NTH * 4;              // [2][BC][HPAD] received h
-  float *stg = hb + 2 * BC * HPAD;               // [2][BC][Hc] this CTA's h slice
-  uint64_t *mb = reinterpret_cast<uint64_t *>(stg + 2 * BC * Hc);
-  int *toff_s = reinterpret_cast<int *>(mb + 2);
+  float *hb = sm + 8 * 4 * NTH * 4;              // [NH][2][BH][HPAD] received h
+  float *stg = hb + 2 * NH * BH * HPAD;          // [NH][2][BH][Hc] this CTA's h slice
+  uint64_t *mb = reinterpret_cast<uint64_t *>(stg + 2 * NH * BH * Hc);  // [NH][2]
+  int *toff_s = reinterpret_cast<int *>(mb + 2 * NH);
   const int T = a.ix.T;
   const bool toff_sm = T + 1 <= kClTokCap;
   const int *toff = toff_sm ? toff_s : a.ix.tok_off;
@@ -178,174 +199,182 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_fwd_cl_kernel(RecArgs a) {
   }
   if (toff_sm)
     for (int i = t; i <= T; i += NTH) toff_s[i] = a.ix.tok_off[i];
-  int len[BC];
-#pragma unroll
-  for (int b = 0; b < BC; ++b) len[b] = (r0 + b < a.ix.b) ? a.ix.row_len[r0 + b] : 0;
-  const int Tg = len[0];
+  const int Tg = (r0 < a.ix.b) ? a.ix.row_len[r0] : 0;
   if (t == 0) {
-    mbar_init1(smem_addr(&mb[0]));
-    mbar_init1(smem_addr(&mb[1]));
+    for (int i = 0; i < 2 * NH; ++i) mbar_init1(smem_addr(&mb[i]));
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   cluster_barrier_all();  // barriers initialised everywhere before any remote store
-  if (t == 0) {
-    if (Tg >= 2) mbar_arm(smem_addr(&mb[0]), Gm::kXBytes);
-    if (Tg >= 3) mbar_arm(smem_addr(&mb[1]), Gm::kXBytes);
-  }
+  if (t == 0)
+    for (int h = 0; h < NH; ++h) {
+      if (Tg >= 2) mbar_arm(smem_addr(&mb[2 * h]), Gm::kXBytes);
+      if (Tg >= 3) mbar_arm(smem_addr(&mb[2 * h + 1]), Gm::kXBytes);
+    }
 
   float *__restrict__ Z = a.Z[d];
   float *__restrict__ Cs = a.Cst[d];
   float *__restrict__ Y = a.Y;
-  // lane ownership after the reduction: rows kl*RPL + rr with all four gates,
-  // or (NPL == 2) row kl/2 with gates 2*(kl&1), 2*(kl&1)+1
+  // lane ownership after the reduction (rows counted within a half): rows
+  // kl*RPL + rr with all four gates, or (NPL == 2) row kl/2 with gates
+  // 2*(kl&1), 2*(kl&1)+1
   auto own_row = [&](int rr) { return NPL >= 4 ? kl * RPL + rr : kl >> 1; };
   auto own_gate = [&](int j) { return NPL >= 4 ? (j & 3) : 2 * (kl & 1) + j; };
-  int olen[RPL];  // lengths of the owned rows (read directly: a runtime index into len[] would live in local memory)
+  int olen[NH][RPL];  // lengths of the owned rows (read directly: a runtime index into an array would live in local memory)
 #pragma unroll
-  for (int rr = 0; rr < RPL; ++rr) {
-    const int r = r0 + own_row(rr);
-    olen[rr] = r < a.ix.b ? a.ix.row_len[r] : 0;
-  }
-  auto tok_at = [&](int rr, int s) {
-    const int tt = d == 0 ? s : olen[rr] - 1 - s;
-    return toff[tt] + r0 + own_row(rr);
+  for (int h = 0; h < NH; ++h)
+#pragma unroll
+    for (int rr = 0; rr < RPL; ++rr) {
+      const int r = r0 + h * BH + own_row(rr);
+      olen[h][rr] = r < a.ix.b ? a.ix.row_len[r] : 0;
+    }
+  auto tok_at = [&](int h, int rr, int s) {
+    const int tt = d == 0 ? s : olen[h][rr] - 1 - s;
+    return toff[tt] + r0 + h * BH + own_row(rr);
   };
-  auto zx_at = [&](int j, int s) {  // owned pre-activation j of step s (0 once the row has ended)
+  auto zx_at = [&](int h, int j, int s) {  // owned pre-activation j of step s (0 once the row has ended)
     const int rr = NPL >= 4 ? j / 4 : 0;
-    return (s < olen[rr]) ? Z[(size_t)tok_at(rr, s) * G + own_gate(j) * H + gu] : 0.f;
+    return (s < olen[h][rr]) ? Z[(size_t)tok_at(h, rr, s) * G + own_gate(j) * H + gu] : 0.f;
   };
-  float zn[NPL];
+  // the next step's pre-activations are loaded into registers one step ahead
+  // (a shared-memory ring with asynchronous copies measured slower here)
+  float zn[NH][NPL], cst[NH][RPL];
 #pragma unroll
-  for (int j = 0; j < NPL; ++j) zn[j] = zx_at(j, 0);
-  float cst[RPL];
+  for (int h = 0; h < NH; ++h) {
 #pragma unroll
-  for (int rr = 0; rr < RPL; ++rr) cst[rr] = 0.f;
-  bool ok = true;
+    for (int j = 0; j < NPL; ++j) zn[h][j] = zx_at(h, j, 0);
+#pragma unroll
+    for (int rr = 0; rr < RPL; ++rr) cst[h][rr] = 0.f;
+  }
+  bool ok = true, stop = false;
 
-  for (int s = 0; s < Tg; ++s) {
-    float zc[NPL];
+  for (int s = 0; s < Tg && !stop; ++s) {
 #pragma unroll
-    for (int j = 0; j < NPL; ++j) zc[j] = zn[j];
-    if (s + 1 < Tg) {
+    for (int h = 0; h < NH; ++h) {
+      float zc[NPL];
 #pragma unroll
-      for (int j = 0; j < NPL; ++j) zn[j] = zx_at(j, s + 1);
-    }
-    float acc[NV];
+      for (int j = 0; j < NPL; ++j) zc[j] = zn[h][j];
+      if (s + 1 < Tg) {
 #pragma unroll
-    for (int i = 0; i < NV; ++i) acc[i] = 0.f;
-    if (s > 0) {  // h_{-1} = 0
-      const int e = s - 1;
-      ok = mbar_wait_bounded(smem_addr(&mb[e & 1]), (e >> 1) & 1) && ok;
-      if (t == 0 && e + 2 <= Tg - 2) mbar_arm(smem_addr(&mb[e & 1]), Gm::kXBytes);
-      const float *hv = hb + (e & 1) * BC * HPAD + kb + 4 * kl;
+        for (int j = 0; j < NPL; ++j) zn[h][j] = zx_at(h, j, s + 1);
+      }
+      float acc[NV];
 #pragma unroll
-      for (int k4 = 0; k4 < 8; ++k4) {
+      for (int i = 0; i < NV; ++i) acc[i] = 0.f;
+      if (s > 0) {  // h_{-1} = 0
+        const int e = s - 1;
+        ok = mbar_wait_bounded(smem_addr(&mb[2 * h + (e & 1)]), (e >> 1) & 1) && ok;
+        if (t == 0 && e + 2 <= Tg - 2) mbar_arm(smem_addr(&mb[2 * h + (e & 1)]), Gm::kXBytes);
+        const float *hv = hb + (2 * h + (e & 1)) * BH * HPAD + kb + 4 * kl;
 #pragma unroll
-        for (int b = 0; b < BC; ++b) {
-          const float4 h4 = *reinterpret_cast<const float4 *>(hv + b * HPAD + 4 * k4);
+        for (int k4 = 0; k4 < 8; ++k4) {
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            float x = fmaf(w[q][4 * k4], h4.x, acc[b * 4 + q]);
-            x = fmaf(w[q][4 * k4 + 1], h4.y, x);
-            x = fmaf(w[q][4 * k4 + 2], h4.z, x);
-            acc[b * 4 + q] = fmaf(w[q][4 * k4 + 3], h4.w, x);
+          for (int b = 0; b < BH; ++b) {
+            const float4 h4 = *reinterpret_cast<const float4 *>(hv + b * HPAD + 4 * k4);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              float x = fmaf(w[q][4 * k4], h4.x, acc[b * 4 + q]);
+              x = fmaf(w[q][4 * k4 + 1], h4.y, x);
+              x = fmaf(w[q][4 * k4 + 2], h4.z, x);
+              acc[b * 4 + q] = fmaf(w[q][4 * k4 + 3], h4.w, x);
+            }
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          float4 wv[4];
+#pragma unroll
+          for (int q = 0; q < 4; ++q) wv[q] = Ws4[(j * 4 + q) * NTH + t];
+#pragma unroll
+          for (int b = 0; b < BH; ++b) {
+            const float4 h4 = *reinterpret_cast<const float4 *>(hv + b * HPAD + 32 + 4 * j);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              float x = fmaf(wv[q].x, h4.x, acc[b * 4 + q]);
+              x = fmaf(wv[q].y, h4.y, x);
+              x = fmaf(wv[q].z, h4.z, x);
+              acc[b * 4 + q] = fmaf(wv[q].w, h4.w, x);
+            }
           }
         }
       }
+      reduce_scatter_lanes<NV, KS>(acc, lane);
+      float *sg = stg + (2 * h + (s & 1)) * BH * Hc;
+      if constexpr (NPL >= 4) {
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        float4 wv[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) wv[q] = Ws4[(j * 4 + q) * NTH + t];
-#pragma unroll
-        for (int b = 0; b < BC; ++b) {
-          const float4 h4 = *reinterpret_cast<const float4 *>(hv + b * HPAD + 32 + 4 * j);
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            float x = fmaf(wv[q].x, h4.x, acc[b * 4 + q]);
-            x = fmaf(wv[q].y, h4.y, x);
-            x = fmaf(wv[q].z, h4.z, x);
-            acc[b * 4 + q] = fmaf(wv[q].w, h4.w, x);
+        for (int rr = 0; rr < RPL; ++rr) {
+          float hval = 0.f;
+          if (s < olen[h][rr]) {
+            const float ig = sigm_cl(acc[rr * 4] + zc[rr * 4]);
+            const float fg = sigm_cl(acc[rr * 4 + 1] + zc[rr * 4 + 1]);
+            const float gg = tanh_cl(acc[rr * 4 + 2] + zc[rr * 4 + 2]);
+            const float og = sigm_cl(acc[rr * 4 + 3] + zc[rr * 4 + 3]);
+            cst[h][rr] = fmaf(fg, cst[h][rr], ig * gg);
+            hval = og * tanh_cl(cst[h][rr]);
+            const size_t tk = (size_t)tok_at(h, rr, s);
+            float *zr = Z + tk * G + gu;
+            zr[0] = ig;
+            zr[H] = fg;
+            zr[2 * H] = gg;
+            zr[3 * H] = og;
+            Cs[tk * H + gu] = cst[h][rr];
+            Y[tk * DH + d * H + gu] = hval;
+          }
+          sg[own_row(rr) * Hc + u] = hval;
+        }
+      } else {
+        const int pr = kl & 1;  // pr 0: (i, f), pr 1: (g, o)
+        const float a0 = pr ? tanh_cl(acc[0] + zc[0]) : sigm_cl(acc[0] + zc[0]);
+        const float a1 = sigm_cl(acc[1] + zc[1]);
+        const float x0 = __shfl_xor_sync(0xffffffffu, a0, 1), x1 = __shfl_xor_sync(0xffffffffu, a1, 1);
+        const float ig = pr ? x0 : a0, fg = pr ? x1 : a1, gg = pr ? a0 : x0, og = pr ? a1 : x1;
+        float hval = 0.f;
+        if (s < olen[h][0]) {
+          cst[h][0] = fmaf(fg, cst[h][0], ig * gg);
+          hval = og * tanh_cl(cst[h][0]);
+          const size_t tk = (size_t)tok_at(h, 0, s);
+          Z[tk * G + (2 * pr) * H + gu] = a0;
+          Z[tk * G + (2 * pr + 1) * H + gu] = a1;
+          if (pr) {
+            Cs[tk * H + gu] = cst[h][0];
+            Y[tk * DH + d * H + gu] = hval;
           }
         }
+        if (!pr) sg[own_row(0) * Hc + u] = hval;
       }
-    }
-    reduce_scatter_lanes<NV, KS>(acc, lane);
-    float *sg = stg + (s & 1) * BC * Hc;
-    if constexpr (NPL >= 4) {
-#pragma unroll
-      for (int rr = 0; rr < RPL; ++rr) {
-        const int b = own_row(rr);
-        float h = 0.f;
-        if (s < olen[rr]) {
-          const float ig = sigm_cl(acc[rr * 4] + zc[rr * 4]);
-          const float fg = sigm_cl(acc[rr * 4 + 1] + zc[rr * 4 + 1]);
-          const float gg = tanhf(acc[rr * 4 + 2] + zc[rr * 4 + 2]);
-          const float og = sigm_cl(acc[rr * 4 + 3] + zc[rr * 4 + 3]);
-          cst[rr] = fmaf(fg, cst[rr], ig * gg);
-          h = og * tanhf(cst[rr]);
-          const size_t tk = (size_t)tok_at(rr, s);
-          float *zr = Z + tk * G + gu;
-          zr[0] = ig;
-          zr[H] = fg;
-          zr[2 * H] = gg;
-          zr[3 * H] = og;
-          Cs[tk * H + gu] = cst[rr];
-          Y[tk * DH + d * H + gu] = h;
+      if (__syncthreads_or(!ok)) {
+        if (t == 0) atomicOr(a.status, kErrExchange);
+        stop = true;
+        break;
+      }
+      if (s + 1 < Tg) {  // exchange s of half h: this CTA's slice to every CTA of the cluster
+        const uint32_t dst0 = smem_addr(hb + (2 * h + (s & 1)) * BH * HPAD), mbl = smem_addr(&mb[2 * h + (s & 1)]);
+        for (int n = t; n < CS * SEND4; n += NTH) {
+          const int peer = n / SEND4, rem = n % SEND4, b = rem / (Hc / 4), u4 = rem % (Hc / 4);
+          const float4 v = *reinterpret_cast<const float4 *>(sg + b * Hc + 4 * u4);
+          const int k = (int)c * Hc + 4 * u4;
+          const uint32_t dst = dst0 + 4u * (uint32_t)(b * HPAD + k + (k >> 6) * 4);
+          st_async4(peer_addr(dst, peer), v, peer_addr(mbl, peer));
         }
-        sg[b * Hc + u] = h;
-      }
-    } else {
-      const int b = own_row(0), pr = kl & 1;  // pr 0: (i, f), pr 1: (g, o)
-      const float a0 = pr ? tanhf(acc[0] + zc[0]) : sigm_cl(acc[0] + zc[0]);
-      const float a1 = sigm_cl(acc[1] + zc[1]);
-      const float x0 = __shfl_xor_sync(0xffffffffu, a0, 1), x1 = __shfl_xor_sync(0xffffffffu, a1, 1);
-      const float ig = pr ? x0 : a0, fg = pr ? x1 : a1, gg = pr ? a0 : x0, og = pr ? a1 : x1;
-      float h = 0.f;
-      if (s < olen[0]) {
-        cst[0] = fmaf(fg, cst[0], ig * gg);
-        h = og * tanhf(cst[0]);
-        const size_t tk = (size_t)tok_at(0, s);
-        Z[tk * G + (2 * pr) * H + gu] = a0;
-        Z[tk * G + (2 * pr + 1) * H + gu] = a1;
-        if (pr) {
-          Cs[tk * H + gu] = cst[0];
-          Y[tk * DH + d * H + gu] = h;
-        }
-      }
-      if (!pr) sg[b * Hc + u] = h;
-    }
-    if (__syncthreads_or(!ok)) {
-      if (t == 0) atomicOr(a.status, kErrExchange);
-      break;
-    }
-    if (s + 1 < Tg) {  // exchange s: this CTA's h_s slice to every CTA of the cluster
-      const uint32_t dst0 = smem_addr(hb + (s & 1) * BC * HPAD), mbl = smem_addr(&mb[s & 1]);
-      for (int n = t; n < CS * SEND4; n += NTH) {
-        const int peer = n / SEND4, rem = n % SEND4, b = rem / (Hc / 4), u4 = rem % (Hc / 4);
-        const float4 v = *reinterpret_cast<const float4 *>(sg + b * Hc + 4 * u4);
-        const int k = (int)c * Hc + 4 * u4;
-        const uint32_t dst = dst0 + 4u * (uint32_t)(b * HPAD + k + (k >> 6) * 4);
-        st_async4(peer_addr(dst, peer), v, peer_addr(mbl, peer));
       }
     }
   }
   cluster_barrier_all();  // no CTA leaves while a peer may still address its shared memory
 }
 
-template <int H, int CS, int BC>
+template <int H, int CS, int BC, int NH>
 __global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a) {
-  using Gm = ClGeom<H, CS, BC>;
-  constexpr int Hc = Gm::Hc, RSL = Gm::RSL, G = 4 * H, NTH = kClThreads, DZS = Gm::DZS;
-  constexpr int NV = 4 * BC, NPL = NV / RSL;  // partials per thread, per lane after the reduction
+  using Gm = ClGeom<H, CS, BC, NH>;
+  constexpr int Hc = Gm::Hc, RSL = Gm::RSL, BH = Gm::BH, G = 4 * H, NTH = kClThreads, DZS = Gm::DZS;
+  constexpr int NV = 4 * BH, NPL = NV / RSL;  // partials per thread, per lane after the reduction
   static_assert(NPL % 4 == 0, "a lane finishes whole float4 column groups");
-  constexpr int PAIRS = Hc * BC, PPT = (PAIRS + NTH - 1) / NTH;
+  constexpr int PAIRS = Hc * BH, PPT = Gm::PPT;  // (unit, row) pairs of a half
   extern __shared__ __align__(16) float sm[];
   float4 *Wb4 = reinterpret_cast<float4 *>(sm);  // [32][NTH] rows 32..63 of each row slice
-  float *dzs = sm + 32 * NTH * 4;                // [2][DZS] dz of this CTA's gate rows
-  float *red = dzs + 2 * DZS;                    // [2][CS][BC][Hc] received partials of W_hh^T dz
-  uint64_t *mb = reinterpret_cast<uint64_t *>(red + 2 * CS * BC * Hc);
-  int *toff_s = reinterpret_cast<int *>(mb + 2);
+  float *dzs = sm + 32 * NTH * 4;                // [NH][2][DZS] dz of this CTA's gate rows
+  float *red = dzs + 2 * NH * DZS;               // [NH][2][CS][BH][Hc] received partials of W_hh^T dz
+  float *ring = red + 2 * NH * CS * BH * Hc;     // [NH][2][NTH][PPT][8] phase B inputs of this and the next step
+  uint64_t *mb = reinterpret_cast<uint64_t *>(ring + 2 * NH * NTH * PPT * 8);  // [NH][2]
+  int *toff_s = reinterpret_cast<int *>(mb + 2 * NH);
   const int T = a.ix.T;
   const bool toff_sm = T + 1 <= kClTokCap;
   const int *toff = toff_sm ? toff_s : a.ix.tok_off;
@@ -358,7 +387,7 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a) {
   const int d = cid / n_groups, grp = cid % n_groups, r0 = grp * BC;
   const int DH = a.dirs * H;
   const float *__restrict__ Whh = a.Whh[d];
-  auto dz_at = [&](int r, int b) { return r * BC + (r >> 6) * 4 + b; };
+  auto dz_at = [&](int r, int b) { return r * BH + (r >> 6) * 4 + b; };
 
   // local gate row r = q * Hc + uu is global row q * H + c * Hc + uu
   float wr[32][4];
@@ -378,159 +407,178 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a) {
   }
   if (toff_sm)
     for (int i = t; i <= T; i += NTH) toff_s[i] = a.ix.tok_off[i];
-  int len[BC];
-#pragma unroll
-  for (int b = 0; b < BC; ++b) len[b] = (r0 + b < a.ix.b) ? a.ix.row_len[r0 + b] : 0;
-  const int Tg = len[0];
+  const int Tg = (r0 < a.ix.b) ? a.ix.row_len[r0] : 0;
   if (t == 0) {
-    mbar_init1(smem_addr(&mb[0]));
-    mbar_init1(smem_addr(&mb[1]));
+    for (int i = 0; i < 2 * NH; ++i) mbar_init1(smem_addr(&mb[i]));
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   cluster_barrier_all();
-  if (t == 0) {
-    if (Tg >= 2) mbar_arm(smem_addr(&mb[0]), Gm::kXBytes);
-    if (Tg >= 3) mbar_arm(smem_addr(&mb[1]), Gm::kXBytes);
-  }
+  if (t == 0)
+    for (int h = 0; h < NH; ++h) {
+      if (Tg >= 2) mbar_arm(smem_addr(&mb[2 * h]), Gm::kXBytes);
+      if (Tg >= 3) mbar_arm(smem_addr(&mb[2 * h + 1]), Gm::kXBytes);
+    }
 
   float *__restrict__ Z = a.Z[d];
   const float *__restrict__ Cs = a.Cst[d];
   const float *__restrict__ dY = a.dY;
-  // phase B pairs (unit, row): pair index i -> unit i % Hc, row i / Hc
-  int plen[PPT];  // row lengths of the pairs (0 for pairs past the end)
+  // phase B pairs of half h: pair index i -> unit i % Hc, row h*BH + i / Hc
+  int plen[NH][PPT];  // row lengths of the pairs (0 for pairs past the end)
 #pragma unroll
-  for (int p = 0; p < PPT; ++p) {
-    const int i = t + p * NTH, r = r0 + i / Hc;
-    plen[p] = (i < PAIRS && r < a.ix.b) ? a.ix.row_len[r] : 0;
-  }
-  auto tok_at = [&](int p, int s) {
-    const int tt = d == 0 ? s : plen[p] - 1 - s;
-    return toff[tt] + r0 + (t + p * NTH) / Hc;
-  };
-  float gn[PPT][4], cn[PPT], cpn[PPT], dyn[PPT], dc[PPT];
-  auto fetch = [&](int p, int s) {
-    const int i = t + p * NTH;
-    const int gu = (int)c * Hc + i % Hc;
-    if (i < PAIRS && s >= 0 && s < plen[p]) {
-      const size_t tk = (size_t)tok_at(p, s);
-#pragma unroll
-      for (int q = 0; q < 4; ++q) gn[p][q] = Z[tk * G + q * H + gu];
-      cn[p] = Cs[tk * H + gu];
-      cpn[p] = s > 0 ? Cs[(size_t)tok_at(p, s - 1) * H + gu] : 0.f;
-      dyn[p] = dY[tk * DH + d * H + gu];
-    }
-  };
-#pragma unroll
-  for (int p = 0; p < PPT; ++p) {
-    dc[p] = 0.f;
-    fetch(p, Tg - 1);
-  }
-  bool ok = true;
-
-  for (int it = 0; it < Tg; ++it) {
-    const int s = Tg - 1 - it;
-    if (it > 0) {
-      const int e = it - 1;
-      ok = mbar_wait_bounded(smem_addr(&mb[e & 1]), (e >> 1) & 1) && ok;
-      if (t == 0 && e + 2 <= Tg - 2) mbar_arm(smem_addr(&mb[e & 1]), Gm::kXBytes);
-    }
-    float *dzb = dzs + (it & 1) * DZS;
-    // phase B
+  for (int h = 0; h < NH; ++h)
 #pragma unroll
     for (int p = 0; p < PPT; ++p) {
-      const int i = t + p * NTH;
-      if (i >= PAIRS) continue;
-      const int uu = i % Hc, b = i / Hc, gu = (int)c * Hc + uu;
-      const float ig = gn[p][0], fg = gn[p][1], gg = gn[p][2], og = gn[p][3];
-      const float ct = cn[p], cp = cpn[p], dy = dyn[p];
-      fetch(p, s - 1);  // a row that starts later still needs its first step fetched
-      if (s < plen[p]) {
-        float dh_rec = 0.f;
-        if (s + 1 < plen[p]) {
-          const float *rp = red + (size_t)((it - 1) & 1) * CS * BC * Hc + b * Hc + uu;
+      const int i = t + p * NTH, r = r0 + h * BH + i / Hc;
+      plen[h][p] = (i < PAIRS && r < a.ix.b) ? a.ix.row_len[r] : 0;
+    }
+  auto tok_at = [&](int h, int p, int s) {
+    const int tt = d == 0 ? s : plen[h][p] - 1 - s;
+    return toff[tt] + r0 + h * BH + (t + p * NTH) / Hc;
+  };
+  // phase B inputs of step s (gates, c_t, c_{t-1}, dY) into ring slot s & 1
+  auto slot_of = [&](int h, int p, int s) { return ring + (((size_t)(2 * h + (s & 1)) * NTH + t) * PPT + p) * 8; };
+  auto issue = [&](int h, int p, int s) {
+    const int i = t + p * NTH;
+    const int gu = (int)c * Hc + i % Hc;
+    if (i < PAIRS && s >= 0 && s < plen[h][p]) {
+      float *sl = slot_of(h, p, s);
+      const size_t tk = (size_t)tok_at(h, p, s);
 #pragma unroll
-          for (int cc = 0; cc < CS; ++cc) dh_rec += rp[cc * BC * Hc];
+      for (int q = 0; q < 4; ++q) cp_async4_cl(sl + q, Z + tk * G + q * H + gu);
+      cp_async4_cl(sl + 4, Cs + tk * H + gu);
+      if (s > 0) cp_async4_cl(sl + 5, Cs + (size_t)tok_at(h, p, s - 1) * H + gu);
+      else sl[5] = 0.f;
+      cp_async4_cl(sl + 6, dY + tk * DH + d * H + gu);
+    }
+  };
+  float dc[NH][PPT];
+#pragma unroll
+  for (int h = 0; h < NH; ++h)
+#pragma unroll
+    for (int p = 0; p < PPT; ++p) {
+      dc[h][p] = 0.f;
+      issue(h, p, Tg - 1);
+    }
+  cp_commit_cl();
+  bool ok = true, stop = false;
+
+  for (int it = 0; it < Tg && !stop; ++it) {
+    const int s = Tg - 1 - it;
+    cp_wait_all_cl();  // this step's inputs, requested one step ago
+#pragma unroll
+    for (int h = 0; h < NH; ++h)
+#pragma unroll
+      for (int p = 0; p < PPT; ++p) issue(h, p, s - 1);  // a row that starts later gets its first step too
+    cp_commit_cl();
+#pragma unroll
+    for (int h = 0; h < NH; ++h) {
+      if (it > 0) {
+        const int e = it - 1;
+        ok = mbar_wait_bounded(smem_addr(&mb[2 * h + (e & 1)]), (e >> 1) & 1) && ok;
+        if (t == 0 && e + 2 <= Tg - 2) mbar_arm(smem_addr(&mb[2 * h + (e & 1)]), Gm::kXBytes);
+      }
+      float *dzb = dzs + (2 * h + (it & 1)) * DZS;
+      // phase B
+#pragma unroll
+      for (int p = 0; p < PPT; ++p) {
+        const int i = t + p * NTH;
+        if (i >= PAIRS) continue;
+        const int uu = i % Hc, b = i / Hc, gu = (int)c * Hc + uu;
+        if (s < plen[h][p]) {
+          const float4 g4 = *reinterpret_cast<const float4 *>(slot_of(h, p, s));
+          const float4 x4 = *reinterpret_cast<const float4 *>(slot_of(h, p, s) + 4);
+          const float ig = g4.x, fg = g4.y, gg = g4.z, og = g4.w;
+          const float ct = x4.x, cp = x4.y, dy = x4.z;
+          float dh_rec = 0.f;
+          if (s + 1 < plen[h][p]) {
+            const float *rp = red + (size_t)(2 * h + ((it - 1) & 1)) * CS * BH * Hc + b * Hc + uu;
+#pragma unroll
+            for (int cc = 0; cc < CS; ++cc) dh_rec += rp[cc * BH * Hc];
+          }
+          const float dh = dy + dh_rec;
+          const float tch = tanh_cl(ct);
+          const float dcv = fmaf(dh * og, 1.f - tch * tch, dc[h][p]);
+          const float dzi = dcv * gg * ig * (1.f - ig);
+          const float dzf = dcv * cp * fg * (1.f - fg);
+          const float dzg = dcv * ig * (1.f - gg * gg);
+          const float dzo = dh * tch * og * (1.f - og);
+          dc[h][p] = dcv * fg;
+          const size_t tk = (size_t)tok_at(h, p, s);
+          float *zr = Z + tk * G + gu;
+          zr[0] = dzi;
+          zr[H] = dzf;
+          zr[2 * H] = dzg;
+          zr[3 * H] = dzo;
+          dzb[dz_at(uu, b)] = dzi;
+          dzb[dz_at(Hc + uu, b)] = dzf;
+          dzb[dz_at(2 * Hc + uu, b)] = dzg;
+          dzb[dz_at(3 * Hc + uu, b)] = dzo;
+        } else {
+#pragma unroll
+          for (int q = 0; q < 4; ++q) dzb[dz_at(q * Hc + uu, b)] = 0.f;
         }
-        const float dh = dy + dh_rec;
-        const float tch = tanhf(ct);
-        const float dcv = fmaf(dh * og, 1.f - tch * tch, dc[p]);
-        const float dzi = dcv * gg * ig * (1.f - ig);
-        const float dzf = dcv * cp * fg * (1.f - fg);
-        const float dzg = dcv * ig * (1.f - gg * gg);
-        const float dzo = dh * tch * og * (1.f - og);
-        dc[p] = dcv * fg;
-        const size_t tk = (size_t)tok_at(p, s);
-        float *zr = Z + tk * G + gu;
-        zr[0] = dzi;
-        zr[H] = dzf;
-        zr[2 * H] = dzg;
-        zr[3 * H] = dzo;
-        dzb[dz_at(uu, b)] = dzi;
-        dzb[dz_at(Hc + uu, b)] = dzf;
-        dzb[dz_at(2 * Hc + uu, b)] = dzg;
-        dzb[dz_at(3 * Hc + uu, b)] = dzo;
-      } else {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) dzb[dz_at(q * Hc + uu, b)] = 0.f;
       }
-    }
-    if (__syncthreads_or(!ok)) {
-      if (t == 0) atomicOr(a.status, kErrExchange);
-      break;
-    }
-    if (it + 1 >= Tg) break;  // dh_{-1} is not needed
-    // phase A: partial W_hh^T dz over this thread's 64 rows, columns k0..k0+3
-    float acc[NV];
-#pragma unroll
-    for (int i = 0; i < NV; ++i) acc[i] = 0.f;
-#pragma unroll
-    for (int j = 0; j < 64; ++j) {
-      const int r = rs * 64 + j;
-      float wv[4];
-      if (j < 32) {
-#pragma unroll
-        for (int cc = 0; cc < 4; ++cc) wv[cc] = wr[j][cc];
-      } else {
-        const float4 v = Wb4[(j - 32) * NTH + t];
-        wv[0] = v.x;
-        wv[1] = v.y;
-        wv[2] = v.z;
-        wv[3] = v.w;
+      if (__syncthreads_or(!ok)) {
+        if (t == 0) atomicOr(a.status, kErrExchange);
+        stop = true;
+        break;
       }
+      if (it + 1 >= Tg) continue;  // dh_{-1} is not needed
+      // phase A: partial W_hh^T dz over this thread's 64 rows, columns k0..k0+3
+      float acc[NV];
 #pragma unroll
-      for (int m = 0; m < BC / 4; ++m) {
-        const float4 z4 = *reinterpret_cast<const float4 *>(dzb + dz_at(r, 4 * m));
-        const float zz[4] = {z4.x, z4.y, z4.z, z4.w};
+      for (int i = 0; i < NV; ++i) acc[i] = 0.f;
 #pragma unroll
-        for (int bb = 0; bb < 4; ++bb)
+      for (int j = 0; j < 64; ++j) {
+        const int r = rs * 64 + j;
+        float wv[4];
+        if (j < 32) {
 #pragma unroll
-          for (int cc = 0; cc < 4; ++cc)
-            acc[(4 * m + bb) * 4 + cc] = fmaf(wv[cc], zz[bb], acc[(4 * m + bb) * 4 + cc]);
+          for (int cc = 0; cc < 4; ++cc) wv[cc] = wr[j][cc];
+        } else {
+          const float4 v = Wb4[(j - 32) * NTH + t];
+          wv[0] = v.x;
+          wv[1] = v.y;
+          wv[2] = v.z;
+          wv[3] = v.w;
+        }
+#pragma unroll
+        for (int m = 0; m < BH / 4; ++m) {
+          const float4 z4 = *reinterpret_cast<const float4 *>(dzb + dz_at(r, 4 * m));
+          const float zz[4] = {z4.x, z4.y, z4.z, z4.w};
+#pragma unroll
+          for (int bb = 0; bb < 4; ++bb)
+#pragma unroll
+            for (int cc = 0; cc < 4; ++cc)
+              acc[(4 * m + bb) * 4 + cc] = fmaf(wv[cc], zz[bb], acc[(4 * m + bb) * 4 + cc]);
+        }
       }
-    }
-    reduce_scatter_lanes<NV, RSL>(acc, lane);
-    // lane holds rows rs*(NPL/4) .. + NPL/4 - 1, columns k0..k0+3 -> the owner of those units
-    const uint32_t owner = (uint32_t)(k0 / Hc);
-    const int uo = k0 % Hc;
-    const uint32_t dst0 = smem_addr(red + (size_t)(it & 1) * CS * BC * Hc + (size_t)c * BC * Hc + uo);
-    const uint32_t rmb = peer_addr(smem_addr(&mb[it & 1]), owner);
+      reduce_scatter_lanes<NV, RSL>(acc, lane);
+      // lane holds rows rs*(NPL/4) .. + NPL/4 - 1 of the half, columns k0..k0+3 -> the owner of those units
+      const uint32_t owner = (uint32_t)(k0 / Hc);
+      const int uo = k0 % Hc;
+      const uint32_t dst0 =
+          smem_addr(red + (size_t)(2 * h + (it & 1)) * CS * BH * Hc + (size_t)c * BH * Hc + uo);
+      const uint32_t rmb = peer_addr(smem_addr(&mb[2 * h + (it & 1)]), owner);
 #pragma unroll
-    for (int rr = 0; rr < NPL / 4; ++rr) {
-      const int b = rs * (NPL / 4) + rr;
-      st_async4(peer_addr(dst0 + 4u * (uint32_t)(b * Hc), owner),
-                make_float4(acc[rr * 4], acc[rr * 4 + 1], acc[rr * 4 + 2], acc[rr * 4 + 3]), rmb);
+      for (int rr = 0; rr < NPL / 4; ++rr) {
+        const int b = rs * (NPL / 4) + rr;
+        st_async4(peer_addr(dst0 + 4u * (uint32_t)(b * Hc), owner),
+                  make_float4(acc[rr * 4], acc[rr * 4 + 1], acc[rr * 4 + 2], acc[rr * 4 + 3]), rmb);
+      }
     }
   }
+  cp_wait_all_cl();
   cluster_barrier_all();
 }
 
 // ---------------------------------------------------------------------------
 namespace {
 
-template <int H, int CS, int BC>
+template <int H, int CS, int BC, int NH>
 size_t cl_smem(bool bwd, int T) {
-  using Gm = ClGeom<H, CS, BC>;
-  return (bwd ? Gm::bwd_floats() : Gm::fwd_floats()) * 4 + cl_tail_bytes(T);
+  using Gm = ClGeom<H, CS, BC, NH>;
+  return (bwd ? Gm::bwd_floats() : Gm::fwd_floats()) * 4 + cl_tail_bytes(NH, T);
 }
 
 template <typename K>
@@ -557,20 +605,20 @@ cudaLaunchConfig_t cl_config(K, int cs, int clusters, size_t smem, cudaStream_t 
   return cfg;
 }
 
-template <int H, int CS, int BC>
+template <int H, int CS, int BC, int NH>
 cudaError_t launch_cl(const RecArgs &a, bool bwd, cudaStream_t s) {
   if (a.ix.b <= 0 || a.ix.T <= 0) return cudaSuccess;
-  const size_t smem = cl_smem<H, CS, BC>(bwd, a.ix.T);
+  const size_t smem = cl_smem<H, CS, BC, NH>(bwd, a.ix.T);
   const int clusters = ((a.ix.b + BC - 1) / BC) * a.dirs;
   cudaLaunchAttribute attr;
   if (bwd) {
-    auto k = lstm_bwd_cl_kernel<H, CS, BC>;
+    auto k = lstm_bwd_cl_kernel<H, CS, BC, NH>;
     cudaError_t e = cl_prepare(k, CS, smem);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = cl_config(k, CS, clusters, smem, s, &attr);
     return cudaLaunchKernelEx(&cfg, k, a);
   }
-  auto k = lstm_fwd_cl_kernel<H, CS, BC>;
+  auto k = lstm_fwd_cl_kernel<H, CS, BC, NH>;
   cudaError_t e = cl_prepare(k, CS, smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = cl_config(k, CS, clusters, smem, s, &attr);
@@ -579,21 +627,21 @@ cudaError_t launch_cl(const RecArgs &a, bool bwd, cudaStream_t s) {
 
 // Clusters of the forward and the BPTT kernel that can be resident at once
 // (0: the configuration cannot launch on this device).
-template <int H, int CS, int BC>
+template <int H, int CS, int BC, int NH>
 int cl_resident(int T) {
   int lo = 1 << 30;
   for (int bwd = 0; bwd < 2; ++bwd) {
-    const size_t smem = cl_smem<H, CS, BC>(bwd != 0, T);
+    const size_t smem = cl_smem<H, CS, BC, NH>(bwd != 0, T);
     cudaLaunchAttribute attr;
     int n = 0;
     cudaError_t e;
     if (bwd) {
-      auto k = lstm_bwd_cl_kernel<H, CS, BC>;
+      auto k = lstm_bwd_cl_kernel<H, CS, BC, NH>;
       e = cl_prepare(k, CS, smem);
       cudaLaunchConfig_t cfg = cl_config(k, CS, 1, smem, 0, &attr);
       if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, k, &cfg);
     } else {
-      auto k = lstm_fwd_cl_kernel<H, CS, BC>;
+      auto k = lstm_fwd_cl_kernel<H, CS, BC, NH>;
       e = cl_prepare(k, CS, smem);
       cudaLaunchConfig_t cfg = cl_config(k, CS, 1, smem, 0, &attr);
       if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, k, &cfg);
@@ -617,11 +665,11 @@ int plan_cl_rows(int H, int b, int dirs) {
   const int T = kClTokCap - 1;
   int r4 = 0, r8 = 0;
   if (H == 256) {
-    r4 = cl_resident<256, 4, 4>(T);
-    r8 = cl_resident<256, 4, 8>(T);
+    r4 = cl_resident<256, 4, 4, 1>(T);
+    r8 = cl_resident<256, 4, 8, 1>(T);
   } else if (H == 512) {
-    r4 = cl_resident<512, 16, 4>(T);
-    r8 = cl_resident<512, 16, 8>(T);
+    r4 = cl_resident<512, 16, 4, 1>(T);
+    r8 = cl_resident<512, 16, 8, 1>(T);
   }
   if (r4 > 0 && ((b + 3) / 4) * dirs <= r4) return 4;
   if (r8 > 0) return 8;
@@ -629,8 +677,8 @@ int plan_cl_rows(int H, int b, int dirs) {
 }
 
 cudaError_t launch_lstm_cl(const RecArgs &a, int bc, bool bwd, cudaStream_t s) {
-  if (a.H == 256) return bc == 4 ? launch_cl<256, 4, 4>(a, bwd, s) : launch_cl<256, 4, 8>(a, bwd, s);
-  if (a.H == 512) return bc == 4 ? launch_cl<512, 16, 4>(a, bwd, s) : launch_cl<512, 16, 8>(a, bwd, s);
+  if (a.H == 256) return bc == 4 ? launch_cl<256, 4, 4, 1>(a, bwd, s) : launch_cl<256, 4, 8, 1>(a, bwd, s);
+  if (a.H == 512) return bc == 4 ? launch_cl<512, 16, 4, 1>(a, bwd, s) : launch_cl<512, 16, 8, 1>(a, bwd, s);
   return cudaErrorInvalidValue;
 }
 
