@@ -372,7 +372,7 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a) {
   float4 *Wb4 = reinterpret_cast<float4 *>(sm);  // [32][NTH] rows 32..63 of each row slice
   float *dzs = sm + 32 * NTH * 4;                // [NH][2][DZS] dz of this CTA's gate rows
   float *red = dzs + 2 * NH * DZS;               // [NH][2][CS][BH][Hc] received partials of W_hh^T dz
-  float *ring = red + 2 * NH * CS * BH * Hc;     // [NH][2][NTH][PPT][8] phase B inputs of this and the next step
+  float *ring = red + 2 * NH * CS * BH * Hc;     // [NH][2][PPT][8][NTH] phase B inputs of this and the next step
   uint64_t *mb = reinterpret_cast<uint64_t *>(ring + 2 * NH * NTH * PPT * 8);  // [NH][2]
   int *toff_s = reinterpret_cast<int *>(mb + 2 * NH);
   const int T = a.ix.T;
@@ -435,8 +435,10 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a) {
     const int tt = d == 0 ? s : plen[h][p] - 1 - s;
     return toff[tt] + r0 + h * BH + (t + p * NTH) / Hc;
   };
-  // phase B inputs of step s (gates, c_t, c_{t-1}, dY) into ring slot s & 1
-  auto slot_of = [&](int h, int p, int s) { return ring + (((size_t)(2 * h + (s & 1)) * NTH + t) * PPT + p) * 8; };
+  // phase B inputs of step s (gates, c_t, c_{t-1}, dY) into ring slot s & 1;
+  // value v of a thread sits at slot + v * NTH, so a warp's copies and reads
+  // touch consecutive words (no bank conflicts)
+  auto slot_of = [&](int h, int p, int s) { return ring + ((size_t)(2 * h + (s & 1)) * PPT + p) * 8 * NTH + t; };
   auto issue = [&](int h, int p, int s) {
     const int i = t + p * NTH;
     const int gu = (int)c * Hc + i % Hc;
@@ -444,11 +446,11 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a) {
       float *sl = slot_of(h, p, s);
       const size_t tk = (size_t)tok_at(h, p, s);
 #pragma unroll
-      for (int q = 0; q < 4; ++q) cp_async4_cl(sl + q, Z + tk * G + q * H + gu);
-      cp_async4_cl(sl + 4, Cs + tk * H + gu);
-      if (s > 0) cp_async4_cl(sl + 5, Cs + (size_t)tok_at(h, p, s - 1) * H + gu);
-      else sl[5] = 0.f;
-      cp_async4_cl(sl + 6, dY + tk * DH + d * H + gu);
+      for (int q = 0; q < 4; ++q) cp_async4_cl(sl + q * NTH, Z + tk * G + q * H + gu);
+      cp_async4_cl(sl + 4 * NTH, Cs + tk * H + gu);
+      if (s > 0) cp_async4_cl(sl + 5 * NTH, Cs + (size_t)tok_at(h, p, s - 1) * H + gu);
+      else sl[5 * NTH] = 0.f;
+      cp_async4_cl(sl + 6 * NTH, dY + tk * DH + d * H + gu);
     }
   };
   float dc[NH][PPT];
@@ -485,10 +487,9 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a) {
         if (i >= PAIRS) continue;
         const int uu = i % Hc, b = i / Hc, gu = (int)c * Hc + uu;
         if (s < plen[h][p]) {
-          const float4 g4 = *reinterpret_cast<const float4 *>(slot_of(h, p, s));
-          const float4 x4 = *reinterpret_cast<const float4 *>(slot_of(h, p, s) + 4);
-          const float ig = g4.x, fg = g4.y, gg = g4.z, og = g4.w;
-          const float ct = x4.x, cp = x4.y, dy = x4.z;
+          const float *sl = slot_of(h, p, s);
+          const float ig = sl[0], fg = sl[NTH], gg = sl[2 * NTH], og = sl[3 * NTH];
+          const float ct = sl[4 * NTH], cp = sl[5 * NTH], dy = sl[6 * NTH];
           float dh_rec = 0.f;
           if (s + 1 < plen[h][p]) {
             const float *rp = red + (size_t)(2 * h + ((it - 1) & 1)) * CS * BH * Hc + b * Hc + uu;
@@ -525,6 +526,8 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a) {
       }
       if (it + 1 >= Tg) continue;  // dh_{-1} is not needed
       // phase A: partial W_hh^T dz over this thread's 64 rows, columns k0..k0+3
+      // (a [batch row][gate row] dz layout made phase B cheaper but this loop
+      // slower, a net loss)
       float acc[NV];
 #pragma unroll
       for (int i = 0; i < NV; ++i) acc[i] = 0.f;

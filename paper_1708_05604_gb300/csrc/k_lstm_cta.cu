@@ -110,7 +110,7 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
   extern __shared__ __align__(16) float sm[];
   float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [SKK/4][16][NTH]
   float *hs = sm + SKK * 16 * NTH;               // [2][BC][8 slices][HS]
-  float *zr = hs + 2 * BC * 8 * HS;              // [BC][kRing][NTH][2] Zx of upcoming steps
+  float *zr = hs + 2 * BC * 8 * HS;              // [BC][kRing][2][NTH] Zx of upcoming steps (value-major: no bank conflicts)
   const int T = a.ix.T;
   const bool toff_sm = T + 1 <= kTokCap;
   int *toff_s = reinterpret_cast<int *>(zr + BC * kRing * NTH * 2);
@@ -160,9 +160,9 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
   auto issue = [&](int b, int s) {  // Zx of step s of row b into its ring slot
     if (s < len[b]) {
       const int tk = tok_at(b, s);
-      float *slot = zr + (((size_t)b * kRing + s % kRing) * NTH + t) * 2;
+      float *slot = zr + ((size_t)b * kRing + s % kRing) * 2 * NTH + t;
       cp_async4(slot, Z + (size_t)tk * G + zo0);
-      cp_async4(slot + 1, Z + (size_t)tk * G + zo1);
+      cp_async4(slot + NTH, Z + (size_t)tk * G + zo1);
     }
   };
 #pragma unroll
@@ -178,8 +178,8 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
 #pragma unroll
     for (int b = 0; b < BC; ++b) {
       if (s >= len[b]) continue;  // uniform over the CTA
-      const float *slot = zr + (((size_t)b * kRing + s % kRing) * NTH + t) * 2;
-      const float zc0 = slot[0], zc1 = slot[1];
+      const float *slot = zr + ((size_t)b * kRing + s % kRing) * 2 * NTH + t;
+      const float zc0 = slot[0], zc1 = slot[NTH];
       const int tc = tok_at(b, s);
       issue(b, s + kPF);
       const float *hv = hs + (p * BC + b) * 8 * HS + ks * HS;
@@ -241,7 +241,7 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
   float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [SKK/4][16][NTH]
   float *dzs = sm + SKK * 16 * NTH;              // [BC][H][4] unit-major dz
   float *red = dzs + BC * G;                     // [BC][NW][H] per-warp column partials
-  float *ring = red + BC * NW * H;               // [BC][kRing][NTH][8] inputs of upcoming steps
+  float *ring = red + BC * NW * H;               // [BC][kRing][8][NTH] inputs of upcoming steps (value-major)
   const int T = a.ix.T;
   const bool toff_sm = T + 1 <= kTokCap;
   int *toff_s = reinterpret_cast<int *>(ring + BC * kRing * NTH * 8);
@@ -288,13 +288,13 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
   auto issue = [&](int b, int s) {
     if (s >= 0 && s < len[b]) {
       const int tk = tok_at(b, s);
-      float *slot = ring + (((size_t)b * kRing + s % kRing) * NTH + t) * 8;
+      float *slot = ring + ((size_t)b * kRing + s % kRing) * 8 * NTH + t;
 #pragma unroll
-      for (int g = 0; g < 4; ++g) cp_async4(slot + g, Z + (size_t)tk * G + g * H + unit);
-      cp_async4(slot + 4, Cs + (size_t)tk * H + unit);
-      if (s > 0) cp_async4(slot + 5, Cs + (size_t)tok_at(b, s - 1) * H + unit);
-      else slot[5] = 0.f;
-      cp_async4(slot + 6, dY + (size_t)tk * DH + d * H + unit);
+      for (int g = 0; g < 4; ++g) cp_async4(slot + g * NTH, Z + (size_t)tk * G + g * H + unit);
+      cp_async4(slot + 4 * NTH, Cs + (size_t)tk * H + unit);
+      if (s > 0) cp_async4(slot + 5 * NTH, Cs + (size_t)tok_at(b, s - 1) * H + unit);
+      else slot[5 * NTH] = 0.f;
+      cp_async4(slot + 6 * NTH, dY + (size_t)tk * DH + d * H + unit);
     }
   };
 #pragma unroll
@@ -316,10 +316,10 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
 #pragma unroll
         for (int wi = 0; wi < NW; ++wi) dh_rec += rp[wi * H];
       }
-      const float *slot = ring + (((size_t)b * kRing + s % kRing) * NTH + t) * 8;
-      const float ig = slot[0], fg = slot[1], gg = slot[2], og = slot[3];
-      const float ct = slot[4], cp = slot[5];
-      const float dh = slot[6] + dh_rec;
+      const float *slot = ring + ((size_t)b * kRing + s % kRing) * 8 * NTH + t;
+      const float ig = slot[0], fg = slot[NTH], gg = slot[2 * NTH], og = slot[3 * NTH];
+      const float ct = slot[4 * NTH], cp = slot[5 * NTH];
+      const float dh = slot[6 * NTH] + dh_rec;
       const int tk = tok_at(b, s);
       issue(b, s - kPF);
       const float tch = tanhf(ct);
