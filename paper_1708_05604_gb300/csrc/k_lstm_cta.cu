@@ -45,7 +45,11 @@ constexpr int kTokCap = 8192;  // time offsets staged in shared memory up to thi
 constexpr int kPF = 4;         // steps of per-step global inputs kept in flight
 constexpr int kRing = kPF + 1; // ring slots: a copy never lands in the slot read this step
 
-__device__ __forceinline__ float sigm(float x) { return 1.f / (1.f + expf(-x)); }
+// Gate nonlinearities from the exponential intrinsic: sigma(x) = 1 / (1 + e^-x)
+// and tanh(x) = 1 - 2 / (1 + e^2x) (absolute error a few 1e-8; both saturate
+// correctly when the exponential overflows to +inf or underflows to 0).
+__device__ __forceinline__ float sigm(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
+__device__ __forceinline__ float tanh_g(float x) { return 1.f - __fdividef(2.f, 1.f + __expf(2.f * x)); }
 
 // Per-thread asynchronous copies (global -> shared) for the step inputs:
 // one commit group per step, so waiting for all but the newest kPF-1 groups
@@ -212,14 +216,14 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
       float v0, v1;
       reduce_scatter8(acc, lane, v0, v1);
       // lane pair 0 holds (i, f), pair 1 holds (g, o) of `unit`
-      const float a0 = pair ? tanhf(v0 + zc0) : sigm(v0 + zc0);
+      const float a0 = pair ? tanh_g(v0 + zc0) : sigm(v0 + zc0);
       const float a1 = sigm(v1 + zc1);
       Z[(size_t)tc * G + zo0] = a0;
       Z[(size_t)tc * G + zo1] = a1;
       const float x0 = __shfl_xor_sync(0xffffffffu, a0, 1), x1 = __shfl_xor_sync(0xffffffffu, a1, 1);
       const float ig = pair ? x0 : a0, fg = pair ? x1 : a1, gg = pair ? a0 : x0, og = pair ? a1 : x1;
       cst[b] = fmaf(fg, cst[b], ig * gg);
-      const float h = og * tanhf(cst[b]);
+      const float h = og * tanh_g(cst[b]);
       if (pair == 0) {
         hs[((p ^ 1) * BC + b) * 8 * HS + hslot] = h;
       } else {
@@ -322,7 +326,7 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
       const float dh = slot[6 * NTH] + dh_rec;
       const int tk = tok_at(b, s);
       issue(b, s - kPF);
-      const float tch = tanhf(ct);
+      const float tch = tanh_g(ct);
       const float dcv = fmaf(dh * og, 1.f - tch * tch, dc[b]);
       const float dzi = dcv * gg * ig * (1.f - ig);
       const float dzf = dcv * cp * fg * (1.f - fg);
