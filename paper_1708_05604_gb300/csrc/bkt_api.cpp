@@ -481,8 +481,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     L.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, g.splits, M, N, out, s); });
   };
   auto bias_sum = [&](const float *A, int64_t lda, int M, float *out) {
-    int splits = std::min(64, std::max(1, std::min(2 * sm_count / ((M + 255) / 256), NT / 64)));
-    while (splits > 1 && (size_t)splits * M > w.part_floats) --splits;
+    const int splits = bkt::colsum_splits(NT, M, w.part_floats);
     L.run("colsum", [&] { return bkt::launch_colsum(A, lda, NT, M, w.part, splits, s); });
     L.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, splits, 1, M, out, s); });
   };
@@ -566,10 +565,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         } else {
           L.run("transpose_bf16", [&] { return bkt::launch_transpose_bf16(Xl, D, nullptr, NT, D, w.BT, NTp, s); });
           tc_reduce(w.BT, D, grads + lo.w_ih[l * dirs + d]);
-          int splits = std::min(64, std::max(1, std::min(2 * sm_count / ((4 * H + 255) / 256), NT / 64)));
-          while (splits > 1 && (size_t)splits * 4 * H > w.part_floats) --splits;
-          L.run("colsum", [&] { return bkt::launch_colsum(dZ, 4 * H, NT, 4 * H, w.part, splits, s); });
-          L.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, splits, 1, 4 * H, grads + lo.bias(l, d), s); });
+          bias_sum(dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
         }
       }
     } else {

@@ -64,6 +64,10 @@ cudaError_t launch_cast_bf16(const float *src, int64_t lds, int R, int C, void *
 // dst[c][r] = bf16(src[src_row ? src_row[r] : r][c]), zeros where src_row[r] < 0.
 cudaError_t launch_transpose_bf16(const float *src, int64_t lds, const int32_t *src_row, int R, int C, void *dst,
                                   int64_t ldd, cudaStream_t s);
+// P[z][m] = sum of A[r][m] over row chunk z of ceil(R / splits) rows (P
+// holds splits * M floats), then launch_splitk_sum finishes the sums;
+// colsum_splits picks about 256 rows per chunk within part_floats.
+int colsum_splits(int R, int M, size_t part_floats);
 cudaError_t launch_colsum(const float *A, int64_t lda, int R, int M, float *P, int splits, cudaStream_t s);
 // hi[c][r] + lo[c][r] = src[src_row ? src_row[r] : r][c] to 2^-22 relative,
 // hi and lo both tf32 values (zeros where src_row[r] < 0).

@@ -3,7 +3,7 @@
 //   cast_bf16:      fp32 [R x C] -> bf16 [R x C] (row-major, own strides)
 //   transpose_bf16: fp32 [R x C] -> bf16 [C x R] (optionally reading row
 //                   src_row[r] instead of r; a negative index gives zeros)
-//   colsum:         P[z][m] = sum over rows of split z of A[r][m]
+//   colsum:         P[z][m] = sum over the rows of chunk z of A[r][m]
 // The transposes turn token-major activations into the K-contiguous layout
 // the tensor-core GEMM reads, so every contraction over tokens is a plain
 // "A[M x K] B[N x K]^T" product.
@@ -174,22 +174,50 @@ cudaError_t launch_log_softmax_rows(float *x, int64_t ld, int R, int C, cudaStre
   return cudaGetLastError();
 }
 
-__global__ void colsum_kernel(const float *__restrict__ A, int64_t lda, int R, int M, float *__restrict__ P,
-                              int splits) {
-  const int m = blockIdx.x * blockDim.x + threadIdx.x;
-  const int z = blockIdx.y;
-  if (m >= M) return;
-  const int chunk = (R + splits - 1) / splits;
+// P[z][m] = sum of A[r][m] over the rows of chunk z (ceil(R / splits) rows).
+// A block holds 32 columns (coalesced along m); its 8 warps take rows
+// r0 + g, r0 + g + 8, ... with four running sums each, and warp 0 adds the 8
+// group sums in a fixed order.
+__global__ void __launch_bounds__(256) colsum_kernel(const float *__restrict__ A, int64_t lda, int R, int M,
+                                                     float *__restrict__ P, int chunk) {
+  __shared__ float part[8][33];
+  const int tx = threadIdx.x & 31, g = threadIdx.x >> 5;
+  const int m = blockIdx.x * 32 + tx, z = blockIdx.y;
   const int r0 = z * chunk, r1 = min(R, r0 + chunk);
-  float acc = 0.f;
-  for (int r = r0; r < r1; ++r) acc += A[(int64_t)r * lda + m];
-  P[(int64_t)z * M + m] = acc;
+  float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+  if (m < M) {
+    int r = r0 + g;
+    for (; r + 24 < r1; r += 32) {
+      a0 += A[(int64_t)r * lda + m];
+      a1 += A[(int64_t)(r + 8) * lda + m];
+      a2 += A[(int64_t)(r + 16) * lda + m];
+      a3 += A[(int64_t)(r + 24) * lda + m];
+    }
+    if (r < r1) a0 += A[(int64_t)r * lda + m];
+    if (r + 8 < r1) a1 += A[(int64_t)(r + 8) * lda + m];
+    if (r + 16 < r1) a2 += A[(int64_t)(r + 16) * lda + m];
+  }
+  part[g][tx] = (a0 + a1) + (a2 + a3);
+  __syncthreads();
+  if (g == 0 && m < M) {
+    float s = 0.f;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) s += part[k][tx];
+    P[(int64_t)z * M + m] = s;
+  }
+}
+
+int colsum_splits(int R, int M, size_t part_floats) {
+  const size_t cap = M > 0 ? part_floats / (size_t)M : 1;
+  return (int)std::max<size_t>(1, std::min<size_t>(std::min<size_t>((R + 255) / 256, cap), 65535));
 }
 
 cudaError_t launch_colsum(const float *A, int64_t lda, int R, int M, float *P, int splits, cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
-  dim3 grid((M + 255) / 256, splits);
-  colsum_kernel<<<grid, 256, 0, s>>>(A, lda, R, M, P, splits);
+  if (splits < 1 || splits > 65535) return cudaErrorInvalidValue;
+  const int chunk = (R + splits - 1) / splits;
+  dim3 grid((M + 31) / 32, splits);
+  colsum_kernel<<<grid, 256, 0, s>>>(A, lda, R, M, P, chunk);
   return cudaGetLastError();
 }
 

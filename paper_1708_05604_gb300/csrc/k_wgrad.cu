@@ -4,19 +4,45 @@
 // the fixed-order sum of split-K partial tiles, scattered straight into the
 // flat gradient layout.
 #include <algorithm>
+#include <cstdint>
 
 #include "bkt_internal.h"
 
 namespace bkt {
 
-// Sums the split partials in order and scatters column n of row m to
-// out1[m*D1 + n], out2[m*D2 + n - D1] or out3[m] (the ones column).
-__global__ void wgrad_reduce_kernel(const float *__restrict__ P, int splits, int M, int N, int D1, int D2,
-                                    float *__restrict__ out1, float *__restrict__ out2, float *__restrict__ out3) {
+// Sums the split partials P[z][i], i < M*N, in a fixed order and scatters
+// column n of row m to out1[m*D1 + n], out2[m*D2 + n - D1] or out3[m] (the
+// ones column).  A block holds 32 consecutive outputs (coalesced along i);
+// its 8 warps take interleaved groups of splits z = g, g+8, ... with four
+// independent running sums each (so loads overlap instead of waiting on one
+// another), and warp 0 adds the 8 group sums in order: the result depends
+// only on `splits`, never on scheduling.
+__global__ void __launch_bounds__(256) wgrad_reduce_kernel(const float *__restrict__ P, int splits, int M, int N,
+                                                           int D1, int D2, float *__restrict__ out1,
+                                                           float *__restrict__ out2, float *__restrict__ out3) {
+  __shared__ float part[8][33];
   const int64_t total = (int64_t)M * N;
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+  const int tx = threadIdx.x & 31, g = threadIdx.x >> 5;
+  const int64_t i = (int64_t)blockIdx.x * 32 + tx;
+  float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+  if (i < total) {
+    int z = g;
+    for (; z + 24 < splits; z += 32) {
+      a0 += P[(int64_t)z * total + i];
+      a1 += P[(int64_t)(z + 8) * total + i];
+      a2 += P[(int64_t)(z + 16) * total + i];
+      a3 += P[(int64_t)(z + 24) * total + i];
+    }
+    if (z < splits) a0 += P[(int64_t)z * total + i];
+    if (z + 8 < splits) a1 += P[(int64_t)(z + 8) * total + i];
+    if (z + 16 < splits) a2 += P[(int64_t)(z + 16) * total + i];
+  }
+  part[g][tx] = (a0 + a1) + (a2 + a3);
+  __syncthreads();
+  if (g == 0 && i < total) {
     float s = 0.f;
-    for (int z = 0; z < splits; ++z) s += P[(int64_t)z * total + i];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) s += part[k][tx];
     const int m = (int)(i / N), n = (int)(i % N);
     if (n < D1) out1[(int64_t)m * D1 + n] = s;
     else if (n < D1 + D2) out2[(int64_t)m * D2 + (n - D1)] = s;
@@ -24,55 +50,95 @@ __global__ void wgrad_reduce_kernel(const float *__restrict__ P, int splits, int
   }
 }
 
+static cudaError_t launch_reduce(const float *P, int splits, int M, int N, int D1, int D2, float *o1, float *o2,
+                                 float *o3, cudaStream_t s) {
+  const int64_t total = (int64_t)M * N;
+  if (total <= 0) return cudaSuccess;
+  const int64_t blocks = (total + 31) / 32;
+  if (blocks > 0x7fffffff) return cudaErrorInvalidConfiguration;
+  wgrad_reduce_kernel<<<(unsigned)blocks, 256, 0, s>>>(P, splits, M, N, D1, D2, o1, o2, o3);
+  return cudaGetLastError();
+}
+
 // Narrow case G[m][n] = sum_k A[k][m] [X[k] | 1][n] with X of D <= 16
-// columns: one thread per m keeps D+1 sums over its token range (A read
-// coalesced along m, X rows broadcast), partials P[z][m][n] as above.
-template <int D>
-__global__ void narrow_wgrad_kernel(const float *__restrict__ A, int64_t lda, int M, const float *__restrict__ X,
-                                    int K, float *__restrict__ P, int splits) {
-  const int m = blockIdx.x * blockDim.x + threadIdx.x;
+// columns, partials P[z][m][n] over token chunk z.  A bandwidth-bound pass
+// over A: with M and lda multiples of 4 a thread keeps 4 (D+1) sums for four
+// consecutive columns and 16 float4 loads of A in flight (X rows are
+// broadcast across the warp); otherwise one column per thread.
+template <int D, int VEC>
+__global__ void __launch_bounds__(128) narrow_wgrad_kernel(const float *__restrict__ A, int64_t lda, int M,
+                                                           const float *__restrict__ X, int K,
+                                                           float *__restrict__ P, int splits) {
+  constexpr int U = 16;
+  const int m0 = (blockIdx.x * blockDim.x + threadIdx.x) * VEC;
   const int z = blockIdx.y;
-  if (m >= M) return;
+  if (m0 >= M) return;
   const int chunk = (K + splits - 1) / splits;
   const int k0 = z * chunk, k1 = min(K, k0 + chunk);
-  float acc[D + 1];
+  float acc[VEC][D + 1];
 #pragma unroll
-  for (int j = 0; j <= D; ++j) acc[j] = 0.f;
-  // eight independent loads of A in flight per thread
-  int k = k0;
-  for (; k + 8 <= k1; k += 8) {
-    float a[8];
+  for (int c = 0; c < VEC; ++c)
 #pragma unroll
-    for (int u = 0; u < 8; ++u) a[u] = A[(int64_t)(k + u) * lda + m];
-#pragma unroll
-    for (int u = 0; u < 8; ++u) {
-#pragma unroll
-      for (int j = 0; j < D; ++j) acc[j] = fmaf(a[u], __ldg(X + (int64_t)(k + u) * D + j), acc[j]);
-      acc[D] += a[u];
+    for (int j = 0; j <= D; ++j) acc[c][j] = 0.f;
+  auto load = [&](int k, float (&v)[VEC]) {
+    if constexpr (VEC == 4) {
+      const float4 a = __ldg(reinterpret_cast<const float4 *>(A + (int64_t)k * lda + m0));
+      v[0] = a.x;
+      v[1] = a.y;
+      v[2] = a.z;
+      v[3] = a.w;
+    } else {
+      v[0] = __ldg(A + (int64_t)k * lda + m0);
     }
+  };
+  auto add = [&](int k, const float (&v)[VEC]) {
+#pragma unroll
+    for (int j = 0; j < D; ++j) {
+      const float x = __ldg(X + (int64_t)k * D + j);
+#pragma unroll
+      for (int c = 0; c < VEC; ++c) acc[c][j] = fmaf(v[c], x, acc[c][j]);
+    }
+#pragma unroll
+    for (int c = 0; c < VEC; ++c) acc[c][D] += v[c];
+  };
+  int k = k0;
+  for (; k + U <= k1; k += U) {
+    float v[U][VEC];
+#pragma unroll
+    for (int u = 0; u < U; ++u) load(k + u, v[u]);
+#pragma unroll
+    for (int u = 0; u < U; ++u) add(k + u, v[u]);
   }
   for (; k < k1; ++k) {
-    const float a = A[(int64_t)k * lda + m];
-#pragma unroll
-    for (int j = 0; j < D; ++j) acc[j] = fmaf(a, __ldg(X + (int64_t)k * D + j), acc[j]);
-    acc[D] += a;
+    float v[VEC];
+    load(k, v);
+    add(k, v);
   }
-  float *out = P + ((int64_t)z * M + m) * (D + 1);
 #pragma unroll
-  for (int j = 0; j <= D; ++j) out[j] = acc[j];
+  for (int c = 0; c < VEC; ++c) {
+    float *out = P + ((int64_t)z * M + m0 + c) * (D + 1);
+#pragma unroll
+    for (int j = 0; j <= D; ++j) out[j] = acc[c][j];
+  }
 }
 
 cudaError_t launch_narrow_wgrad(const float *A, int64_t lda, int M, const float *X, int D, int K, float *P,
                                 size_t part_floats, int sm_count, float *out_w, float *out_b, cudaStream_t s) {
   if (M <= 0 || K <= 0) return cudaSuccess;
-  const int mb = (M + 255) / 256;
-  int splits = std::max(1, std::min(2 * sm_count / mb, K / 32));
+  const bool vec = (M % 4 == 0) && (lda % 4 == 0) && (reinterpret_cast<uintptr_t>(A) % 16 == 0);
+  const int per_thread = vec ? 4 : 1;
+  const int mb = (M / per_thread + 127) / 128;
+  // about two blocks of 128 threads per SM, each with at least 64 tokens
+  int splits = std::max(1, std::min(2 * sm_count / mb, K / 64));
   splits = std::min(splits, 1024);
   while (splits > 1 && (size_t)splits * M * (D + 1) > part_floats) --splits;
   dim3 grid(mb, splits);
   switch (D) {
-#define BKT_NW(DD) \
-  case DD: narrow_wgrad_kernel<DD><<<grid, 256, 0, s>>>(A, lda, M, X, K, P, splits); break;
+#define BKT_NW(DD)                                                                                  \
+  case DD:                                                                                          \
+    if (vec) narrow_wgrad_kernel<DD, 4><<<grid, 128, 0, s>>>(A, lda, M, X, K, P, splits);           \
+    else narrow_wgrad_kernel<DD, 1><<<grid, 128, 0, s>>>(A, lda, M, X, K, P, splits);               \
+    break;
     BKT_NW(1) BKT_NW(2) BKT_NW(3) BKT_NW(4) BKT_NW(5) BKT_NW(6) BKT_NW(7) BKT_NW(8)
     BKT_NW(9) BKT_NW(10) BKT_NW(11) BKT_NW(12) BKT_NW(13) BKT_NW(14) BKT_NW(15) BKT_NW(16)
 #undef BKT_NW
@@ -80,18 +146,11 @@ cudaError_t launch_narrow_wgrad(const float *A, int64_t lda, int M, const float 
   }
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  const int64_t total = (int64_t)M * (D + 1);
-  int blocks = (int)std::min<int64_t>(4096, (total + 255) / 256);
-  wgrad_reduce_kernel<<<blocks, 256, 0, s>>>(P, splits, M, D + 1, D, 0, out_w, nullptr, out_b);
-  return cudaGetLastError();
+  return launch_reduce(P, splits, M, D + 1, D, 0, out_w, nullptr, out_b, s);
 }
 
 cudaError_t launch_splitk_sum(const float *P, int splits, int M, int N, float *out, cudaStream_t s) {
-  const int64_t total = (int64_t)M * N;
-  if (total <= 0) return cudaSuccess;
-  int blocks = (int)std::min<int64_t>(4096, (total + 255) / 256);
-  wgrad_reduce_kernel<<<blocks, 256, 0, s>>>(P, splits, M, N, N, 0, out, nullptr, nullptr);
-  return cudaGetLastError();
+  return launch_reduce(P, splits, M, N, N, 0, out, nullptr, nullptr, s);
 }
 
 }  // namespace bkt
