@@ -63,56 +63,69 @@ static cudaError_t launch_reduce(const float *P, int splits, int M, int N, int D
 // Narrow case G[m][n] = sum_k A[k][m] [X[k] | 1][n] with X of D <= 16
 // columns, partials P[z][m][n] over token chunk z.  A bandwidth-bound pass
 // over A: with M and lda multiples of 4 a thread keeps 4 (D+1) sums for four
-// consecutive columns and 16 float4 loads of A in flight (X rows are
-// broadcast across the warp); otherwise one column per thread.
+// consecutive columns (otherwise one column).  Tokens go in groups of 16
+// (predicated, no serial tail), and the loads of the next group are issued
+// before the current one is summed, so a thread always has a group of A in
+// flight; X rows are broadcast across the warp.
 template <int D, int VEC>
 __global__ void __launch_bounds__(128) narrow_wgrad_kernel(const float *__restrict__ A, int64_t lda, int M,
                                                            const float *__restrict__ X, int K,
-                                                           float *__restrict__ P, int splits) {
+                                                           float *__restrict__ P, int chunk) {
   constexpr int U = 16;
   const int m0 = (blockIdx.x * blockDim.x + threadIdx.x) * VEC;
   const int z = blockIdx.y;
   if (m0 >= M) return;
-  const int chunk = (K + splits - 1) / splits;
   const int k0 = z * chunk, k1 = min(K, k0 + chunk);
   float acc[VEC][D + 1];
 #pragma unroll
   for (int c = 0; c < VEC; ++c)
 #pragma unroll
     for (int j = 0; j <= D; ++j) acc[c][j] = 0.f;
-  auto load = [&](int k, float (&v)[VEC]) {
-    if constexpr (VEC == 4) {
-      const float4 a = __ldg(reinterpret_cast<const float4 *>(A + (int64_t)k * lda + m0));
-      v[0] = a.x;
-      v[1] = a.y;
-      v[2] = a.z;
-      v[3] = a.w;
-    } else {
-      v[0] = __ldg(A + (int64_t)k * lda + m0);
+  auto load_group = [&](int k, float (&v)[U][VEC]) {
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (k + u < k1) {
+        if constexpr (VEC == 4) {
+          const float4 a = __ldg(reinterpret_cast<const float4 *>(A + (int64_t)(k + u) * lda + m0));
+          v[u][0] = a.x;
+          v[u][1] = a.y;
+          v[u][2] = a.z;
+          v[u][3] = a.w;
+        } else {
+          v[u][0] = __ldg(A + (int64_t)(k + u) * lda + m0);
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < VEC; ++c) v[u][c] = 0.f;
+      }
     }
   };
-  auto add = [&](int k, const float (&v)[VEC]) {
+  auto add_group = [&](int k, const float (&v)[U][VEC]) {
 #pragma unroll
-    for (int j = 0; j < D; ++j) {
-      const float x = __ldg(X + (int64_t)k * D + j);
+    for (int u = 0; u < U; ++u) {
+      if (k + u < k1) {
 #pragma unroll
-      for (int c = 0; c < VEC; ++c) acc[c][j] = fmaf(v[c], x, acc[c][j]);
+        for (int j = 0; j < D; ++j) {
+          const float x = __ldg(X + (int64_t)(k + u) * D + j);
+#pragma unroll
+          for (int c = 0; c < VEC; ++c) acc[c][j] = fmaf(v[u][c], x, acc[c][j]);
+        }
+#pragma unroll
+        for (int c = 0; c < VEC; ++c) acc[c][D] += v[u][c];
+      }
     }
-#pragma unroll
-    for (int c = 0; c < VEC; ++c) acc[c][D] += v[c];
   };
+  float va[U][VEC], vb[U][VEC];
   int k = k0;
-  for (; k + U <= k1; k += U) {
-    float v[U][VEC];
-#pragma unroll
-    for (int u = 0; u < U; ++u) load(k + u, v[u]);
-#pragma unroll
-    for (int u = 0; u < U; ++u) add(k + u, v[u]);
-  }
-  for (; k < k1; ++k) {
-    float v[VEC];
-    load(k, v);
-    add(k, v);
+  if (k < k1) load_group(k, va);
+  while (k < k1) {
+    if (k + U < k1) load_group(k + U, vb);
+    add_group(k, va);
+    k += U;
+    if (k >= k1) break;
+    if (k + U < k1) load_group(k + U, va);
+    add_group(k, vb);
+    k += U;
   }
 #pragma unroll
   for (int c = 0; c < VEC; ++c) {
@@ -128,16 +141,19 @@ cudaError_t launch_narrow_wgrad(const float *A, int64_t lda, int M, const float 
   const bool vec = (M % 4 == 0) && (lda % 4 == 0) && (reinterpret_cast<uintptr_t>(A) % 16 == 0);
   const int per_thread = vec ? 4 : 1;
   const int mb = (M / per_thread + 127) / 128;
-  // about two blocks of 128 threads per SM, each with at least 64 tokens
-  int splits = std::max(1, std::min(2 * sm_count / mb, K / 64));
+  // at least four blocks of 128 threads per SM when the batch allows (a
+  // thread streams 64 tokens or more; chunks are whole 16-token groups)
+  int splits = std::max(1, std::max(std::min(4 * sm_count / mb, K / 64), K / 2048));
   splits = std::min(splits, 1024);
   while (splits > 1 && (size_t)splits * M * (D + 1) > part_floats) --splits;
+  const int chunk = (((K + splits - 1) / splits) + 15) & ~15;
+  splits = (K + chunk - 1) / chunk;
   dim3 grid(mb, splits);
   switch (D) {
 #define BKT_NW(DD)                                                                                  \
   case DD:                                                                                          \
-    if (vec) narrow_wgrad_kernel<DD, 4><<<grid, 128, 0, s>>>(A, lda, M, X, K, P, splits);           \
-    else narrow_wgrad_kernel<DD, 1><<<grid, 128, 0, s>>>(A, lda, M, X, K, P, splits);               \
+    if (vec) narrow_wgrad_kernel<DD, 4><<<grid, 128, 0, s>>>(A, lda, M, X, K, P, chunk);            \
+    else narrow_wgrad_kernel<DD, 1><<<grid, 128, 0, s>>>(A, lda, M, X, K, P, chunk);                \
     break;
     BKT_NW(1) BKT_NW(2) BKT_NW(3) BKT_NW(4) BKT_NW(5) BKT_NW(6) BKT_NW(7) BKT_NW(8)
     BKT_NW(9) BKT_NW(10) BKT_NW(11) BKT_NW(12) BKT_NW(13) BKT_NW(14) BKT_NW(15) BKT_NW(16)
