@@ -71,6 +71,7 @@ __global__ void __launch_bounds__(512) ctc_tables_kernel(DevIdx ix, const float 
   const int SP = ix.S_max + 4;
   float *buf0 = sm, *buf1 = sm + SP;
   float *wmax = sm + 2 * SP;  // [2][32]
+  int *toff = reinterpret_cast<int *>(wmax + 64);  // [L] packed offsets of this row's time steps
   const int nw = blockDim.x >> 5;
   const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
   const int32_t *lab = labels + ix.row_lab_off[r];
@@ -111,12 +112,15 @@ __global__ void __launch_bounds__(512) ctc_tables_kernel(DevIdx ix, const float 
     buf0[i] = -CUDART_INF_F;
     buf1[i] = -CUDART_INF_F;
   }
+  // the time offsets live in shared memory: an emission prefetch is then one
+  // global load, not two dependent ones
+  for (int i = tid; i < L; i += blockDim.x) toff[i] = ix.tok_off[i];
   __syncthreads();
 
   const float *lprow = logp + (int64_t)r * C;  // token (t, r) = tok_off[t] + r
   auto emis = [&](int step, int j) -> float {
     const int t = fwd ? step : L - 1 - step;
-    return __ldg(lprow + (int64_t)ix.tok_off[t] * C + ext[j]);
+    return __ldg(lprow + (int64_t)toff[t] * C + ext[j]);
   };
   const int d1 = fwd ? -1 : 1, d2 = fwd ? -2 : 2;
 
@@ -175,7 +179,7 @@ __global__ void __launch_bounds__(512) ctc_tables_kernel(DevIdx ix, const float 
         lm = fmaxf(lm, v);
         em[j][u] = (step + kPre < L) ? emis(step + kPre, j) : 0.f;
       }
-      M += (double)mprev;
+      if (u == 0 && tid == 0) M += (double)mprev;  // fp64 is slow here: once per re-anchoring, one thread
       if (u == kPre - 1 || step == L - 1) {  // uniform over the CTA
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) lm = fmaxf(lm, __shfl_xor_sync(0xffffffffu, lm, o));
@@ -214,7 +218,16 @@ cudaError_t launch_ctc_tables(const DevIdx &ix, const float *logp, int C, int bl
   while (spt < 4 && (S + spt - 1) / spt > 512) spt *= 2;
   if ((S + spt - 1) / spt > 512) return cudaErrorInvalidValue;
   int threads = ((S + spt - 1) / spt + 31) / 32 * 32;
-  const size_t smem = (size_t)(2 * (S + 4) + 64) * sizeof(float);
+  const size_t smem = (size_t)(2 * (S + 4) + 64 + ix.T) * sizeof(float);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaSuccess;
+    switch (spt) {
+      case 1: e = cudaFuncSetAttribute(ctc_tables_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); break;
+      case 2: e = cudaFuncSetAttribute(ctc_tables_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); break;
+      default: e = cudaFuncSetAttribute(ctc_tables_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); break;
+    }
+    if (e != cudaSuccess) return e;
+  }
   dim3 grid(ix.b, 2);
   switch (spt) {
     case 1: ctc_tables_kernel<1><<<grid, threads, smem, s>>>(ix, logp, C, blank, labels, alpha, beta, loss, row_ok, status); break;
