@@ -41,8 +41,14 @@ extern "C" {
 #define BKT_ECUDA 3    /* a CUDA runtime call failed (message has the name) */
 #define BKT_EDEVICE 4  /* a device-side input check failed (label >= classes or == blank) */
 
-#define BKT_GEMM_FP32 0 /* all contractions in fp32 (SIMT FMA) */
-#define BKT_GEMM_BF16 1 /* token-axis contractions: bf16 operands, fp32 accumulation */
+#define BKT_GEMM_FP32 0 /* fp32 contractions (tensor cores with split-precision 3xTF32 operands) */
+#define BKT_GEMM_BF16 1 /* projection, dX and token-axis contractions: bf16 operands, fp32 accumulation */
+
+/* Emission order of an epoch's mini-batches (bkt_plan_buckets_ordered). */
+#define BKT_ORDER_ASCENDING 0       /* shortest bucket first (Section IV.A) */
+#define BKT_ORDER_DESCENDING 1      /* longest bucket first */
+#define BKT_ORDER_SHUFFLE_BUCKETS 2 /* buckets in a seeded random order, each kept together */
+#define BKT_ORDER_SHUFFLE_BATCHES 3 /* all mini-batches in a seeded random order */
 
 /* ------------------------------------------------------------------ */
 /* Bucketing planner (host only; no GPU needed).                       */
@@ -57,7 +63,7 @@ typedef struct bkt_plan_view {
   const int32_t *order;         /* [n] sequence ids (0..n-1) in emission order */
   int32_t n_batches;
   const int32_t *batch_off;     /* [n_batches+1] batch k is order[batch_off[k] .. batch_off[k+1]) */
-  const int32_t *batch_bucket;  /* [n_batches] bucket index of each batch, non-decreasing */
+  const int32_t *batch_bucket;  /* [n_batches] bucket index of each batch (non-decreasing for BKT_ORDER_ASCENDING) */
   int64_t padded_timesteps;     /* sum over batches of |batch| * max length in the batch */
   int64_t unpadded_timesteps;   /* sum of all lengths */
 } bkt_plan_view;
@@ -80,6 +86,25 @@ typedef struct bkt_plan_view {
 int bkt_plan_buckets(const int32_t *lengths, int64_t n, int32_t n_buckets,
                      int32_t batch, uint64_t seed, uint64_t epoch,
                      bkt_plan **out);
+
+/* As bkt_plan_buckets, with the batches emitted in `batch_order` (one of
+ * BKT_ORDER_*; Section V names bucket-ordering strategies as future work).
+ * Bounds, bucket contents, the in-bucket shuffles and the cut into batches
+ * are those of bkt_plan_buckets; only the order in which the batches are
+ * emitted changes (order[] is rewritten so every batch stays contiguous):
+ *   ASCENDING       buckets 0, 1, ..., Q-1 (identical to bkt_plan_buckets);
+ *   DESCENDING      buckets Q-1, ..., 0, batches of a bucket in cut order;
+ *   SHUFFLE_BUCKETS the bucket sequence permuted by Fisher-Yates over the Q
+ *                   bucket indices (k = Q-1 down to 1, j = next() mod (k+1)),
+ *                   drawing from the same SplitMix64 stream after the
+ *                   in-bucket shuffles; batches of a bucket in cut order;
+ *   SHUFFLE_BATCHES the sequence of all batches (in ascending cut order)
+ *                   permuted the same way, k = n_batches-1 down to 1.
+ * padded_timesteps and dp_cost do not depend on the order.  An unknown
+ * batch_order is BKT_EINVAL.                                            */
+int bkt_plan_buckets_ordered(const int32_t *lengths, int64_t n, int32_t n_buckets,
+                             int32_t batch, uint64_t seed, uint64_t epoch,
+                             int32_t batch_order, bkt_plan **out);
 
 /* Fills *view with pointers into the plan (valid until bkt_plan_free). */
 int bkt_plan_get(const bkt_plan *plan, bkt_plan_view *view);

@@ -66,6 +66,10 @@ def _load():
                                 ctypes.c_uint64, ctypes.c_uint64, i32p, i64p, i32p,
                                 i32p, i32p, i32p, i64p]
         lib.or_plan.restype = ctypes.c_int
+        lib.or_plan_ordered.argtypes = [i32p, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
+                                        ctypes.c_uint64, ctypes.c_uint64, ctypes.c_int32, i32p,
+                                        i64p, i32p, i32p, i32p, i32p, i64p]
+        lib.or_plan_ordered.restype = ctypes.c_int
         lib.or_ctc.argtypes = [f64p, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
                                i32p, ctypes.c_int32, f64p]
         lib.or_ctc.restype = ctypes.c_double
@@ -121,8 +125,13 @@ def dynamic_bucketing(f, Q: int):
     return bests, int(cost.value)
 
 
-def plan(lengths, n_buckets: int, batch: int, seed: int, epoch: int = 0) -> dict:
-    """The epoch plan: bounds, dp cost, emission order and mini-batches."""
+PLAN_ORDERS = {"ascending": 0, "descending": 1, "shuffle_buckets": 2, "shuffle_batches": 3}
+
+
+def plan(lengths, n_buckets: int, batch: int, seed: int, epoch: int = 0,
+         batch_order: str = "ascending") -> dict:
+    """The epoch plan: bounds, dp cost, emission order and mini-batches
+    (or_plan for "ascending", or_plan_ordered otherwise)."""
     lib = _load()
     L = np.ascontiguousarray(lengths, dtype=np.int32)
     n = L.size
@@ -133,11 +142,16 @@ def plan(lengths, n_buckets: int, batch: int, seed: int, epoch: int = 0) -> dict
     nb = ctypes.c_int32(0)
     cost = ctypes.c_int64(0)
     padded = ctypes.c_int64(0)
-    rc = lib.or_plan(_p(L, ctypes.c_int32), n, n_buckets, batch,
-                     ctypes.c_uint64(seed), ctypes.c_uint64(epoch),
-                     _p(bounds, ctypes.c_int32), ctypes.byref(cost),
-                     _p(order, ctypes.c_int32), _p(boff, ctypes.c_int32),
-                     _p(bbuck, ctypes.c_int32), ctypes.byref(nb), ctypes.byref(padded))
+    tail = (_p(bounds, ctypes.c_int32), ctypes.byref(cost), _p(order, ctypes.c_int32),
+            _p(boff, ctypes.c_int32), _p(bbuck, ctypes.c_int32), ctypes.byref(nb),
+            ctypes.byref(padded))
+    if batch_order == "ascending":
+        rc = lib.or_plan(_p(L, ctypes.c_int32), n, n_buckets, batch, ctypes.c_uint64(seed),
+                         ctypes.c_uint64(epoch), *tail)
+    else:
+        rc = lib.or_plan_ordered(_p(L, ctypes.c_int32), n, n_buckets, batch,
+                                 ctypes.c_uint64(seed), ctypes.c_uint64(epoch),
+                                 PLAN_ORDERS[batch_order], *tail)
     if rc:
         raise OracleError(rc, "plan")
     k = nb.value

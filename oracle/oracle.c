@@ -19,6 +19,10 @@
  *                       first bucket whose upper bound holds its length,
  *                       shuffle inside each bucket, cut mini-batches, emit the
  *                       buckets shortest first.
+ *   or_plan_ordered     the same plan with the batches emitted in another
+ *                       order (Section V leaves bucket-ordering strategies to
+ *                       future work): descending buckets, a shuffled bucket
+ *                       sequence, or all batches shuffled.
  *   or_ctc              CTC (Graves et al. 2006, the paper's ref. [15]):
  *                       log-space forward/backward variables and the gradient
  *                       of -ln p with respect to the unnormalised outputs.
@@ -30,6 +34,8 @@
  *                       padding ever enters the arithmetic (eq. 1-2 are the
  *                       padded cost this removes).
  *   or_sgd              theta <- theta - lr * g.
+ *   or_adadelta         ADADELTA (Zeiler 2012, the paper's ref. [21], its
+ *                       Algorithm 1), the update rule of Section III.B step 4.
  *
  * Numerics: all arithmetic is in double; exp/log/tanh are the C library's.
  */
@@ -142,19 +148,25 @@ int or_dynamic_bucketing(const int64_t *f, int32_t n, int32_t Q,
  *      IV.A: the shorter sequences are fed first).  Each bucket is cut into
  *      consecutive mini-batches of `batch` entries; its last one may be
  *      partial and is kept.  batch_off[b]..batch_off[b+1] indexes order.
+ *   5. (or_plan_ordered) mode 0 keeps that order; mode 1 emits the buckets
+ *      longest first; mode 2 permutes the bucket sequence 0..Q-1 by
+ *      Fisher-Yates (k = Q-1 .. 1, j = next() mod (k+1)) drawing on from
+ *      the same stream; mode 3 permutes all batches (in the order of step
+ *      4) the same way.  Batches stay whole; order is rewritten to match.
  * Capacities: bounds[Q], order[n], batch_off[n+1], batch_bucket[n].    */
-int or_plan(const int32_t *lengths, int64_t n, int32_t Q, int32_t batch,
-            uint64_t seed, uint64_t epoch, int32_t *bounds, int64_t *dp_cost,
-            int32_t *order, int32_t *batch_off, int32_t *batch_bucket,
-            int32_t *n_batches, int64_t *padded_timesteps) {
+int or_plan_ordered(const int32_t *lengths, int64_t n, int32_t Q,
+                    int32_t batch, uint64_t seed, uint64_t epoch,
+                    int32_t mode, int32_t *bounds, int64_t *dp_cost,
+                    int32_t *order, int32_t *batch_off, int32_t *batch_bucket,
+                    int32_t *n_batches, int64_t *padded_timesteps) {
   int32_t lmax = 0, q;
-  int64_t i, *f, pos = 0, padded = 0;
+  int64_t i, *f, padded = 0;
   int32_t nb = 0;
   int32_t *bucket_of, *bucket_start, *bucket_fill;
   uint64_t state;
   int rc;
   if (!lengths || n < 1 || Q < 1 || batch < 1 || !bounds || !order ||
-      !batch_off || !batch_bucket || !n_batches)
+      !batch_off || !batch_bucket || !n_batches || mode < 0 || mode > 3)
     return OR_EINVAL;
   for (i = 0; i < n; i++) {
     if (lengths[i] < 1) return OR_EINVAL;
@@ -215,14 +227,80 @@ int or_plan(const int32_t *lengths, int64_t n, int32_t Q, int32_t batch,
     }
   }
   batch_off[nb] = (int32_t)n;
-  pos = n;
-  (void)pos;
   *n_batches = nb;
   if (padded_timesteps) *padded_timesteps = padded;
   free(bucket_of);
   free(bucket_start);
   free(bucket_fill);
+  if (mode != 0) {
+    /* The batches above are in ascending cut order.  seq lists them in
+     * emission order; then order, batch_off and batch_bucket are rebuilt
+     * from it. */
+    int32_t *seq = (int32_t *)malloc(sizeof(int32_t) * (size_t)nb);
+    int32_t *qseq = (int32_t *)malloc(sizeof(int32_t) * (size_t)Q);
+    int32_t *old_order = (int32_t *)malloc(sizeof(int32_t) * (size_t)n);
+    int32_t *old_off = (int32_t *)malloc(sizeof(int32_t) * (size_t)(nb + 1));
+    int32_t *old_bucket = (int32_t *)malloc(sizeof(int32_t) * (size_t)(nb > 0 ? nb : 1));
+    int32_t b, w = 0, k;
+    if (!seq || !qseq || !old_order || !old_off || !old_bucket) {
+      free(seq);
+      free(qseq);
+      free(old_order);
+      free(old_off);
+      free(old_bucket);
+      return OR_ENOMEM;
+    }
+    memcpy(old_order, order, sizeof(int32_t) * (size_t)n);
+    memcpy(old_off, batch_off, sizeof(int32_t) * (size_t)(nb + 1));
+    if (nb > 0) memcpy(old_bucket, batch_bucket, sizeof(int32_t) * (size_t)nb);
+    if (mode == 3) {
+      /* every batch, shuffled by Fisher-Yates from the same stream */
+      for (b = 0; b < nb; b++) seq[b] = b;
+      for (k = nb - 1; k >= 1; k--) {
+        int32_t j = (int32_t)(or_splitmix64(&state) % (uint64_t)(k + 1));
+        int32_t t = seq[k];
+        seq[k] = seq[j];
+        seq[j] = t;
+      }
+    } else {
+      /* a sequence of buckets, each bucket's batches in cut order */
+      for (q = 0; q < Q; q++) qseq[q] = (mode == 1) ? Q - 1 - q : q;
+      if (mode == 2) {
+        for (k = Q - 1; k >= 1; k--) {
+          int32_t j = (int32_t)(or_splitmix64(&state) % (uint64_t)(k + 1));
+          int32_t t = qseq[k];
+          qseq[k] = qseq[j];
+          qseq[j] = t;
+        }
+      }
+      for (q = 0; q < Q; q++)
+        for (b = 0; b < nb; b++)
+          if (old_bucket[b] == qseq[q]) seq[w++] = b;
+    }
+    w = 0;
+    for (b = 0; b < nb; b++) {
+      int32_t src = seq[b], r;
+      batch_off[b] = w;
+      batch_bucket[b] = old_bucket[src];
+      for (r = old_off[src]; r < old_off[src + 1]; r++) order[w++] = old_order[r];
+    }
+    batch_off[nb] = (int32_t)n;
+    free(seq);
+    free(qseq);
+    free(old_order);
+    free(old_off);
+    free(old_bucket);
+  }
   return OR_OK;
+}
+
+int or_plan(const int32_t *lengths, int64_t n, int32_t Q, int32_t batch,
+            uint64_t seed, uint64_t epoch, int32_t *bounds, int64_t *dp_cost,
+            int32_t *order, int32_t *batch_off, int32_t *batch_bucket,
+            int32_t *n_batches, int64_t *padded_timesteps) {
+  return or_plan_ordered(lengths, n, Q, batch, seed, epoch, 0, bounds, dp_cost,
+                         order, batch_off, batch_bucket, n_batches,
+                         padded_timesteps);
 }
 
 /* ------------------------------------------------------------------ */

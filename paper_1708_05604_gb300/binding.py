@@ -20,7 +20,7 @@ BKT_OK, BKT_EINVAL, BKT_ENOMEM, BKT_ECUDA, BKT_EDEVICE = 0, 1, 2, 3, 4
 BKT_GEMM_FP32, BKT_GEMM_BF16 = 0, 1
 
 # Every symbol include/bkt.h declares.
-EXPORTS = ("bkt_plan_buckets", "bkt_plan_get", "bkt_plan_free", "bkt_param_count",
+EXPORTS = ("bkt_plan_buckets", "bkt_plan_buckets_ordered", "bkt_plan_get", "bkt_plan_free", "bkt_param_count",
            "bkt_ctx_create", "bkt_ctx_destroy", "bkt_lstm_ctc_step", "bkt_lstm_ctc_step_static",
            "bkt_sgd_update",
            "bkt_ctx_sync_status", "bkt_ctx_set_timing", "bkt_ctx_kernel_times",
@@ -78,6 +78,9 @@ def lib() -> ctypes.CDLL:
         vp = ctypes.c_void_p
         L.bkt_plan_buckets.argtypes = [i32p, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
                                        ctypes.c_uint64, ctypes.c_uint64, ctypes.POINTER(vp)]
+        L.bkt_plan_buckets_ordered.argtypes = [i32p, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
+                                               ctypes.c_uint64, ctypes.c_uint64, ctypes.c_int32,
+                                               ctypes.POINTER(vp)]
         L.bkt_plan_get.argtypes = [vp, ctypes.POINTER(PlanView)]
         L.bkt_plan_free.argtypes = [vp]
         L.bkt_plan_free.restype = None
@@ -96,7 +99,7 @@ def lib() -> ctypes.CDLL:
         L.bkt_ctx_kernel_times.argtypes = [vp, ctypes.POINTER(KernelTime), ctypes.c_int32, i32p]
         L.bkt_last_error.argtypes = []
         L.bkt_last_error.restype = ctypes.c_char_p
-        for name in ("bkt_plan_buckets", "bkt_plan_get", "bkt_ctx_create", "bkt_lstm_ctc_step",
+        for name in ("bkt_plan_buckets", "bkt_plan_buckets_ordered", "bkt_plan_get", "bkt_ctx_create", "bkt_lstm_ctc_step",
                      "bkt_lstm_ctc_step_static",
                      "bkt_sgd_update", "bkt_ctx_sync_status", "bkt_ctx_set_timing",
                      "bkt_ctx_kernel_times"):
@@ -132,12 +135,18 @@ def _stream_handle(stream) -> ctypes.c_void_p:
 
 
 # ---------------------------------------------------------------------------
-def plan_buckets(lengths, n_buckets: int, batch: int, seed: int, epoch: int = 0) -> dict:
-    """bkt_plan_buckets + bkt_plan_get, copied into numpy arrays."""
+BATCH_ORDERS = {"ascending": 0, "descending": 1, "shuffle_buckets": 2, "shuffle_batches": 3}
+
+
+def plan_buckets(lengths, n_buckets: int, batch: int, seed: int, epoch: int = 0,
+                 batch_order: str = "ascending") -> dict:
+    """bkt_plan_buckets_ordered + bkt_plan_get, copied into numpy arrays
+    (batch_order: a key of BATCH_ORDERS; "ascending" is bkt_plan_buckets)."""
     L = _i32(lengths)
     h = ctypes.c_void_p()
-    _check(lib().bkt_plan_buckets(_ptr(L, ctypes.c_int32), L.size, n_buckets, batch,
-                                  ctypes.c_uint64(seed), ctypes.c_uint64(epoch), ctypes.byref(h)))
+    _check(lib().bkt_plan_buckets_ordered(_ptr(L, ctypes.c_int32), L.size, n_buckets, batch,
+                                          ctypes.c_uint64(seed), ctypes.c_uint64(epoch),
+                                          BATCH_ORDERS[batch_order], ctypes.byref(h)))
     try:
         v = PlanView()
         _check(lib().bkt_plan_get(h, ctypes.byref(v)))

@@ -59,9 +59,11 @@ struct bkt_plan {
   int64_t dp_cost = 0, padded = 0, unpadded = 0;
 };
 
-extern "C" int bkt_plan_buckets(const int32_t *lengths, int64_t n, int32_t Q, int32_t batch,
-                                uint64_t seed, uint64_t epoch, bkt_plan **out) {
+extern "C" int bkt_plan_buckets_ordered(const int32_t *lengths, int64_t n, int32_t Q, int32_t batch,
+                                        uint64_t seed, uint64_t epoch, int32_t batch_order, bkt_plan **out) {
   if (!out) return set_err(BKT_EINVAL, "bkt_plan_buckets: out is NULL");
+  if (batch_order < BKT_ORDER_ASCENDING || batch_order > BKT_ORDER_SHUFFLE_BATCHES)
+    return set_err(BKT_EINVAL, "bkt_plan_buckets: unknown batch order %d", batch_order);
   *out = nullptr;
   if (!lengths || n < 1) return set_err(BKT_EINVAL, "bkt_plan_buckets: no lengths");
   if (Q < 1 || batch < 1) return set_err(BKT_EINVAL, "bkt_plan_buckets: n_buckets and batch must be >= 1");
@@ -141,16 +143,52 @@ extern "C" int bkt_plan_buckets(const int32_t *lengths, int64_t n, int32_t Q, in
         std::swap(lst[k], lst[j]);
       }
     }
+    // mini-batches: consecutive chunks of each bucket, buckets ascending
+    std::vector<int64_t> cut_s, cut_e;
+    std::vector<int32_t> cut_q;
     for (int32_t q = 0; q < Q; ++q) {
       for (int64_t s = start[q]; s < start[q + 1]; s += batch) {
         const int64_t e = std::min<int64_t>(s + batch, start[q + 1]);
         int32_t mx = 0;
         for (int64_t r = s; r < e; ++r) mx = std::max(mx, lengths[p->order[r]]);
-        p->batch_off.push_back((int32_t)s);
-        p->batch_bucket.push_back(q);
+        cut_s.push_back(s);
+        cut_e.push_back(e);
+        cut_q.push_back(q);
         p->padded += (e - s) * (int64_t)mx;
       }
     }
+    // emission order of the batches (the bucket-ordering strategies that
+    // Section V leaves to future work); the shuffles continue the stream
+    const int64_t nb = (int64_t)cut_q.size();
+    std::vector<int64_t> seq(nb);
+    for (int64_t b = 0; b < nb; ++b) seq[b] = b;
+    if (batch_order == BKT_ORDER_DESCENDING || batch_order == BKT_ORDER_SHUFFLE_BUCKETS) {
+      std::vector<int32_t> qs(Q);
+      for (int32_t q = 0; q < Q; ++q) qs[q] = batch_order == BKT_ORDER_DESCENDING ? Q - 1 - q : q;
+      if (batch_order == BKT_ORDER_SHUFFLE_BUCKETS)
+        for (int64_t k = Q - 1; k >= 1; --k) {
+          const int64_t j = (int64_t)(splitmix64_next(state) % (uint64_t)(k + 1));
+          std::swap(qs[k], qs[j]);
+        }
+      int64_t w = 0;
+      for (int32_t qi = 0; qi < Q; ++qi)
+        for (int64_t b = 0; b < nb; ++b)
+          if (cut_q[b] == qs[qi]) seq[w++] = b;
+    } else if (batch_order == BKT_ORDER_SHUFFLE_BATCHES) {
+      for (int64_t k = nb - 1; k >= 1; --k) {
+        const int64_t j = (int64_t)(splitmix64_next(state) % (uint64_t)(k + 1));
+        std::swap(seq[k], seq[j]);
+      }
+    }
+    std::vector<int32_t> emitted(n);
+    int64_t pos = 0;
+    for (int64_t i = 0; i < nb; ++i) {
+      const int64_t b = seq[i];
+      p->batch_off.push_back((int32_t)pos);
+      p->batch_bucket.push_back(cut_q[b]);
+      for (int64_t r = cut_s[b]; r < cut_e[b]; ++r) emitted[pos++] = p->order[r];
+    }
+    p->order.swap(emitted);
     p->batch_off.push_back((int32_t)n);
     p->unpadded = total;
   } catch (const std::bad_alloc &) {
@@ -159,6 +197,11 @@ extern "C" int bkt_plan_buckets(const int32_t *lengths, int64_t n, int32_t Q, in
   }
   *out = p;
   return BKT_OK;
+}
+
+extern "C" int bkt_plan_buckets(const int32_t *lengths, int64_t n, int32_t Q, int32_t batch,
+                                uint64_t seed, uint64_t epoch, bkt_plan **out) {
+  return bkt_plan_buckets_ordered(lengths, n, Q, batch, seed, epoch, BKT_ORDER_ASCENDING, out);
 }
 
 extern "C" int bkt_plan_get(const bkt_plan *p, bkt_plan_view *v) {

@@ -59,6 +59,27 @@ def test_planner_bit_exact_vs_oracle(lib, wname, Q, seed):
         assert a["unpadded_timesteps"] == int(L.sum())
 
 
+@pytest.mark.parametrize("mode", ["descending", "shuffle_buckets", "shuffle_batches"])
+@pytest.mark.parametrize("wname,Q", PLAN_CASES[::2])
+def test_ordered_planner_bit_exact_vs_oracle(lib, wname, Q, mode):
+    w = synth.WORKLOADS[wname]
+    L = synth.draw_lengths(np.random.default_rng(5), w.n_seqs, w.length_dist)
+    for epoch in (0, 4):
+        a = binding.plan_buckets(L, Q, w.batch, seed=5, epoch=epoch, batch_order=mode)
+        b = oracle.plan(L, Q, w.batch, seed=5, epoch=epoch, batch_order=mode)
+        for k in ("bounds", "order", "batch_off", "batch_bucket"):
+            assert np.array_equal(a[k], b[k]), (k, wname, Q, mode, epoch)
+        assert a["padded_timesteps"] == b["padded_timesteps"]
+
+
+def test_ordered_planner_rejects_unknown_order(lib):
+    L = np.array([1, 2, 3], np.int32)
+    h = ctypes.c_void_p()
+    rc = lib.bkt_plan_buckets_ordered(L.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)), 3, 2, 2,
+                                      ctypes.c_uint64(0), ctypes.c_uint64(0), 7, ctypes.byref(h))
+    assert rc == binding.BKT_EINVAL and not h.value
+
+
 @pytest.mark.parametrize("seed", range(30))
 def test_planner_small_random_vs_oracle(lib, seed):
     rng = np.random.default_rng(500 + seed)

@@ -169,3 +169,89 @@ def test_plan_empty_bucket_and_q_equals_lmax():
     _check_plan(p, L, 10, 3)
     with pytest.raises(oracle.OracleError):
         oracle.plan(L, 11, 3, seed=3, epoch=0)
+
+
+# ---------------------------------------------------------------------------
+# Batch-order variants (bucket-ordering strategies, Section V future work).
+
+def _batches(p):
+    o, off = p["order"], p["batch_off"]
+    return [tuple(o[off[k]:off[k + 1]].tolist()) for k in range(p["n_batches"])]
+
+
+ORDERS = ["descending", "shuffle_buckets", "shuffle_batches"]
+
+
+@pytest.mark.parametrize("mode", ORDERS)
+@pytest.mark.parametrize("Q,B", [(1, 16), (4, 7), (8, 64), (3, 1)])
+def test_ordered_plan_permutes_whole_batches(mode, Q, B):
+    """Every order emits exactly the ascending plan's batches (same members,
+    same internal order), with the same bounds, dp cost and padding."""
+    rng = np.random.default_rng(11)
+    L = rng.integers(20, 201, size=300).astype(np.int32)
+    a = oracle.plan(L, Q, B, seed=5, epoch=2)
+    p = oracle.plan(L, Q, B, seed=5, epoch=2, batch_order=mode)
+    assert np.array_equal(a["bounds"], p["bounds"])
+    assert a["dp_cost"] == p["dp_cost"] and a["padded_timesteps"] == p["padded_timesteps"]
+    assert a["n_batches"] == p["n_batches"]
+    ba, bp = _batches(a), _batches(p)
+    assert sorted(ba) == sorted(bp)
+    bucket_of = {b: q for b, q in zip(ba, a["batch_bucket"].tolist())}
+    assert [bucket_of[b] for b in bp] == p["batch_bucket"].tolist()
+    if mode != "shuffle_batches":
+        # buckets stay together, each bucket's batches in cut order
+        seq = p["batch_bucket"].tolist()
+        runs = [q for i, q in enumerate(seq) if i == 0 or seq[i - 1] != q]
+        assert len(runs) == len(set(runs))
+        for q in set(seq):
+            assert [b for b in bp if bucket_of[b] == q] == [b for b in ba if bucket_of[b] == q]
+        if mode == "descending":
+            assert runs == sorted(runs, reverse=True)
+
+
+def test_ordered_plan_ascending_is_the_plain_plan():
+    L = np.random.default_rng(3).integers(1, 60, size=200).astype(np.int32)
+    for e in range(3):
+        a = oracle.plan(L, 5, 9, seed=1, epoch=e)
+        b = oracle.plan(L, 5, 9, seed=1, epoch=e, batch_order="ascending")
+        assert _batches(a) == _batches(b)
+
+
+def test_shuffle_batches_is_fisher_yates_on_the_continued_stream():
+    """Definition check: after the in-bucket shuffles (sum over buckets of
+    m_q - 1 draws), the same SplitMix64 stream permutes the list of batches
+    with Fisher-Yates, k = n_batches-1 .. 1, j = next() mod (k+1)."""
+    L = np.random.default_rng(4).integers(1, 50, size=150).astype(np.int32)
+    Q, B, seed, epoch = 4, 6, 9, 1
+    a = oracle.plan(L, Q, B, seed=seed, epoch=epoch)
+    p = oracle.plan(L, Q, B, seed=seed, epoch=epoch, batch_order="shuffle_batches")
+    sizes = np.bincount(a["batch_bucket"], weights=np.diff(a["batch_off"]), minlength=Q)
+    used = int(sum(max(int(m) - 1, 0) for m in sizes))
+    nb = a["n_batches"]
+    state0 = (seed + (epoch + 1) * 0x9E3779B97F4A7C15) % (1 << 64)
+    draws = oracle.splitmix64_stream(state0, used + nb)[used:]
+    seq = list(range(nb))
+    for i, k in enumerate(range(nb - 1, 0, -1)):
+        j = draws[i] % (k + 1)
+        seq[k], seq[j] = seq[j], seq[k]
+    ba = _batches(a)
+    assert _batches(p) == [ba[s] for s in seq]
+
+
+@pytest.mark.parametrize("mode", ["shuffle_buckets", "shuffle_batches"])
+def test_order_shuffles_are_uniform_enough(mode):
+    """Over many epochs each bucket (batch) takes every position about equally
+    often, and the order changes with the epoch."""
+    L = np.repeat(np.arange(1, 5, dtype=np.int32), 3)   # 4 buckets of 3 equal lengths
+    Q, B = 4, 3                                          # one batch per bucket
+    counts = np.zeros((4, 4))
+    for e in range(2000):
+        p = oracle.plan(L, Q, B, seed=77, epoch=e, batch_order=mode)
+        for pos, q in enumerate(p["batch_bucket"].tolist()):
+            counts[q, pos] += 1
+    assert counts.min() > 2000 / 4 * 0.8 and counts.max() < 2000 / 4 * 1.2
+
+
+def test_ordered_plan_rejects_unknown_order():
+    with pytest.raises(KeyError):
+        oracle.plan(np.array([1, 2, 3], np.int32), 2, 2, seed=0, batch_order="zigzag")
