@@ -4,7 +4,8 @@
 One "step" = one training epoch over the synthetic workload: plan the
 buckets (bkt_plan_buckets: histogram, dynamic program, per-epoch reshuffle),
 then for every mini-batch one bkt_lstm_ctc_step (packed layout, LSTM forward,
-output + log-softmax, CTC, BPTT, weight gradients) and one bkt_sgd_update.
+output + log-softmax, CTC, BPTT, weight gradients) and one bkt_sgd_update
+(or, with --optimizer adadelta, the paper's update rule bkt_adadelta_update).
 The metric is unpadded timesteps per second (sum of sequence lengths
 processed / time).  Inputs are resident in HBM when the timed region starts;
 L2 is flushed (a 256 MiB write) between timed steps, outside their events.
@@ -48,6 +49,7 @@ def parse():
     ap.add_argument("--compare-buckets", default="1",
                     help="extra bucket counts timed briefly for epoch time vs Q ('' = none)")
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--optimizer", default="sgd", choices=["sgd", "adadelta"])
     ap.add_argument("--cpu-baseline-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -230,6 +232,8 @@ def run_native(args, world, rank, local):
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
     unpadded = int(ds.lengths.sum())
 
+    opt = binding.Adadelta(params) if args.optimizer == "adadelta" else None
+
     def epoch(e, Q, dataset=dd, loss_buf=loss):
         plan = binding.plan_buckets(ds.lengths, Q, w.batch, seed=args.seed, epoch=e)
         order, off = plan["order"], plan["batch_off"]
@@ -237,7 +241,10 @@ def run_native(args, world, rank, local):
             ids = order[off[k]:off[k + 1]]
             lv = loss_buf[off[k]:off[k + 1]]
             ctx.step(dataset, ids, params, grads, lv, stream)
-            binding.sgd_update(params, grads, LR, stream)
+            if opt is None:
+                binding.sgd_update(params, grads, LR, stream)
+            else:
+                opt.step(grads, stream)
         return plan
 
     def timed(Q, steps, warmup, e0=0, with_timer=False, clocks=None):
@@ -341,6 +348,7 @@ def run_native(args, world, rank, local):
 
     line = {
         "metric": "unpadded timesteps/sec (LSTM+CTC fwd+bwd+SGD epoch, 1 GPU)",
+        "optimizer": args.optimizer,
         "value": value, "unit": "timesteps/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32" if not w.gemm_bf16 else "bf16+f32",

@@ -9,8 +9,8 @@
  *   - bkt_lstm_ctc_step: the training step of Section IV (an LSTM, ref. [1],
  *     trained with the CTC cost, ref. [15]) over one length-bucketed
  *     mini-batch, forward + back-propagation through time, on one GPU.
- *   - bkt_sgd_update: the parameter update.  (The paper's update rule is
- *     ADADELTA, Section III.B step 4; this step uses plain SGD.)
+ *   - bkt_adadelta_update: the paper's parameter update rule, ADADELTA
+ *     (Section III.B step 4, ref. [21]); bkt_sgd_update: plain SGD.
  *
  * Conventions
  *   - Every entry point returns an int status (BKT_OK = 0).  On failure
@@ -209,6 +209,23 @@ int bkt_lstm_ctc_step_static(const bkt_model_cfg *cfg, const bkt_batch *batch,
  * vectors when both are 16-byte aligned), enqueued on `stream`.          */
 int bkt_sgd_update(float *params, const float *grads, int64_t n, float lr,
                    void *stream);
+
+/* ADADELTA (Zeiler 2012, the paper's ref. [21], Algorithm 1; the update
+ * rule of Section III.B step 4), for i < n:
+ *   eg2[i]  = rho * eg2[i] + (1 - rho) * grads[i]^2
+ *   dx      = sqrt(edx2[i] + eps) / sqrt(eg2[i] + eps) * grads[i]
+ *   edx2[i] = rho * edx2[i] + (1 - rho) * dx^2
+ *   params[i] -= lr * dx
+ * (Zeiler's rule is lr = 1; the paper names no constants, the usual ones
+ * are rho = 0.95, eps = 1e-6.)  All arrays are device fp32 of n entries;
+ * eg2 and edx2 are the caller's running averages, zero before the first
+ * update, and are updated in place.  IEEE square roots and division; one
+ * element per thread, 16-byte vectors when all four arrays are 16-byte
+ * aligned.  BKT_EINVAL: n < 0, a NULL array with n > 0, rho outside
+ * [0, 1), eps <= 0 or lr < 0.  Enqueued on `stream`.                    */
+int bkt_adadelta_update(float *params, const float *grads, float *eg2,
+                        float *edx2, int64_t n, float rho, float eps,
+                        float lr, void *stream);
 
 /* Waits for the work this ctx enqueued, then returns BKT_OK or the first
  * device-side error (BKT_EDEVICE) raised since the previous call, and

@@ -80,6 +80,9 @@ def _load():
         lib.or_lstm_ctc_step.restype = ctypes.c_int
         lib.or_sgd.argtypes = [f64p, f64p, ctypes.c_int64, ctypes.c_double]
         lib.or_sgd.restype = None
+        lib.or_adadelta.argtypes = [f64p, f64p, f64p, f64p, ctypes.c_int64, ctypes.c_double,
+                                    ctypes.c_double, ctypes.c_double]
+        lib.or_adadelta.restype = None
         _lib = lib
         return lib
 
@@ -220,3 +223,16 @@ def sgd(params, grads, lr: float) -> np.ndarray:
     g = np.ascontiguousarray(grads, dtype=np.float64)
     lib.or_sgd(_p(p, ctypes.c_double), _p(g, ctypes.c_double), p.size, lr)
     return p
+
+
+def adadelta(params, grads, eg2, edx2, rho: float = 0.95, eps: float = 1e-6,
+             lr: float = 1.0):
+    """One ADADELTA update; returns new (params, eg2, edx2) as float64."""
+    lib = _load()
+    p = np.array(params, dtype=np.float64, copy=True)
+    g = np.ascontiguousarray(grads, dtype=np.float64)
+    a = np.array(eg2, dtype=np.float64, copy=True)
+    b = np.array(edx2, dtype=np.float64, copy=True)
+    lib.or_adadelta(_p(p, ctypes.c_double), _p(g, ctypes.c_double), _p(a, ctypes.c_double),
+                    _p(b, ctypes.c_double), p.size, rho, eps, lr)
+    return p, a, b

@@ -655,3 +655,25 @@ void or_sgd(double *params, const double *grads, int64_t n, double lr) {
   int64_t i;
   for (i = 0; i < n; i++) params[i] -= lr * grads[i];
 }
+
+/* ADADELTA, Zeiler 2012 (ref. [21]), Algorithm 1, one update for i < n:
+ *   accumulate gradient:  E[g^2] <- rho E[g^2] + (1 - rho) g^2
+ *   compute update:       dx = -(RMS[dx]_{t-1} / RMS[g]_t) g,
+ *                         RMS[y] = sqrt(E[y^2] + eps)
+ *   accumulate updates:   E[dx^2] <- rho E[dx^2] + (1 - rho) dx^2
+ *   apply update:         x <- x + lr dx   (lr = 1 in the algorithm; a
+ *                         learning-rate factor scales the applied step only)
+ */
+void or_adadelta(double *x, const double *g, double *eg2, double *edx2,
+                 int64_t n, double rho, double eps, double lr) {
+  int64_t i;
+  for (i = 0; i < n; i++) {
+    double rms_g, rms_dx, dx;
+    eg2[i] = rho * eg2[i] + (1.0 - rho) * g[i] * g[i];
+    rms_g = sqrt(eg2[i] + eps);
+    rms_dx = sqrt(edx2[i] + eps);
+    dx = -(rms_dx / rms_g) * g[i];
+    edx2[i] = rho * edx2[i] + (1.0 - rho) * dx * dx;
+    x[i] += lr * dx;
+  }
+}

@@ -22,7 +22,7 @@ BKT_GEMM_FP32, BKT_GEMM_BF16 = 0, 1
 # Every symbol include/bkt.h declares.
 EXPORTS = ("bkt_plan_buckets", "bkt_plan_buckets_ordered", "bkt_plan_get", "bkt_plan_free", "bkt_param_count",
            "bkt_ctx_create", "bkt_ctx_destroy", "bkt_lstm_ctc_step", "bkt_lstm_ctc_step_static",
-           "bkt_sgd_update",
+           "bkt_sgd_update", "bkt_adadelta_update",
            "bkt_ctx_sync_status", "bkt_ctx_set_timing", "bkt_ctx_kernel_times",
            "bkt_last_error")
 
@@ -94,6 +94,8 @@ def lib() -> ctypes.CDLL:
         L.bkt_lstm_ctc_step_static.argtypes = [ctypes.POINTER(ModelCfg), ctypes.POINTER(Batch), vp,
                                                vp, vp, vp]
         L.bkt_sgd_update.argtypes = [vp, vp, ctypes.c_int64, ctypes.c_float, vp]
+        L.bkt_adadelta_update.argtypes = [vp, vp, vp, vp, ctypes.c_int64, ctypes.c_float,
+                                          ctypes.c_float, ctypes.c_float, vp]
         L.bkt_ctx_sync_status.argtypes = [vp]
         L.bkt_ctx_set_timing.argtypes = [vp, ctypes.c_int32]
         L.bkt_ctx_kernel_times.argtypes = [vp, ctypes.POINTER(KernelTime), ctypes.c_int32, i32p]
@@ -101,7 +103,7 @@ def lib() -> ctypes.CDLL:
         L.bkt_last_error.restype = ctypes.c_char_p
         for name in ("bkt_plan_buckets", "bkt_plan_buckets_ordered", "bkt_plan_get", "bkt_ctx_create", "bkt_lstm_ctc_step",
                      "bkt_lstm_ctc_step_static",
-                     "bkt_sgd_update", "bkt_ctx_sync_status", "bkt_ctx_set_timing",
+                     "bkt_sgd_update", "bkt_adadelta_update", "bkt_ctx_sync_status", "bkt_ctx_set_timing",
                      "bkt_ctx_kernel_times"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
@@ -179,6 +181,34 @@ def sgd_update(params, grads, lr: float, stream=None):
     _check(lib().bkt_sgd_update(ctypes.c_void_p(params.data_ptr()),
                                 ctypes.c_void_p(grads.data_ptr()), params.numel(),
                                 ctypes.c_float(lr), _stream_handle(stream)))
+
+
+def adadelta_update(params, grads, eg2, edx2, rho: float = 0.95, eps: float = 1e-6,
+                    lr: float = 1.0, stream=None):
+    """bkt_adadelta_update on four CUDA fp32 tensors of equal size (eg2 and
+    edx2 are the running averages, zero before the first update)."""
+    n = params.numel()
+    for t in (params, grads, eg2, edx2):
+        assert t.is_cuda and t.numel() == n
+    _check(lib().bkt_adadelta_update(ctypes.c_void_p(params.data_ptr()),
+                                     ctypes.c_void_p(grads.data_ptr()),
+                                     ctypes.c_void_p(eg2.data_ptr()),
+                                     ctypes.c_void_p(edx2.data_ptr()), n, ctypes.c_float(rho),
+                                     ctypes.c_float(eps), ctypes.c_float(lr),
+                                     _stream_handle(stream)))
+
+
+class Adadelta:
+    """ADADELTA state for one flat parameter tensor (Section III.B step 4)."""
+
+    def __init__(self, params, rho: float = 0.95, eps: float = 1e-6, lr: float = 1.0):
+        import torch
+        self.params, self.rho, self.eps, self.lr = params, rho, eps, lr
+        self.eg2 = torch.zeros_like(params)
+        self.edx2 = torch.zeros_like(params)
+
+    def step(self, grads, stream=None):
+        adadelta_update(self.params, grads, self.eg2, self.edx2, self.rho, self.eps, self.lr, stream)
 
 
 def _batch(lengths, x_offsets, label_lengths, label_offsets, x_ptr: int, labels_ptr: int):

@@ -962,6 +962,18 @@ extern "C" int bkt_ctx_sync_status(bkt_ctx *c) {
   return BKT_OK;
 }
 
+extern "C" int bkt_adadelta_update(float *params, const float *grads, float *eg2, float *edx2, int64_t n,
+                                   float rho, float eps, float lr, void *stream) {
+  if (n < 0 || (n > 0 && (!params || !grads || !eg2 || !edx2)))
+    return set_err(BKT_EINVAL, "bkt_adadelta_update: bad arguments");
+  if (!(rho >= 0.f && rho < 1.f) || !(eps > 0.f) || !(lr >= 0.f))
+    return set_err(BKT_EINVAL, "bkt_adadelta_update: need 0 <= rho < 1, eps > 0, lr >= 0");
+  if (n == 0) return BKT_OK;
+  cudaError_t e = bkt::launch_adadelta(params, grads, eg2, edx2, n, rho, eps, lr, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_err("adadelta kernel launch", e);
+  return BKT_OK;
+}
+
 extern "C" int bkt_sgd_update(float *params, const float *grads, int64_t n, float lr, void *stream) {
   if (n < 0 || (n > 0 && (!params || !grads))) return set_err(BKT_EINVAL, "bkt_sgd_update: bad arguments");
   if (n == 0) return BKT_OK;

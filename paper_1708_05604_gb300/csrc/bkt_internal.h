@@ -162,6 +162,9 @@ cudaError_t launch_lstm_cta(const RecArgs &a, int bc, bool bwd, cudaStream_t s);
 
 // a13
 cudaError_t launch_sgd(float *p, const float *g, int64_t n, float lr, cudaStream_t s);
+// a13, ADADELTA: see bkt_adadelta_update in bkt.h
+cudaError_t launch_adadelta(float *p, const float *g, float *eg2, float *edx2, int64_t n, float rho, float eps,
+                            float lr, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
 // Device buffers of one step (see the step engine in bkt_api.cpp).

@@ -1,0 +1,157 @@
+"""Multi-epoch training with per-epoch rebucketing and reshuffling.
+
+Section III.B step 3 rebuilds the buckets and reshuffles them every epoch;
+step 4 trains with ADADELTA (ref. [21]); Section IV.A holds out 5% of the
+sequences for validation and feeds shorter buckets first; Fig. 3 plots the
+validation loss against wall-clock time for several bucket counts Q and
+Fig. 4 the epoch time against Q.  This driver runs that loop on one GPU on
+a synthetic workload and reports, per epoch, the training time, the mean
+training loss and the mean validation loss per sequence.
+
+  python -m paper_1708_05604_gb300.train --workload lstm1_bi_h128 \\
+      --buckets 1,2,3,4,6 --epochs 3 [--optimizer adadelta|sgd]
+      [--batch-order ascending|descending|shuffle_buckets|shuffle_batches]
+
+Every step runs in the library (bkt_plan_buckets_ordered, bkt_lstm_ctc_step,
+bkt_adadelta_update / bkt_sgd_update); this module only sequences the calls.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import sys
+import time
+
+import numpy as np
+
+
+def split_validation(n: int, frac: float, seed: int):
+    """(train ids, validation ids): a seeded random `frac` of 0..n-1 held out
+    (at least one sequence when frac > 0), both sorted ascending."""
+    k = int(round(n * frac))
+    if frac > 0:
+        k = max(1, min(k, n - 1))
+    perm = np.random.default_rng(seed).permutation(n)
+    return np.sort(perm[k:]).astype(np.int64), np.sort(perm[:k]).astype(np.int64)
+
+
+def epoch_batches(lengths, train_ids, n_buckets: int, batch: int, seed: int, epoch: int,
+                  batch_order: str = "ascending"):
+    """The epoch's mini-batches as arrays of dataset ids: the plan is made on
+    the training sequences alone (their lengths in train_ids order)."""
+    from . import binding
+    lengths = np.asarray(lengths)
+    plan = binding.plan_buckets(lengths[train_ids], n_buckets, batch, seed, epoch, batch_order)
+    order, off = plan["order"], plan["batch_off"]
+    return [train_ids[order[off[k]:off[k + 1]]] for k in range(plan["n_batches"])], plan
+
+
+def validation_batches(lengths, val_ids, batch: int):
+    """Held-out sequences sorted by length (longest first), cut into batches."""
+    lengths = np.asarray(lengths)
+    o = val_ids[np.argsort(-lengths[val_ids], kind="stable")]
+    return [o[i:i + batch] for i in range(0, o.size, batch)]
+
+
+def train(workload: str, n_buckets: int, epochs: int, optimizer: str = "adadelta",
+          batch_order: str = "ascending", seed: int = 0, val_frac: float = 0.05,
+          lr: float | None = None, n_seqs: int | None = None, max_len: int | None = None,
+          params0=None, device: str = "cuda", log=None) -> dict:
+    """Trains `epochs` epochs; returns the per-epoch record and final params."""
+    import torch
+
+    from . import binding, build, synth
+
+    build.build()
+    w = synth.WORKLOADS[workload]
+    cfg = w.model_cfg()
+    ds = synth.make_workload(w, seed=seed, n_seqs=n_seqs, max_len=max_len)
+    train_ids, val_ids = split_validation(ds.n, val_frac, seed + 17)
+    P = binding.param_count(cfg)
+    if params0 is None:
+        params0 = synth.draw_params(np.random.default_rng(seed + 1), P)
+    dev = torch.device(device)
+    params = torch.from_numpy(np.ascontiguousarray(params0, np.float32)).to(dev)
+    grads = torch.zeros_like(params)
+    dd = binding.DeviceDataset(ds, device=dev)
+    cap = int(np.sort(ds.lengths)[-w.batch:].sum())
+    ctx = binding.Ctx(cfg, cap, w.batch, max(1, int(ds.label_lengths.max())))
+    loss = torch.zeros(ds.n, dtype=torch.float32, device=dev)
+    if optimizer == "adadelta":
+        opt = binding.Adadelta(params, lr=1.0 if lr is None else lr)
+        update = opt.step
+    elif optimizer == "sgd":
+        step_lr = 1e-3 if lr is None else lr
+        update = lambda g, stream=None: binding.sgd_update(params, g, step_lr, stream)
+    else:
+        raise ValueError(f"unknown optimizer {optimizer!r}")
+    stream = torch.cuda.current_stream(dev)
+    vbatches = validation_batches(ds.lengths, val_ids, w.batch)
+
+    def validate():
+        total = 0.0
+        for ids in vbatches:
+            lv = torch.zeros(ids.size, dtype=torch.float32, device=dev)
+            ctx.step(dd, ids, params, grads, lv, stream)
+            total += float(lv.double().sum())
+        return total / max(1, val_ids.size)
+
+    record = {"workload": workload, "n_buckets": n_buckets, "optimizer": optimizer,
+              "batch_order": batch_order, "n_train": int(train_ids.size),
+              "n_val": int(val_ids.size), "epochs": []}
+    wall = 0.0
+    v0 = validate()
+    ctx.sync_status()
+    record["val_loss_initial"] = v0
+    for e in range(epochs):
+        batches, plan = epoch_batches(ds.lengths, train_ids, n_buckets, w.batch, seed, e,
+                                      batch_order)
+        torch.cuda.synchronize(dev)
+        t0 = time.perf_counter()
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev0.record(stream)
+        pos = 0
+        for ids in batches:
+            lv = loss[pos:pos + ids.size]
+            ctx.step(dd, ids, params, grads, lv, stream)
+            update(grads, stream)
+            pos += ids.size
+        ev1.record(stream)
+        torch.cuda.synchronize(dev)
+        host_s = time.perf_counter() - t0
+        ms = ev0.elapsed_time(ev1)
+        ctx.sync_status()
+        wall += host_s
+        tl = float(loss[:pos].double().sum()) / max(1, pos)
+        vl = validate()
+        rec = {"epoch": e, "epoch_ms": ms, "host_s": host_s, "wall_s": wall,
+               "train_loss": tl, "val_loss": vl, "n_batches": plan["n_batches"],
+               "padded_efficiency": plan["unpadded_timesteps"] / plan["padded_timesteps"],
+               "timesteps": int(plan["unpadded_timesteps"])}
+        record["epochs"].append(rec)
+        if log:
+            log(rec)
+    record["params"] = params.cpu().numpy()
+    return record
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--workload", default="lstm1_bi_h128")
+    ap.add_argument("--buckets", default="1,2,3,4,6")
+    ap.add_argument("--epochs", type=int, default=3)
+    ap.add_argument("--optimizer", default="adadelta", choices=["adadelta", "sgd"])
+    ap.add_argument("--batch-order", default="ascending",
+                    choices=["ascending", "descending", "shuffle_buckets", "shuffle_batches"])
+    ap.add_argument("--lr", type=float, default=None)
+    ap.add_argument("--seed", type=int, default=0)
+    a = ap.parse_args(argv)
+    for Q in [int(q) for q in a.buckets.split(",") if q]:
+        r = train(a.workload, Q, a.epochs, a.optimizer, a.batch_order, a.seed, lr=a.lr)
+        r.pop("params")
+        print(json.dumps(r), flush=True)
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -8,6 +8,7 @@ import math
 import numpy as np
 import pytest
 
+import oracle
 from paper_1708_05604_gb300 import binding, synth
 
 from gpu_util import BF16_TOL, FP32_TOL, compare, gpu_step, oracle_step
@@ -153,6 +154,40 @@ def test_sgd_update():
     binding.sgd_update(tp[1:], tg[1:], 0.5)
     torch.cuda.synchronize()
     check(p[1:], g[1:], 0.5, tp[1:].cpu().numpy())
+
+
+def test_adadelta_update_vs_oracle():
+    """ADADELTA (ref. [21]) against the oracle, one update at a time from the
+    same fp32 state.  Error budget of the kernel's fp32 arithmetic, in units
+    u = 2^-24 of relative error: E[g^2] is an fma of a rounded product (2u);
+    dx takes two sums, two IEEE square roots, one IEEE division and one
+    product on top (<= 5u); E[dx^2] squares it (10u) and adds two roundings
+    (12u); the parameter moves by lr dx (5u of lr |dx|) plus one rounding of
+    the result.  Bounds used: 4u, 16u and 8u (|p| + lr |dx|)."""
+    import torch
+    rng = np.random.default_rng(3)
+    rho, eps, lr = 0.95, 1e-6, 1.0
+    u = 2.0 ** -24
+    for n, offset in ((1, 0), (7409, 0), (100003, 0), (5000, 1)):
+        p = torch.from_numpy(rng.standard_normal(n + offset).astype(np.float32)).cuda()[offset:]
+        a = torch.zeros(n + offset, device="cuda")[offset:]
+        b = torch.zeros(n + offset, device="cuda")[offset:]
+        for step in range(5):
+            g = torch.from_numpy((rng.standard_normal(n) * 10.0 ** rng.uniform(-3, 1)).astype(np.float32)).cuda()
+            p0, a0, b0, g0 = (t.cpu().numpy().astype(np.float64) for t in (p, a, b, g))
+            binding.adadelta_update(p, g, a, b, rho, eps, lr)
+            torch.cuda.synchronize()
+            xe, ae, be = oracle.adadelta(p0, g0, a0, b0, np.float32(rho), np.float32(eps), lr)
+            gx, ga, gb = (t.cpu().numpy().astype(np.float64) for t in (p, a, b))
+            dx = np.abs(xe - p0) / lr
+            assert np.all(np.abs(gx - xe) <= 8 * u * (np.abs(xe) + lr * dx) + 1e-37), (n, step)
+            assert np.all(np.abs(ga - ae) <= 4 * u * np.abs(ae) + 1e-37), (n, step)
+            assert np.all(np.abs(gb - be) <= 16 * u * np.abs(be) + 1e-37), (n, step)
+    # argument checks
+    t = torch.zeros(4, device="cuda")
+    for bad in ((1.0, 1e-6, 1.0), (0.9, 0.0, 1.0), (0.9, 1e-6, -1.0)):
+        with pytest.raises(binding.BktError):
+            binding.adadelta_update(t, t, t, t, *bad)
 
 
 def test_argument_errors():
