@@ -174,6 +174,24 @@ def roofline_for(name, launches, total_ms, work, peaks, peak_src, clocks):
             "algorithmic_flops_per_launch": per_launch, "avg_launch_ms": avg_s * 1e3}
 
 
+def recorded_traffic(kernel: str, workload: str, buckets: int):
+    """DRAM bytes per launch of `kernel` from the ncu record committed under
+    profiles/ for this workload, or None when there is none or the kernel's
+    source has changed since it was taken (sha256 of the source file)."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", f"traffic_{workload}.json")
+    try:
+        rec = json.load(open(path))
+        if rec.get("kernel") != kernel or int(rec.get("buckets", -1)) != buckets:
+            return None, None
+        src = open(os.path.join(ROOT, rec["source"]), "rb").read()
+        if hashlib.sha256(src).hexdigest() != rec.get("source_sha256"):
+            return None, None
+        return float(rec["dram_bytes_per_launch"]), os.path.relpath(path, ROOT)
+    except (OSError, ValueError, KeyError):
+        return None, None
+
+
 def kernel_work(cfg, plan, ds):
     """Algorithmic work per launch of the main kernels, averaged over the
     epoch's batches: name -> (kind, per-launch amount)."""
@@ -309,6 +327,9 @@ def run_native(args, world, rank, local):
         roof = roofline_for(name, n, t, work, peaks, peak_src, clk)
         if roof:
             roof["share_of_kernel_time"] = t / total_k
+            tb, tsrc = recorded_traffic(name, w.name, args.buckets)
+            roof["traffic"] = tb
+            roof["traffic_source"] = tsrc
             break
     kernel_table = [{"kernel": nm, "launches": n, "total_ms": round(t, 3),
                      "share": round(t / total_k, 4)} for nm, n, t in ktimes_sorted]
