@@ -54,6 +54,14 @@ __device__ __forceinline__ float lse2(float a, float b) {
 
 constexpr int kPre = 8;  // emission prefetch depth (steps)
 
+// Read-only global load issued where it is written: a volatile asm statement
+// keeps the compiler from sinking a prefetch next to its use kPre steps later.
+__device__ __forceinline__ float ld_prefetch(const float *p) {
+  float v;
+  asm volatile("ld.global.nc.f32 %0, [%1];" : "=f"(v) : "l"(p));
+  return v;
+}
+
 }  // namespace
 
 template <int SPT>
@@ -120,7 +128,7 @@ __global__ void __launch_bounds__(512) ctc_tables_kernel(DevIdx ix, const float 
   const float *lprow = logp + (int64_t)r * C;  // token (t, r) = tok_off[t] + r
   auto emis = [&](int step, int j) -> float {
     const int t = fwd ? step : L - 1 - step;
-    return __ldg(lprow + (int64_t)toff[t] * C + ext[j]);
+    return ld_prefetch(lprow + (int64_t)toff[t] * C + ext[j]);
   };
   const int d1 = fwd ? -1 : 1, d2 = fwd ? -2 : 2;
 
