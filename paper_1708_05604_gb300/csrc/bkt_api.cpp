@@ -391,12 +391,16 @@ size_t max_reduce_block(const Layout &lo) {
 }
 
 // Enqueues every kernel of one step (a4 gather .. a12) on `s`.
+// `side` (with its two events) is an optional second stream: the output
+// layer's weight gradient runs there, overlapping dY and the top layer's BPTT.
 int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepBufs &w, const bkt::RecGeom *geom,
                     const bkt::DevIdx &ix, const bkt_batch *bt, const float *params, float *grads, float *loss,
-                    cudaStream_t s, bkt::KernelTimer *timer, int sm_count) {
+                    cudaStream_t s, bkt::KernelTimer *timer, int sm_count, cudaStream_t side = nullptr,
+                    cudaEvent_t fork_ev = nullptr, cudaEvent_t join_ev = nullptr) {
   const int H = lo.H, dirs = lo.dirs, DH = dirs * H, C = lo.C, NT = ix.n_tok;
   const bool bf16 = cfg.gemm_precision == BKT_GEMM_BF16;
   Launch L{timer, s};
+  Launch Ls{timer, side ? side : s};
 
   // ---- a4: packed time-major input
   L.run("layout_gather", [&] { return bkt::launch_layout(ix, bt->x, lo.D0, w.X, w.tok_t, w.tok_r, w.prev_tok, s); });
@@ -504,11 +508,12 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
   // fp32 contractions over tokens on the tensor cores (3xTF32): the
   // token-major operands are transposed and split into hi + lo parts first
   const int NTq = (NT + 7) & ~7;
-  auto split_A = [&](const float *A, int64_t lda, int M) {
-    L.run("transpose_split", [&] { return bkt::launch_transpose_split(A, lda, nullptr, NT, M, w.AT, w.ATl, NTq, s); });
+  auto split_A_on = [&](Launch &X, const float *A, int64_t lda, int M) {
+    X.run("transpose_split", [&] { return bkt::launch_transpose_split(A, lda, nullptr, NT, M, w.AT, w.ATl, NTq, X.s); });
   };
-  auto tf32_reduce = [&](int M, const float *B, int64_t ldb, const int32_t *gather, int N, float *out) {
-    L.run("transpose_split", [&] { return bkt::launch_transpose_split(B, ldb, gather, NT, N, w.BTf, w.BTl, NTq, s); });
+  auto split_A = [&](const float *A, int64_t lda, int M) { split_A_on(L, A, lda, M); };
+  auto tf32_reduce_on = [&](Launch &X, int M, const float *B, int64_t ldb, const int32_t *gather, int N, float *out) {
+    X.run("transpose_split", [&] { return bkt::launch_transpose_split(B, ldb, gather, NT, N, w.BTf, w.BTl, NTq, X.s); });
     bkt::TcGemmArgs g{};
     g.M = M;
     g.N = N;
@@ -520,24 +525,39 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     g.P = w.part;
     g.splits = bkt::tf32x3_splits(M, N, NT, sm_count, w.part_floats);
     g.err = w.status;
-    L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.ATl, w.BTl, s); });
-    L.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, g.splits, M, N, out, s); });
+    X.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.ATl, w.BTl, X.s); });
+    X.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, g.splits, M, N, out, X.s); });
   };
-  auto bias_sum = [&](const float *A, int64_t lda, int M, float *out) {
+  auto tf32_reduce = [&](int M, const float *B, int64_t ldb, const int32_t *gather, int N, float *out) {
+    tf32_reduce_on(L, M, B, ldb, gather, N, out);
+  };
+  auto bias_sum_on = [&](Launch &X, const float *A, int64_t lda, int M, float *out) {
     const int splits = bkt::colsum_splits(NT, M, w.part_floats);
-    L.run("colsum", [&] { return bkt::launch_colsum(A, lda, NT, M, w.part, splits, s); });
-    L.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, splits, 1, M, out, s); });
+    X.run("colsum", [&] { return bkt::launch_colsum(A, lda, NT, M, w.part, splits, X.s); });
+    X.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, splits, 1, M, out, X.s); });
   };
+  auto bias_sum = [&](const float *A, int64_t lda, int M, float *out) { bias_sum_on(L, A, lda, M, out); };
   // [dW_ih | db] of the first layer: dz^T [X | 1] with X of in_dim columns
   auto narrow = [&](const float *dZ, const float *X, int D, float *ow, float *ob) {
     L.run("narrow_wgrad", [&] {
       return bkt::launch_narrow_wgrad(dZ, 4 * H, 4 * H, X, D, NT, w.part, w.part_floats, sm_count, ow, ob, s);
     });
   };
-  // [dW_out | db_out] = dlogit^T [Y | 1]
-  split_A(w.logit, C, C);
-  tf32_reduce(C, Ytop, DH, nullptr, DH, grads + lo.w_out);
-  bias_sum(w.logit, C, C, grads + lo.b_out);
+  // [dW_out | db_out] = dlogit^T [Y | 1]; with a side stream it overlaps dY
+  // and the top layer's BPTT, and is joined before the weight-gradient
+  // section reuses AT, BT and the partial-sum buffer
+  if (side) {
+    cudaError_t e = cudaEventRecord(fork_ev, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(side, fork_ev, 0);
+    if (e != cudaSuccess) return cuda_err("fork to the side stream", e);
+  }
+  split_A_on(Ls, w.logit, C, C);
+  tf32_reduce_on(Ls, C, Ytop, DH, nullptr, DH, grads + lo.w_out);
+  bias_sum_on(Ls, w.logit, C, C, grads + lo.b_out);
+  if (side) {
+    cudaError_t e = cudaEventRecord(join_ev, side);
+    if (e != cudaSuccess) return cuda_err("cudaEventRecord(join)", e);
+  }
   {
     // dY = dlogit W_out on the tensor cores: dlogit split with its rows padded
     // to a multiple of 4 floats (TMA strides), W_out split transposed
@@ -575,6 +595,10 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     ra.status = w.status;
     ra.dY = w.dY;
     L.run("lstm_bwd", [&] { return bkt::launch_lstm_bwd(ra, geom[l], s); });
+    if (side && l == lo.L - 1) {
+      cudaError_t e = cudaStreamWaitEvent(s, join_ev, 0);
+      if (e != cudaSuccess) return cuda_err("join the side stream", e);
+    }
     const int D = lo.D(l);
     const float *Xl = (l == 0) ? w.X : w.Y[l - 1];
     if (bf16) {
@@ -676,6 +700,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     }
   }
   if (L.failed) return cuda_err(L.failed, L.err);
+  if (Ls.failed) return cuda_err(Ls.failed, Ls.err);
   return BKT_OK;
 }
 
@@ -772,10 +797,15 @@ struct bkt_ctx {
   bool stage_used[kStageSlots] = {};
   int stage_next = 0;
   cudaStream_t last_stream = nullptr;
+  cudaStream_t side = nullptr;  // output-layer weight gradient overlaps BPTT here
+  cudaEvent_t fork_ev = nullptr, join_ev = nullptr;
   EventTimer timer;
   bkt::RecGeom geom[bkt::kMaxLayers] = {};
 
   ~bkt_ctx() {
+    if (fork_ev) cudaEventDestroy(fork_ev);
+    if (join_ev) cudaEventDestroy(join_ev);
+    if (side) cudaStreamDestroy(side);
     for (int i = 0; i < kStageSlots; ++i)
       if (stage_ev[i]) cudaEventDestroy(stage_ev[i]);
     if (stage) cudaFreeHost(stage);
@@ -907,6 +937,15 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
       return cuda_err("cudaEventCreate", e);
     }
   }
+  {
+    cudaError_t e2 = cudaStreamCreateWithFlags(&c->side, cudaStreamNonBlocking);
+    if (e2 == cudaSuccess) e2 = cudaEventCreateWithFlags(&c->fork_ev, cudaEventDisableTiming);
+    if (e2 == cudaSuccess) e2 = cudaEventCreateWithFlags(&c->join_ev, cudaEventDisableTiming);
+    if (e2 != cudaSuccess) {
+      delete c;
+      return cuda_err("side stream", e2);
+    }
+  }
   for (int l = 0; l < lo.L; ++l) c->geom[l] = bkt::plan_recurrent(lo.H, max_batch, lo.dirs, c->sm_count);
   *out = c;
   return BKT_OK;
@@ -1019,7 +1058,7 @@ extern "C" int bkt_lstm_ctc_step(bkt_ctx *c, const bkt_batch *bt, const float *p
   c->stage_used[slot] = true;
   c->last_stream = s;
   return enqueue_kernels(c->cfg, c->lo, c->w, c->geom, ix, bt, params, grads, loss, s,
-                         c->timer.on ? &c->timer : nullptr, c->sm_count);
+                         c->timer.on ? &c->timer : nullptr, c->sm_count, c->side, c->fork_ev, c->join_ev);
 }
 
 // ---------------------------------------------------------------------------
