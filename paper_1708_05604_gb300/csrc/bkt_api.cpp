@@ -511,7 +511,6 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
   auto split_A_on = [&](Launch &X, const float *A, int64_t lda, int M) {
     X.run("transpose_split", [&] { return bkt::launch_transpose_split(A, lda, nullptr, NT, M, w.AT, w.ATl, NTq, X.s); });
   };
-  auto split_A = [&](const float *A, int64_t lda, int M) { split_A_on(L, A, lda, M); };
   auto tf32_reduce_on = [&](Launch &X, int M, const float *B, int64_t ldb, const int32_t *gather, int N, float *out) {
     X.run("transpose_split", [&] { return bkt::launch_transpose_split(B, ldb, gather, NT, N, w.BTf, w.BTl, NTq, X.s); });
     bkt::TcGemmArgs g{};
@@ -528,24 +527,14 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     X.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.ATl, w.BTl, X.s); });
     X.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, g.splits, M, N, out, X.s); });
   };
-  auto tf32_reduce = [&](int M, const float *B, int64_t ldb, const int32_t *gather, int N, float *out) {
-    tf32_reduce_on(L, M, B, ldb, gather, N, out);
-  };
   auto bias_sum_on = [&](Launch &X, const float *A, int64_t lda, int M, float *out) {
     const int splits = bkt::colsum_splits(NT, M, w.part_floats);
     X.run("colsum", [&] { return bkt::launch_colsum(A, lda, NT, M, w.part, splits, X.s); });
     X.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, splits, 1, M, out, X.s); });
   };
-  auto bias_sum = [&](const float *A, int64_t lda, int M, float *out) { bias_sum_on(L, A, lda, M, out); };
-  // [dW_ih | db] of the first layer: dz^T [X | 1] with X of in_dim columns
-  auto narrow = [&](const float *dZ, const float *X, int D, float *ow, float *ob) {
-    L.run("narrow_wgrad", [&] {
-      return bkt::launch_narrow_wgrad(dZ, 4 * H, 4 * H, X, D, NT, w.part, w.part_floats, sm_count, ow, ob, s);
-    });
-  };
   // [dW_out | db_out] = dlogit^T [Y | 1]; with a side stream it overlaps dY
-  // and the top layer's BPTT, and is joined before the weight-gradient
-  // section reuses AT, BT and the partial-sum buffer
+  // and the top layer's BPTT (the side stream runs all weight gradients in
+  // order and is joined at the end of the step)
   if (side) {
     cudaError_t e = cudaEventRecord(fork_ev, s);
     if (e == cudaSuccess) e = cudaStreamWaitEvent(side, fork_ev, 0);
@@ -554,10 +543,6 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
   split_A_on(Ls, w.logit, C, C);
   tf32_reduce_on(Ls, C, Ytop, DH, nullptr, DH, grads + lo.w_out);
   bias_sum_on(Ls, w.logit, C, C, grads + lo.b_out);
-  if (side) {
-    cudaError_t e = cudaEventRecord(join_ev, side);
-    if (e != cudaSuccess) return cuda_err("cudaEventRecord(join)", e);
-  }
   {
     // dY = dlogit W_out on the tensor cores: dlogit split with its rows padded
     // to a multiple of 4 floats (TMA strides), W_out split transposed
@@ -580,7 +565,16 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.Ll, w.Wl, s); });
   }
 
-  // ---- a11, a12: BPTT and weight gradients, top layer first
+  // ---- a11, a12: BPTT and weight gradients, top layer first.  With a side
+  // stream, a layer's weight gradients run there (after its BPTT) while the
+  // main stream goes on with dX and the BPTT of the layer below; the side
+  // stream's scratch (AT, BT, part) is its own, dX uses separate buffers.
+  auto fork_to_side = [&]() -> int {
+    if (!side) return BKT_OK;
+    cudaError_t e = cudaEventRecord(fork_ev, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(side, fork_ev, 0);
+    return e == cudaSuccess ? BKT_OK : cuda_err("fork to the side stream", e);
+  };
   for (int l = lo.L - 1; l >= 0; --l) {
     bkt::RecArgs ra{};
     ra.ix = ix;
@@ -595,12 +589,15 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     ra.status = w.status;
     ra.dY = w.dY;
     L.run("lstm_bwd", [&] { return bkt::launch_lstm_bwd(ra, geom[l], s); });
-    if (side && l == lo.L - 1) {
-      cudaError_t e = cudaStreamWaitEvent(s, join_ev, 0);
-      if (e != cudaSuccess) return cuda_err("join the side stream", e);
-    }
+    if (int rc = fork_to_side()) return rc;
+    Launch &X = Ls;  // the weight gradients of layer l
     const int D = lo.D(l);
     const float *Xl = (l == 0) ? w.X : w.Y[l - 1];
+    auto narrow_on = [&](const float *dZ, float *ow, float *ob) {
+      X.run("narrow_wgrad", [&] {
+        return bkt::launch_narrow_wgrad(dZ, 4 * H, 4 * H, Xl, D, NT, w.part, w.part_floats, sm_count, ow, ob, X.s);
+      });
+    };
     if (bf16) {
       const int NTp = (NT + 7) & ~7;
       auto tc_reduce = [&](const void *B, int N, float *out) {
@@ -615,24 +612,24 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         g.P = w.part;
         g.splits = bkt::tc_splits(g.M, g.N, NT, sm_count, w.part_floats);
         g.err = w.status;
-        L.run("gemm_tc", [&] { return bkt::launch_gemm_bf16_tc(g, s); });
-        L.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, g.splits, g.M, g.N, out, s); });
+        X.run("gemm_tc", [&] { return bkt::launch_gemm_bf16_tc(g, X.s); });
+        X.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, g.splits, g.M, g.N, out, X.s); });
       };
       for (int d = 0; d < dirs; ++d) {
         const float *dZ = w.Z[l * dirs + d];
         // dW_hh = dz^T h_{t-1} on the tensor cores (both operands transposed to bf16)
-        L.run("transpose_bf16", [&] { return bkt::launch_transpose_bf16(dZ, 4 * H, nullptr, NT, 4 * H, w.dZT, NTp, s); });
-        L.run("transpose_bf16", [&] {
-          return bkt::launch_transpose_bf16(w.Y[l] + d * H, DH, w.prev_tok[d], NT, H, w.BT, NTp, s);
+        X.run("transpose_bf16", [&] { return bkt::launch_transpose_bf16(dZ, 4 * H, nullptr, NT, 4 * H, w.dZT, NTp, X.s); });
+        X.run("transpose_bf16", [&] {
+          return bkt::launch_transpose_bf16(w.Y[l] + d * H, DH, w.prev_tok[d], NT, H, w.BT, NTp, X.s);
         });
         tc_reduce(w.BT, H, grads + lo.w_hh(l, d));
         if (l == 0) {
           // narrow input: [dW_ih | db] = dz^T [X | 1] in fp32
-          narrow(dZ, Xl, D, grads + lo.w_ih[l * dirs + d], grads + lo.bias(l, d));
+          narrow_on(dZ, grads + lo.w_ih[l * dirs + d], grads + lo.bias(l, d));
         } else {
-          L.run("transpose_bf16", [&] { return bkt::launch_transpose_bf16(Xl, D, nullptr, NT, D, w.BT, NTp, s); });
+          X.run("transpose_bf16", [&] { return bkt::launch_transpose_bf16(Xl, D, nullptr, NT, D, w.BT, NTp, X.s); });
           tc_reduce(w.BT, D, grads + lo.w_ih[l * dirs + d]);
-          bias_sum(dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
+          bias_sum_on(X, dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
         }
       }
     } else {
@@ -640,14 +637,14 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         // dW_hh = dz^T h_{t-1}; h_{t-1} of token (t, r) is the row's previous
         // token in its direction (zeros at the start)
         const float *dZ = w.Z[l * dirs + d];
-        split_A(dZ, 4 * H, 4 * H);
-        tf32_reduce(4 * H, w.Y[l] + d * H, DH, w.prev_tok[d], H, grads + lo.w_hh(l, d));
+        split_A_on(X, dZ, 4 * H, 4 * H);
+        tf32_reduce_on(X, 4 * H, w.Y[l] + d * H, DH, w.prev_tok[d], H, grads + lo.w_hh(l, d));
         if (l == 0) {
-          // narrow input: [dW_ih | db] = dz^T [X | 1] on the FMA pipe
-          narrow(dZ, Xl, D, grads + lo.w_ih[l * dirs + d], grads + lo.bias(l, d));
+          // narrow input: [dW_ih | db] = dz^T [X | 1] streamed over dz
+          narrow_on(dZ, grads + lo.w_ih[l * dirs + d], grads + lo.bias(l, d));
         } else {
-          tf32_reduce(4 * H, Xl, D, nullptr, D, grads + lo.w_ih[l * dirs + d]);
-          bias_sum(dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
+          tf32_reduce_on(X, 4 * H, Xl, D, nullptr, D, grads + lo.w_ih[l * dirs + d]);
+          bias_sum_on(X, dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
         }
       }
     }
@@ -675,9 +672,11 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     } else if (l > 0) {
       // dX = dz W_ih in fp32 on the tensor cores (3xTF32): dz rows are
       // K-contiguous already, W_ih is transposed while it is split
+      float *dxa = w.DXh ? w.DXh : w.AT, *dxl = w.DXl ? w.DXl : w.ATl;
+      if (side && !w.DXh) return set_err(BKT_EINVAL, "internal: dX buffers missing for the side stream");
       for (int d = 0; d < dirs; ++d) {
         L.run("split_rows", [&] {
-          return bkt::launch_split_rows(w.Z[l * dirs + d], 4 * H, NT, 4 * H, w.AT, w.ATl, 4 * H, s);
+          return bkt::launch_split_rows(w.Z[l * dirs + d], 4 * H, NT, 4 * H, dxa, dxl, 4 * H, s);
         });
         L.run("transpose_split", [&] {
           return bkt::launch_transpose_split(params + lo.w_ih[l * dirs + d], DH, nullptr, 4 * H, DH, w.Wh, w.Wl,
@@ -687,7 +686,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         g.M = NT;
         g.N = DH;
         g.K = 4 * H;
-        g.A = w.AT;
+        g.A = dxa;
         g.lda = 4 * H;
         g.B = w.Wh;
         g.ldb = 4 * H;
@@ -695,9 +694,14 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         g.ldd = DH;
         g.accumulate = d > 0;
         g.err = w.status;
-        L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.ATl, w.Wl, s); });
+        L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, dxl, w.Wl, s); });
       }
     }
+  }
+  if (side) {  // every gradient is written before the step's work on `s` ends
+    cudaError_t e = cudaEventRecord(join_ev, side);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s, join_ev, 0);
+    if (e != cudaSuccess) return cuda_err("join the side stream", e);
   }
   if (L.failed) return cuda_err(L.failed, L.err);
   if (Ls.failed) return cuda_err(Ls.failed, Ls.err);
@@ -895,6 +899,10 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
     const size_t WW = std::max(Cp * DHp, (lo.L > 1 && cfg->gemm_precision != BKT_GEMM_BF16) ? 4 * (size_t)H * DHp : 0);
     BKT_ALLOC(w.Wh, WW);
     BKT_ALLOC(w.Wl, WW);
+    if (lo.L > 1 && cfg->gemm_precision != BKT_GEMM_BF16) {  // dX operands beside the side stream's AT
+      BKT_ALLOC(w.DXh, NT * 4 * (size_t)H);
+      BKT_ALLOC(w.DXl, NT * 4 * (size_t)H);
+    }
   }
   if (cfg->gemm_precision == BKT_GEMM_BF16) {
     const size_t NTp = (NT + 7) & ~size_t(7);

@@ -175,6 +175,7 @@ struct StepBufs {
   float *Z[2 * kMaxLayers];                   // per layer*dirs+dir: Zx / gates / dz [NT x 4H]
   float *Cst[2 * kMaxLayers];                 // cell states [NT x H]
   float *logit;                               // log-probabilities / dlogit [NT x C]
+  float *DXh, *DXl;                           // split dz for dX while the side stream holds AT (or null)
   float *alpha, *beta;                        // CTC tables, sum_i L_i (2 U_i + 1) each
   float *dY;                                  // dloss/dY of the current layer [NT x dirs*H]
   float *part;                                // split-K partial sums
