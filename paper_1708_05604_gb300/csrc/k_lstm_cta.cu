@@ -310,10 +310,16 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
   }
   for (int s = Tg - 1; s >= 0; --s) {
     cp_wait_all_but_newest();
-    // phase B: dz of unit j from dh = dY + recurrent part
+    // phase B: dz of unit j from dh = dY + recurrent part.  The prefetch of
+    // step s - kPF is issued for every row, active or not: steps run
+    // backwards, so a shorter row becomes active only later and needs its
+    // first kPF steps in flight by then.
 #pragma unroll
     for (int b = 0; b < BC; ++b) {
-      if (s >= len[b]) continue;  // uniform over the CTA
+      if (s >= len[b]) {  // uniform over the CTA
+        issue(b, s - kPF);
+        continue;
+      }
       float dh_rec = 0.f;
       if (s + 1 < len[b]) {
         const float *rp = red + (size_t)b * NW * H + unit;

@@ -71,6 +71,51 @@ def test_step_parity_odd_shapes(layers, bi, H):
     compare(cfg, lg, gg, lo, go, FP32_TOL)
 
 
+def _ctx_for(cfg, ds, max_batch):
+    """A ctx sized for `max_batch` rows: its recurrent geometry is planned for
+    that many rows, so a small batch runs the wide-batch kernel variant."""
+    return binding.Ctx(cfg, max(int(ds.lengths.sum()), 64 * max_batch), max_batch,
+                       max(1, int(ds.label_lengths.max())))
+
+
+@pytest.mark.parametrize("wname,lengths,max_batch", [
+    # 8 rows per 4-CTA cluster, rows ending at different steps, a partial second group
+    ("lstm3_bi_h256_bf16", [26, 24, 21, 21, 17, 12, 9, 7, 5, 3, 2], 128),
+    # 8 rows per 16-CTA cluster
+    ("lstm2_uni_h512", [22, 20, 19, 14, 11, 8, 6, 4, 2, 1], 32),
+    # two rows per single-CTA block (rows x directions > SMs)
+    ("lstm1_bi_h128", [45, 44, 30, 30, 22, 13, 8, 3, 1], 100),
+    ("lstm1_uni_h32", [40, 33, 20, 12, 6, 2, 1], 200),
+])
+def test_step_parity_wide_batch_kernels(wname, lengths, max_batch):
+    """Element-wise parity of the kernel variants that full-size batches use,
+    on oracle-sized batches (fp32 contractions, so the 1e-4 bound applies)."""
+    w = synth.WORKLOADS[wname]
+    rng = np.random.default_rng(4)
+    ds = synth.make_dataset(lengths, 4, rng)
+    cfg = dict(w.model_cfg(), gemm_bf16=False)
+    params = synth.draw_params(rng, binding.param_count(cfg))
+    ctx = _ctx_for(cfg, ds, max_batch)
+    lg, gg = gpu_step(cfg, ds, params, ctx=ctx)
+    lo, go = oracle_step(cfg, ds, params)
+    compare(cfg, lg, gg, lo, go, FP32_TOL)
+
+
+@pytest.mark.parametrize("H", [32, 256])
+def test_step_parity_longer_than_shared_time_index(H):
+    """A sequence longer than the 8,192 time offsets the recurrent kernels
+    stage in shared memory (they then read them from global memory), with a
+    long label (CTC with four extended-label positions per thread)."""
+    cfg = {"n_layers": 1, "bidirectional": H == 32, "in_dim": 4, "hidden": H, "n_classes": 81,
+           "blank": 0}
+    rng = np.random.default_rng(8)
+    ds = synth.make_dataset([8300, 37, 5], 10, rng)
+    params = synth.draw_params(rng, binding.param_count(cfg))
+    lg, gg = gpu_step(cfg, ds, params)
+    lo, go = oracle_step(cfg, ds, params)
+    compare(cfg, lg, gg, lo, go, FP32_TOL)
+
+
 def test_edge_cases_one_step():
     """Length-1 sequence, empty label, repeated labels, no alignment, equal lengths."""
     cfg = synth.WORKLOADS["lstm1_bi_h128"].model_cfg()
