@@ -15,7 +15,17 @@ import pytest
 pytestmark = pytest.mark.gpu
 
 
-def test_static_step_matches_ctx_step(cuda_device):
+STATIC_CASES = [
+    ("lstm1_bi_h128", None, 180),
+    # two fp32 layers: dX on the tensor cores shares scratch with the weight
+    # gradients here, while the ctx path runs them on two streams
+    ("lstm1_bi_h128", {"n_layers": 2, "hidden": 64}, 120),
+    ("lstm3_bi_h256_bf16", None, 50),
+]
+
+
+@pytest.mark.parametrize("wname,override,max_len", STATIC_CASES)
+def test_static_step_matches_ctx_step(cuda_device, wname, override, max_len):
     import torch
 
     from paper_1708_05604_gb300 import binding, build, synth
@@ -23,9 +33,9 @@ def test_static_step_matches_ctx_step(cuda_device):
     from gpu_util import FP32_TOL, compare, gpu_step
 
     build.build()
-    w = synth.WORKLOADS["lstm1_bi_h128"]
-    cfg = w.model_cfg()
-    ds = synth.make_workload(w, seed=4, n_seqs=14, max_len=180)
+    w = synth.WORKLOADS[wname]
+    cfg = dict(w.model_cfg(), **(override or {}))
+    ds = synth.make_workload(w, seed=4, n_seqs=14, max_len=max_len)
     params_np = synth.draw_params(np.random.default_rng(8), binding.param_count(cfg))
     dd = binding.DeviceDataset(ds)
     params = torch.from_numpy(params_np).cuda()
