@@ -593,9 +593,15 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     Launch &X = Ls;  // the weight gradients of layer l
     const int D = lo.D(l);
     const float *Xl = (l == 0) ? w.X : w.Y[l - 1];
+    // layer 1's narrow [dW_ih | db] goes to the main stream (own partials)
+    // when it has nothing else left, beside the side stream's dW_hh work
+    const bool narrow_main = side && l == 0 && w.part2;
     auto narrow_on = [&](const float *dZ, float *ow, float *ob) {
-      X.run("narrow_wgrad", [&] {
-        return bkt::launch_narrow_wgrad(dZ, 4 * H, 4 * H, Xl, D, NT, w.part, w.part_floats, sm_count, ow, ob, X.s);
+      Launch &Y = narrow_main ? L : X;
+      float *P = narrow_main ? w.part2 : w.part;
+      const size_t PF = narrow_main ? w.part2_floats : w.part_floats;
+      Y.run("narrow_wgrad", [&] {
+        return bkt::launch_narrow_wgrad(dZ, 4 * H, 4 * H, Xl, D, NT, P, PF, sm_count, ow, ob, Y.s);
       });
     };
     if (bf16) {
@@ -903,6 +909,9 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
       BKT_ALLOC(w.DXh, NT * 4 * (size_t)H);
       BKT_ALLOC(w.DXl, NT * 4 * (size_t)H);
     }
+    // layer 1's narrow weight gradient: up to 1024 token chunks of 4H x (in_dim+1) partials
+    w.part2_floats = (size_t)1024 * 4 * H * (cfg->in_dim + 1);
+    BKT_ALLOC(w.part2, w.part2_floats);
   }
   if (cfg->gemm_precision == BKT_GEMM_BF16) {
     const size_t NTp = (NT + 7) & ~size_t(7);

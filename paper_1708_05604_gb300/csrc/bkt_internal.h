@@ -176,6 +176,8 @@ struct StepBufs {
   float *Cst[2 * kMaxLayers];                 // cell states [NT x H]
   float *logit;                               // log-probabilities / dlogit [NT x C]
   float *DXh, *DXl;                           // split dz for dX while the side stream holds AT (or null)
+  float *part2;                               // partials of layer 1's narrow weight gradient on the main stream (or null)
+  size_t part2_floats;
   float *alpha, *beta;                        // CTC tables, sum_i L_i (2 U_i + 1) each
   float *dY;                                  // dloss/dY of the current layer [NT x dirs*H]
   float *part;                                // split-K partial sums
