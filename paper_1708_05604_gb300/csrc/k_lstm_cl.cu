@@ -44,6 +44,10 @@ namespace bkt {
 namespace {
 
 constexpr int kClThreads = 256;
+#ifndef BKT_CL_FWD_REG_COLS
+#define BKT_CL_FWD_REG_COLS 32
+#endif
+constexpr int kClFwdRegCols = BKT_CL_FWD_REG_COLS;  // multiple of 4, at most 64
 constexpr int kClTokCap = 8192;  // time offsets staged in shared memory up to this T
 constexpr int kClPolls = 1 << 22;
 constexpr int32_t kErrExchange = 4;
@@ -142,9 +146,8 @@ struct ClGeom {
   static_assert(Hc * KS == kClThreads && (H / 4) * RSL == kClThreads, "256 threads per CTA");
   static_assert(Hc % 4 == 0 && BH % 4 == 0 && BC == BH * NH, "float4 exchange");
   static constexpr int PPT = (Hc * BH + kClThreads - 1) / kClThreads;  // BPTT pairs per thread and half
-  static size_t fwd_floats() {
-    return (size_t)8 * 4 * kClThreads * 4 + 2 * NH * BH * (HPAD + Hc);
-  }
+  static constexpr int RKF = kClFwdRegCols;   // forward: W columns of a 64-column slice kept in registers
+  static size_t fwd_floats() { return (size_t)(64 - RKF) * 4 * kClThreads + 2 * NH * BH * (HPAD + Hc); }
   static size_t bwd_floats() {
     return (size_t)32 * kClThreads * 4 + 2 * NH * (DZS + (size_t)CS * BH * Hc) + (size_t)2 * NH * kClThreads * PPT * 8;
   }
@@ -166,8 +169,9 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_fwd_cl_kernel(RecArgs a) {
   constexpr int RPL = NPL >= 4 ? NPL / 4 : 1;  // rows of a half finished per lane
   constexpr int SEND4 = BH * Hc / 4;           // float4 sent to each CTA per half and step
   extern __shared__ __align__(16) float sm[];
-  float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [8][4][NTH] columns 32..63 of each slice
-  float *hb = sm + 8 * 4 * NTH * 4;              // [NH][2][BH][HPAD] received h
+  constexpr int RK = Gm::RKF, SK4 = (64 - RK) / 4;  // register columns, shared float4 columns
+  float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [SK4][4][NTH] columns RK..63 of each slice
+  float *hb = sm + SK4 * 4 * NTH * 4;            // [NH][2][BH][HPAD] received h
   float *stg = hb + 2 * NH * BH * HPAD;          // [NH][2][BH][Hc] this CTA's h slice
   uint64_t *mb = reinterpret_cast<uint64_t *>(stg + 2 * NH * BH * Hc);  // [NH][2]
   int *toff_s = reinterpret_cast<int *>(mb + 2 * NH);
@@ -185,15 +189,15 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_fwd_cl_kernel(RecArgs a) {
   const int DH = a.dirs * H;
   const float *__restrict__ Whh = a.Whh[d];
 
-  float w[4][32];
+  float w[4][RK];
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     const float *row = Whh + (size_t)(q * H + gu) * H + kb;
 #pragma unroll
-    for (int k = 0; k < 32; ++k) w[q][k] = __ldg(row + k);
+    for (int k = 0; k < RK; ++k) w[q][k] = __ldg(row + k);
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const float *p = row + 32 + 4 * j;
+    for (int j = 0; j < SK4; ++j) {
+      const float *p = row + RK + 4 * j;
       Ws4[(j * 4 + q) * NTH + t] = make_float4(__ldg(p), __ldg(p + 1), __ldg(p + 2), __ldg(p + 3));
     }
   }
@@ -266,7 +270,7 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_fwd_cl_kernel(RecArgs a) {
         if (t == 0 && e + 2 <= Tg - 2) mbar_arm(smem_addr(&mb[2 * h + (e & 1)]), Gm::kXBytes);
         const float *hv = hb + (2 * h + (e & 1)) * BH * HPAD + kb + 4 * kl;
 #pragma unroll
-        for (int k4 = 0; k4 < 8; ++k4) {
+        for (int k4 = 0; k4 < RK / 4; ++k4) {
 #pragma unroll
           for (int b = 0; b < BH; ++b) {
             const float4 h4 = *reinterpret_cast<const float4 *>(hv + b * HPAD + 4 * k4);
@@ -280,13 +284,13 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_fwd_cl_kernel(RecArgs a) {
           }
         }
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
+        for (int j = 0; j < SK4; ++j) {
           float4 wv[4];
 #pragma unroll
           for (int q = 0; q < 4; ++q) wv[q] = Ws4[(j * 4 + q) * NTH + t];
 #pragma unroll
           for (int b = 0; b < BH; ++b) {
-            const float4 h4 = *reinterpret_cast<const float4 *>(hv + b * HPAD + 32 + 4 * j);
+            const float4 h4 = *reinterpret_cast<const float4 *>(hv + b * HPAD + RK + 4 * j);
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
               float x = fmaf(wv[q].x, h4.x, acc[b * 4 + q]);
