@@ -51,17 +51,20 @@ constexpr int kRing = kPF + 1; // ring slots: a copy never lands in the slot rea
 __device__ __forceinline__ float sigm(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
 __device__ __forceinline__ float tanh_g(float x) { return 1.f - __fdividef(2.f, 1.f + __expf(2.f * x)); }
 
-// Per-thread asynchronous copies (global -> shared) for the step inputs:
-// one commit group per step, so waiting for all but the newest kPF-1 groups
-// makes the oldest step's values visible to the issuing thread.
-__device__ __forceinline__ void cp_async4(float *dst, const float *src) {
-  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
+// The step inputs are whole rows (Zx or gates, cell states, dY), copied to a
+// shared-memory ring in 16-byte asynchronous pieces by all threads together:
+// one commit group per step.  A thread reads pieces other threads copied, so
+// a step's group is completed one step early (wait_group kPF-2 at the top of
+// the previous step) and published by that step's closing barrier.
+__device__ __forceinline__ void cp_async16(float *dst, const float *src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
                "l"(src)
                : "memory");
 }
 __device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void cp_wait_all_but_newest() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(kPF - 1) : "memory");
+template <int N>
+__device__ __forceinline__ void cp_wait_pending() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
 // Reduce-scatter over the 8 lanes of a k-slice group (lane bits 0..2): on
@@ -114,10 +117,10 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
   extern __shared__ __align__(16) float sm[];
   float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [SKK/4][16][NTH]
   float *hs = sm + SKK * 16 * NTH;               // [2][BC][8 slices][HS]
-  float *zr = hs + 2 * BC * 8 * HS;              // [BC][kRing][2][NTH] Zx of upcoming steps (value-major: no bank conflicts)
+  float *zr = hs + 2 * BC * 8 * HS;              // [BC][kRing][4H] Zx rows of upcoming steps
   const int T = a.ix.T;
   const bool toff_sm = T + 1 <= kTokCap;
-  int *toff_s = reinterpret_cast<int *>(zr + BC * kRing * NTH * 2);
+  int *toff_s = reinterpret_cast<int *>(zr + BC * kRing * G);
   const int *toff = toff_sm ? toff_s : a.ix.tok_off;
   const int t = threadIdx.x, lane = t & 31;
   const int ks = lane & 7, rg = (t >> 5) * 4 + (lane >> 3);
@@ -161,12 +164,11 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
     return toff[tt] + r0 + b;
   };
   float cst[BC];
-  auto issue = [&](int b, int s) {  // Zx of step s of row b into its ring slot
+  auto issue = [&](int b, int s) {  // the Zx row of step s of row b into its ring slot
     if (s < len[b]) {
-      const int tk = tok_at(b, s);
-      float *slot = zr + ((size_t)b * kRing + s % kRing) * 2 * NTH + t;
-      cp_async4(slot, Z + (size_t)tk * G + zo0);
-      cp_async4(slot + NTH, Z + (size_t)tk * G + zo1);
+      const float *src = Z + (size_t)tok_at(b, s) * G;
+      float *slot = zr + ((size_t)b * kRing + s % kRing) * G;
+      for (int i = t; i < G / 4; i += NTH) cp_async16(slot + 4 * i, src + 4 * i);
     }
   };
 #pragma unroll
@@ -176,14 +178,16 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
     for (int b = 0; b < BC; ++b) issue(b, j);
     cp_commit();
   }
+  cp_wait_pending<kPF - 1>();  // step 0's rows
+  __syncthreads();
   for (int s = 0; s < Tg; ++s) {
     const int p = s & 1;
-    cp_wait_all_but_newest();
+    cp_wait_pending<kPF - 2>();  // step s + 1's rows, published by this step's barrier
 #pragma unroll
     for (int b = 0; b < BC; ++b) {
       if (s >= len[b]) continue;  // uniform over the CTA
-      const float *slot = zr + ((size_t)b * kRing + s % kRing) * 2 * NTH + t;
-      const float zc0 = slot[0], zc1 = slot[NTH];
+      const float *slot = zr + ((size_t)b * kRing + s % kRing) * G;
+      const float zc0 = slot[zo0], zc1 = slot[zo1];
       const int tc = tok_at(b, s);
       issue(b, s + kPF);
       const float *hv = hs + (p * BC + b) * 8 * HS + ks * HS;
@@ -245,10 +249,10 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
   float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [SKK/4][16][NTH]
   float *dzs = sm + SKK * 16 * NTH;              // [BC][H][4] unit-major dz
   float *red = dzs + BC * G;                     // [BC][NW][H] per-warp column partials
-  float *ring = red + BC * NW * H;               // [BC][kRing][8][NTH] inputs of upcoming steps (value-major)
+  float *ring = red + BC * NW * H;               // [BC][kRing][7H] input rows of upcoming steps
   const int T = a.ix.T;
   const bool toff_sm = T + 1 <= kTokCap;
-  int *toff_s = reinterpret_cast<int *>(ring + BC * kRing * NTH * 8);
+  int *toff_s = reinterpret_cast<int *>(ring + BC * kRing * 7 * H);
   const int *toff = toff_sm ? toff_s : a.ix.tok_off;
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   const int ks = lane & 7, rgl = lane >> 3, rg = warp * 4 + rgl;
@@ -287,18 +291,23 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
     const int tt = d == 0 ? s : len[b] - 1 - s;
     return toff[tt] + r0 + b;
   };
-  // phase B inputs of `unit` (gates, c_t, c_{t-1}, dY), kPF steps ahead
+  // phase B inputs of step s, kPF steps ahead: the gate row [4H], c_t [H],
+  // c_{t-1} [H] (zeros at the start) and dY [H] of the row, in 16-byte pieces
   float dc[BC];
   auto issue = [&](int b, int s) {
     if (s >= 0 && s < len[b]) {
       const int tk = tok_at(b, s);
-      float *slot = ring + ((size_t)b * kRing + s % kRing) * 8 * NTH + t;
-#pragma unroll
-      for (int g = 0; g < 4; ++g) cp_async4(slot + g * NTH, Z + (size_t)tk * G + g * H + unit);
-      cp_async4(slot + 4 * NTH, Cs + (size_t)tk * H + unit);
-      if (s > 0) cp_async4(slot + 5 * NTH, Cs + (size_t)tok_at(b, s - 1) * H + unit);
-      else slot[5 * NTH] = 0.f;
-      cp_async4(slot + 6 * NTH, dY + (size_t)tk * DH + d * H + unit);
+      const int tp = s > 0 ? tok_at(b, s - 1) : -1;
+      float *slot = ring + ((size_t)b * kRing + s % kRing) * 7 * H;
+      for (int i = t; i < 7 * H / 4; i += NTH) {
+        const int q = 4 * i;  // float offset in the slot
+        if (q < 4 * H) cp_async16(slot + q, Z + (size_t)tk * G + q);
+        else if (q < 5 * H) cp_async16(slot + q, Cs + (size_t)tk * H + (q - 4 * H));
+        else if (q < 6 * H) {
+          if (tp >= 0) cp_async16(slot + q, Cs + (size_t)tp * H + (q - 5 * H));
+          else *reinterpret_cast<float4 *>(slot + q) = make_float4(0.f, 0.f, 0.f, 0.f);
+        } else cp_async16(slot + q, dY + (size_t)tk * DH + d * H + (q - 6 * H));
+      }
     }
   };
 #pragma unroll
@@ -308,30 +317,25 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
     for (int b = 0; b < BC; ++b) issue(b, Tg - 1 - j);
     cp_commit();
   }
+  cp_wait_pending<kPF - 1>();  // the first step's rows
+  __syncthreads();
   for (int s = Tg - 1; s >= 0; --s) {
-    cp_wait_all_but_newest();
-    // phase B: dz of unit j from dh = dY + recurrent part.  The prefetch of
-    // step s - kPF is issued for every row, active or not: steps run
-    // backwards, so a shorter row becomes active only later and needs its
-    // first kPF steps in flight by then.
+    cp_wait_pending<kPF - 2>();  // step s - 1's rows, published by this step's barriers
+    // phase B: dz of unit j from dh = dY + recurrent part
 #pragma unroll
     for (int b = 0; b < BC; ++b) {
-      if (s >= len[b]) {  // uniform over the CTA
-        issue(b, s - kPF);
-        continue;
-      }
+      if (s >= len[b]) continue;  // uniform over the CTA
       float dh_rec = 0.f;
       if (s + 1 < len[b]) {
         const float *rp = red + (size_t)b * NW * H + unit;
 #pragma unroll
         for (int wi = 0; wi < NW; ++wi) dh_rec += rp[wi * H];
       }
-      const float *slot = ring + ((size_t)b * kRing + s % kRing) * 8 * NTH + t;
-      const float ig = slot[0], fg = slot[NTH], gg = slot[2 * NTH], og = slot[3 * NTH];
-      const float ct = slot[4 * NTH], cp = slot[5 * NTH];
-      const float dh = slot[6 * NTH] + dh_rec;
+      const float *slot = ring + ((size_t)b * kRing + s % kRing) * 7 * H;
+      const float ig = slot[unit], fg = slot[H + unit], gg = slot[2 * H + unit], og = slot[3 * H + unit];
+      const float ct = slot[4 * H + unit], cp = slot[5 * H + unit];
+      const float dh = slot[6 * H + unit] + dh_rec;
       const int tk = tok_at(b, s);
-      issue(b, s - kPF);
       const float tch = tanh_g(ct);
       const float dcv = fmaf(dh * og, 1.f - tch * tch, dc[b]);
       const float dzi = dcv * gg * ig * (1.f - ig);
@@ -344,6 +348,11 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
       Z[(size_t)tk * G + (2 * pair) * H + unit] = z0;
       Z[(size_t)tk * G + (2 * pair + 1) * H + unit] = z1;
     }
+    // the prefetch of step s - kPF, for every row active or not: steps run
+    // backwards, so a shorter row becomes active only later and needs its
+    // first kPF steps in flight by then
+#pragma unroll
+    for (int b = 0; b < BC; ++b) issue(b, s - kPF);
     cp_commit();
     __syncthreads();
     // phase A: column partials of W_hh^T dz over this warp's 16 x 4 rows
@@ -402,8 +411,8 @@ namespace {
 size_t cta_smem_bytes(bool bwd, int H, int RKK, int BC, int T) {
   const int KPT = H / 8, SKK = KPT - RKK, NTH = 2 * H;
   const size_t wf = (size_t)SKK * 16 * NTH;
-  const size_t f = bwd ? wf + (size_t)BC * 4 * H + (size_t)BC * (NTH / 32) * H + (size_t)BC * kRing * NTH * 8
-                       : wf + (size_t)2 * BC * 8 * (KPT + 4) + (size_t)BC * kRing * NTH * 2;
+  const size_t f = bwd ? wf + (size_t)BC * 4 * H + (size_t)BC * (NTH / 32) * H + (size_t)BC * kRing * 7 * H
+                       : wf + (size_t)2 * BC * 8 * (KPT + 4) + (size_t)BC * kRing * 4 * H;
   const size_t i = (T + 1 <= kTokCap) ? (size_t)(T + 1) : 0;
   return (f + i) * 4 + 16;
 }
