@@ -86,19 +86,35 @@ extern "C" int bkt_plan_buckets_ordered(const int32_t *lengths, int64_t n, int32
     std::vector<int64_t> F(nf, 0);
     for (int64_t i = 0; i < n; ++i) F[lengths[i]] += 1;
     for (int32_t l = 1; l < nf; ++l) F[l] += F[l - 1];
-    // dp rows q-1 and q, back-pointers for every q.
+    // dp rows q-1 and q, back-pointers for every q.  The charge
+    // w(j, i) = i (F[i] - F[j]) satisfies the quadrangle inequality
+    // (w(a,c) + w(b,d) - w(a,d) - w(b,c) = (c - d)(F[b] - F[a]) <= 0 for
+    // a <= b <= c <= d), so the largest minimising j of row i is
+    // non-decreasing in i and a divide-and-conquer over i finds, for every i,
+    // the same minimum and the same largest argmin as the full scan (j
+    // descending, strict "<"), in O(Q n log n) instead of O(Q n^2).
     std::vector<int64_t> prev_row(nf, kDpInf), row(nf, kDpInf);
     std::vector<int32_t> back((size_t)(Q + 1) * nf, -1);
     prev_row[0] = 0;
+    struct Range {
+      int32_t lo, hi, jlo, jhi;
+    };
+    std::vector<Range> todo;
     for (int32_t q = 1; q <= Q; ++q) {
       std::fill(row.begin(), row.end(), kDpInf);
       int32_t *bq = back.data() + (size_t)q * nf;
       // dp[q-1][j] is finite only for j >= q-1.
-      for (int32_t i = q; i < nf; ++i) {
+      todo.clear();
+      if (q < nf) todo.push_back({q, nf - 1, q - 1, nf - 2});
+      while (!todo.empty()) {
+        const Range r = todo.back();
+        todo.pop_back();
+        if (r.lo > r.hi) continue;
+        const int32_t i = r.lo + (r.hi - r.lo) / 2;
         const int64_t Fi = F[i];
         int64_t best = kDpInf;
         int32_t arg = -1;
-        for (int32_t j = i - 1; j >= q - 1; --j) {
+        for (int32_t j = std::min(i - 1, r.jhi); j >= std::max(q - 1, r.jlo); --j) {
           const int64_t v = (int64_t)i * (Fi - F[j]) + prev_row[j];
           if (v < best) {  // strict: ties keep the larger j
             best = v;
@@ -107,6 +123,9 @@ extern "C" int bkt_plan_buckets_ordered(const int32_t *lengths, int64_t n, int32
         }
         row[i] = best;
         bq[i] = arg;
+        const int32_t split = arg >= 0 ? arg : r.jlo;
+        todo.push_back({r.lo, i - 1, r.jlo, split});
+        todo.push_back({i + 1, r.hi, split, r.jhi});
       }
       std::swap(prev_row, row);
     }

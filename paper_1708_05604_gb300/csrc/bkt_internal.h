@@ -7,7 +7,30 @@
 
 #include "bkt.h"
 
+#include <map>
+#include <mutex>
+#include <utility>
+
 namespace bkt {
+
+// Raises `func`'s dynamic shared-memory limit to at least `bytes` on the
+// current device, calling the runtime only when the limit must grow (a
+// cudaFuncSetAttribute per launch costs microseconds of host time per
+// kernel, many times per step).  `cluster16` also allows 16-CTA clusters.
+inline cudaError_t ensure_smem(const void *func, size_t bytes, bool cluster16 = false) {
+  static std::mutex mu;
+  static std::map<std::pair<int, const void *>, size_t> granted;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = granted.find({dev, func});
+  if (it != granted.end() && it->second >= bytes) return cudaSuccess;
+  e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+  if (e == cudaSuccess && cluster16) e = cudaFuncSetAttribute(func, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e == cudaSuccess) granted[{dev, func}] = bytes;
+  return e;
+}
 
 // Device-side view of one packed mini-batch.  Rows are the batch's sequences
 // sorted by length, longest first (stable), so the sequences still running at

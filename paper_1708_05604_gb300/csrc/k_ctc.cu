@@ -228,12 +228,9 @@ cudaError_t launch_ctc_tables(const DevIdx &ix, const float *logp, int C, int bl
   int threads = ((S + spt - 1) / spt + 31) / 32 * 32;
   const size_t smem = (size_t)(2 * (S + 4) + 64 + ix.T) * sizeof(float);
   if (smem > 48 * 1024) {
-    cudaError_t e = cudaSuccess;
-    switch (spt) {
-      case 1: e = cudaFuncSetAttribute(ctc_tables_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); break;
-      case 2: e = cudaFuncSetAttribute(ctc_tables_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); break;
-      default: e = cudaFuncSetAttribute(ctc_tables_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); break;
-    }
+    const void *k = spt == 1 ? (const void *)ctc_tables_kernel<1>
+                             : spt == 2 ? (const void *)ctc_tables_kernel<2> : (const void *)ctc_tables_kernel<4>;
+    cudaError_t e = ensure_smem(k, smem);
     if (e != cudaSuccess) return e;
   }
   dim3 grid(ix.b, 2);

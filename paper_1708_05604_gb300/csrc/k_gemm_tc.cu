@@ -442,7 +442,7 @@ cudaError_t launch_gemm_bf16_tc(const TcGemmArgs &g, cudaStream_t s) {
   CUtensorMap ta, tb;
   if (!make_map(&ta, g.A, (uint64_t)g.K, (uint64_t)g.M, g.lda, TBM)) return cudaErrorInvalidValue;
   if (!make_map(&tb, g.B, (uint64_t)g.K, (uint64_t)g.N, g.ldb, TBN)) return cudaErrorInvalidValue;
-  cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kTcSmem);
+  cudaError_t e = ensure_smem((const void *)gemm_bf16_tc_kernel, kTcSmem);
   if (e != cudaSuccess) return e;
   dim3 grid((g.M + TBM - 1) / TBM, (g.N + TBN - 1) / TBN, g.P ? g.splits : 1);
   if (grid.y > 65535u || grid.z > 65535u) return cudaErrorInvalidConfiguration;
@@ -475,7 +475,7 @@ cudaError_t launch_gemm_tf32x3_tc(const TcGemmArgs &g, const void *A_lo, const v
       !make_map(&tbh, g.B, (uint64_t)g.K, (uint64_t)g.N, g.ldb, FBN, true) ||
       !make_map(&tbl, B_lo, (uint64_t)g.K, (uint64_t)g.N, g.ldb, FBN, true))
     return cudaErrorInvalidValue;
-  cudaError_t e = cudaFuncSetAttribute(gemm_tf32x3_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFSmem);
+  cudaError_t e = ensure_smem((const void *)gemm_tf32x3_tc_kernel, kFSmem);
   if (e != cudaSuccess) return e;
   dim3 grid((g.M + FBM - 1) / FBM, (g.N + FBN - 1) / FBN, g.P ? g.splits : 1);
   if (grid.y > 65535u || grid.z > 65535u) return cudaErrorInvalidConfiguration;

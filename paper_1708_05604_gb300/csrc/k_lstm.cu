@@ -392,12 +392,8 @@ template <typename K>
 cudaError_t launch_rec(K kernel, const RecArgs &a, const RecGeom &g, bool bwd, cudaStream_t s) {
   const int ng = (a.ix.b + g.bc - 1) / g.bc;
   const size_t smem = rec_smem_bytes(bwd, g.w_smem != 0, a.H, g.cs, g.bc, a.ix.T);
-  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e = ensure_smem((const void *)kernel, smem, g.cs > 8);
   if (e != cudaSuccess) return e;
-  if (g.cs > 8) {
-    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    if (e != cudaSuccess) return e;
-  }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(ng * a.dirs * g.cs, 1, 1);
   cfg.blockDim = dim3(g.threads, 1, 1);

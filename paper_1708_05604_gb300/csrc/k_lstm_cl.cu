@@ -590,10 +590,7 @@ size_t cl_smem(bool bwd, int T) {
 
 template <typename K>
 cudaError_t cl_prepare(K kernel, int cs, size_t smem) {
-  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
-  if (cs > 8) e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  return e;
+  return ensure_smem((const void *)kernel, smem, cs > 8);
 }
 
 template <typename K>

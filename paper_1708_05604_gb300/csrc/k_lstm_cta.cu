@@ -422,13 +422,11 @@ cudaError_t launch_cta(const RecArgs &a, bool bwd, cudaStream_t s) {
   const size_t smem = cta_smem_bytes(bwd, H, RKK, BC, a.ix.T);
   const int ng = (a.ix.b + BC - 1) / BC;
   if (bwd) {
-    cudaError_t e = cudaFuncSetAttribute(lstm_bwd_cta_kernel<H, RKK, BC>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = ensure_smem((const void *)lstm_bwd_cta_kernel<H, RKK, BC>, smem);
     if (e != cudaSuccess) return e;
     lstm_bwd_cta_kernel<H, RKK, BC><<<ng * a.dirs, 2 * H, smem, s>>>(a);
   } else {
-    cudaError_t e = cudaFuncSetAttribute(lstm_fwd_cta_kernel<H, RKK, BC>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = ensure_smem((const void *)lstm_fwd_cta_kernel<H, RKK, BC>, smem);
     if (e != cudaSuccess) return e;
     lstm_fwd_cta_kernel<H, RKK, BC><<<ng * a.dirs, 2 * H, smem, s>>>(a);
   }

@@ -113,3 +113,33 @@ def test_param_count_matches_oracle_layout(lib):
             cfg["n_layers"], cfg["bidirectional"], cfg["in_dim"], cfg["hidden"], cfg["n_classes"])
     bad = dict(synth.WORKLOADS["lstm1_uni_h32"].model_cfg(), blank=81)
     assert binding.param_count(bad) == 0
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_planner_tie_heavy_histograms_vs_oracle(lib, seed):
+    """Histograms built to create equal-cost bound tuples (flat counts,
+    repeated blocks, lengths in arithmetic steps), every Q up to the longest
+    length: the library's bounds, cost and plan equal the oracle's."""
+    rng = np.random.default_rng(900 + seed)
+    kind = seed % 3
+    if kind == 0:      # every length once: many tuples of equal cost
+        L = np.arange(1, int(rng.integers(2, 60)) + 1, dtype=np.int32)
+    elif kind == 1:    # a repeated block of counts
+        block = rng.integers(1, 4, size=int(rng.integers(2, 6)))
+        counts = np.tile(block, int(rng.integers(2, 12)))
+        L = np.repeat(np.arange(1, counts.size + 1), counts).astype(np.int32)
+    else:              # lengths on a coarse grid with equal counts
+        step = int(rng.integers(2, 7))
+        vals = np.arange(step, step * int(rng.integers(3, 25)) + 1, step)
+        L = np.repeat(vals, int(rng.integers(1, 4))).astype(np.int32)
+    rng.shuffle(L)
+    lmax = int(L.max())
+    for Q in sorted(set([1, 2, 3, lmax // 2, lmax - 1, lmax]) - {0}):
+        if Q < 1 or Q > lmax:
+            continue
+        a = binding.plan_buckets(L, Q, 4, seed=seed, epoch=1)
+        b = oracle.plan(L, Q, 4, seed=seed, epoch=1)
+        assert np.array_equal(a["bounds"], b["bounds"]), (Q, a["bounds"], b["bounds"])
+        assert a["dp_cost"] == b["dp_cost"]
+        for k in ("order", "batch_off", "batch_bucket"):
+            assert np.array_equal(a[k], b[k])
