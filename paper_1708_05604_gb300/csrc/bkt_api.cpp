@@ -524,13 +524,43 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
   });
 
   // ---- a10: output layer backward
-  // fp32 contractions over tokens on the tensor cores (3xTF32): the
-  // token-major operands are transposed and split into hi + lo parts first
+  // fp32 contractions over tokens on the tensor cores (3xTF32).  Small
+  // aligned outputs read the token-major operands directly (split and
+  // swizzled while loading); otherwise the operands are transposed and split
+  // first and the TMA-fed GEMM runs (measured on GB300: the fused kernel moves
+  // more bytes through shared memory per slab, so it wins only while the
+  // transposes dominate, e.g. dW_hh at H = 128: 43 us against 66 us)
   const int NTq = (NT + 7) & ~7;
-  auto split_A_on = [&](Launch &X, const float *A, int64_t lda, int M) {
-    X.run("transpose_split", [&] { return bkt::launch_transpose_split(A, lda, nullptr, NT, M, w.AT, w.ATl, NTq, X.s); });
-  };
-  auto tf32_reduce_on = [&](Launch &X, int M, const float *B, int64_t ldb, const int32_t *gather, int N, float *out) {
+  // the transposed split of A left in AT by the last fallback call: dW_ih of
+  // a layer above the first reuses the one its dW_hh made (nothing else
+  // writes AT between them)
+  const float *at_src = nullptr;
+  auto tn_reduce_on = [&](Launch &X, const float *A, int64_t lda, int M, const float *B, int64_t ldb,
+                          const int32_t *gather, int N, float *out) {
+    const bool fused = ((lda | ldb | M | N) & 3) == 0 &&
+                       ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(B)) & 15) == 0 &&
+                       (int64_t)M * N <= 128 * 1024;
+    if (fused) {
+      bkt::TnGemmArgs g{};
+      g.M = M;
+      g.N = N;
+      g.K = NT;
+      g.A = A;
+      g.lda = lda;
+      g.B = B;
+      g.ldb = ldb;
+      g.gather = gather;
+      g.P = w.part;
+      g.splits = bkt::tf32x3_tn_splits(M, N, NT, sm_count, w.part_floats);
+      g.err = w.status;
+      X.run("gemm_tf32x3_tn", [&] { return bkt::launch_gemm_tf32x3_tn(g, X.s); });
+      X.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, g.splits, M, N, out, X.s); });
+      return;
+    }
+    if (at_src != A) {
+      X.run("transpose_split", [&] { return bkt::launch_transpose_split(A, lda, nullptr, NT, M, w.AT, w.ATl, NTq, X.s); });
+      at_src = A;
+    }
     X.run("transpose_split", [&] { return bkt::launch_transpose_split(B, ldb, gather, NT, N, w.BTf, w.BTl, NTq, X.s); });
     bkt::TcGemmArgs g{};
     g.M = M;
@@ -559,8 +589,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     if (e == cudaSuccess) e = cudaStreamWaitEvent(side, fork_ev, 0);
     if (e != cudaSuccess) return cuda_err("fork to the side stream", e);
   }
-  split_A_on(Ls, w.logit, C, C);
-  tf32_reduce_on(Ls, C, Ytop, DH, nullptr, DH, grads + lo.w_out);
+  tn_reduce_on(Ls, w.logit, C, C, Ytop, DH, nullptr, DH, grads + lo.w_out);
   bias_sum_on(Ls, w.logit, C, C, grads + lo.b_out);
   {
     // dY = dlogit W_out on the tensor cores: dlogit split with its rows padded
@@ -662,13 +691,12 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         // dW_hh = dz^T h_{t-1}; h_{t-1} of token (t, r) is the row's previous
         // token in its direction (zeros at the start)
         const float *dZ = w.Z[l * dirs + d];
-        split_A_on(X, dZ, 4 * H, 4 * H);
-        tf32_reduce_on(X, 4 * H, w.Y[l] + d * H, DH, w.prev_tok[d], H, grads + lo.w_hh(l, d));
+        tn_reduce_on(X, dZ, 4 * H, 4 * H, w.Y[l] + d * H, DH, w.prev_tok[d], H, grads + lo.w_hh(l, d));
         if (l == 0) {
           // narrow input: [dW_ih | db] = dz^T [X | 1] streamed over dz
           narrow_on(dZ, grads + lo.w_ih[l * dirs + d], grads + lo.bias(l, d));
         } else {
-          tf32_reduce_on(X, 4 * H, Xl, D, nullptr, D, grads + lo.w_ih[l * dirs + d]);
+          tn_reduce_on(X, dZ, 4 * H, 4 * H, Xl, D, nullptr, D, grads + lo.w_ih[l * dirs + d]);
           bias_sum_on(X, dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
         }
       }
@@ -699,6 +727,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
       // K-contiguous already, W_ih is transposed while it is split
       float *dxa = w.DXh ? w.DXh : w.AT, *dxl = w.DXl ? w.DXl : w.ATl;
       if (side && !w.DXh) return set_err(BKT_EINVAL, "internal: dX buffers missing for the side stream");
+      if (dxa == w.AT) at_src = nullptr;  // AT is overwritten here
       for (int d = 0; d < dirs; ++d) {
         L.run("split_rows", [&] {
           return bkt::launch_split_rows(w.Z[l * dirs + d], 4 * H, NT, 4 * H, dxa, dxl, 4 * H, s);

@@ -125,6 +125,22 @@ cudaError_t launch_gemm_bf16_tc(const TcGemmArgs &g, cudaStream_t s);
 // multiples of 4, 16-byte aligned); D (or partials) as for the bf16 GEMM.
 int tf32x3_splits(int M, int N, int K, int sm_count, size_t part_floats);
 cudaError_t launch_gemm_tf32x3_tc(const TcGemmArgs &g, const void *A_lo, const void *B_lo, cudaStream_t s);
+// The same 3xTF32 contraction over the token axis with token-major operands,
+// split and swizzled while loading: D[m][n] = sum_k A[k*lda + m] B[g(k)*ldb + n]
+// (g = gather, or the identity when null; a negative entry gives a zero row).
+// Writes partials P[split][M][N] (D with ldd when splits == 1 and P is null);
+// no alignment requirement.
+struct TnGemmArgs {
+  int M, N, K;
+  const float *A; int64_t lda;
+  const float *B; int64_t ldb;
+  const int32_t *gather;
+  float *D; int64_t ldd;
+  float *P; int splits;
+  int32_t *err;
+};
+int tf32x3_tn_splits(int M, int N, int K, int sm_count, size_t part_floats);
+cudaError_t launch_gemm_tf32x3_tn(const TnGemmArgs &g, cudaStream_t s);
 
 // a8: log-space CTC forward (alpha) and backward (beta-hat) tables, one CTA
 // per (row, direction); writes the per-sequence loss and the row's flag.
