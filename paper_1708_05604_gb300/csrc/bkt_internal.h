@@ -128,8 +128,8 @@ cudaError_t launch_gemm_tf32x3_tc(const TcGemmArgs &g, const void *A_lo, const v
 // The same 3xTF32 contraction over the token axis with token-major operands,
 // split and swizzled while loading: D[m][n] = sum_k A[k*lda + m] B[g(k)*ldb + n]
 // (g = gather, or the identity when null; a negative entry gives a zero row).
-// Writes partials P[split][M][N] (D with ldd when splits == 1 and P is null);
-// no alignment requirement.
+// Writes partials P[split][M][N] (D with ldd when splits == 1 and P is null).
+// lda, ldb, M and N must be multiples of 4 and A, B 16-byte aligned.
 struct TnGemmArgs {
   int M, N, K;
   const float *A; int64_t lda;

@@ -392,65 +392,72 @@ __global__ void __launch_bounds__(128, 1)
 // ---------------------------------------------------------------------------
 // 3xTF32 contraction over the token axis with token-major operands:
 //   D[m][n] = sum_k A[k][m] * B[g(k)][n]
-// (A [K x M], B [rows x N], both fp32 row-major with M or N contiguous; g an
-// optional row gather, -1 giving a zero row), as the weight gradients need
-// (k = token), without transposed and split copies of the operands.
+// (A [K x M], B [rows x N], both fp32 row-major with M or N contiguous and
+// 16-byte aligned rows, M and N multiples of 4; g an optional row gather, -1
+// giving a zero row), as the weight gradients need (k = token), without
+// transposed and split copies of the operands.
 //
-// Per 32-token slab: asynchronous copies bring the raw rows of both tiles
-// (32 x 128 floats each, as they lie in global memory) into a kTnRaw-slot
-// ring kTnRaw slabs ahead (16-byte pieces when rows are 16-byte aligned, else
-// 4-byte ones; rows outside the operands are zero-filled by a zero source
-// size).
-// Then all 256 threads split each value into tf32 hi + lo (both rounded to
-// nearest, as in the transposed split) and store the four tiles K-major in
-// the 128-byte swizzled layout TMA would produce (16-byte chunk c of row r at
-// chunk position c ^ (r & 7)) in the MMA stage, make the stores visible to
-// the tensor core (fence.proxy.async) and meet at a barrier; thread 0 issues
-// the twelve MMAs of the slab and commits them to the stage's empty barrier,
-// which the threads wait on (bounded) before the stage is refilled.  Shared
-// memory holds one MMA stage (64 KB) and four raw slabs (128 KB): measured on
-// GB300, copies issued four slabs ahead beat overlapping the MMAs of one slab
-// with the conversion of the next.  The gather indices of the CTA's token range (up to kTnMaxChunk; the
-// split rule keeps ranges shorter) are staged in shared memory first, so a
-// copy's address waits on no global load.  The epilogue splits the 128
-// accumulator columns between the two warps of each TMEM lane quarter.
+// Eight converter warps and one MMA warp.  Per 32-token slab the converters
+// copy the raw rows of both tiles (32 x 128 floats each, as they lie in
+// global memory) into a kTnRaw-slot ring with asynchronous 16-byte copies
+// (rows outside the operands zero-filled by a zero source size), then split
+// each value into tf32 hi + lo and store the four tiles K-major in the
+// 128-byte swizzled layout TMA would produce (16-byte chunk c of row r at
+// chunk position c ^ (r & 7)) in one of two MMA stages, make the stores
+// visible to the tensor core (fence.proxy.async) and arrive on the stage's
+// full barrier.  The MMA warp waits on it, issues the twelve MMAs and commits
+// them to the stage's empty barrier, which the converters wait on before
+// refilling the stage; so the MMAs of one slab run while the next is
+// converted (issuing them from a converter warp held its warp for the MMAs'
+// duration).  The split truncates: hi = x with the low 13 mantissa bits
+// cleared, lo = (x - hi) likewise, |x - hi - lo| <= 2^-20 |x| (three
+// instructions per value; rounding both parts cost five).  One 256-thread
+// barrier per slab both publishes the slab's copies and frees the previous
+// raw slot, whose refill is issued right after it.  A thread's gather
+// indices are loaded (from clamped positions, never selected on) two slabs
+// before its copies use them; the loop is unrolled over two slabs to keep
+// those registers statically named.  Every wait is bounded; on expiry the
+// CTA records an error flag.  The epilogue splits the 128 accumulator columns
+// between the two converter warps of each TMEM lane quarter.
 namespace {
 
-constexpr int kTnThreads = 256;
-constexpr int kTnStages = 1;                      // converted (MMA) stages
-constexpr int kTnRaw = 4;                         // raw slabs in flight
+constexpr int kTnConv = 256;                      // converter threads (warps 0-7)
+constexpr int kTnThreads = kTnConv + 32;          // + the MMA warp
+constexpr int kTnStages = 2;                      // converted (MMA) stages
+constexpr int kTnRaw = 3;                         // raw slabs in flight
 constexpr uint32_t kTnRawTile = FBK * 128 * 4;    // 16 KB: 32 rows x 128 floats
 constexpr uint32_t kTnRawSlab = 2 * kTnRawTile;   // A and B
-constexpr int kTnMaxChunk = 4096;
-constexpr size_t kTnSmem = 1024 + (size_t)kTnStages * kFStage + (size_t)kTnRaw * kTnRawSlab + 256 +
-                           kTnMaxChunk * sizeof(int32_t);
+constexpr size_t kTnSmem = 1024 + (size_t)kTnStages * kFStage + (size_t)kTnRaw * kTnRawSlab + 256;
 
-// x = h + l with h, l tf32 values, both rounded to nearest (ties away from
-// zero, by adding half an ulp to the bit pattern and truncating):
-// |x - h - l| <= 2^-22 |x|.
-__device__ __forceinline__ void split_tf32(float x, float &h, float &l) {
-  h = __uint_as_float((__float_as_uint(x) + 0x1000u) & 0xFFFFE000u);
-  l = __uint_as_float((__float_as_uint(x - h) + 0x1000u) & 0xFFFFE000u);
+__device__ __forceinline__ void split_tf32_trunc(float x, float &h, float &l) {
+  h = __uint_as_float(__float_as_uint(x) & 0xFFFFE000u);
+  l = __uint_as_float(__float_as_uint(x - h) & 0xFFFFE000u);
 }
-// Asynchronous global -> shared copies; `bytes` of the source are read and
-// the rest of the piece is zero-filled (0: nothing is read).
+// Asynchronous 16-byte global -> shared copy; `bytes` of the source are read
+// and the rest is zero-filled (0: nothing is read).
 __device__ __forceinline__ void cpa16(uint32_t dst, const void *src, uint32_t bytes) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(bytes));
 }
-__device__ __forceinline__ void cpa4(uint32_t dst, const void *src, uint32_t bytes) {
-  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(dst), "l"(src), "r"(bytes));
+// Barrier 1 over the converter warps; returns whether any passed `fail`.
+__device__ __forceinline__ bool conv_barrier_or(bool fail) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n barrier.cta.red.or.pred q, 1, %2, p;\n selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(r)
+      : "r"((uint32_t)fail), "n"(kTnConv)
+      : "memory");
+  return r != 0;
 }
 
 }  // namespace
 
-template <bool VEC>
 __global__ void __launch_bounds__(kTnThreads, 1) gemm_tf32x3_tn_kernel(TnGemmArgs g) {
   extern __shared__ uint8_t tc_smem_raw[];
   uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(tc_smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t *raw = base + kTnStages * kFStage;                              // [kTnRaw][A | B][32][128]
-  uint64_t *bars = reinterpret_cast<uint64_t *>(raw + kTnRaw * kTnRawSlab);  // empty[S], done
-  uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + kTnStages + 1);
-  int32_t *gsm = reinterpret_cast<int32_t *>(raw + kTnRaw * kTnRawSlab + 256);  // [kTnMaxChunk] B rows
+  uint8_t *raw = base + kTnStages * kFStage;                                 // [kTnRaw][A | B][32][128]
+  uint64_t *bars = reinterpret_cast<uint64_t *>(raw + kTnRaw * kTnRawSlab);  // full[S], empty[S], done
+  uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 2 * kTnStages + 1);
+  int *abort_s = reinterpret_cast<int *>(tslot + 1);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int m0 = blockIdx.x * FBM, n0 = blockIdx.y * FBN;
   const int nkb = (g.K + FBK - 1) / FBK;
@@ -459,12 +466,15 @@ __global__ void __launch_bounds__(kTnThreads, 1) gemm_tf32x3_tn_kernel(TnGemmArg
   const int nk = max(0, min(nkb, kb0 + chunk) - kb0);
   const int kbase = kb0 * FBK;
   const int ntok = max(0, min(nk * FBK, g.K - kbase));
-  const bool gstage = ntok <= kTnMaxChunk;
-  const uint32_t empty0 = su32(bars), done = su32(bars + kTnStages);
+  const uint32_t full0 = su32(bars), empty0 = su32(bars + kTnStages), done = su32(bars + 2 * kTnStages);
 
   if (tid == 0) {
-    for (int s = 0; s < kTnStages; ++s) mbar_init(empty0 + 8 * s, 1);
+    for (int s = 0; s < kTnStages; ++s) {
+      mbar_init(full0 + 8 * s, kTnConv / 32);
+      mbar_init(empty0 + 8 * s, 1);
+    }
     mbar_init(done, 1);
+    *abort_s = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) {
@@ -472,86 +482,98 @@ __global__ void __launch_bounds__(kTnThreads, 1) gemm_tf32x3_tn_kernel(TnGemmArg
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  // B row of each of this CTA's tokens (-1: zero row)
-  if (gstage)
-    for (int i = tid; i < ntok; i += kTnThreads) gsm[i] = g.gather ? g.gather[kbase + i] : kbase + i;
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tslot;
 
-  // raw slab i -> ring slot i % kTnRaw: row k of A holds A[kbase+k][m0 .. m0+127], of B the gathered row
-  auto issue = [&](int i) {
-    const uint32_t slot = su32(raw + (i % kTnRaw) * kTnRawSlab);
-    if (VEC) {
-      // 32 rows x 32 pieces per tile: this thread's pieces are rows
-      // warp + 8 j, columns 4 lane .. 4 lane + 3
-      const int c4 = 4 * lane;
-      const bool a_col = m0 + c4 < g.M, b_col = n0 + c4 < g.N;
-      const float *acol = g.A + (m0 + c4), *bcol = g.B + (n0 + c4);
+  if (warp == kTnConv / 32) {  // the MMA warp
+    if (lane == 0) {
+      int issued = 0;
+      for (int i = 0; i < nk; ++i) {
+        const int s = i % kTnStages;
+        if (!mbar_wait(full0 + 8 * s, (i / kTnStages) & 1)) {
+          *abort_s = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t ah = su32(base + s * kFStage), al = ah + kFTile, bh = ah + 2 * kFTile, bl = ah + 3 * kFTile;
+#pragma unroll
+        for (int kk = 0; kk < FBK / 8; ++kk) {
+          const uint32_t o = kk * 32;
+          tc_mma_tf32(tmem, sw128_desc(ah + o), sw128_desc(bh + o), kIdescTf32, (i > 0 || kk > 0) ? 1u : 0u);
+          tc_mma_tf32(tmem, sw128_desc(ah + o), sw128_desc(bl + o), kIdescTf32, 1u);
+          tc_mma_tf32(tmem, sw128_desc(al + o), sw128_desc(bh + o), kIdescTf32, 1u);
+        }
+        tc_commit(empty0 + 8 * s);
+        ++issued;
+      }
+      // the final commit tracks every MMA issued above
+      if (issued > 0) tc_commit(done);
+      else mbar_arrive(done);
+    }
+    __syncwarp();
+  } else {  // converters
+    // copy geometry: rows warp + 8 j (j < 4) of a slab, columns 4 lane .. +3
+    const int c4 = 4 * lane;
+    const bool a_col = m0 + c4 < g.M, b_col = n0 + c4 < g.N;
+    const float *acol = g.A + (m0 + c4), *bcol = g.B + (n0 + c4);
+    auto rows_of = [&](int i, int (&br)[4]) {  // B rows of this thread's copies of slab i (validity checked at use)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int kl = i * FBK + warp + 8 * j;
+        br[j] = (g.gather && ntok > 0) ? __ldg(g.gather + kbase + min(kl, ntok - 1)) : kbase + kl;
+      }
+    };
+    auto issue = [&](int i, const int (&br)[4]) {  // raw slab i -> ring slot i % kTnRaw
+      const uint32_t slot = su32(raw + (i % kTnRaw) * kTnRawSlab);
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const int k = warp + 8 * j;
         const int kl = i * FBK + k;
-        const bool kin = kl < ntok;
         const uint32_t dst = slot + (uint32_t)(k * 128 + c4) * 4;
+        const bool kin = kl < ntok;
         const bool av = kin && a_col;
         cpa16(dst, av ? acol + (int64_t)(kbase + kl) * g.lda : g.A, av ? 16u : 0u);
-        const int br = !kin ? -1 : gstage ? gsm[kl] : g.gather ? g.gather[kbase + kl] : kbase + kl;
-        const bool bv = br >= 0 && b_col;
-        cpa16(dst + kTnRawTile, bv ? bcol + (int64_t)br * g.ldb : g.B, bv ? 16u : 0u);
+        const bool bv = kin && br[j] >= 0 && b_col;
+        cpa16(dst + kTnRawTile, bv ? bcol + (int64_t)br[j] * g.ldb : g.B, bv ? 16u : 0u);
       }
-    } else {
-#pragma unroll 4
-      for (int j = 0; j < 16; ++j) {
-        const int e = tid + kTnThreads * j;  // element of the 32 x 128 tile
-        const int k = e >> 7, c = e & 127;
-        const int kl = i * FBK + k;
-        const bool kin = kl < ntok;
-        const int am = m0 + c, bn = n0 + c;
-        const bool av = kin && am < g.M;
-        cpa4(slot + (uint32_t)(k * 128 + c) * 4, av ? g.A + (int64_t)(kbase + kl) * g.lda + am : g.A, av ? 4u : 0u);
-        const int br = !kin ? -1 : gstage ? gsm[kl] : g.gather ? g.gather[kbase + kl] : kbase + kl;
-        const bool bv = br >= 0 && bn < g.N;
-        cpa4(slot + kTnRawTile + (uint32_t)(k * 128 + c) * 4, bv ? g.B + (int64_t)br * g.ldb + bn : g.B,
-             bv ? 4u : 0u);
-      }
-    }
-    asm volatile("cp.async.commit_group;" ::: "memory");
-  };
+      asm volatile("cp.async.commit_group;" ::: "memory");
+    };
 
-  // conversion geometry: warp w covers rows 32 (w & 3) .. +31 and k chunks
-  // 4 (w >> 2) .. +3; lane l takes rows r0 .. r0+3 with r0 = 32 (w & 3) + 4 rb,
-  // rb = l & 7, and chunk kc = 4 (w >> 2) + ((rb >> 1) + (l >> 3)) mod 4, so
-  // that the eight lanes of each quarter warp (one 128-bit shared access
-  // phase) read eight distinct raw 16-byte positions and write eight
-  // distinct swizzled chunk positions
-  const int rb = lane & 7;
-  const int r0 = 32 * (warp & 3) + 4 * rb, kc = 4 * (warp >> 2) + (((rb >> 1) + (lane >> 3)) & 3);
-  bool abort_run = false;
-  int issued = 0;
-  for (int i = 0; i < kTnRaw; ++i) {
-    if (i < nk) issue(i);
-    else asm volatile("cp.async.commit_group;" ::: "memory");
-  }
-  for (int i = 0; i < nk; ++i) {
-    const int s = i % kTnStages;
-    asm volatile("cp.async.wait_group %0;" ::"n"(kTnRaw - 1) : "memory");  // raw slab i (own pieces)
-    bool ok = true;
-    if (i >= kTnStages) ok = mbar_wait(empty0 + 8 * s, ((i / kTnStages) - 1) & 1);
-    __syncthreads();  // raw slab i complete for all threads
-    {
-      // this thread: rows r0 .. r0+3 of both tiles, k chunk kc (4 tokens);
-      // read as four 16-byte rows of the raw slab, written as four 16-byte
-      // K-major chunks
+    // conversion geometry: warp w covers rows 32 (w & 3) .. +31 and k chunks
+    // 4 (w >> 2) .. +3; lane l takes rows r0 .. r0+3 with r0 = 32 (w & 3) + 4 rb,
+    // rb = l & 7, and chunk kc = 4 (w >> 2) + ((rb >> 1) + (l >> 3)) mod 4, so
+    // that the eight lanes of each quarter warp (one 128-bit shared access
+    // phase) read eight distinct raw 16-byte positions and write eight
+    // distinct swizzled chunk positions
+    const int rb = lane & 7;
+    const int r0 = 32 * (warp & 3) + 4 * rb, kc = 4 * (warp >> 2) + (((rb >> 1) + (lane >> 3)) & 3);
+    bool fail = false;
+
+    // slab i: its copies done and the previous raw slot free (one barrier),
+    // refill that slot with slab i-1+kTnRaw, load the rows of slab i+kTnRaw+1,
+    // convert slab i into stage i % 2 and hand it to the MMA warp
+    auto slab = [&](int i, int (&br)[4]) -> bool {
+      const int s = i % kTnStages;
+      asm volatile("cp.async.wait_group %0;" ::"n"(kTnRaw - 2) : "memory");  // raw slab i (own pieces)
+      if (conv_barrier_or(fail)) return false;
+      if (i > 0) {
+        issue(i - 1 + kTnRaw, br);  // past the last slab: zero-filled pieces, never converted
+        rows_of(i + 1 + kTnRaw, br);
+      }
+      if (i >= kTnStages && !mbar_wait(empty0 + 8 * s, ((i / kTnStages) - 1) & 1)) {
+        fail = true;
+        return true;
+      }
       const float *ra = reinterpret_cast<const float *>(raw + (i % kTnRaw) * kTnRawSlab);
-      const float *rb = ra + FBK * 128;
+      const float *rbp = ra + FBK * 128;
       uint8_t *st = base + s * kFStage;
       float4 va[4], vb[4];
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk) {
         va[kk] = *reinterpret_cast<const float4 *>(ra + (4 * kc + kk) * 128 + r0);
-        vb[kk] = *reinterpret_cast<const float4 *>(rb + (4 * kc + kk) * 128 + r0);
+        vb[kk] = *reinterpret_cast<const float4 *>(rbp + (4 * kc + kk) * 128 + r0);
       }
 #pragma unroll
       for (int mm = 0; mm < 4; ++mm) {
@@ -559,70 +581,69 @@ __global__ void __launch_bounds__(kTnThreads, 1) gemm_tf32x3_tn_kernel(TnGemmArg
         const uint32_t off = (uint32_t)r * 128u + ((uint32_t)(kc ^ (r & 7)) << 4);
         auto el = [](const float4 &v, int q) { return q == 0 ? v.x : q == 1 ? v.y : q == 2 ? v.z : v.w; };
         float4 ah, al, bh, bl;
-        split_tf32(el(va[0], mm), ah.x, al.x);
-        split_tf32(el(va[1], mm), ah.y, al.y);
-        split_tf32(el(va[2], mm), ah.z, al.z);
-        split_tf32(el(va[3], mm), ah.w, al.w);
-        split_tf32(el(vb[0], mm), bh.x, bl.x);
-        split_tf32(el(vb[1], mm), bh.y, bl.y);
-        split_tf32(el(vb[2], mm), bh.z, bl.z);
-        split_tf32(el(vb[3], mm), bh.w, bl.w);
+        split_tf32_trunc(el(va[0], mm), ah.x, al.x);
+        split_tf32_trunc(el(va[1], mm), ah.y, al.y);
+        split_tf32_trunc(el(va[2], mm), ah.z, al.z);
+        split_tf32_trunc(el(va[3], mm), ah.w, al.w);
+        split_tf32_trunc(el(vb[0], mm), bh.x, bl.x);
+        split_tf32_trunc(el(vb[1], mm), bh.y, bl.y);
+        split_tf32_trunc(el(vb[2], mm), bh.z, bl.z);
+        split_tf32_trunc(el(vb[3], mm), bh.w, bl.w);
         *reinterpret_cast<float4 *>(st + off) = ah;
         *reinterpret_cast<float4 *>(st + kFTile + off) = al;
         *reinterpret_cast<float4 *>(st + 2 * kFTile + off) = bh;
         *reinterpret_cast<float4 *>(st + 3 * kFTile + off) = bl;
       }
-    }
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    if (__syncthreads_or(!ok)) {  // stage s converted; raw slot free again
-      abort_run = true;
-      break;
-    }
-    if (tid == 0) {
-      tc_fence_after();
-      const uint32_t ah = su32(base + s * kFStage), al = ah + kFTile, bh = ah + 2 * kFTile, bl = ah + 3 * kFTile;
-#pragma unroll
-      for (int kk = 0; kk < FBK / 8; ++kk) {
-        const uint32_t o = kk * 32;
-        tc_mma_tf32(tmem, sw128_desc(ah + o), sw128_desc(bh + o), kIdescTf32, (i > 0 || kk > 0) ? 1u : 0u);
-        tc_mma_tf32(tmem, sw128_desc(ah + o), sw128_desc(bl + o), kIdescTf32, 1u);
-        tc_mma_tf32(tmem, sw128_desc(al + o), sw128_desc(bh + o), kIdescTf32, 1u);
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) mbar_arrive(full0 + 8 * s);
+      return true;
+    };
+
+    int brA[4], brB[4];  // rows of the slabs copied at odd and even slabs
+    {
+#pragma unroll 1
+      for (int i = 0; i < kTnRaw; ++i) {
+        rows_of(i, brA);
+        issue(i, brA);
       }
-      tc_commit(empty0 + 8 * s);
-      ++issued;
     }
-    if (i + kTnRaw < nk) issue(i + kTnRaw);
-    else asm volatile("cp.async.commit_group;" ::: "memory");
-  }
-  asm volatile("cp.async.wait_all;" ::: "memory");
-  if (tid == 0) {
-    // the final commit tracks every MMA issued above
-    if (issued > 0) tc_commit(done);
-    else mbar_arrive(done);
+    rows_of(kTnRaw, brB);      // copied at slab 1
+    rows_of(kTnRaw + 1, brA);  // copied at slab 2
+    for (int i = 0; i < nk; i += 2) {
+      if (!slab(i, brA)) break;
+      if (i + 1 < nk && !slab(i + 1, brB)) break;
+    }
+    if (fail) *abort_s = 1;
+    asm volatile("cp.async.wait_all;" ::: "memory");
   }
 
   const bool ready = mbar_wait(done, 0);
   tc_fence_after();
-  const int quarter = warp & 3, half = warp >> 2;
-  const int m = m0 + quarter * 32 + lane;
-  const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
-  const bool write = ready && !abort_run && m < g.M;
-  float *out = g.P ? g.P + (int64_t)blockIdx.z * g.M * g.N + (int64_t)m * g.N : g.D + (int64_t)m * g.ldd;
+  __syncthreads();
+  const bool aborted = *abort_s != 0;
+  if (warp < kTnConv / 32) {
+    const int quarter = warp & 3, half = warp >> 2;
+    const int m = m0 + quarter * 32 + lane;
+    const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
+    const bool write = ready && !aborted && m < g.M;
+    float *out = g.P ? g.P + (int64_t)blockIdx.z * g.M * g.N + (int64_t)m * g.N : g.D + (int64_t)m * g.ldd;
 #pragma unroll 1
-  for (int cc = half * (FBN / 2); cc < (half + 1) * (FBN / 2); cc += 32) {
-    uint32_t v[32];
-    __syncwarp();
-    tmem_ld32(trow + cc, v);
-    if (!write) continue;
-    const int nb = n0 + cc;
+    for (int cc = half * (FBN / 2); cc < (half + 1) * (FBN / 2); cc += 32) {
+      uint32_t v[32];
+      __syncwarp();
+      tmem_ld32(trow + cc, v);
+      if (!write) continue;
+      const int nb = n0 + cc;
 #pragma unroll
-    for (int j = 0; j < 32; ++j)
-      if (nb + j < g.N) out[nb + j] = nk > 0 ? __uint_as_float(v[j]) : 0.f;
+      for (int j = 0; j < 32; ++j)
+        if (nb + j < g.N) out[nb + j] = nk > 0 ? __uint_as_float(v[j]) : 0.f;
+    }
   }
   tc_fence_before();
   __syncthreads();
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(FBN) : "memory");
-  if (tid == 0 && (abort_run || !ready) && g.err) atomicOr(g.err, 2);
+  if (tid == 0 && (aborted || !ready) && g.err) atomicOr(g.err, 2);
 }
 
 // ---------------------------------------------------------------------------
@@ -726,17 +747,16 @@ int tf32x3_tn_splits(int M, int N, int K, int sm_count, size_t part_floats) {
 cudaError_t launch_gemm_tf32x3_tn(const TnGemmArgs &g, cudaStream_t s) {
   if (g.M <= 0 || g.N <= 0) return cudaSuccess;
   if (g.K <= 0 || g.splits < 1 || (!g.P && (!g.D || g.splits != 1)) || !g.A || !g.B) return cudaErrorInvalidValue;
-  // 16-byte pieces when every row of both tiles starts 16-byte aligned and
-  // no piece straddles the end of a row
-  const bool vec = ((g.lda | g.ldb | g.M | g.N) & 3) == 0 &&
-                   ((reinterpret_cast<uintptr_t>(g.A) | reinterpret_cast<uintptr_t>(g.B)) & 15) == 0;
-  const void *k = vec ? (const void *)gemm_tf32x3_tn_kernel<true> : (const void *)gemm_tf32x3_tn_kernel<false>;
-  cudaError_t e = ensure_smem(k, kTnSmem);
+  // 16-byte pieces: every row of both tiles starts 16-byte aligned and no
+  // piece straddles the end of a row
+  if (((g.lda | g.ldb | g.M | g.N) & 3) != 0 ||
+      ((reinterpret_cast<uintptr_t>(g.A) | reinterpret_cast<uintptr_t>(g.B)) & 15) != 0)
+    return cudaErrorInvalidValue;
+  cudaError_t e = ensure_smem((const void *)gemm_tf32x3_tn_kernel, kTnSmem);
   if (e != cudaSuccess) return e;
   dim3 grid((g.M + FBM - 1) / FBM, (g.N + FBN - 1) / FBN, g.splits);
   if (grid.y > 65535u || grid.z > 65535u) return cudaErrorInvalidConfiguration;
-  if (vec) gemm_tf32x3_tn_kernel<true><<<grid, kTnThreads, kTnSmem, s>>>(g);
-  else gemm_tf32x3_tn_kernel<false><<<grid, kTnThreads, kTnSmem, s>>>(g);
+  gemm_tf32x3_tn_kernel<<<grid, kTnThreads, kTnSmem, s>>>(g);
   return cudaGetLastError();
 }
 
