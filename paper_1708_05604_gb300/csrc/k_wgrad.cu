@@ -63,61 +63,63 @@ static cudaError_t launch_reduce(const float *P, int splits, int M, int N, int D
 // Narrow case G[m][n] = sum_k A[k][m] [X[k] | 1][n] with X of D <= 16
 // columns, partials P[z][m][n] over token chunk z.  A bandwidth-bound pass
 // over A: with M and lda multiples of 4 a thread keeps 4 (D+1) sums for four
-// consecutive columns (otherwise one column).  Tokens go in groups of 16
-// (predicated, no serial tail), and the loads of the next group are issued
-// before the current one is summed, so a thread always has a group of A in
-// flight; X rows are broadcast across the warp.
+// consecutive columns (otherwise one column).  The block first stages its
+// chunk's rows [X | 1] in shared memory, zero past the chunk's end; tokens
+// then go in groups of 16 whose A rows are loaded from clamped (always
+// valid) rows one group ahead, and a group is summed with plain FMAs against
+// the staged rows: no branch and no select stands between a load and the
+// loads behind it (a warp issues in order), the ones column forms the bias
+// sum and the zero rows cancel the clamped tail.
 template <int D, int VEC>
 __global__ void __launch_bounds__(128) narrow_wgrad_kernel(const float *__restrict__ A, int64_t lda, int M,
                                                            const float *__restrict__ X, int K,
                                                            float *__restrict__ P, int chunk) {
-  constexpr int U = 16;
-  const int m0 = (blockIdx.x * blockDim.x + threadIdx.x) * VEC;
+  constexpr int U = 16, DX = D + 1;
+  extern __shared__ float xs[];  // [chunk][D + 1]
   const int z = blockIdx.y;
-  if (m0 >= M) return;
   const int k0 = z * chunk, k1 = min(K, k0 + chunk);
-  float acc[VEC][D + 1];
+  for (int i = threadIdx.x; i < chunk * DX; i += blockDim.x) {
+    const int k = k0 + i / DX, j = i % DX;
+    xs[i] = k < k1 ? (j < D ? X[(int64_t)k * D + j] : 1.f) : 0.f;
+  }
+  __syncthreads();
+  const int m0 = (blockIdx.x * blockDim.x + threadIdx.x) * VEC;
+  if (m0 >= M) return;
+  float acc[VEC][DX];
 #pragma unroll
   for (int c = 0; c < VEC; ++c)
 #pragma unroll
-    for (int j = 0; j <= D; ++j) acc[c][j] = 0.f;
+    for (int j = 0; j < DX; ++j) acc[c][j] = 0.f;
+  const float *acol = A + m0;
   auto load_group = [&](int k, float (&v)[U][VEC]) {
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      if (k + u < k1) {
-        if constexpr (VEC == 4) {
-          const float4 a = __ldg(reinterpret_cast<const float4 *>(A + (int64_t)(k + u) * lda + m0));
-          v[u][0] = a.x;
-          v[u][1] = a.y;
-          v[u][2] = a.z;
-          v[u][3] = a.w;
-        } else {
-          v[u][0] = __ldg(A + (int64_t)(k + u) * lda + m0);
-        }
+      const float *row = acol + (int64_t)min(k + u, k1 - 1) * lda;
+      if constexpr (VEC == 4) {
+        const float4 a = __ldg(reinterpret_cast<const float4 *>(row));
+        v[u][0] = a.x;
+        v[u][1] = a.y;
+        v[u][2] = a.z;
+        v[u][3] = a.w;
       } else {
-#pragma unroll
-        for (int c = 0; c < VEC; ++c) v[u][c] = 0.f;
+        v[u][0] = __ldg(row);
       }
     }
   };
   auto add_group = [&](int k, const float (&v)[U][VEC]) {
+    const float *xr = xs + (k - k0) * DX;
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      if (k + u < k1) {
+    for (int u = 0; u < U; ++u)
 #pragma unroll
-        for (int j = 0; j < D; ++j) {
-          const float x = __ldg(X + (int64_t)(k + u) * D + j);
+      for (int j = 0; j < DX; ++j) {
+        const float x = xr[u * DX + j];
 #pragma unroll
-          for (int c = 0; c < VEC; ++c) acc[c][j] = fmaf(v[u][c], x, acc[c][j]);
-        }
-#pragma unroll
-        for (int c = 0; c < VEC; ++c) acc[c][D] += v[u][c];
+        for (int c = 0; c < VEC; ++c) acc[c][j] = fmaf(v[u][c], x, acc[c][j]);
       }
-    }
   };
   float va[U][VEC], vb[U][VEC];
   int k = k0;
-  if (k < k1) load_group(k, va);
+  load_group(k, va);
   while (k < k1) {
     if (k + U < k1) load_group(k + U, vb);
     add_group(k, va);
@@ -129,32 +131,43 @@ __global__ void __launch_bounds__(128) narrow_wgrad_kernel(const float *__restri
   }
 #pragma unroll
   for (int c = 0; c < VEC; ++c) {
-    float *out = P + ((int64_t)z * M + m0 + c) * (D + 1);
+    float *out = P + ((int64_t)z * M + m0 + c) * DX;
 #pragma unroll
-    for (int j = 0; j <= D; ++j) out[j] = acc[c][j];
+    for (int j = 0; j < DX; ++j) out[j] = acc[c][j];
   }
 }
 
 cudaError_t launch_narrow_wgrad(const float *A, int64_t lda, int M, const float *X, int D, int K, float *P,
                                 size_t part_floats, int sm_count, float *out_w, float *out_b, cudaStream_t s) {
   if (M <= 0 || K <= 0) return cudaSuccess;
+  if (D < 1 || D > 16) return cudaErrorInvalidValue;
   const bool vec = (M % 4 == 0) && (lda % 4 == 0) && (reinterpret_cast<uintptr_t>(A) % 16 == 0);
   const int per_thread = vec ? 4 : 1;
   const int mb = (M / per_thread + 127) / 128;
   // at least four blocks of 128 threads per SM when the batch allows (a
-  // thread streams 64 tokens or more; chunks are whole 16-token groups)
+  // thread streams 64 tokens or more; chunks are whole 16-token groups), and
+  // a chunk's [X | 1] rows within 48 KB of shared memory
+  const int max_chunk = std::max(16, (int)((48 * 1024 / (4 * (D + 1))) & ~15));
   int splits = std::max(1, std::max(std::min(4 * sm_count / mb, K / 64), K / 2048));
+  splits = std::max(splits, (K + max_chunk - 1) / max_chunk);
   splits = std::min(splits, 1024);
   while (splits > 1 && (size_t)splits * M * (D + 1) > part_floats) --splits;
   const int chunk = (((K + splits - 1) / splits) + 15) & ~15;
   splits = (K + chunk - 1) / chunk;
+  const size_t smem = (size_t)chunk * (D + 1) * sizeof(float);
   dim3 grid(mb, splits);
   switch (D) {
-#define BKT_NW(DD)                                                                                  \
-  case DD:                                                                                          \
-    if (vec) narrow_wgrad_kernel<DD, 4><<<grid, 128, 0, s>>>(A, lda, M, X, K, P, chunk);            \
-    else narrow_wgrad_kernel<DD, 1><<<grid, 128, 0, s>>>(A, lda, M, X, K, P, chunk);                \
-    break;
+#define BKT_NW(DD)                                                                                           \
+  case DD: {                                                                                                 \
+    const void *kv = vec ? (const void *)narrow_wgrad_kernel<DD, 4> : (const void *)narrow_wgrad_kernel<DD, 1>; \
+    if (smem > 48 * 1024) {                                                                                  \
+      cudaError_t e = ensure_smem(kv, smem);                                                                 \
+      if (e != cudaSuccess) return e;                                                                        \
+    }                                                                                                        \
+    if (vec) narrow_wgrad_kernel<DD, 4><<<grid, 128, smem, s>>>(A, lda, M, X, K, P, chunk);                 \
+    else narrow_wgrad_kernel<DD, 1><<<grid, 128, smem, s>>>(A, lda, M, X, K, P, chunk);                     \
+    break;                                                                                                   \
+  }
     BKT_NW(1) BKT_NW(2) BKT_NW(3) BKT_NW(4) BKT_NW(5) BKT_NW(6) BKT_NW(7) BKT_NW(8)
     BKT_NW(9) BKT_NW(10) BKT_NW(11) BKT_NW(12) BKT_NW(13) BKT_NW(14) BKT_NW(15) BKT_NW(16)
 #undef BKT_NW
