@@ -421,6 +421,25 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
   Launch L{timer, s};
   Launch Ls{timer, side ? side : s};
 
+  // ---- W_out in the two split forms the output layer needs (rows for the
+  // logits, transposed for dY); they depend on the parameters only, so with
+  // a side stream they run beside the forward pass
+  const int DHp = (DH + 3) & ~3;  // split rows padded to 16 bytes for TMA
+  const int Cp = (C + 3) & ~3;
+  if (side) {
+    cudaError_t e = cudaEventRecord(fork_ev, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(side, fork_ev, 0);
+    if (e != cudaSuccess) return cuda_err("fork to the side stream", e);
+  }
+  Ls.run("split_rows", [&] { return bkt::launch_split_rows(params + lo.w_out, DH, C, DH, w.Woh, w.Wol, DHp, Ls.s); });
+  Ls.run("transpose_split", [&] {
+    return bkt::launch_transpose_split(params + lo.w_out, DH, nullptr, C, DH, w.WoTh, w.WoTl, Cp, Ls.s);
+  });
+  if (side) {
+    cudaError_t e = cudaEventRecord(join_ev, side);
+    if (e != cudaSuccess) return cuda_err("record on the side stream", e);
+  }
+
   // ---- a4: packed time-major input
   L.run("layout_gather", [&] { return bkt::launch_layout(ix, bt->x, lo.D0, w.X, w.tok_t, w.tok_r, w.prev_tok, s); });
 
@@ -493,12 +512,15 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
 
   // ---- a7: output layer and log-softmax
   // logits = Y W_out^T + b_out on the tensor cores (3xTF32; both operands are
-  // already K-contiguous, so they are split without transposing), then a
-  // log-softmax pass in place
+  // already K-contiguous, so they are split without transposing); the
+  // GEMM's epilogue holds whole rows (C <= 128 columns in one tile) and
+  // writes their log-softmax
   float *Ytop = w.Y[lo.L - 1];
-  const int DHp = (DH + 3) & ~3;  // split rows padded to 16 bytes for TMA
   L.run("split_rows", [&] { return bkt::launch_split_rows(Ytop, DH, NT, DH, w.BTf, w.BTl, DHp, s); });
-  L.run("split_rows", [&] { return bkt::launch_split_rows(params + lo.w_out, DH, C, DH, w.Wh, w.Wl, DHp, s); });
+  if (side) {
+    cudaError_t e = cudaStreamWaitEvent(s, join_ev, 0);  // the W_out splits
+    if (e != cudaSuccess) return cuda_err("wait for the side stream", e);
+  }
   {
     bkt::TcGemmArgs g{};
     g.M = NT;
@@ -506,21 +528,21 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     g.K = DH;
     g.A = w.BTf;
     g.lda = DHp;
-    g.B = w.Wh;
+    g.B = w.Woh;
     g.ldb = DHp;
     g.D = w.logit;
     g.ldd = C;
     g.bias = params + lo.b_out;
+    g.logsoftmax = 1;
     g.err = w.status;
-    L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.BTl, w.Wl, s); });
+    L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.BTl, w.Wol, s); });
   }
-  L.run("log_softmax", [&] { return bkt::launch_log_softmax_rows(w.logit, C, NT, C, s); });
   // ---- a8, a9: CTC
   L.run("ctc_tables", [&] {
     return bkt::launch_ctc_tables(ix, w.logit, C, cfg.blank, bt->labels, w.alpha, w.beta, loss, w.row_ok, w.status, s);
   });
-  L.run("ctc_grad", [&] {
-    return bkt::launch_ctc_grad(ix, w.logit, C, cfg.blank, bt->labels, w.alpha, w.beta, w.row_ok, s);
+  L.run("ctc_grad", [&] {  // dlogit in place, and its split for dY
+    return bkt::launch_ctc_grad(ix, w.logit, C, cfg.blank, bt->labels, w.alpha, w.beta, w.row_ok, w.Lh, w.Ll, Cp, s);
   });
 
   // ---- a10: output layer backward
@@ -592,25 +614,21 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
   tn_reduce_on(Ls, w.logit, C, C, Ytop, DH, nullptr, DH, grads + lo.w_out);
   bias_sum_on(Ls, w.logit, C, C, grads + lo.b_out);
   {
-    // dY = dlogit W_out on the tensor cores: dlogit split with its rows padded
-    // to a multiple of 4 floats (TMA strides), W_out split transposed
-    const int Cp = (C + 3) & ~3;
-    L.run("split_rows", [&] { return bkt::launch_split_rows(w.logit, C, NT, C, w.Lh, w.Ll, Cp, s); });
-    L.run("transpose_split", [&] {
-      return bkt::launch_transpose_split(params + lo.w_out, DH, nullptr, C, DH, w.Wh, w.Wl, Cp, s);
-    });
+    // dY = dlogit W_out on the tensor cores: dlogit split by the CTC gradient
+    // (rows padded to a multiple of 4 floats, TMA strides), W_out split
+    // transposed at the step's start
     bkt::TcGemmArgs g{};
     g.M = NT;
     g.N = DH;
     g.K = C;
     g.A = w.Lh;
     g.lda = Cp;
-    g.B = w.Wh;
+    g.B = w.WoTh;
     g.ldb = Cp;
     g.D = w.dY;
     g.ldd = DH;
     g.err = w.status;
-    L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.Ll, w.Wl, s); });
+    L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.Ll, w.WoTl, s); });
   }
 
   // ---- a11, a12: BPTT and weight gradients, top layer first.  With a side
@@ -953,6 +971,10 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
     const size_t WW = std::max(Cp * DHp, (lo.L > 1 && cfg->gemm_precision != BKT_GEMM_BF16) ? 4 * (size_t)H * DHp : 0);
     BKT_ALLOC(w.Wh, WW);
     BKT_ALLOC(w.Wl, WW);
+    BKT_ALLOC(w.Woh, (size_t)lo.C * DHp);
+    BKT_ALLOC(w.Wol, (size_t)lo.C * DHp);
+    BKT_ALLOC(w.WoTh, (size_t)DH * Cp);
+    BKT_ALLOC(w.WoTl, (size_t)DH * Cp);
     if (lo.L > 1 && cfg->gemm_precision != BKT_GEMM_BF16) {  // dX operands beside the side stream's AT
       BKT_ALLOC(w.DXh, NT * 4 * (size_t)H);
       BKT_ALLOC(w.DXl, NT * 4 * (size_t)H);
@@ -1220,6 +1242,10 @@ int bkt::step_on_scratch(const bkt_model_cfg *cfg, const bkt_batch *bt, const fl
     const size_t WW = std::max(Cp * DHp, (lo.L > 1 && cfg->gemm_precision != BKT_GEMM_BF16) ? 4 * (size_t)H * DHp : 0);
     w.Wh = cv.take<float>(WW);
     w.Wl = cv.take<float>(WW);
+    w.Woh = cv.take<float>((size_t)lo.C * DHp);
+    w.Wol = cv.take<float>((size_t)lo.C * DHp);
+    w.WoTh = cv.take<float>((size_t)DH * Cp);
+    w.WoTl = cv.take<float>((size_t)DH * Cp);
   }
   if (cfg->gemm_precision == BKT_GEMM_BF16) {
     const size_t NTp = (NT + 7) & ~size_t(7);

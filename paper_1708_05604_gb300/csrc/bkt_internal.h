@@ -99,8 +99,6 @@ cudaError_t launch_transpose_split(const float *src, int64_t lds, const int32_t 
 // The same split without transposing (row-major, destination stride ldd).
 cudaError_t launch_split_rows(const float *src, int64_t lds, int R, int C, float *hi, float *lo, int64_t ldd,
                               cudaStream_t s);
-// x[r][:C] <- log-softmax(x[r][:C]) in place (C <= 128).
-cudaError_t launch_log_softmax_rows(float *x, int64_t ld, int R, int C, cudaStream_t s);
 
 // bf16 tensor-core GEMM (k_gemm_tc.cu):
 //   D[m][n] (+)= sum_k A[m][k] B[n][k] (+ bias[n]); A, B bf16 with K contiguous
@@ -117,6 +115,7 @@ struct TcGemmArgs {
   int accumulate;
   float *P; int splits;
   int32_t *err;
+  int logsoftmax;  // 3xTF32 GEMM only: replace each output row by its log-softmax (N <= 128, no split)
 };
 int tc_splits(int M, int N, int K, int sm_count, size_t part_floats);
 cudaError_t launch_gemm_bf16_tc(const TcGemmArgs &g, cudaStream_t s);
@@ -149,10 +148,11 @@ cudaError_t launch_ctc_tables(const DevIdx &ix, const float *logp, int C, int bl
                               float *loss, int32_t *row_ok, int32_t *status,
                               cudaStream_t s);
 
-// a9: dlogit = softmax - posterior, written over logp in place.
-cudaError_t launch_ctc_grad(const DevIdx &ix, float *logp_dlogit, int C, int blank,
-                            const int32_t *labels, const float *alpha, const float *beta,
-                            const int32_t *row_ok, cudaStream_t s);
+// a9: dlogit = softmax - posterior, written over logp in place, and also as
+// tf32 hi + lo parts [n_tok x ld_split] for the dY GEMM (when dl_hi is set).
+cudaError_t launch_ctc_grad(const DevIdx &ix, float *logp_dlogit, int C, int blank, const int32_t *labels,
+                            const float *alpha, const float *beta, const int32_t *row_ok, float *dl_hi, float *dl_lo,
+                            int64_t ld_split, cudaStream_t s);
 
 // Geometry of the recurrent kernels for one layer.
 //   mode 1: one CTA per bc rows holds all of W_hh (H in {32, 64, 128});
@@ -230,6 +230,8 @@ struct StepBufs {
   float *BTf, *BTl;                           // [dirs*H x NTq] transposed X, h_{t-1} or Y, hi and lo
   float *Lh, *Ll;                             // [NT x Cp] dlogit split, rows padded to Cp = C rounded to 4
   float *Wh, *Wl;                             // [Cp x dirs*H] W_out split (or its transpose)
+  float *Woh, *Wol;                           // [C x DHp] W_out split for the logits (made at the step's start)
+  float *WoTh, *WoTl;                         // [dirs*H x Cp] W_out transposed and split for dY
   // bf16 GEMM path only (null otherwise)
   void *Yb;                                   // [NT x dirs*H] bf16 layer input of a projection
   void *dZb;                                  // [NT x 4H] bf16 dz (input-gradient GEMM)

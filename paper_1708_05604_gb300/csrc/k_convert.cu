@@ -140,40 +140,6 @@ cudaError_t launch_split_rows(const float *src, int64_t lds, int R, int C, float
   return cudaGetLastError();
 }
 
-// In-place log-softmax over the C columns of each row, one warp per row.
-__global__ void log_softmax_rows_kernel(float *__restrict__ x, int64_t ld, int R, int C) {
-  const int lane = threadIdx.x & 31;
-  const int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (r >= R) return;
-  float *row = x + (int64_t)r * ld;
-  float v[4];
-  float mx = -INFINITY;
-#pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    const int c = lane + 32 * j;
-    v[j] = c < C ? row[c] : -INFINITY;
-    mx = fmaxf(mx, v[j]);
-  }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-  float se = 0.f;
-#pragma unroll
-  for (int j = 0; j < 4; ++j) se += (lane + 32 * j < C) ? expf(v[j] - mx) : 0.f;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
-  const float lz = mx + logf(se);
-#pragma unroll
-  for (int j = 0; j < 4; ++j)
-    if (lane + 32 * j < C) row[lane + 32 * j] = v[j] - lz;
-}
-
-cudaError_t launch_log_softmax_rows(float *x, int64_t ld, int R, int C, cudaStream_t s) {
-  if (R <= 0) return cudaSuccess;
-  if (C > 128) return cudaErrorInvalidValue;
-  log_softmax_rows_kernel<<<(R + 7) / 8, 256, 0, s>>>(x, ld, R, C);
-  return cudaGetLastError();
-}
-
 // P[z][m] = sum of A[r][m] over the rows of chunk z (ceil(R / splits) rows).
 // A block holds 32 columns (coalesced along m); its 8 warps take rows
 // r0 + g, r0 + g + 8, ... with four running sums each, and warp 0 adds the 8

@@ -342,14 +342,18 @@ cudaError_t launch_ctc_tables(const DevIdx &ix, const float *logp, int C, int bl
 //   v(s) = a_t(s) + bh_t(s) - log2(e) lp_t(l'_s)  (log2 of alpha_t(s) beta_t(s), offset)
 //   gamma(s) = 2^(v(s) - lse2_s v)
 //   dlogit[k] = exp(lp_t(k)) - sum_{s: l'_s = k} gamma(s)
-// written over the log-probabilities in place.  Blank mass is a warp sum;
-// label mass goes through a per-warp shared row.  Rows without an alignment
-// (or with a bad label) get zeros.
+// written over the log-probabilities in place, and (when dl_hi is set) as
+// the tf32 hi + lo split the dY GEMM reads, rows padded to ld_split (both
+// parts rounded to nearest: |x - hi - lo| <= 2^-22 |x|).  Blank mass is a
+// warp sum; label mass goes through a per-warp shared row.  Rows without an
+// alignment (or with a bad label) get zeros.
 __global__ void __launch_bounds__(256) ctc_grad_kernel(DevIdx ix, float *__restrict__ lp_dl, int C, int blank,
                                                        const int32_t *__restrict__ labels,
                                                        const float *__restrict__ alpha,
                                                        const float *__restrict__ beta,
-                                                       const int32_t *__restrict__ row_ok) {
+                                                       const int32_t *__restrict__ row_ok,
+                                                       float *__restrict__ dl_hi, float *__restrict__ dl_lo,
+                                                       int64_t ld_split) {
   __shared__ float acc[8][kMaxClasses];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int tok = blockIdx.x * 8 + w;
@@ -405,13 +409,27 @@ __global__ void __launch_bounds__(256) ctc_grad_kernel(DevIdx ix, float *__restr
 #pragma unroll
   for (int j = 0; j < 4; ++j)
     if (lane + 32 * j < C) row[lane + 32 * j] = out[j];
+  if (dl_hi) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int k = lane + 32 * j;
+      if (k < (int)ld_split) {  // the padding columns get zeros
+        const float x = k < C ? out[j] : 0.f;
+        const float hv = __uint_as_float((__float_as_uint(x) + 0x1000u) & 0xFFFFE000u);
+        const float lv = __uint_as_float((__float_as_uint(x - hv) + 0x1000u) & 0xFFFFE000u);
+        dl_hi[(int64_t)tok * ld_split + k] = hv;
+        dl_lo[(int64_t)tok * ld_split + k] = lv;
+      }
+    }
+  }
 }
 
 cudaError_t launch_ctc_grad(const DevIdx &ix, float *lp_dl, int C, int blank, const int32_t *labels,
-                            const float *alpha, const float *beta, const int32_t *row_ok, cudaStream_t s) {
-  if (C > kMaxClasses) return cudaErrorInvalidValue;
+                            const float *alpha, const float *beta, const int32_t *row_ok, float *dl_hi, float *dl_lo,
+                            int64_t ld_split, cudaStream_t s) {
+  if (C > kMaxClasses || (dl_hi && (ld_split < C || ld_split > kMaxClasses || !dl_lo))) return cudaErrorInvalidValue;
   const int blocks = (ix.n_tok + 7) / 8;
-  ctc_grad_kernel<<<blocks, 256, 0, s>>>(ix, lp_dl, C, blank, labels, alpha, beta, row_ok);
+  ctc_grad_kernel<<<blocks, 256, 0, s>>>(ix, lp_dl, C, blank, labels, alpha, beta, row_ok, dl_hi, dl_lo, ld_split);
   return cudaGetLastError();
 }
 

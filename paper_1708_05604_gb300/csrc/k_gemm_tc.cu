@@ -354,6 +354,36 @@ __global__ void __launch_bounds__(128, 1)
     ld = g.ldd;
   }
   const bool vec = ((ld & 3) == 0) && ((reinterpret_cast<uintptr_t>(g.P ? g.P : g.D) & 15) == 0);
+  if (g.logsoftmax) {
+    // the whole row (N <= FBN columns, one tile) is in this thread's TMEM
+    // lane: bias, then x - max - ln sum exp(x - max) over the N columns
+    float x[FBN];
+#pragma unroll
+    for (int c0 = 0; c0 < FBN; c0 += 32) {
+      uint32_t v[32];
+      __syncwarp();
+      tmem_ld32(trow + c0, v);
+#pragma unroll
+      for (int j = 0; j < 32; ++j) x[c0 + j] = __uint_as_float(v[j]);
+    }
+    if (write) {
+      float mx = -INFINITY;
+#pragma unroll
+      for (int j = 0; j < FBN; ++j)
+        if (j < g.N) {
+          x[j] = (nk > 0 ? x[j] : 0.f) + (g.bias ? g.bias[j] : 0.f);
+          mx = fmaxf(mx, x[j]);
+        }
+      float se = 0.f;
+#pragma unroll
+      for (int j = 0; j < FBN; ++j)
+        if (j < g.N) se += expf(x[j] - mx);
+      const float lz = mx + logf(se);
+#pragma unroll
+      for (int j = 0; j < FBN; ++j)
+        if (j < g.N) out[j] = x[j] - lz;
+    }
+  } else
 #pragma unroll 1
   for (int c0 = 0; c0 < FBN; c0 += 32) {
     uint32_t v[32];
@@ -726,6 +756,7 @@ cudaError_t launch_gemm_tf32x3_tc(const TcGemmArgs &g, const void *A_lo, const v
                                                   15) ||
       (g.P && g.splits < 1) || (!g.P && !g.D))
     return cudaErrorInvalidValue;
+  if (g.logsoftmax && (g.P || g.N > FBN || g.accumulate)) return cudaErrorInvalidValue;
   CUtensorMap tah, tal, tbh, tbl;
   if (!make_map(&tah, g.A, (uint64_t)g.K, (uint64_t)g.M, g.lda, FBM, true) ||
       !make_map(&tal, A_lo, (uint64_t)g.K, (uint64_t)g.M, g.lda, FBM, true) ||
