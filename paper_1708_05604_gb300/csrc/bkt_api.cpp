@@ -546,12 +546,12 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
   });
 
   // ---- a10: output layer backward
-  // fp32 contractions over tokens on the tensor cores (3xTF32).  Small
-  // aligned outputs read the token-major operands directly (split and
-  // swizzled while loading); otherwise the operands are transposed and split
-  // first and the TMA-fed GEMM runs (measured on GB300: the fused kernel moves
-  // more bytes through shared memory per slab, so it wins only while the
-  // transposes dominate, e.g. dW_hh at H = 128: 43 us against 66 us)
+  // fp32 contractions over tokens on the tensor cores (3xTF32).  Operands
+  // with 16-byte aligned rows are read token-major by the fused kernel
+  // (split and swizzled while loading); others (dlogit: C = 81 columns) are
+  // transposed and split first for the TMA-fed GEMM.  Measured on GB300:
+  // dW_hh at H = 128, 32 us fused against 66 us; at H = 512, 1.22 ms
+  // against 1.31 ms.
   const int NTq = (NT + 7) & ~7;
   // the transposed split of A left in AT by the last fallback call: dW_ih of
   // a layer above the first reuses the one its dW_hh made (nothing else
@@ -560,8 +560,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
   auto tn_reduce_on = [&](Launch &X, const float *A, int64_t lda, int M, const float *B, int64_t ldb,
                           const int32_t *gather, int N, float *out) {
     const bool fused = ((lda | ldb | M | N) & 3) == 0 &&
-                       ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(B)) & 15) == 0 &&
-                       (int64_t)M * N <= 128 * 1024;
+                       ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(B)) & 15) == 0;
     if (fused) {
       bkt::TnGemmArgs g{};
       g.M = M;

@@ -427,56 +427,45 @@ __global__ void __launch_bounds__(128, 1)
 // giving a zero row), as the weight gradients need (k = token), without
 // transposed and split copies of the operands.
 //
-// Eight converter warps and one MMA warp.  Per 32-token slab the converters
-// copy the raw rows of both tiles (32 x 128 floats each, as they lie in
-// global memory) into a kTnRaw-slot ring with asynchronous 16-byte copies
-// (rows outside the operands zero-filled by a zero source size), then split
-// each value into tf32 hi + lo and store the four tiles K-major in the
-// 128-byte swizzled layout TMA would produce (16-byte chunk c of row r at
-// chunk position c ^ (r & 7)) in one of two MMA stages, make the stores
-// visible to the tensor core (fence.proxy.async) and arrive on the stage's
-// full barrier.  The MMA warp waits on it, issues the twelve MMAs and commits
-// them to the stage's empty barrier, which the converters wait on before
-// refilling the stage; so the MMAs of one slab run while the next is
-// converted (issuing them from a converter warp held its warp for the MMAs'
-// duration).  The split truncates: hi = x with the low 13 mantissa bits
-// cleared, lo = (x - hi) likewise, |x - hi - lo| <= 2^-20 |x| (three
-// instructions per value; rounding both parts cost five).  One 256-thread
-// barrier per slab both publishes the slab's copies and frees the previous
-// raw slot, whose refill is issued right after it.  A thread's gather
-// indices are loaded (from clamped positions, never selected on) two slabs
-// before its copies use them; the loop is unrolled over two slabs to keep
-// those registers statically named.  Every wait is bounded; on expiry the
-// CTA records an error flag.  The epilogue splits the 128 accumulator columns
+// Eight converter warps and one MMA warp.  Per 32-token slab a converter
+// thread loads a 4 x 4 block of each tile (tokens 4 kc .. 4 kc + 3 of the
+// slab, rows r0 .. r0 + 3) as four 16-byte vectors, two slabs ahead, into
+// registers; out-of-range rows read a zero vector in global memory instead,
+// so no instruction consumes a loaded value before its slab is converted (a
+// warp issues in order).  Converting a slab transposes the block in
+// registers, splits each value into tf32 hi + lo (truncating: hi = x with the
+// low 13 mantissa bits cleared, lo = (x - hi) likewise, |x - hi - lo| <=
+// 2^-20 |x|) and stores four 16-byte K-major chunks per tile in the 128-byte
+// swizzled layout TMA would produce (chunk c of row r at chunk position
+// c ^ (r & 7)), into one of kTnStages MMA stages; the warp then makes its
+// stores visible to the tensor core (fence.proxy.async) and arrives on the
+// stage's full barrier.  The MMA warp waits on it, issues the twelve MMAs and
+// commits them to the stage's empty barrier, which the converter warps wait
+// on before refilling the stage.  Converter warps never wait for each other.
+// A thread's gather indices are loaded two slabs before the vectors they
+// address; the loop is unrolled over two slabs to keep the prefetch
+// registers statically named.  Every wait is bounded; on expiry the CTA
+// records an error flag.  The epilogue splits the 128 accumulator columns
 // between the two converter warps of each TMEM lane quarter.
 namespace {
 
 constexpr int kTnConv = 256;                      // converter threads (warps 0-7)
 constexpr int kTnThreads = kTnConv + 32;          // + the MMA warp
-constexpr int kTnStages = 2;                      // converted (MMA) stages
-constexpr int kTnRaw = 3;                         // raw slabs in flight
-constexpr uint32_t kTnRawTile = FBK * 128 * 4;    // 16 KB: 32 rows x 128 floats
-constexpr uint32_t kTnRawSlab = 2 * kTnRawTile;   // A and B
-constexpr size_t kTnSmem = 1024 + (size_t)kTnStages * kFStage + (size_t)kTnRaw * kTnRawSlab + 256;
+constexpr int kTnStages = 3;                      // converted (MMA) stages
+constexpr size_t kTnSmem = 1024 + (size_t)kTnStages * kFStage + 256;
+
+__device__ __align__(16) float g_tn_zero[4];      // the zero vector out-of-range rows read
 
 __device__ __forceinline__ void split_tf32_trunc(float x, float &h, float &l) {
   h = __uint_as_float(__float_as_uint(x) & 0xFFFFE000u);
   l = __uint_as_float(__float_as_uint(x - h) & 0xFFFFE000u);
 }
-// Asynchronous 16-byte global -> shared copy; `bytes` of the source are read
-// and the rest is zero-filled (0: nothing is read).
-__device__ __forceinline__ void cpa16(uint32_t dst, const void *src, uint32_t bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(bytes));
-}
-// Barrier 1 over the converter warps; returns whether any passed `fail`.
-__device__ __forceinline__ bool conv_barrier_or(bool fail) {
-  uint32_t r;
-  asm volatile(
-      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n barrier.cta.red.or.pred q, 1, %2, p;\n selp.u32 %0, 1, 0, q;\n}\n"
-      : "=r"(r)
-      : "r"((uint32_t)fail), "n"(kTnConv)
-      : "memory");
-  return r != 0;
+// A read-only 16-byte load issued where it is written (volatile: not moved
+// toward its use two slabs later).
+__device__ __forceinline__ float4 ldg4_pinned(const float *p) {
+  float4 v;
+  asm volatile("ld.global.nc.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "l"(p));
+  return v;
 }
 
 }  // namespace
@@ -484,8 +473,7 @@ __device__ __forceinline__ bool conv_barrier_or(bool fail) {
 __global__ void __launch_bounds__(kTnThreads, 1) gemm_tf32x3_tn_kernel(TnGemmArgs g) {
   extern __shared__ uint8_t tc_smem_raw[];
   uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(tc_smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t *raw = base + kTnStages * kFStage;                                 // [kTnRaw][A | B][32][128]
-  uint64_t *bars = reinterpret_cast<uint64_t *>(raw + kTnRaw * kTnRawSlab);  // full[S], empty[S], done
+  uint64_t *bars = reinterpret_cast<uint64_t *>(base + kTnStages * kFStage);  // full[S], empty[S], done
   uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 2 * kTnStages + 1);
   int *abort_s = reinterpret_cast<int *>(tslot + 1);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -544,67 +532,45 @@ __global__ void __launch_bounds__(kTnThreads, 1) gemm_tf32x3_tn_kernel(TnGemmArg
     }
     __syncwarp();
   } else {  // converters
-    // copy geometry: rows warp + 8 j (j < 4) of a slab, columns 4 lane .. +3
-    const int c4 = 4 * lane;
-    const bool a_col = m0 + c4 < g.M, b_col = n0 + c4 < g.N;
-    const float *acol = g.A + (m0 + c4), *bcol = g.B + (n0 + c4);
-    auto rows_of = [&](int i, int (&br)[4]) {  // B rows of this thread's copies of slab i (validity checked at use)
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int kl = i * FBK + warp + 8 * j;
-        br[j] = (g.gather && ntok > 0) ? __ldg(g.gather + kbase + min(kl, ntok - 1)) : kbase + kl;
-      }
-    };
-    auto issue = [&](int i, const int (&br)[4]) {  // raw slab i -> ring slot i % kTnRaw
-      const uint32_t slot = su32(raw + (i % kTnRaw) * kTnRawSlab);
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int k = warp + 8 * j;
-        const int kl = i * FBK + k;
-        const uint32_t dst = slot + (uint32_t)(k * 128 + c4) * 4;
-        const bool kin = kl < ntok;
-        const bool av = kin && a_col;
-        cpa16(dst, av ? acol + (int64_t)(kbase + kl) * g.lda : g.A, av ? 16u : 0u);
-        const bool bv = kin && br[j] >= 0 && b_col;
-        cpa16(dst + kTnRawTile, bv ? bcol + (int64_t)br[j] * g.ldb : g.B, bv ? 16u : 0u);
-      }
-      asm volatile("cp.async.commit_group;" ::: "memory");
-    };
-
-    // conversion geometry: warp w covers rows 32 (w & 3) .. +31 and k chunks
-    // 4 (w >> 2) .. +3; lane l takes rows r0 .. r0+3 with r0 = 32 (w & 3) + 4 rb,
-    // rb = l & 7, and chunk kc = 4 (w >> 2) + ((rb >> 1) + (l >> 3)) mod 4, so
-    // that the eight lanes of each quarter warp (one 128-bit shared access
-    // phase) read eight distinct raw 16-byte positions and write eight
-    // distinct swizzled chunk positions
+    // geometry: warp w covers rows 32 (w & 3) .. +31 and k chunks 4 (w >> 2)
+    // .. +3; lane l takes rows r0 .. r0+3 with r0 = 32 (w & 3) + 4 rb, rb =
+    // l & 7, and chunk kc = 4 (w >> 2) + ((rb >> 1) + (l >> 3)) mod 4, so
+    // that the eight lanes of each quarter warp (one 128-bit shared store
+    // phase) write eight distinct swizzled chunk positions
     const int rb = lane & 7;
     const int r0 = 32 * (warp & 3) + 4 * rb, kc = 4 * (warp >> 2) + (((rb >> 1) + (lane >> 3)) & 3);
-    bool fail = false;
-
-    // slab i: its copies done and the previous raw slot free (one barrier),
-    // refill that slot with slab i-1+kTnRaw, load the rows of slab i+kTnRaw+1,
-    // convert slab i into stage i % 2 and hand it to the MMA warp
-    auto slab = [&](int i, int (&br)[4]) -> bool {
-      const int s = i % kTnStages;
-      asm volatile("cp.async.wait_group %0;" ::"n"(kTnRaw - 2) : "memory");  // raw slab i (own pieces)
-      if (conv_barrier_or(fail)) return false;
-      if (i > 0) {
-        issue(i - 1 + kTnRaw, br);  // past the last slab: zero-filled pieces, never converted
-        rows_of(i + 1 + kTnRaw, br);
+    const bool a_in = m0 + r0 < g.M, b_in = n0 + r0 < g.N;  // M, N multiples of 4: a block is in or out
+    const float *acol = g.A + (m0 + r0), *bcol = g.B + (n0 + r0);
+    // B rows of this thread's tokens of slab i (gather read at clamped
+    // positions; validity is checked where the rows are used); a uniform
+    // branch, so that no select waits for the loaded indices
+    const bool gathered = g.gather && ntok > 0;
+    auto rows_of = [&](int i, int (&br)[4]) {
+      if (gathered) {
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) br[kk] = __ldg(g.gather + kbase + min(i * FBK + 4 * kc + kk, ntok - 1));
+      } else {
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) br[kk] = kbase + i * FBK + 4 * kc + kk;
       }
-      if (i >= kTnStages && !mbar_wait(empty0 + 8 * s, ((i / kTnStages) - 1) & 1)) {
-        fail = true;
-        return true;
-      }
-      const float *ra = reinterpret_cast<const float *>(raw + (i % kTnRaw) * kTnRawSlab);
-      const float *rbp = ra + FBK * 128;
-      uint8_t *st = base + s * kFStage;
-      float4 va[4], vb[4];
+    };
+    auto load = [&](int i, const int (&br)[4], float4 (&va)[4], float4 (&vb)[4]) {
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk) {
-        va[kk] = *reinterpret_cast<const float4 *>(ra + (4 * kc + kk) * 128 + r0);
-        vb[kk] = *reinterpret_cast<const float4 *>(rbp + (4 * kc + kk) * 128 + r0);
+        const int kl = i * FBK + 4 * kc + kk;
+        const bool kin = kl < ntok;
+        va[kk] = ldg4_pinned(kin && a_in ? acol + (int64_t)(kbase + kl) * g.lda : g_tn_zero);
+        vb[kk] = ldg4_pinned(kin && b_in && br[kk] >= 0 ? bcol + (int64_t)br[kk] * g.ldb : g_tn_zero);
       }
+    };
+    bool fail = false;
+    auto slab = [&](int i, float4 (&va)[4], float4 (&vb)[4], int (&br)[4]) -> bool {
+      const int s = i % kTnStages;
+      if (i >= kTnStages && !mbar_wait(empty0 + 8 * s, ((i / kTnStages) - 1) & 1)) {
+        fail = true;
+        return false;
+      }
+      uint8_t *st = base + s * kFStage;
 #pragma unroll
       for (int mm = 0; mm < 4; ++mm) {
         const int r = r0 + mm;
@@ -627,25 +593,25 @@ __global__ void __launch_bounds__(kTnThreads, 1) gemm_tf32x3_tn_kernel(TnGemmArg
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       __syncwarp();
       if (lane == 0) mbar_arrive(full0 + 8 * s);
+      // the vectors of slab i + 2 (rows loaded two slabs ago), then the rows of slab i + 4
+      load(i + 2, br, va, vb);
+      rows_of(i + 4, br);
       return true;
     };
 
-    int brA[4], brB[4];  // rows of the slabs copied at odd and even slabs
-    {
-#pragma unroll 1
-      for (int i = 0; i < kTnRaw; ++i) {
-        rows_of(i, brA);
-        issue(i, brA);
-      }
-    }
-    rows_of(kTnRaw, brB);      // copied at slab 1
-    rows_of(kTnRaw + 1, brA);  // copied at slab 2
+    float4 a0[4], b0[4], a1[4], b1[4];  // slabs of even and odd index
+    int r_even[4], r_odd[4];
+    rows_of(0, r_even);
+    load(0, r_even, a0, b0);
+    rows_of(1, r_odd);
+    load(1, r_odd, a1, b1);
+    rows_of(2, r_even);
+    rows_of(3, r_odd);
     for (int i = 0; i < nk; i += 2) {
-      if (!slab(i, brA)) break;
-      if (i + 1 < nk && !slab(i + 1, brB)) break;
+      if (!slab(i, a0, b0, r_even)) break;
+      if (i + 1 < nk && !slab(i + 1, a1, b1, r_odd)) break;
     }
     if (fail) *abort_s = 1;
-    asm volatile("cp.async.wait_all;" ::: "memory");
   }
 
   const bool ready = mbar_wait(done, 0);
