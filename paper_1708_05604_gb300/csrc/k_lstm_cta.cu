@@ -164,9 +164,17 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
     return toff[tt] + r0 + b;
   };
   float cst[BC];
-  auto issue = [&](int b, int s) {  // the Zx row of step s of row b into its ring slot
+  // token of step s of row b at a clamped (always valid) time; meaningful
+  // only while s < len[b].  The prefetch reads it one step before its copy
+  // needs it, so the copy's address waits on no load (a warp issues in order)
+  auto tok_clamped = [&](int b, int s) {
+    const int last = max(len[b] - 1, 0);
+    const int tt = d == 0 ? min(s, last) : max(last - s, 0);
+    return toff[tt] + r0 + b;
+  };
+  auto issue_at = [&](int b, int s, int tk) {  // the Zx row of step s of row b (token tk) into its ring slot
     if (s < len[b]) {
-      const float *src = Z + (size_t)tok_at(b, s) * G;
+      const float *src = Z + (size_t)tk * G;
       float *slot = zr + ((size_t)b * kRing + s % kRing) * G;
       for (int i = t; i < G / 4; i += NTH) cp_async16(slot + 4 * i, src + 4 * i);
     }
@@ -175,9 +183,12 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
   for (int b = 0; b < BC; ++b) cst[b] = 0.f;
   for (int j = 0; j < kPF; ++j) {
 #pragma unroll
-    for (int b = 0; b < BC; ++b) issue(b, j);
+    for (int b = 0; b < BC; ++b) issue_at(b, j, tok_clamped(b, j));
     cp_commit();
   }
+  int tk_pf[BC];  // token of step s + kPF
+#pragma unroll
+  for (int b = 0; b < BC; ++b) tk_pf[b] = tok_clamped(b, kPF);
   cp_wait_pending<kPF - 1>();  // step 0's rows
   __syncthreads();
   for (int s = 0; s < Tg; ++s) {
@@ -189,7 +200,8 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
       const float *slot = zr + ((size_t)b * kRing + s % kRing) * G;
       const float zc0 = slot[zo0], zc1 = slot[zo1];
       const int tc = tok_at(b, s);
-      issue(b, s + kPF);
+      issue_at(b, s + kPF, tk_pf[b]);
+      tk_pf[b] = tok_clamped(b, s + kPF + 1);
       const float *hv = hs + (p * BC + b) * 8 * HS + ks * HS;
       float acc[16];
 #pragma unroll
@@ -294,10 +306,17 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
   // phase B inputs of step s, kPF steps ahead: the gate row [4H], c_t [H],
   // c_{t-1} [H] (zeros at the start) and dY [H] of the row, in 16-byte pieces
   float dc[BC];
-  auto issue = [&](int b, int s) {
+  // token of step s of row b at a clamped (always valid) time; meaningful
+  // only while 0 <= s < len[b].  The prefetch reads the tokens of its step
+  // one step before its copies need them, so no copy address waits on a load
+  auto tok_clamped = [&](int b, int s) {
+    const int last = max(len[b] - 1, 0);
+    const int tt = d == 0 ? min(max(s, 0), last) : max(last - max(s, 0), 0);
+    return toff[tt] + r0 + b;
+  };
+  auto issue = [&](int b, int s, int tk, int tp) {  // tp: token of step s - 1 (used when s > 0)
     if (s >= 0 && s < len[b]) {
-      const int tk = tok_at(b, s);
-      const int tp = s > 0 ? tok_at(b, s - 1) : -1;
+      if (s == 0) tp = -1;
       float *slot = ring + ((size_t)b * kRing + s % kRing) * 7 * H;
       for (int i = t; i < 7 * H / 4; i += NTH) {
         const int q = 4 * i;  // float offset in the slot
@@ -314,8 +333,14 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
   for (int b = 0; b < BC; ++b) dc[b] = 0.f;
   for (int j = 0; j < kPF; ++j) {
 #pragma unroll
-    for (int b = 0; b < BC; ++b) issue(b, Tg - 1 - j);
+    for (int b = 0; b < BC; ++b) issue(b, Tg - 1 - j, tok_clamped(b, Tg - 1 - j), tok_clamped(b, Tg - 2 - j));
     cp_commit();
+  }
+  int tk_pf[BC], tp_pf[BC];  // tokens of steps s - kPF and s - kPF - 1
+#pragma unroll
+  for (int b = 0; b < BC; ++b) {
+    tk_pf[b] = tok_clamped(b, Tg - 1 - kPF);
+    tp_pf[b] = tok_clamped(b, Tg - 2 - kPF);
   }
   cp_wait_pending<kPF - 1>();  // the first step's rows
   __syncthreads();
@@ -352,7 +377,11 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_bwd_cta_kernel(RecArgs a) {
     // backwards, so a shorter row becomes active only later and needs its
     // first kPF steps in flight by then
 #pragma unroll
-    for (int b = 0; b < BC; ++b) issue(b, s - kPF);
+    for (int b = 0; b < BC; ++b) {
+      issue(b, s - kPF, tk_pf[b], tp_pf[b]);
+      tk_pf[b] = tp_pf[b];  // the next step's token is this one's predecessor
+      tp_pf[b] = tok_clamped(b, s - kPF - 2);
+    }
     cp_commit();
     __syncthreads();
     // phase A: column partials of W_hh^T dz over this warp's 16 x 4 rows
