@@ -342,11 +342,14 @@ cudaError_t launch_ctc_tables(const DevIdx &ix, const float *logp, int C, int bl
 //   v(s) = a_t(s) + bh_t(s) - log2(e) lp_t(l'_s)  (log2 of alpha_t(s) beta_t(s), offset)
 //   gamma(s) = 2^(v(s) - lse2_s v)
 //   dlogit[k] = exp(lp_t(k)) - sum_{s: l'_s = k} gamma(s)
+// For labels of up to 256 extended positions each lane keeps the v(s) of its
+// positions in registers, so the tables, labels and emissions are read once.
 // written over the log-probabilities in place, and (when dl_hi is set) as
 // the tf32 hi + lo split the dY GEMM reads, rows padded to ld_split (both
 // parts rounded to nearest: |x - hi - lo| <= 2^-22 |x|).  Blank mass is a
 // warp sum; label mass goes through a per-warp shared row.  Rows without an
 // alignment (or with a bad label) get zeros.
+template <int JC>  // JC > 0: v(s) of positions s = lane + 32 j (j < JC) kept in registers (S <= 32 JC)
 __global__ void __launch_bounds__(256) ctc_grad_kernel(DevIdx ix, float *__restrict__ lp_dl, int C, int blank,
                                                        const int32_t *__restrict__ labels,
                                                        const float *__restrict__ alpha,
@@ -372,37 +375,73 @@ __global__ void __launch_bounds__(256) ctc_grad_kernel(DevIdx ix, float *__restr
     const float *a = alpha + ix.row_ctc_off[r] + (int64_t)t * S;
     const float *b = beta + ix.row_ctc_off[r] + (int64_t)t * S;
     const float lpb = row[blank];
-    float mx = -CUDART_INF_F;
-    for (int s = lane; s < S; s += 32) {
-      const float e = (s & 1) ? row[lab[(s - 1) >> 1]] : lpb;
-      mx = fmaxf(mx, a[s] + b[s] - kLog2e * e);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    float se = 0.f;
-    for (int s = lane; s < S; s += 32) {
-      const float e = (s & 1) ? row[lab[(s - 1) >> 1]] : lpb;
-      se += exp2f(a[s] + b[s] - kLog2e * e - mx);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
-    const float lz = mx + log2f(se);
     float blank_mass = 0.f;
     __syncwarp();
-    for (int s = lane; s < S; s += 32) {
-      const int k = (s & 1) ? lab[(s - 1) >> 1] : blank;
-      const float e = (s & 1) ? row[k] : lpb;
-      const float g = exp2f(a[s] + b[s] - kLog2e * e - lz);
-      if (s & 1) atomicAdd(&acc[w][k], g);
-      else blank_mass += g;
+    if (JC > 0) {
+      // one pass of loads: label, emission and both tables of each position
+      float v[JC > 0 ? JC : 1];
+      int k[JC > 0 ? JC : 1];
+      float mx = -CUDART_INF_F;
+#pragma unroll
+      for (int j = 0; j < JC; ++j) {
+        const int s = lane + 32 * j;
+        k[j] = blank;
+        v[j] = -CUDART_INF_F;
+        if (s < S) {  // positions past S read nothing
+          if (s & 1) k[j] = lab[(s - 1) >> 1];
+          const float e = (s & 1) ? row[k[j]] : lpb;
+          v[j] = a[s] + b[s] - kLog2e * e;
+        }
+        mx = fmaxf(mx, v[j]);
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      float se = 0.f;
+#pragma unroll
+      for (int j = 0; j < JC; ++j) se += exp2f(v[j] - mx);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
+      const float lz = mx + log2f(se);
+#pragma unroll
+      for (int j = 0; j < JC; ++j) {
+        const int s = lane + 32 * j;
+        if (s < S) {
+          const float gm = exp2f(v[j] - lz);
+          if (s & 1) atomicAdd(&acc[w][k[j]], gm);
+          else blank_mass += gm;
+        }
+      }
+    } else {
+      float mx = -CUDART_INF_F;
+      for (int s = lane; s < S; s += 32) {
+        const float e = (s & 1) ? row[lab[(s - 1) >> 1]] : lpb;
+        mx = fmaxf(mx, a[s] + b[s] - kLog2e * e);
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      float se = 0.f;
+      for (int s = lane; s < S; s += 32) {
+        const float e = (s & 1) ? row[lab[(s - 1) >> 1]] : lpb;
+        se += exp2f(a[s] + b[s] - kLog2e * e - mx);
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) se += __shfl_xor_sync(0xffffffffu, se, o);
+      const float lz = mx + log2f(se);
+      for (int s = lane; s < S; s += 32) {
+        const int kk = (s & 1) ? lab[(s - 1) >> 1] : blank;
+        const float e = (s & 1) ? row[kk] : lpb;
+        const float gm = exp2f(a[s] + b[s] - kLog2e * e - lz);
+        if (s & 1) atomicAdd(&acc[w][kk], gm);
+        else blank_mass += gm;
+      }
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) blank_mass += __shfl_xor_sync(0xffffffffu, blank_mass, o);
     __syncwarp();
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      const int k = lane + 32 * j;
-      out[j] = expf(lpk[j]) - acc[w][k] - (k == blank ? blank_mass : 0.f);
+      const int kk = lane + 32 * j;
+      out[j] = expf(lpk[j]) - acc[w][kk] - (kk == blank ? blank_mass : 0.f);
     }
   }
   __syncwarp();
@@ -412,13 +451,13 @@ __global__ void __launch_bounds__(256) ctc_grad_kernel(DevIdx ix, float *__restr
   if (dl_hi) {
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      const int k = lane + 32 * j;
-      if (k < (int)ld_split) {  // the padding columns get zeros
-        const float x = k < C ? out[j] : 0.f;
+      const int kk = lane + 32 * j;
+      if (kk < (int)ld_split) {  // the padding columns get zeros
+        const float x = kk < C ? out[j] : 0.f;
         const float hv = __uint_as_float((__float_as_uint(x) + 0x1000u) & 0xFFFFE000u);
         const float lv = __uint_as_float((__float_as_uint(x - hv) + 0x1000u) & 0xFFFFE000u);
-        dl_hi[(int64_t)tok * ld_split + k] = hv;
-        dl_lo[(int64_t)tok * ld_split + k] = lv;
+        dl_hi[(int64_t)tok * ld_split + kk] = hv;
+        dl_lo[(int64_t)tok * ld_split + kk] = lv;
       }
     }
   }
@@ -429,7 +468,11 @@ cudaError_t launch_ctc_grad(const DevIdx &ix, float *lp_dl, int C, int blank, co
                             int64_t ld_split, cudaStream_t s) {
   if (C > kMaxClasses || (dl_hi && (ld_split < C || ld_split > kMaxClasses || !dl_lo))) return cudaErrorInvalidValue;
   const int blocks = (ix.n_tok + 7) / 8;
-  ctc_grad_kernel<<<blocks, 256, 0, s>>>(ix, lp_dl, C, blank, labels, alpha, beta, row_ok, dl_hi, dl_lo, ld_split);
+  // labels up to 256 extended positions keep each position's value in registers
+  if (ix.S_max <= 32 * 8)
+    ctc_grad_kernel<8><<<blocks, 256, 0, s>>>(ix, lp_dl, C, blank, labels, alpha, beta, row_ok, dl_hi, dl_lo, ld_split);
+  else
+    ctc_grad_kernel<0><<<blocks, 256, 0, s>>>(ix, lp_dl, C, blank, labels, alpha, beta, row_ok, dl_hi, dl_lo, ld_split);
   return cudaGetLastError();
 }
 
