@@ -1,6 +1,14 @@
-// k_gemm_tc.cu -- bf16 GEMM on the 5th-generation tensor cores for the
-// contractions of the bf16 path (input projection of layers > 1, weight
-// gradients, input gradients):
+// k_gemm_tc.cu -- GEMMs on the 5th-generation tensor cores (tcgen05, TMEM
+// accumulators):
+//   gemm_bf16_tc_kernel    bf16 operands fed by TMA: the bf16 path's input
+//                          projections, weight gradients and input gradients;
+//   gemm_tf32x3_tc_kernel  fp32 split into tf32 hi + lo (3 MMAs per product),
+//                          operands fed by TMA: the fp32 path's logits (with
+//                          a log-softmax epilogue), dY, projections and dX,
+//                          and weight gradients with unaligned operand rows;
+//   gemm_tf32x3_tn_kernel  the same split, read token-major and split while
+//                          loading: the fp32 path's weight gradients.
+// The bf16 kernel:
 //   D[m][n] (+)= sum_k A[m][k] * B[n][k]  (+ bias[n]),   fp32 accumulation
 // A [M x K] and B [N x K] are bf16 with K contiguous (row-major); D is fp32.
 //
