@@ -42,41 +42,55 @@ cudaError_t launch_layout(const DevIdx &ix, const float *x, int in_dim, float *X
 }
 
 // ---------------------------------------------------------------------------
-// a5 with a narrow input.  Thread n of a CTA owns output column n of one
-// direction: W row n (in_dim values) and b[n] stay in registers while the CTA
-// walks a chunk of tokens; each token row of X is read once per CTA
-// (broadcast) and the [tok x 4H] output is written coalesced along n.
+// a5 with a narrow input.  A CTA stages its chunk of token rows of X in
+// shared memory; thread i owns output columns 4i .. 4i+3 of one direction
+// (their W rows and biases in registers) and writes each token's four values
+// as one 16-byte store, coalesced along n; no FMA waits on a global load.
 constexpr int kProjTok = 64;
 
 template <int D>
 __global__ void __launch_bounds__(128) proj_narrow_kernel(const float *__restrict__ X, int n_tok,
                                                          const float *__restrict__ params, int64_t w_off,
                                                          int64_t w_stride, int H, float *Z0, float *Z1) {
+  __shared__ float xs[kProjTok * D];
   const int d = blockIdx.z;
-  const int n = blockIdx.x * 128 + threadIdx.x;
   const int G = 4 * H;
-  if (n >= G) return;
-  const float *W = params + w_off + d * w_stride;
-  const float *bias = W + (int64_t)G * D + (int64_t)G * H;
-  float w[D];
-#pragma unroll
-  for (int k = 0; k < D; ++k) w[k] = W[(int64_t)n * D + k];
-  const float bn = bias[n];
-  float *Z = d == 0 ? Z0 : Z1;
   const int t0 = blockIdx.y * kProjTok;
   const int t1 = min(n_tok, t0 + kProjTok);
-  for (int tok = t0; tok < t1; ++tok) {
-    float z = bn;
+  for (int i = threadIdx.x; i < (t1 - t0) * D; i += blockDim.x) xs[i] = X[(int64_t)t0 * D + i];
+  __syncthreads();
+  const int n0 = 4 * (blockIdx.x * 128 + threadIdx.x);  // this thread's outputs n0 .. n0+3 (4H % 4 == 0)
+  if (n0 >= G) return;
+  const float *W = params + w_off + d * w_stride;
+  const float *bias = W + (int64_t)G * D + (int64_t)G * H;
+  float w[4][D], bn[4];
 #pragma unroll
-    for (int k = 0; k < D; ++k) z = fmaf(w[k], __ldg(X + (int64_t)tok * D + k), z);
-    Z[(int64_t)tok * G + n] = z;
+  for (int c = 0; c < 4; ++c) {
+#pragma unroll
+    for (int k = 0; k < D; ++k) w[c][k] = W[(int64_t)(n0 + c) * D + k];
+    bn[c] = bias[n0 + c];
+  }
+  float *Z = d == 0 ? Z0 : Z1;
+  for (int tok = t0; tok < t1; ++tok) {
+    const float *x = xs + (tok - t0) * D;
+    float4 z = make_float4(bn[0], bn[1], bn[2], bn[3]);
+#pragma unroll
+    for (int k = 0; k < D; ++k) {
+      const float xk = x[k];
+      z.x = fmaf(w[0][k], xk, z.x);
+      z.y = fmaf(w[1][k], xk, z.y);
+      z.z = fmaf(w[2][k], xk, z.z);
+      z.w = fmaf(w[3][k], xk, z.w);
+    }
+    *reinterpret_cast<float4 *>(Z + (int64_t)tok * G + n0) = z;
   }
 }
 
 cudaError_t launch_proj_narrow(const float *X, int n_tok, int in_dim, const float *params, int64_t w_off,
                                int64_t w_stride, int H, int dirs, float *const *Z, cudaStream_t s) {
-  dim3 grid((4 * H + 127) / 128, (n_tok + kProjTok - 1) / kProjTok, dirs);
+  dim3 grid((H + 127) / 128, (n_tok + kProjTok - 1) / kProjTok, dirs);  // 4H outputs, 4 per thread
   float *Z1 = dirs > 1 ? Z[1] : Z[0];
+  if (((reinterpret_cast<uintptr_t>(Z[0]) | reinterpret_cast<uintptr_t>(Z1)) & 15) != 0) return cudaErrorInvalidValue;
   switch (in_dim) {
 #define BKT_CASE(D) \
   case D:           \
