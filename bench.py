@@ -7,8 +7,18 @@ then for every mini-batch one bkt_lstm_ctc_step (packed layout, LSTM forward,
 output + log-softmax, CTC, BPTT, weight gradients) and one bkt_sgd_update
 (or, with --optimizer adadelta, the paper's update rule bkt_adadelta_update).
 The metric is unpadded timesteps per second (sum of sequence lengths
-processed / time).  Inputs are resident in HBM when the timed region starts;
-L2 is flushed (a 256 MiB write) between timed steps, outside their events.
+processed / time), plus the epoch time against the bucket count (the
+quantity of the paper's Fig. 4).  Inputs are resident in HBM when the timed
+region starts; L2 is flushed (a 256 MiB write) between timed steps, outside
+their events.
+
+The default workload is the full-epoch sweep: a 3-layer bidirectional LSTM
+(H = 256, bf16 tensor-core contractions, fp32 recurrence) with 81-class CTC
+over 32,768 sequences of bimodal length (lognormal medians 150 and 900,
+sigma 0.5, clipped to [20, 3000]), batch 128, timed at Q = 8 buckets with
+single epochs at Q = 1, 2, 4, 16 and 32.  Every kernel's achieved rate
+against its roofline comes from the library's per-launch work accounting
+(bkt_ctx_kernel_times), measured in separate epochs.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl native|reference]
 
@@ -21,6 +31,7 @@ from __future__ import annotations
 
 import argparse
 import json
+import math
 import os
 import statistics
 import subprocess
@@ -33,12 +44,14 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
-DEFAULT_WORKLOAD = "lstm1_bi_h128"
-DEFAULT_BUCKETS = 4
+DEFAULT_WORKLOAD = "lstm3_bi_h256_bf16_bimodal"
+DEFAULT_BUCKETS = 8
+DEFAULT_COMPARE = "1,2,4,16,32"
 LR = 1e-3
+METRIC = "unpadded timesteps/sec (LSTM+CTC fwd+bwd, 1 GPU) and epoch time vs bucket count"
 
 
-def parse():
+def parse(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
@@ -46,14 +59,14 @@ def parse():
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--buckets", type=int, default=DEFAULT_BUCKETS)
-    ap.add_argument("--compare-buckets", default="1",
+    ap.add_argument("--compare-buckets", default=DEFAULT_COMPARE,
                     help="extra bucket counts timed briefly for epoch time vs Q ('' = none)")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--optimizer", default="sgd", choices=["sgd", "adadelta"])
     ap.add_argument("--cpu-baseline-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    return ap.parse_args()
+    return ap.parse_args(argv)
 
 
 # ---------------------------------------------------------------------------
@@ -150,28 +163,56 @@ def max_over_ranks(world, v: float) -> float:
 
 
 # ---------------------------------------------------------------------------
-def roofline_for(name, launches, total_ms, work, peaks, peak_src, clocks):
-    """Achieved algorithmic rate of one kernel vs its bound."""
-    avg_s = total_ms / 1e3 / max(1, launches)
-    w = work.get(name)
-    if w is None:
+# What bounds each kernel of the step (everything not listed moves data: HBM).
+#   alu            fp32 FMA pipe of the whole GPU (the recurrent matvecs)
+#   tensor_bf16    tcgen05 kind::f16 with bf16 operands
+#   tensor_tf32x3  tcgen05 kind::tf32, three MMAs per split-precision product
+KERNEL_BOUND = {"lstm_fwd": "alu", "lstm_bwd": "alu", "gemm_tc": "tensor_bf16",
+                "gemm_tf32x3": "tensor_tf32x3", "gemm_tf32x3_tn": "tensor_tf32x3"}
+TF32_PER_BF16 = 1.1 / 2.25   # nominal dense tf32 : bf16 tensor rate
+
+
+def roofline_for(stat: dict, peaks: dict, peak_src: str, clocks: dict, n_sm: int = 152):
+    """Achieved algorithmic rate of one kernel (its totals over the timer
+    epochs: launches, total_ms, flops, bytes, serial_steps) against the peak
+    of what bounds it; None when the kernel carries no work."""
+    name, ms = stat["name"], stat["total_ms"]
+    if ms <= 0 or stat["launches"] <= 0:
         return None
-    kind, per_launch = w
-    if kind == "hbm":
-        ach = per_launch / avg_s / 1e9
+    bound = KERNEL_BOUND.get(name, "hbm")
+    sec = ms / 1e3
+    out = {"kernel": name, "launches": stat["launches"], "avg_launch_ms": ms / stat["launches"]}
+    if bound == "hbm":
+        if stat["bytes"] <= 0:
+            return None
         peak = peaks["hbm_gbs"]
-        return {"kernel": name, "bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
-                "frac": ach / peak, "traffic": None, "peak_source": f"hbm_gbs of {peak_src}",
-                "algorithmic_bytes_per_launch": per_launch, "avg_launch_ms": avg_s * 1e3}
-    # fp32 FMA pipe of the whole GPU at the SM clock seen under load
-    sm_mhz = clocks.get("sm_mhz") or peaks.get("sm_max_mhz", 2070.0)
-    n_sm = w[2] if len(w) > 2 else 152
-    peak = n_sm * 128 * 2 * sm_mhz * 1e6 / 1e12
-    ach = per_launch / avg_s / 1e12
-    return {"kernel": name, "bound": "alu", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
-            "frac": ach / peak, "traffic": None,
-            "peak_source": f"{n_sm} SMs x 128 fp32 FMA/clk x 2 x {sm_mhz:.0f} MHz (sampled median)",
-            "algorithmic_flops_per_launch": per_launch, "avg_launch_ms": avg_s * 1e3}
+        out.update(bound="hbm", achieved=stat["bytes"] / sec / 1e9, peak=peak, unit="GB/s",
+                   peak_source=f"hbm_gbs of {peak_src}",
+                   algorithmic_bytes_per_launch=stat["bytes"] / stat["launches"])
+    else:
+        if stat["flops"] <= 0:
+            return None
+        if bound == "alu":
+            sm_mhz = clocks.get("sm_mhz") or peaks.get("sm_max_mhz", 2070.0)
+            peak = n_sm * 128 * 2 * sm_mhz * 1e6 / 1e12
+            src = f"{n_sm} SMs x 128 fp32 FMA/clk x 2 x {sm_mhz:.0f} MHz (sampled median)"
+            b = "alu"
+        elif bound == "tensor_bf16":
+            peak = peaks.get("bf16_tflops_sustained") or peaks["bf16_tflops"]
+            src = f"bf16_tflops_sustained of {peak_src} (kernel timed inside a long step)"
+            b = "tensor"
+        else:
+            base = peaks.get("bf16_tflops_sustained") or peaks["bf16_tflops"]
+            peak = base * TF32_PER_BF16 / 3.0
+            src = (f"bf16_tflops_sustained of {peak_src} x {TF32_PER_BF16:.3f} (nominal tf32:bf16) / 3 "
+                   "(three tf32 MMAs per split-precision product)")
+            b = "tensor"
+        out.update(bound=b, achieved=stat["flops"] / sec / 1e12, peak=peak, unit="TFLOP/s",
+                   peak_source=src, algorithmic_flops_per_launch=stat["flops"] / stat["launches"])
+    out["frac"] = out["achieved"] / out["peak"]
+    if stat.get("serial_steps", 0) > 0:
+        out["us_per_step"] = ms * 1e3 / stat["serial_steps"]
+    return out
 
 
 def recorded_traffic(kernel: str, workload: str, buckets: int):
@@ -192,35 +233,10 @@ def recorded_traffic(kernel: str, workload: str, buckets: int):
         return None, None
 
 
-def kernel_work(cfg, plan, ds):
-    """Algorithmic work per launch of the main kernels, averaged over the
-    epoch's batches: name -> (kind, per-launch amount)."""
-    H, C = cfg["hidden"], cfg["n_classes"]
-    dirs = 2 if cfg["bidirectional"] else 1
-    Lc = cfg["n_layers"]
-    n_tok, n_b = 0, plan["n_batches"]
-    ext_cells = 0
-    for k in range(n_b):
-        ids = plan["order"][plan["batch_off"][k]:plan["batch_off"][k + 1]]
-        L = ds.lengths[ids]
-        n_tok += int(L.sum())
-        ext_cells += int((L * (2 * ds.label_lengths[ids] + 1)).sum())
-    tok_pb = n_tok / n_b
-    cells_pb = ext_cells / n_b
-    # recurrent kernels: W_hh matvec, 8 H^2 flops per token and direction
-    # (forward), twice that counted once per direction in the backward
-    rec = 8.0 * H * H * tok_pb * dirs
-    work = {
-        "lstm_fwd": ("alu", rec),
-        "lstm_bwd": ("alu", rec),
-        # CTC tables: each cell written once (fp32), emissions read once per cell
-        "ctc_tables": ("hbm", 2 * 4.0 * cells_pb * 2),
-        # posterior: alpha + beta read, logp row read + dlogit row written
-        "ctc_grad": ("hbm", 4.0 * (2 * cells_pb + 2 * C * tok_pb)),
-        "proj_narrow": ("hbm", 4.0 * tok_pb * (cfg["in_dim"] + 4 * H * dirs)),
-        "layout_gather": ("hbm", 4.0 * tok_pb * (2 * cfg["in_dim"] + 4)),
-    }
-    return work, tok_pb
+def budget_count(ms_per_epoch: float, budget_ms: float, lo: int, hi: int) -> int:
+    """How many epochs of `ms_per_epoch` fit in `budget_ms`, within [lo, hi]."""
+    n = int(math.ceil(budget_ms / max(ms_per_epoch, 1e-3)))
+    return max(lo, min(hi, n))
 
 
 # ---------------------------------------------------------------------------
@@ -233,6 +249,7 @@ def run_native(args, world, rank, local):
     binding.lib()
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
+    n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
     w = synth.WORKLOADS[args.workload]
     cfg = w.model_cfg()
     ds = synth.make_workload(w, seed=args.seed)
@@ -289,55 +306,62 @@ def run_native(args, world, rank, local):
         barrier(world)
         torch.cuda.synchronize(dev)
         ms = [a.elapsed_time(b) for a, b in evs]
-        ktimes = ctx.kernel_times() if with_timer else []
+        kstats = ctx.kernel_stats() if with_timer else []
         if with_timer:
             ctx.set_timing(False)
         ctx.sync_status()
-        return ms, plans, ktimes
+        return ms, plans, kstats
 
     clocks = Clocks(local if not os.environ.get("CUDA_VISIBLE_DEVICES") else 0)
     ms, plans, _ = timed(args.buckets, args.steps, args.warmup, clocks=clocks)
-    # per-kernel durations come from separate epochs: the per-launch event
-    # records they need would otherwise sit inside the timed epochs
-    timer_steps = max(3, args.steps // 2)
-    _, tplans, ktimes = timed(args.buckets, timer_steps, 0, e0=args.warmup, with_timer=True)
     ms_step = sum(ms) / len(ms)
     ms_max = max_over_ranks(world, ms_step)
     value = world * unpadded / (ms_max / 1e3)
     pe = [p["unpadded_timesteps"] / p["padded_timesteps"] for p in plans]
     clk = clocks.summary()
+    infeasible = ctx.infeasible_count()
+
+    # per-kernel durations and work come from separate epochs: the per-launch
+    # event records they need would otherwise sit inside the timed epochs
+    timer_steps = budget_count(ms_step, 3000.0, 1, max(1, args.steps // 2))
+    _, _, kstats = timed(args.buckets, timer_steps, 0, e0=args.warmup, with_timer=True)
 
     # epoch time vs bucket count (short runs)
     by_q = {str(args.buckets): {"ms_per_epoch": ms_step, "padded_efficiency": float(np.mean(pe)),
-                                "dp_cost": plans[0]["dp_cost"], "n_batches": plans[0]["n_batches"]}}
+                                "dp_cost": plans[0]["dp_cost"], "n_batches": plans[0]["n_batches"],
+                                "serial_steps": serial_steps(plans[0], ds), "epochs": len(ms)}}
+    q_steps = budget_count(ms_step, 2000.0, 1, max(1, args.steps // 3))
     for qs in [q for q in args.compare_buckets.split(",") if q.strip()]:
         q = int(qs)
         if q == args.buckets:
             continue
-        m2, p2, _ = timed(q, max(2, args.steps // 3), 1, e0=1000)
+        m2, p2, _ = timed(q, q_steps, 0, e0=1000)
         by_q[str(q)] = {"ms_per_epoch": sum(m2) / len(m2),
                         "padded_efficiency": float(np.mean([p["unpadded_timesteps"] / p["padded_timesteps"]
                                                             for p in p2])),
-                        "dp_cost": p2[0]["dp_cost"], "n_batches": p2[0]["n_batches"]}
+                        "dp_cost": p2[0]["dp_cost"], "n_batches": p2[0]["n_batches"],
+                        "serial_steps": serial_steps(p2[0], ds), "epochs": len(m2)}
+    by_q = dict(sorted(by_q.items(), key=lambda kv: int(kv[0])))
 
-    # kernel launches in the timed region and the dominant kernel's roofline
-    per_epoch = sum(n for _, n, _ in ktimes) / timer_steps + plans[0]["n_batches"]
+    # kernel launches in the timed region, per-kernel rooflines, the dominant one
+    per_epoch = sum(k["launches"] for k in kstats) / timer_steps + plans[0]["n_batches"]
     launches = round(per_epoch * args.steps)
     peaks, peak_src = measured_peaks()
-    work, tok_pb = kernel_work(cfg, plans[0], ds)
-    ktimes_sorted = sorted(ktimes, key=lambda t: -t[2])
-    total_k = sum(t for _, _, t in ktimes) or 1.0
-    roof = None
-    for name, n, t in ktimes_sorted:
-        roof = roofline_for(name, n, t, work, peaks, peak_src, clk)
-        if roof:
-            roof["share_of_kernel_time"] = t / total_k
-            tb, tsrc = recorded_traffic(name, w.name, args.buckets)
-            roof["traffic"] = tb
-            roof["traffic_source"] = tsrc
-            break
-    kernel_table = [{"kernel": nm, "launches": n, "total_ms": round(t, 3),
-                     "share": round(t / total_k, 4)} for nm, n, t in ktimes_sorted]
+    total_k = sum(k["total_ms"] for k in kstats) or 1.0
+    rooflines = []
+    for k in sorted(kstats, key=lambda k: -k["total_ms"]):
+        r = roofline_for(k, peaks, peak_src, clk, n_sm)
+        if r:
+            r["share_of_kernel_time"] = k["total_ms"] / total_k
+            rooflines.append(r)
+    roof = dict(rooflines[0]) if rooflines else None
+    if roof:
+        tb, tsrc = recorded_traffic(roof["kernel"], w.name, args.buckets)
+        roof["traffic"] = tb
+        roof["traffic_source"] = tsrc
+    kernel_table = [{"kernel": k["name"], "launches": k["launches"], "total_ms": round(k["total_ms"], 3),
+                     "share": round(k["total_ms"] / total_k, 4)}
+                    for k in sorted(kstats, key=lambda k: -k["total_ms"])]
 
     # end to end through the public API with host buffers
     e2e = None
@@ -350,8 +374,10 @@ def run_native(args, world, rank, local):
         dd2 = binding.DeviceDataset.__new__(binding.DeviceDataset)
         dd2.__dict__.update(dd.__dict__)
         dd2.x, dd2.labels = x_dev, lab_dev
+        e2e_warm = min(args.warmup, 1)
+        e2e_steps = budget_count(ms_step, 15000.0, 2, max(2, args.steps))
         e2e_ms = []
-        for i in range(args.warmup + max(2, args.steps // 2)):
+        for i in range(e2e_warm + e2e_steps):
             flush.zero_()
             torch.cuda.synchronize(dev)
             t0 = time.perf_counter()
@@ -360,11 +386,11 @@ def run_native(args, world, rank, local):
             epoch(5000 + i, args.buckets, dataset=dd2)
             loss_host.copy_(loss, non_blocking=True)
             torch.cuda.synchronize(dev)
-            if i >= args.warmup:
+            if i >= e2e_warm:
                 e2e_ms.append((time.perf_counter() - t0) * 1e3)
         e_ms = max_over_ranks(world, sum(e2e_ms) / len(e2e_ms))
         e2e = {"value": world * unpadded / (e_ms / 1e3), "unit": "timesteps/s",
-               "ms_per_step": e_ms,
+               "ms_per_step": e_ms, "steps": len(e2e_ms),
                "h2d_bytes_per_step": int(x_host.numel() * 4 + lab_host.numel() * 4),
                "d2h_bytes_per_step": int(loss_host.numel() * 4)}
 
@@ -373,7 +399,7 @@ def run_native(args, world, rank, local):
         cpu = cpu_baseline(args, w, ds, params0, plans[0], args.cpu_baseline_seconds)
 
     line = {
-        "metric": "unpadded timesteps/sec (LSTM+CTC fwd+bwd+SGD epoch, 1 GPU)",
+        "metric": METRIC,
         "optimizer": args.optimizer,
         "value": value, "unit": "timesteps/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True,
@@ -382,14 +408,16 @@ def run_native(args, world, rank, local):
         "config": {"workload": w.name, "layers": w.n_layers, "bidirectional": w.bidirectional,
                    "hidden": w.hidden, "n_seqs": w.n_seqs, "batch": w.batch,
                    "buckets": args.buckets, "unpadded_timesteps_per_epoch": unpadded,
-                   "step": "one epoch: plan + every batch's fwd/bwd/CTC + SGD",
+                   "step": "one epoch: plan + every batch's fwd/bwd/CTC + SGD, rebucketed and reshuffled",
                    "l2": "flushed between timed steps (256 MiB write, outside the events)",
                    "parallelism": "replicas" if world > 1 else "1 GPU"},
         "padded_efficiency": float(np.mean(pe)),
+        "infeasible_sequences_per_epoch": infeasible / max(1, args.steps),
         "epoch_time_vs_buckets": by_q,
         "clocks": clk,
         "gpu_launches": int(launches),
         "roofline": roof,
+        "rooflines": rooflines,
         "kernels": kernel_table,
         "e2e": e2e,
         "cpu_baseline": cpu,
@@ -397,6 +425,13 @@ def run_native(args, world, rank, local):
     if rank == 0:
         print(json.dumps(line), flush=True)
     ctx.close()
+
+
+def serial_steps(plan, ds) -> int:
+    """Sum over the plan's batches of the longest length: the recurrence's
+    serial time steps per layer and direction in one epoch."""
+    off, order = plan["batch_off"], plan["order"]
+    return int(sum(int(ds.lengths[order[off[k]:off[k + 1]]].max()) for k in range(plan["n_batches"])))
 
 
 class _Null:
@@ -465,10 +500,11 @@ def run_reference(args, world, rank):
         tot_n += n
     value = tot_steps / tot_s
     line = {"impl": "reference",
-            "metric": "unpadded timesteps/sec (LSTM+CTC fwd+bwd+SGD epoch, 1 GPU)",
+            "metric": METRIC,
             "value": value, "unit": "timesteps/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": tot_s / args.steps * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "gpu_launches": 0,
             "data": "synthetic (seeded; stands in for the paper's handwriting set)",
             "config": {"workload": w.name, "buckets": args.buckets,
                        "step": f"bounded sample: sequences of the epoch order for {per_step:.1f} s"},

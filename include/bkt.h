@@ -40,6 +40,9 @@ extern "C" {
 #define BKT_ENOMEM 2   /* host or device allocation failed */
 #define BKT_ECUDA 3    /* a CUDA runtime call failed (message has the name) */
 #define BKT_EDEVICE 4  /* a device-side input check failed (label >= classes or == blank) */
+#define BKT_ETIMEOUT 5 /* a bounded device-side wait (tensor-core pipeline or recurrent
+                          cluster exchange) reached its iteration cap; the kernel left
+                          its loop, its results are invalid, the context stays usable */
 
 #define BKT_GEMM_FP32 0 /* fp32 contractions (tensor cores with split-precision 3xTF32 operands) */
 #define BKT_GEMM_BF16 1 /* projection, dX and token-axis contractions: bf16 operands, fp32 accumulation */
@@ -192,6 +195,8 @@ int bkt_lstm_ctc_step(bkt_ctx *ctx, const bkt_batch *batch,
  *     BKT_EINVAL with the needed and available bytes in bkt_last_error().
  *   - The first call on a device looks up the array's address on that
  *     device, so make that first call before any stream capture.
+ *   - The array used is the current device's; a stream of another device
+ *     returns BKT_EINVAL before anything is enqueued.
  *   - All calls share the one array, and it keeps the previous call's
  *     contents (the device error flags are cleared at the start of each
  *     call).  Calls whose GPU work overlaps, on different streams or from
@@ -227,10 +232,37 @@ int bkt_adadelta_update(float *params, const float *grads, float *eg2,
                         float *edx2, int64_t n, float rho, float eps,
                         float lr, void *stream);
 
-/* Waits for the work this ctx enqueued, then returns BKT_OK or the first
- * device-side error (BKT_EDEVICE) raised since the previous call, and
- * clears it.                                                             */
+/* Waits for the work this ctx enqueued, then returns BKT_OK or the
+ * device-side errors raised since the previous call, and clears them:
+ * BKT_ETIMEOUT when a bounded wait ran out (it takes precedence),
+ * otherwise BKT_EDEVICE for a label outside 1..C-1.  The message lists
+ * every flag that was set.                                               */
 int bkt_ctx_sync_status(bkt_ctx *ctx);
+
+/* Sequences without any CTC alignment (lengths[i] < label_lengths[i] +
+ * repeated neighbours; ref. [15]): their loss is +inf and they add nothing
+ * to grads, which is not an error.  Waits for the ctx's work, stores in
+ * *count how many such sequences the steps of this ctx met since it was
+ * created or since the previous call, and resets the counter.           */
+int bkt_ctx_infeasible_count(bkt_ctx *ctx, int64_t *count);
+
+/* Failure-detection hooks (off by default; for tests of the bounded waits).
+ *   poll_cap  > 0: every bounded device-side wait of this ctx's kernels
+ *             gives up after poll_cap polls instead of the built-in cap
+ *             (about 4 M polls); values below 256 are raised to 256;
+ *             0 restores the built-in caps.
+ *   withhold  bit 0 (BKT_WITHHOLD_EXCHANGE): CTA 0 of every recurrent
+ *             cluster (H = 256, 512) sends none of its exchange data, so
+ *             its peers' waits run out; bit 1 (BKT_WITHHOLD_TMA): the TMA
+ *             producer of every tensor-core GEMM skips the loads of its
+ *             first k slab, so the MMA issuer's wait runs out.
+ * A step run with a withhold bit set ends with BKT_ETIMEOUT from
+ * bkt_ctx_sync_status and invalid results; every wait is bounded, so it
+ * finishes, and the next step with the hooks off is normal.  BKT_EINVAL
+ * for a negative poll_cap or unknown withhold bits.                      */
+#define BKT_WITHHOLD_EXCHANGE 1
+#define BKT_WITHHOLD_TMA 2
+int bkt_ctx_set_wait_faults(bkt_ctx *ctx, int32_t poll_cap, int32_t withhold);
 
 /* ------------------------------------------------------------------ */
 /* Per-kernel timing with CUDA events on the launching stream.         */
@@ -239,6 +271,17 @@ typedef struct bkt_kernel_time {
   const char *name;  /* static string */
   int64_t launches;
   double total_ms;
+  /* Algorithmic work of all those launches, from their shapes:
+   *   flops         floating-point operations of the contraction or
+   *                 recurrence (2 per multiply-add; a split-precision
+   *                 product counts once);
+   *   bytes         the minimum DRAM bytes the kernel must move (each
+   *                 input read once, each output written once);
+   *   serial_steps  sum over launches of the time steps a launch runs one
+   *                 after another (recurrent and CTC kernels), else 0.   */
+  double flops;
+  double bytes;
+  int64_t serial_steps;
 } bkt_kernel_time;
 
 /* enable != 0: record an event pair around every kernel this ctx launches

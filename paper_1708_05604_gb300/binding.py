@@ -16,15 +16,16 @@ import numpy as np
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libbkt.so")
 
-BKT_OK, BKT_EINVAL, BKT_ENOMEM, BKT_ECUDA, BKT_EDEVICE = 0, 1, 2, 3, 4
+BKT_OK, BKT_EINVAL, BKT_ENOMEM, BKT_ECUDA, BKT_EDEVICE, BKT_ETIMEOUT = 0, 1, 2, 3, 4, 5
+BKT_WITHHOLD_EXCHANGE, BKT_WITHHOLD_TMA = 1, 2
 BKT_GEMM_FP32, BKT_GEMM_BF16 = 0, 1
 
 # Every symbol include/bkt.h declares.
 EXPORTS = ("bkt_plan_buckets", "bkt_plan_buckets_ordered", "bkt_plan_get", "bkt_plan_free", "bkt_param_count",
            "bkt_ctx_create", "bkt_ctx_destroy", "bkt_lstm_ctc_step", "bkt_lstm_ctc_step_static",
            "bkt_sgd_update", "bkt_adadelta_update",
-           "bkt_ctx_sync_status", "bkt_ctx_set_timing", "bkt_ctx_kernel_times",
-           "bkt_last_error")
+           "bkt_ctx_sync_status", "bkt_ctx_infeasible_count", "bkt_ctx_set_wait_faults",
+           "bkt_ctx_set_timing", "bkt_ctx_kernel_times", "bkt_last_error")
 
 i32p = ctypes.POINTER(ctypes.c_int32)
 i64p = ctypes.POINTER(ctypes.c_int64)
@@ -52,7 +53,8 @@ class Batch(ctypes.Structure):
 
 class KernelTime(ctypes.Structure):
     _fields_ = [("name", ctypes.c_char_p), ("launches", ctypes.c_int64),
-                ("total_ms", ctypes.c_double)]
+                ("total_ms", ctypes.c_double), ("flops", ctypes.c_double),
+                ("bytes", ctypes.c_double), ("serial_steps", ctypes.c_int64)]
 
 
 _lock = threading.Lock()
@@ -97,13 +99,16 @@ def lib() -> ctypes.CDLL:
         L.bkt_adadelta_update.argtypes = [vp, vp, vp, vp, ctypes.c_int64, ctypes.c_float,
                                           ctypes.c_float, ctypes.c_float, vp]
         L.bkt_ctx_sync_status.argtypes = [vp]
+        L.bkt_ctx_infeasible_count.argtypes = [vp, i64p]
+        L.bkt_ctx_set_wait_faults.argtypes = [vp, ctypes.c_int32, ctypes.c_int32]
         L.bkt_ctx_set_timing.argtypes = [vp, ctypes.c_int32]
         L.bkt_ctx_kernel_times.argtypes = [vp, ctypes.POINTER(KernelTime), ctypes.c_int32, i32p]
         L.bkt_last_error.argtypes = []
         L.bkt_last_error.restype = ctypes.c_char_p
         for name in ("bkt_plan_buckets", "bkt_plan_buckets_ordered", "bkt_plan_get", "bkt_ctx_create", "bkt_lstm_ctc_step",
                      "bkt_lstm_ctc_step_static",
-                     "bkt_sgd_update", "bkt_adadelta_update", "bkt_ctx_sync_status", "bkt_ctx_set_timing",
+                     "bkt_sgd_update", "bkt_adadelta_update", "bkt_ctx_sync_status",
+                     "bkt_ctx_infeasible_count", "bkt_ctx_set_wait_faults", "bkt_ctx_set_timing",
                      "bkt_ctx_kernel_times"):
             getattr(L, name).restype = ctypes.c_int
         _lib = L
@@ -292,13 +297,33 @@ class Ctx:
     def sync_status(self):
         _check(lib().bkt_ctx_sync_status(self.h))
 
+    def infeasible_count(self) -> int:
+        """bkt_ctx_infeasible_count: sequences without a CTC alignment since
+        the previous call (the counter is reset)."""
+        n = ctypes.c_int64(0)
+        _check(lib().bkt_ctx_infeasible_count(self.h, ctypes.byref(n)))
+        return int(n.value)
+
+    def set_wait_faults(self, poll_cap: int = 0, withhold: int = 0):
+        """bkt_ctx_set_wait_faults: failure-detection hooks (0, 0 = off)."""
+        _check(lib().bkt_ctx_set_wait_faults(self.h, int(poll_cap), int(withhold)))
+
     def set_timing(self, on: bool):
         _check(lib().bkt_ctx_set_timing(self.h, int(bool(on))))
 
     def kernel_times(self) -> list[tuple[str, int, float]]:
+        """(name, launches, total ms) of every kernel timed since timing was
+        switched on."""
+        return [(k["name"], k["launches"], k["total_ms"]) for k in self.kernel_stats()]
+
+    def kernel_stats(self) -> list[dict]:
+        """bkt_ctx_kernel_times with the algorithmic work of each kernel:
+        name, launches, total_ms, flops, bytes, serial_steps."""
         n = ctypes.c_int32(0)
         _check(lib().bkt_ctx_kernel_times(self.h, None, 0, ctypes.byref(n)))
         arr = (KernelTime * max(1, n.value))()
         _check(lib().bkt_ctx_kernel_times(self.h, arr, n.value, ctypes.byref(n)))
-        return [(arr[i].name.decode(), int(arr[i].launches), float(arr[i].total_ms))
+        return [{"name": arr[i].name.decode(), "launches": int(arr[i].launches),
+                 "total_ms": float(arr[i].total_ms), "flops": float(arr[i].flops),
+                 "bytes": float(arr[i].bytes), "serial_steps": int(arr[i].serial_steps)}
                 for i in range(n.value)]

@@ -387,9 +387,9 @@ struct Launch {
   const char *failed = nullptr;
   cudaError_t err = cudaSuccess;
   template <typename F>
-  bool run(const char *name, F &&f) {
+  bool run(const char *name, const bkt::Work &wk, F &&f) {
     if (failed) return false;
-    if (timer) timer->begin(name, s);
+    if (timer) timer->begin(name, wk, s);
     cudaError_t e = f();
     if (timer) timer->end(s);
     if (e != cudaSuccess) {
@@ -400,6 +400,25 @@ struct Launch {
     return true;
   }
 };
+
+// Algorithmic work of a launch (bkt_kernel_time): contraction flops,
+// minimum DRAM bytes, serial time steps.
+bkt::Work flops_w(double f, int64_t steps = 0) {
+  bkt::Work w;
+  w.flops = f;
+  w.steps = steps;
+  return w;
+}
+bkt::Work bytes_w(double b, int64_t steps = 0) {
+  bkt::Work w;
+  w.bytes = b;
+  w.steps = steps;
+  return w;
+}
+// a GEMM of 2 M N K flops; an element-wise pass over R x C values reading
+// `rb` and writing `wb` bytes per value
+bkt::Work gemm_w(double M, double N, double K) { return flops_w(2.0 * M * N * K); }
+bkt::Work pass_w(double R, double C, double rb, double wb) { return bytes_w(R * C * (rb + wb)); }
 
 // Largest M x N block a token reduction writes: [W_out | b_out] or
 // [W_ih | W_hh | b] of one layer and direction.
@@ -415,7 +434,7 @@ size_t max_reduce_block(const Layout &lo) {
 int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepBufs &w, const bkt::RecGeom *geom,
                     const bkt::DevIdx &ix, const bkt_batch *bt, const float *params, float *grads, float *loss,
                     cudaStream_t s, bkt::KernelTimer *timer, int sm_count, cudaStream_t side = nullptr,
-                    cudaEvent_t fork_ev = nullptr, cudaEvent_t join_ev = nullptr) {
+                    cudaEvent_t fork_ev = nullptr, cudaEvent_t join_ev = nullptr, bkt::WaitFaults wf = {}) {
   const int H = lo.H, dirs = lo.dirs, DH = dirs * H, C = lo.C, NT = ix.n_tok;
   const bool bf16 = cfg.gemm_precision == BKT_GEMM_BF16;
   Launch L{timer, s};
@@ -431,8 +450,9 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     if (e == cudaSuccess) e = cudaStreamWaitEvent(side, fork_ev, 0);
     if (e != cudaSuccess) return cuda_err("fork to the side stream", e);
   }
-  Ls.run("split_rows", [&] { return bkt::launch_split_rows(params + lo.w_out, DH, C, DH, w.Woh, w.Wol, DHp, Ls.s); });
-  Ls.run("transpose_split", [&] {
+  Ls.run("split_rows", pass_w(C, DH, 4, 8),
+         [&] { return bkt::launch_split_rows(params + lo.w_out, DH, C, DH, w.Woh, w.Wol, DHp, Ls.s); });
+  Ls.run("transpose_split", pass_w(C, DH, 4, 8), [&] {
     return bkt::launch_transpose_split(params + lo.w_out, DH, nullptr, C, DH, w.WoTh, w.WoTl, Cp, Ls.s);
   });
   if (side) {
@@ -441,21 +461,21 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
   }
 
   // ---- a4: packed time-major input
-  L.run("layout_gather", [&] { return bkt::launch_layout(ix, bt->x, lo.D0, w.X, w.tok_t, w.tok_r, w.prev_tok, s); });
+  L.run("layout_gather", bytes_w((double)NT * (8.0 * lo.D0 + 16.0)), [&] { return bkt::launch_layout(ix, bt->x, lo.D0, w.X, w.tok_t, w.tok_r, w.prev_tok, s); });
 
   // ---- forward, layer by layer
   for (int l = 0; l < lo.L; ++l) {
     float *Zl[2] = {w.Z[l * dirs], dirs > 1 ? w.Z[l * dirs + 1] : nullptr};
     if (l == 0) {
       // a5, narrow input: both directions in one launch
-      L.run("proj_narrow", [&] {
+      L.run("proj_narrow", bytes_w(4.0 * NT * (lo.D0 + 4.0 * H * dirs)), [&] {
         return bkt::launch_proj_narrow(w.X, NT, lo.D0, params, lo.w_ih[0], lo.stride(0), H, dirs, Zl, s);
       });
     } else if (bf16) {
       // a5 on the tensor cores: Zx = bf16(Y_{l-1}) bf16(W_ih)^T + b, fp32 accumulation
-      L.run("cast_bf16", [&] { return bkt::launch_cast_bf16(w.Y[l - 1], DH, NT, DH, w.Yb, DH, s); });
+      L.run("cast_bf16", pass_w(NT, DH, 4, 2), [&] { return bkt::launch_cast_bf16(w.Y[l - 1], DH, NT, DH, w.Yb, DH, s); });
       for (int d = 0; d < dirs; ++d) {
-        L.run("cast_bf16", [&] {
+        L.run("cast_bf16", pass_w(4.0 * H, DH, 4, 2), [&] {
           return bkt::launch_cast_bf16(params + lo.w_ih[l * dirs + d], DH, 4 * H, DH, w.Wb, DH, s);
         });
         bkt::TcGemmArgs g{};
@@ -470,15 +490,17 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         g.ldd = 4 * H;
         g.bias = params + lo.bias(l, d);
         g.err = w.status;
-        L.run("gemm_tc", [&] { return bkt::launch_gemm_bf16_tc(g, s); });
+        g.wf = wf;
+        L.run("gemm_tc", gemm_w(g.M, g.N, g.K), [&] { return bkt::launch_gemm_bf16_tc(g, s); });
       }
     } else {
       // a5 in fp32 on the tensor cores (3xTF32): Zx = Y_{l-1} W_ih^T + b; both
       // operands are K-contiguous, split into hi + lo rows padded to 16 bytes
       const int DHq = (DH + 3) & ~3;
-      L.run("split_rows", [&] { return bkt::launch_split_rows(w.Y[l - 1], DH, NT, DH, w.AT, w.ATl, DHq, s); });
+      L.run("split_rows", pass_w(NT, DH, 4, 8),
+            [&] { return bkt::launch_split_rows(w.Y[l - 1], DH, NT, DH, w.AT, w.ATl, DHq, s); });
       for (int d = 0; d < dirs; ++d) {
-        L.run("split_rows", [&] {
+        L.run("split_rows", pass_w(4.0 * H, DH, 4, 8), [&] {
           return bkt::launch_split_rows(params + lo.w_ih[l * dirs + d], DH, 4 * H, DH, w.Wh, w.Wl, DHq, s);
         });
         bkt::TcGemmArgs g{};
@@ -493,7 +515,8 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         g.ldd = 4 * H;
         g.bias = params + lo.bias(l, d);
         g.err = w.status;
-        L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.ATl, w.Wl, s); });
+        g.wf = wf;
+        L.run("gemm_tf32x3", gemm_w(g.M, g.N, g.K), [&] { return bkt::launch_gemm_tf32x3_tc(g, w.ATl, w.Wl, s); });
       }
     }
     bkt::RecArgs ra{};
@@ -507,7 +530,8 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     }
     ra.Y = w.Y[l];
     ra.status = w.status;
-    L.run("lstm_fwd", [&] { return bkt::launch_lstm_fwd(ra, geom[l], s); });
+    ra.wf = wf;
+    L.run("lstm_fwd", flops_w(8.0 * H * H * (double)NT * dirs, ix.T), [&] { return bkt::launch_lstm_fwd(ra, geom[l], s); });
   }
 
   // ---- a7: output layer and log-softmax
@@ -516,7 +540,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
   // GEMM's epilogue holds whole rows (C <= 128 columns in one tile) and
   // writes their log-softmax
   float *Ytop = w.Y[lo.L - 1];
-  L.run("split_rows", [&] { return bkt::launch_split_rows(Ytop, DH, NT, DH, w.BTf, w.BTl, DHp, s); });
+  L.run("split_rows", pass_w(NT, DH, 4, 8), [&] { return bkt::launch_split_rows(Ytop, DH, NT, DH, w.BTf, w.BTl, DHp, s); });
   if (side) {
     cudaError_t e = cudaStreamWaitEvent(s, join_ev, 0);  // the W_out splits
     if (e != cudaSuccess) return cuda_err("wait for the side stream", e);
@@ -535,13 +559,14 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     g.bias = params + lo.b_out;
     g.logsoftmax = 1;
     g.err = w.status;
-    L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.BTl, w.Wol, s); });
+    g.wf = wf;
+    L.run("gemm_tf32x3", gemm_w(g.M, g.N, g.K), [&] { return bkt::launch_gemm_tf32x3_tc(g, w.BTl, w.Wol, s); });
   }
   // ---- a8, a9: CTC
-  L.run("ctc_tables", [&] {
+  L.run("ctc_tables", bytes_w(16.0 * (double)ix.n_cells, ix.T), [&] {
     return bkt::launch_ctc_tables(ix, w.logit, C, cfg.blank, bt->labels, w.alpha, w.beta, loss, w.row_ok, w.status, s);
   });
-  L.run("ctc_grad", [&] {  // dlogit in place, and its split for dY
+  L.run("ctc_grad", bytes_w(8.0 * (double)ix.n_cells + 8.0 * NT * C + 8.0 * NT * Cp), [&] {  // dlogit in place, and its split for dY
     return bkt::launch_ctc_grad(ix, w.logit, C, cfg.blank, bt->labels, w.alpha, w.beta, w.row_ok, w.Lh, w.Ll, Cp, s);
   });
 
@@ -574,15 +599,19 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
       g.P = w.part;
       g.splits = bkt::tf32x3_tn_splits(M, N, NT, sm_count, w.part_floats);
       g.err = w.status;
-      X.run("gemm_tf32x3_tn", [&] { return bkt::launch_gemm_tf32x3_tn(g, X.s); });
-      X.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, g.splits, M, N, out, X.s); });
+      g.wf = wf;
+      X.run("gemm_tf32x3_tn", gemm_w(M, N, NT), [&] { return bkt::launch_gemm_tf32x3_tn(g, X.s); });
+      X.run("splitk_sum", pass_w(M, N, 4.0 * g.splits, 4),
+            [&] { return bkt::launch_splitk_sum(w.part, g.splits, M, N, out, X.s); });
       return;
     }
     if (at_src != A) {
-      X.run("transpose_split", [&] { return bkt::launch_transpose_split(A, lda, nullptr, NT, M, w.AT, w.ATl, NTq, X.s); });
+      X.run("transpose_split", pass_w(NT, M, 4, 8),
+            [&] { return bkt::launch_transpose_split(A, lda, nullptr, NT, M, w.AT, w.ATl, NTq, X.s); });
       at_src = A;
     }
-    X.run("transpose_split", [&] { return bkt::launch_transpose_split(B, ldb, gather, NT, N, w.BTf, w.BTl, NTq, X.s); });
+    X.run("transpose_split", pass_w(NT, N, 4, 8),
+          [&] { return bkt::launch_transpose_split(B, ldb, gather, NT, N, w.BTf, w.BTl, NTq, X.s); });
     bkt::TcGemmArgs g{};
     g.M = M;
     g.N = N;
@@ -594,13 +623,17 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     g.P = w.part;
     g.splits = bkt::tf32x3_splits(M, N, NT, sm_count, w.part_floats);
     g.err = w.status;
-    X.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.ATl, w.BTl, X.s); });
-    X.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, g.splits, M, N, out, X.s); });
+    g.wf = wf;
+    X.run("gemm_tf32x3", gemm_w(M, N, NT), [&] { return bkt::launch_gemm_tf32x3_tc(g, w.ATl, w.BTl, X.s); });
+    X.run("splitk_sum", pass_w(M, N, 4.0 * g.splits, 4),
+          [&] { return bkt::launch_splitk_sum(w.part, g.splits, M, N, out, X.s); });
   };
   auto bias_sum_on = [&](Launch &X, const float *A, int64_t lda, int M, float *out) {
     const int splits = bkt::colsum_splits(NT, M, w.part_floats);
-    X.run("colsum", [&] { return bkt::launch_colsum(A, lda, NT, M, w.part, splits, X.s); });
-    X.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, splits, 1, M, out, X.s); });
+    X.run("colsum", bytes_w(4.0 * NT * M + 4.0 * splits * M),
+          [&] { return bkt::launch_colsum(A, lda, NT, M, w.part, splits, X.s); });
+    X.run("splitk_sum", pass_w(1, M, 4.0 * splits, 4),
+          [&] { return bkt::launch_splitk_sum(w.part, splits, 1, M, out, X.s); });
   };
   // [dW_out | db_out] = dlogit^T [Y | 1]; with a side stream it overlaps dY
   // and the top layer's BPTT (the side stream runs all weight gradients in
@@ -627,7 +660,8 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     g.D = w.dY;
     g.ldd = DH;
     g.err = w.status;
-    L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, w.Ll, w.WoTl, s); });
+    g.wf = wf;
+    L.run("gemm_tf32x3", gemm_w(g.M, g.N, g.K), [&] { return bkt::launch_gemm_tf32x3_tc(g, w.Ll, w.WoTl, s); });
   }
 
   // ---- a11, a12: BPTT and weight gradients, top layer first.  With a side
@@ -653,7 +687,8 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     ra.Y = w.Y[l];
     ra.status = w.status;
     ra.dY = w.dY;
-    L.run("lstm_bwd", [&] { return bkt::launch_lstm_bwd(ra, geom[l], s); });
+    ra.wf = wf;
+    L.run("lstm_bwd", flops_w(8.0 * H * H * (double)NT * dirs, ix.T), [&] { return bkt::launch_lstm_bwd(ra, geom[l], s); });
     if (int rc = fork_to_side()) return rc;
     Launch &X = Ls;  // the weight gradients of layer l
     const int D = lo.D(l);
@@ -665,7 +700,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
       Launch &Y = narrow_main ? L : X;
       float *P = narrow_main ? w.part2 : w.part;
       const size_t PF = narrow_main ? w.part2_floats : w.part_floats;
-      Y.run("narrow_wgrad", [&] {
+      Y.run("narrow_wgrad", bytes_w(4.0 * NT * (4.0 * H + D)), [&] {
         return bkt::launch_narrow_wgrad(dZ, 4 * H, 4 * H, Xl, D, NT, P, PF, sm_count, ow, ob, Y.s);
       });
     };
@@ -683,14 +718,17 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         g.P = w.part;
         g.splits = bkt::tc_splits(g.M, g.N, NT, sm_count, w.part_floats);
         g.err = w.status;
-        X.run("gemm_tc", [&] { return bkt::launch_gemm_bf16_tc(g, X.s); });
-        X.run("splitk_sum", [&] { return bkt::launch_splitk_sum(w.part, g.splits, g.M, g.N, out, X.s); });
+        g.wf = wf;
+        X.run("gemm_tc", gemm_w(g.M, g.N, g.K), [&] { return bkt::launch_gemm_bf16_tc(g, X.s); });
+        X.run("splitk_sum", pass_w(g.M, g.N, 4.0 * g.splits, 4),
+              [&] { return bkt::launch_splitk_sum(w.part, g.splits, g.M, g.N, out, X.s); });
       };
       for (int d = 0; d < dirs; ++d) {
         const float *dZ = w.Z[l * dirs + d];
         // dW_hh = dz^T h_{t-1} on the tensor cores (both operands transposed to bf16)
-        X.run("transpose_bf16", [&] { return bkt::launch_transpose_bf16(dZ, 4 * H, nullptr, NT, 4 * H, w.dZT, NTp, X.s); });
-        X.run("transpose_bf16", [&] {
+        X.run("transpose_bf16", pass_w(NT, 4.0 * H, 4, 2),
+              [&] { return bkt::launch_transpose_bf16(dZ, 4 * H, nullptr, NT, 4 * H, w.dZT, NTp, X.s); });
+        X.run("transpose_bf16", pass_w(NT, H, 4, 2), [&] {
           return bkt::launch_transpose_bf16(w.Y[l] + d * H, DH, w.prev_tok[d], NT, H, w.BT, NTp, X.s);
         });
         tc_reduce(w.BT, H, grads + lo.w_hh(l, d));
@@ -698,7 +736,8 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
           // narrow input: [dW_ih | db] = dz^T [X | 1] in fp32
           narrow_on(dZ, grads + lo.w_ih[l * dirs + d], grads + lo.bias(l, d));
         } else {
-          X.run("transpose_bf16", [&] { return bkt::launch_transpose_bf16(Xl, D, nullptr, NT, D, w.BT, NTp, X.s); });
+          X.run("transpose_bf16", pass_w(NT, D, 4, 2),
+                [&] { return bkt::launch_transpose_bf16(Xl, D, nullptr, NT, D, w.BT, NTp, X.s); });
           tc_reduce(w.BT, D, grads + lo.w_ih[l * dirs + d]);
           bias_sum_on(X, dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
         }
@@ -721,8 +760,9 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     if (l > 0 && bf16) {
       // dX = dz W_ih on the tensor cores, both directions accumulated into dY
       for (int d = 0; d < dirs; ++d) {
-        L.run("cast_bf16", [&] { return bkt::launch_cast_bf16(w.Z[l * dirs + d], 4 * H, NT, 4 * H, w.dZb, 4 * H, s); });
-        L.run("transpose_bf16", [&] {
+        L.run("cast_bf16", pass_w(NT, 4.0 * H, 4, 2),
+              [&] { return bkt::launch_cast_bf16(w.Z[l * dirs + d], 4 * H, NT, 4 * H, w.dZb, 4 * H, s); });
+        L.run("transpose_bf16", pass_w(4.0 * H, DH, 4, 2), [&] {
           return bkt::launch_transpose_bf16(params + lo.w_ih[l * dirs + d], DH, nullptr, 4 * H, DH, w.WTb, 4 * H, s);
         });
         bkt::TcGemmArgs g{};
@@ -737,7 +777,8 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         g.ldd = DH;
         g.accumulate = d > 0;
         g.err = w.status;
-        L.run("gemm_tc", [&] { return bkt::launch_gemm_bf16_tc(g, s); });
+        g.wf = wf;
+        L.run("gemm_tc", gemm_w(g.M, g.N, g.K), [&] { return bkt::launch_gemm_bf16_tc(g, s); });
       }
     } else if (l > 0) {
       // dX = dz W_ih in fp32 on the tensor cores (3xTF32): dz rows are
@@ -746,10 +787,10 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
       if (side && !w.DXh) return set_err(BKT_EINVAL, "internal: dX buffers missing for the side stream");
       if (dxa == w.AT) at_src = nullptr;  // AT is overwritten here
       for (int d = 0; d < dirs; ++d) {
-        L.run("split_rows", [&] {
+        L.run("split_rows", pass_w(NT, 4.0 * H, 4, 8), [&] {
           return bkt::launch_split_rows(w.Z[l * dirs + d], 4 * H, NT, 4 * H, dxa, dxl, 4 * H, s);
         });
-        L.run("transpose_split", [&] {
+        L.run("transpose_split", pass_w(4.0 * H, DH, 4, 8), [&] {
           return bkt::launch_transpose_split(params + lo.w_ih[l * dirs + d], DH, nullptr, 4 * H, DH, w.Wh, w.Wl,
                                              4 * H, s);
         });
@@ -765,7 +806,8 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         g.ldd = DH;
         g.accumulate = d > 0;
         g.err = w.status;
-        L.run("gemm_tf32x3", [&] { return bkt::launch_gemm_tf32x3_tc(g, dxl, w.Wl, s); });
+        g.wf = wf;
+        L.run("gemm_tf32x3", gemm_w(g.M, g.N, g.K), [&] { return bkt::launch_gemm_tf32x3_tc(g, dxl, w.Wl, s); });
       }
     }
   }
@@ -793,12 +835,15 @@ namespace {
 struct EventTimer : bkt::KernelTimer {
   struct Rec {
     const char *name;
+    bkt::Work work;
     cudaEvent_t a, b;
   };
   struct Total {
     const char *name;
     int64_t launches;
     double ms;
+    double flops, bytes;
+    int64_t steps;
   };
   std::vector<Rec> pending;
   std::vector<cudaEvent_t> pool;
@@ -814,10 +859,10 @@ struct EventTimer : bkt::KernelTimer {
     cudaEventCreate(&e);
     return e;
   }
-  void begin(const char *name, cudaStream_t s) override {
+  void begin(const char *name, const bkt::Work &wk, cudaStream_t s) override {
     if (!on) return;
     if (pending.size() >= 32768) fold();
-    Rec r{name, get(), get()};
+    Rec r{name, wk, get(), get()};
     cudaEventRecord(r.a, s);
     pending.push_back(r);
   }
@@ -834,11 +879,14 @@ struct EventTimer : bkt::KernelTimer {
       for (auto &x : totals)
         if (std::strcmp(x.name, r.name) == 0) t = &x;
       if (!t) {
-        totals.push_back(Total{r.name, 0, 0.0});
+        totals.push_back(Total{r.name, 0, 0.0, 0.0, 0.0, 0});
         t = &totals.back();
       }
       t->launches += 1;
       t->ms += ms;
+      t->flops += r.work.flops;
+      t->bytes += r.work.bytes;
+      t->steps += r.work.steps;
       pool.push_back(r.a);
       pool.push_back(r.b);
     }
@@ -875,6 +923,7 @@ struct bkt_ctx {
   cudaStream_t side = nullptr;  // output-layer weight gradient overlaps BPTT here
   cudaEvent_t fork_ev = nullptr, join_ev = nullptr;
   EventTimer timer;
+  bkt::WaitFaults wf{};  // failure-detection hooks (off)
   bkt::RecGeom geom[bkt::kMaxLayers] = {};
 
   ~bkt_ctx() {
@@ -956,7 +1005,7 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
   BKT_ALLOC(w.prev_tok[0], NT);
   BKT_ALLOC(w.prev_tok[1], NT);
   BKT_ALLOC(w.row_ok, (size_t)max_batch);
-  BKT_ALLOC(w.status, 1);
+  BKT_ALLOC(w.status, bkt::kStatusWords);
   {
     const size_t NTq = (NT + 7) & ~size_t(7), MA = std::max<size_t>(4 * H, (size_t)lo.C);
     BKT_ALLOC(w.AT, MA * NTq);
@@ -1006,7 +1055,7 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
     w.idx_dev = p;
   }
 #undef BKT_ALLOC
-  e = cudaMemset(w.status, 0, sizeof(int32_t));
+  e = cudaMemset(w.status, 0, bkt::kStatusWords * sizeof(int32_t));
   if (e != cudaSuccess) {
     delete c;
     return cuda_err("cudaMemset", e);
@@ -1061,6 +1110,9 @@ extern "C" int bkt_ctx_kernel_times(bkt_ctx *c, bkt_kernel_time *out, int32_t ca
       out[n].name = t.name;
       out[n].launches = t.launches;
       out[n].total_ms = t.ms;
+      out[n].flops = t.flops;
+      out[n].bytes = t.bytes;
+      out[n].serial_steps = t.steps;
     }
     ++n;
   }
@@ -1068,22 +1120,53 @@ extern "C" int bkt_ctx_kernel_times(bkt_ctx *c, bkt_kernel_time *out, int32_t ca
   return BKT_OK;
 }
 
-extern "C" int bkt_ctx_sync_status(bkt_ctx *c) {
-  if (!c) return set_err(BKT_EINVAL, "bkt_ctx_sync_status: NULL ctx");
+namespace {
+// Waits for the ctx's work and reads status word `i`; with `clear`, zeroes it.
+int read_status_word(bkt_ctx *c, int i, int32_t *v, bool clear) {
   cudaError_t e = cudaSetDevice(c->device);
   if (e != cudaSuccess) return cuda_err("cudaSetDevice", e);
   e = cudaStreamSynchronize(c->last_stream);
+  if (e == cudaSuccess && c->side) e = cudaStreamSynchronize(c->side);
   if (e != cudaSuccess) return cuda_err("cudaStreamSynchronize", e);
-  int32_t st = 0;
-  e = cudaMemcpy(&st, c->w.status, sizeof st, cudaMemcpyDeviceToHost);
+  e = cudaMemcpy(v, c->w.status + i, sizeof *v, cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return cuda_err("cudaMemcpy(status)", e);
-  if (st != 0) {
-    cudaMemset(c->w.status, 0, sizeof st);
-    return set_err(BKT_EDEVICE, "device check failed (flags 0x%x):%s%s%s", st,
-                   (st & 1) ? " a label is out of range or equals the blank;" : "",
-                   (st & 2) ? " a tensor-core pipeline wait timed out;" : "",
-                   (st & 4) ? " a recurrent cluster exchange wait timed out;" : "");
+  if (clear && *v != 0) {
+    e = cudaMemset(c->w.status + i, 0, sizeof *v);
+    if (e != cudaSuccess) return cuda_err("cudaMemset(status)", e);
   }
+  return BKT_OK;
+}
+}  // namespace
+
+extern "C" int bkt_ctx_sync_status(bkt_ctx *c) {
+  if (!c) return set_err(BKT_EINVAL, "bkt_ctx_sync_status: NULL ctx");
+  int32_t st = 0;
+  if (int rc = read_status_word(c, 0, &st, true)) return rc;
+  if (st != 0) {
+    const bool timeout = (st & (bkt::kErrTcWait | bkt::kErrExchWait)) != 0;
+    return set_err(timeout ? BKT_ETIMEOUT : BKT_EDEVICE, "device check failed (flags 0x%x):%s%s%s", st,
+                   (st & bkt::kErrLabel) ? " a label is out of range or equals the blank;" : "",
+                   (st & bkt::kErrTcWait) ? " a tensor-core pipeline wait timed out;" : "",
+                   (st & bkt::kErrExchWait) ? " a recurrent cluster exchange wait timed out;" : "");
+  }
+  return BKT_OK;
+}
+
+extern "C" int bkt_ctx_infeasible_count(bkt_ctx *c, int64_t *count) {
+  if (!c || !count) return set_err(BKT_EINVAL, "bkt_ctx_infeasible_count: NULL argument");
+  int32_t v = 0;
+  if (int rc = read_status_word(c, 1, &v, true)) return rc;
+  *count = v;
+  return BKT_OK;
+}
+
+extern "C" int bkt_ctx_set_wait_faults(bkt_ctx *c, int32_t poll_cap, int32_t withhold) {
+  if (!c) return set_err(BKT_EINVAL, "bkt_ctx_set_wait_faults: NULL ctx");
+  if (poll_cap < 0 || (withhold & ~(BKT_WITHHOLD_EXCHANGE | BKT_WITHHOLD_TMA)) != 0)
+    return set_err(BKT_EINVAL, "bkt_ctx_set_wait_faults: poll_cap %d or withhold bits 0x%x out of range", poll_cap,
+                   withhold);
+  c->wf.poll_cap = poll_cap == 0 ? 0 : std::max(poll_cap, 256);
+  c->wf.withhold = withhold;
   return BKT_OK;
 }
 
@@ -1143,8 +1226,9 @@ extern "C" int bkt_lstm_ctc_step(bkt_ctx *c, const bkt_batch *bt, const float *p
   if (e != cudaSuccess) return cuda_err("cudaEventRecord(stage)", e);
   c->stage_used[slot] = true;
   c->last_stream = s;
+  ix.n_cells = cells;
   return enqueue_kernels(c->cfg, c->lo, c->w, c->geom, ix, bt, params, grads, loss, s,
-                         c->timer.on ? &c->timer : nullptr, c->sm_count, c->side, c->fork_ev, c->join_ev);
+                         c->timer.on ? &c->timer : nullptr, c->sm_count, c->side, c->fork_ev, c->join_ev, c->wf);
 }
 
 // ---------------------------------------------------------------------------
@@ -1227,7 +1311,7 @@ int bkt::step_on_scratch(const bkt_model_cfg *cfg, const bkt_batch *bt, const fl
   w.prev_tok[0] = cv.take<int32_t>(NT);
   w.prev_tok[1] = cv.take<int32_t>(NT);
   w.row_ok = cv.take<int32_t>((size_t)b);
-  w.status = cv.take<int32_t>(1);
+  w.status = cv.take<int32_t>(kStatusWords);
   w.idx_dev = cv.take<char>(il.bytes);
   {
     const size_t NTq = (NT + 7) & ~size_t(7), MA = std::max<size_t>(4 * H, (size_t)lo.C);
@@ -1271,7 +1355,7 @@ int bkt::step_on_scratch(const bkt_model_cfg *cfg, const bkt_batch *bt, const fl
   const RecGeom g0 = plan_recurrent(lo.H, b, lo.dirs, sm_count);
   for (int l = 0; l < lo.L; ++l) geom[l] = g0;
 
-  cudaError_t e = cudaMemsetAsync(w.status, 0, sizeof(int32_t), s);
+  cudaError_t e = cudaMemsetAsync(w.status, 0, kStatusWords * sizeof(int32_t), s);
   if (e != cudaSuccess) return cuda_err("cudaMemsetAsync(status)", e);
   DevIdx ix;
   {
@@ -1282,5 +1366,6 @@ int bkt::step_on_scratch(const bkt_model_cfg *cfg, const bkt_batch *bt, const fl
     e = cudaMemcpyAsync(w.idx_dev, g_scratch_stage, il.bytes, cudaMemcpyHostToDevice, s);
   }
   if (e != cudaSuccess) return cuda_err("cudaMemcpyAsync(index block)", e);
+  ix.n_cells = cells;
   return enqueue_kernels(*cfg, lo, w, geom, ix, bt, params, grads, loss, s, nullptr, sm_count);
 }

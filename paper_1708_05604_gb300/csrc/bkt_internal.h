@@ -50,12 +50,34 @@ struct DevIdx {
   const int32_t *tok_off;      // [T+1]
   const int32_t *tok_t;        // [n_tok] time index of each packed token
   const int32_t *tok_r;        // [n_tok] row of each packed token
+  int64_t n_cells;             // host bookkeeping: sum_i L_i (2 U_i + 1), the CTC table cells
 };
 
+// Failure-detection hooks of a ctx (bkt_ctx_set_wait_faults): the poll cap
+// of every bounded wait (0: the kernel's built-in cap) and the withhold bits.
+struct WaitFaults {
+  int32_t poll_cap;
+  int32_t withhold;
+};
+constexpr int32_t kWithholdExchange = 1;  // BKT_WITHHOLD_EXCHANGE
+constexpr int32_t kWithholdTma = 2;       // BKT_WITHHOLD_TMA
+
+// Device error flags (word 0 of the status block; word 1 counts sequences
+// without a CTC alignment).
+constexpr int32_t kErrLabel = 1;     // a label outside 1..C-1
+constexpr int32_t kErrTcWait = 2;    // a tensor-core pipeline wait ran out
+constexpr int32_t kErrExchWait = 4;  // a recurrent cluster exchange wait ran out
+constexpr int kStatusWords = 4;
+
 // Records per-kernel CUDA events when timing is on (owned by the ctx).
+// Each launch carries its algorithmic work (see bkt_kernel_time in bkt.h).
+struct Work {
+  double flops = 0, bytes = 0;
+  int64_t steps = 0;
+};
 struct KernelTimer {
   virtual ~KernelTimer() {}
-  virtual void begin(const char *name, cudaStream_t s) = 0;
+  virtual void begin(const char *name, const Work &w, cudaStream_t s) = 0;
   virtual void end(cudaStream_t s) = 0;
 };
 
@@ -116,6 +138,7 @@ struct TcGemmArgs {
   float *P; int splits;
   int32_t *err;
   int logsoftmax;  // 3xTF32 GEMM only: replace each output row by its log-softmax (N <= 128, no split)
+  WaitFaults wf;   // poll cap / withheld first slab (failure-detection tests)
 };
 int tc_splits(int M, int N, int K, int sm_count, size_t part_floats);
 cudaError_t launch_gemm_bf16_tc(const TcGemmArgs &g, cudaStream_t s);
@@ -137,12 +160,14 @@ struct TnGemmArgs {
   float *D; int64_t ldd;
   float *P; int splits;
   int32_t *err;
+  WaitFaults wf;
 };
 int tf32x3_tn_splits(int M, int N, int K, int sm_count, size_t part_floats);
 cudaError_t launch_gemm_tf32x3_tn(const TnGemmArgs &g, cudaStream_t s);
 
 // a8: log-space CTC forward (alpha) and backward (beta-hat) tables, one CTA
-// per (row, direction); writes the per-sequence loss and the row's flag.
+// per (row, direction); writes the per-sequence loss and the row's flag, and
+// counts rows without an alignment in status[1].
 cudaError_t launch_ctc_tables(const DevIdx &ix, const float *logp, int C, int blank,
                               const int32_t *labels, float *alpha, float *beta,
                               float *loss, int32_t *row_ok, int32_t *status,
@@ -182,6 +207,7 @@ struct RecArgs {
   float *Y;            // forward output / backward: h source for nothing
   const float *dY;     // backward: d loss / d Y of this layer [n_tok x dirs*H]
   int32_t *status;     // device error flags (bit 4: a cluster exchange wait timed out)
+  WaitFaults wf;       // poll cap / withheld exchange (failure-detection tests)
 };
 cudaError_t launch_lstm_fwd(const RecArgs &a, const RecGeom &g, cudaStream_t s);
 // a11: BPTT for both directions; Z[d] holds the gates on entry and dz on exit.
@@ -223,7 +249,7 @@ struct StepBufs {
   size_t part_floats;
   int32_t *tok_t, *tok_r, *prev_tok[2];       // [NT] each
   int32_t *row_ok;                            // [b]
-  int32_t *status;                            // device error flags
+  int32_t *status;                            // device error flags [kStatusWords]
   void *idx_dev;                              // per-step index block
   // split-precision (3xTF32) operands of the fp32 contractions over tokens
   float *AT, *ATl;                            // [max(4H, C) x NTq] transposed dz / dlogit, hi and lo

@@ -144,7 +144,7 @@ __global__ void __launch_bounds__(K >= 16 ? 1024 : 512)
   bad = __syncthreads_or(bad);
   if (bad) {
     if (tid == 0 && fwd) {
-      atomicOr(status, 1);
+      atomicOr(status, kErrLabel);
       row_ok[r] = 0;
       loss[ix.row_orig[r]] = CUDART_NAN_F;
     }
@@ -279,6 +279,7 @@ __global__ void __launch_bounds__(K >= 16 ? 1024 : 512)
       const float l2 = lse2b(fin[0], fin[1]);
       const bool ok = l2 > kDead;
       row_ok[r] = ok ? 1 : 0;
+      if (!ok) atomicAdd(status + 1, 1);  // counted in the ctx (no alignment is not an error)
       loss[ix.row_orig[r]] = ok ? (float)(-((double)M + (double)l2) * kLn2) : CUDART_INF_F;
     }
   }

@@ -21,7 +21,8 @@
 // tile rows) and write fp32 to global memory.  The token range can be split
 // over gridDim.z, each split writing its own partial tile.  Every mbarrier
 // wait is bounded: on expiry the CTA records an error flag, still waits for
-// its issued MMAs through the final commit, frees TMEM and exits.
+// its issued MMAs through the final commit, waits (bounded) for the TMA loads
+// it armed, frees TMEM and exits.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -67,10 +68,14 @@ __device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
   return ok != 0;
 }
 // Bounded wait for the phase with the given parity; false on expiry.
-__device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity) {
-  for (uint32_t i = 0; i < kWaitPolls; ++i)
+__device__ __forceinline__ bool mbar_wait(uint32_t a, uint32_t parity, uint32_t cap = kWaitPolls) {
+  for (uint32_t i = 0; i < cap; ++i)
     if (mbar_try(a, parity)) return true;
   return false;
+}
+// The poll cap of a launch: the failure-detection hook's, else the built-in one.
+__device__ __forceinline__ uint32_t wait_cap(const WaitFaults &wf) {
+  return wf.poll_cap > 0 ? (uint32_t)wf.poll_cap : kWaitPolls;
 }
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y, uint32_t mbar) {
   asm volatile(
@@ -172,19 +177,31 @@ __global__ void __launch_bounds__(128, 1)
   tc_fence_after();
   const uint32_t tmem = *tslot;
 
+  const uint32_t cap = wait_cap(g.wf);
   if (warp == 0) {
     if (lane == 0) {  // TMA producer
+      int last_phase[TSTAGES];  // phase of each stage's last armed load (-1: none)
+#pragma unroll
+      for (int s = 0; s < TSTAGES; ++s) last_phase[s] = -1;
       for (int i = 0; i < nk; ++i) {
         const int s = i % TSTAGES;
-        if (i >= TSTAGES && !mbar_wait(empty0 + 8 * s, ((i / TSTAGES) - 1) & 1)) {
+        if (i >= TSTAGES && !mbar_wait(empty0 + 8 * s, ((i / TSTAGES) - 1) & 1, cap)) {
           *abort_s = 1;
           break;
         }
+        if (i == 0 && (g.wf.withhold & kWithholdTma)) continue;  // failure-detection hook
         mbar_expect_tx(full0 + 8 * s, kTxBytes);
         const int kx = (kb0 + i) * TBK;
         tma_load_2d(su32(sA + s * kAStage), &ta, kx, m0, full0 + 8 * s);
         tma_load_2d(su32(sB + s * kBStage), &tb, kx, n0, full0 + 8 * s);
+        last_phase[s] = i / TSTAGES;
       }
+      // after an abort, loads issued to stages the MMA warp never consumed
+      // may still be in flight: wait (bounded) until every armed stage has
+      // landed before the CTA can exit and its shared memory be reused
+#pragma unroll
+      for (int s = 0; s < TSTAGES; ++s)
+        if (last_phase[s] >= 0 && !mbar_wait(full0 + 8 * s, last_phase[s] & 1, cap)) *abort_s = 1;
     }
     __syncwarp();
   } else if (warp == 1) {
@@ -192,7 +209,7 @@ __global__ void __launch_bounds__(128, 1)
       int issued = 0;
       for (int i = 0; i < nk; ++i) {
         const int s = i % TSTAGES;
-        if (!mbar_wait(full0 + 8 * s, (i / TSTAGES) & 1)) {
+        if (!mbar_wait(full0 + 8 * s, (i / TSTAGES) & 1, cap)) {
           *abort_s = 1;
           break;
         }
@@ -212,7 +229,7 @@ __global__ void __launch_bounds__(128, 1)
   }
 
   // epilogue: TMEM -> registers -> global
-  const bool ready = mbar_wait(done, 0);
+  const bool ready = mbar_wait(done, 0, cap);
   if (!ready) *abort_s = 1;
   tc_fence_after();
   const int row = warp * 32 + lane;
@@ -261,7 +278,7 @@ __global__ void __launch_bounds__(128, 1)
   tc_fence_before();
   __syncthreads();
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TBN) : "memory");
-  if (threadIdx.x == 0 && *abort_s && g.err) atomicOr(g.err, 2);
+  if (threadIdx.x == 0 && *abort_s && g.err) atomicOr(g.err, kErrTcWait);
 }
 
 __global__ void __launch_bounds__(128, 1)
@@ -301,14 +318,19 @@ __global__ void __launch_bounds__(128, 1)
   tc_fence_after();
   const uint32_t tmem = *tslot;
 
+  const uint32_t cap = wait_cap(g.wf);
   if (warp == 0) {
     if (lane == 0) {  // TMA producer
+      int last_phase[FSTAGES];  // phase of each stage's last armed load (-1: none)
+#pragma unroll
+      for (int s = 0; s < FSTAGES; ++s) last_phase[s] = -1;
       for (int i = 0; i < nk; ++i) {
         const int s = i % FSTAGES;
-        if (i >= FSTAGES && !mbar_wait(empty0 + 8 * s, ((i / FSTAGES) - 1) & 1)) {
+        if (i >= FSTAGES && !mbar_wait(empty0 + 8 * s, ((i / FSTAGES) - 1) & 1, cap)) {
           *abort_s = 1;
           break;
         }
+        if (i == 0 && (g.wf.withhold & kWithholdTma)) continue;  // failure-detection hook
         uint8_t *st = base + s * kFStage;
         mbar_expect_tx(full0 + 8 * s, kFStage);
         const int kx = (kb0 + i) * FBK;
@@ -316,7 +338,12 @@ __global__ void __launch_bounds__(128, 1)
         tma_load_2d(su32(st + kFTile), &tal, kx, m0, full0 + 8 * s);
         tma_load_2d(su32(st + 2 * kFTile), &tbh, kx, n0, full0 + 8 * s);
         tma_load_2d(su32(st + 3 * kFTile), &tbl, kx, n0, full0 + 8 * s);
+        last_phase[s] = i / FSTAGES;
       }
+      // drain the armed stages before the CTA can exit (see the bf16 kernel)
+#pragma unroll
+      for (int s = 0; s < FSTAGES; ++s)
+        if (last_phase[s] >= 0 && !mbar_wait(full0 + 8 * s, last_phase[s] & 1, cap)) *abort_s = 1;
     }
     __syncwarp();
   } else if (warp == 1) {
@@ -324,7 +351,7 @@ __global__ void __launch_bounds__(128, 1)
       int issued = 0;
       for (int i = 0; i < nk; ++i) {
         const int s = i % FSTAGES;
-        if (!mbar_wait(full0 + 8 * s, (i / FSTAGES) & 1)) {
+        if (!mbar_wait(full0 + 8 * s, (i / FSTAGES) & 1, cap)) {
           *abort_s = 1;
           break;
         }
@@ -346,7 +373,7 @@ __global__ void __launch_bounds__(128, 1)
     __syncwarp();
   }
 
-  const bool ready = mbar_wait(done, 0);
+  const bool ready = mbar_wait(done, 0, cap);
   if (!ready) *abort_s = 1;
   tc_fence_after();
   const int m = m0 + warp * 32 + lane;
@@ -424,7 +451,7 @@ __global__ void __launch_bounds__(128, 1)
   tc_fence_before();
   __syncthreads();
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(FBN) : "memory");
-  if (threadIdx.x == 0 && *abort_s && g.err) atomicOr(g.err, 2);
+  if (threadIdx.x == 0 && *abort_s && g.err) atomicOr(g.err, kErrTcWait);
 }
 
 // ---------------------------------------------------------------------------
@@ -513,12 +540,13 @@ __global__ void __launch_bounds__(kTnThreads, 1) gemm_tf32x3_tn_kernel(TnGemmArg
   tc_fence_after();
   const uint32_t tmem = *tslot;
 
+  const uint32_t cap = wait_cap(g.wf);
   if (warp == kTnConv / 32) {  // the MMA warp
     if (lane == 0) {
       int issued = 0;
       for (int i = 0; i < nk; ++i) {
         const int s = i % kTnStages;
-        if (!mbar_wait(full0 + 8 * s, (i / kTnStages) & 1)) {
+        if (!mbar_wait(full0 + 8 * s, (i / kTnStages) & 1, cap)) {
           *abort_s = 1;
           break;
         }
@@ -574,7 +602,7 @@ __global__ void __launch_bounds__(kTnThreads, 1) gemm_tf32x3_tn_kernel(TnGemmArg
     bool fail = false;
     auto slab = [&](int i, float4 (&va)[4], float4 (&vb)[4], int (&br)[4]) -> bool {
       const int s = i % kTnStages;
-      if (i >= kTnStages && !mbar_wait(empty0 + 8 * s, ((i / kTnStages) - 1) & 1)) {
+      if (i >= kTnStages && !mbar_wait(empty0 + 8 * s, ((i / kTnStages) - 1) & 1, cap)) {
         fail = true;
         return false;
       }
@@ -600,7 +628,8 @@ __global__ void __launch_bounds__(kTnThreads, 1) gemm_tf32x3_tn_kernel(TnGemmArg
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       __syncwarp();
-      if (lane == 0) mbar_arrive(full0 + 8 * s);
+      // (failure-detection hook: the first slab is never published)
+      if (lane == 0 && !(i == 0 && (g.wf.withhold & kWithholdTma))) mbar_arrive(full0 + 8 * s);
       // the vectors of slab i + 2 (rows loaded two slabs ago), then the rows of slab i + 4
       load(i + 2, br, va, vb);
       rows_of(i + 4, br);
@@ -622,7 +651,7 @@ __global__ void __launch_bounds__(kTnThreads, 1) gemm_tf32x3_tn_kernel(TnGemmArg
     if (fail) *abort_s = 1;
   }
 
-  const bool ready = mbar_wait(done, 0);
+  const bool ready = mbar_wait(done, 0, cap);
   tc_fence_after();
   __syncthreads();
   const bool aborted = *abort_s != 0;
@@ -647,7 +676,7 @@ __global__ void __launch_bounds__(kTnThreads, 1) gemm_tf32x3_tn_kernel(TnGemmArg
   tc_fence_before();
   __syncthreads();
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(FBN) : "memory");
-  if (tid == 0 && (aborted || !ready) && g.err) atomicOr(g.err, 2);
+  if (tid == 0 && (aborted || !ready) && g.err) atomicOr(g.err, kErrTcWait);
 }
 
 // ---------------------------------------------------------------------------

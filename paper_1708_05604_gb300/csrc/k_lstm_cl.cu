@@ -31,8 +31,10 @@
 // every read of the buffer it will reuse two steps later, so the data
 // dependence itself orders reuse and no cluster-wide barrier is needed per
 // step.  Every wait is bounded: on expiry the kernel sets bit 4 of the status
-// word, leaves its loop at the next CTA barrier, and all CTAs meet at a final
-// cluster barrier.
+// word, leaves its loop at the next CTA barrier, sleeps 20 us so that stores
+// its peers issued before they gave up can land, and all CTAs meet at a final
+// cluster barrier.  (A peer gives up only after its own bounded wait, at
+// least 256 polls after its last store.)
 #include <cstdint>
 
 #include <algorithm>
@@ -50,7 +52,7 @@ constexpr int kClThreads = 256;
 constexpr int kClFwdRegCols = BKT_CL_FWD_REG_COLS;  // multiple of 4, at most 64
 constexpr int kClTokCap = 8192;  // time offsets staged in shared memory up to this T
 constexpr int kClPolls = 1 << 22;
-constexpr int32_t kErrExchange = 4;
+constexpr int32_t kErrExchange = kErrExchWait;
 
 // Gate nonlinearities from the exponential intrinsic: sigma(x) = 1 / (1 + e^-x)
 // and tanh(x) = 1 - 2 / (1 + e^2x) (absolute error a few 1e-8; both saturate
@@ -81,8 +83,8 @@ __device__ __forceinline__ void mbar_init1(uint32_t mb) {
 __device__ __forceinline__ void mbar_arm(uint32_t mb, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(mb), "r"(bytes) : "memory");
 }
-__device__ __forceinline__ bool mbar_wait_bounded(uint32_t mb, uint32_t parity) {
-  for (int i = 0; i < kClPolls; ++i) {
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t mb, uint32_t parity, int cap) {
+  for (int i = 0; i < cap; ++i) {
     uint32_t done;
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
@@ -250,6 +252,9 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_fwd_cl_kernel(RecArgs a) {
     for (int rr = 0; rr < RPL; ++rr) cst[h][rr] = 0.f;
   }
   bool ok = true, stop = false;
+  const int cap = a.wf.poll_cap > 0 ? a.wf.poll_cap : kClPolls;
+  // failure-detection hook: CTA 0 of the cluster withholds its exchange data
+  const bool withhold = (a.wf.withhold & kWithholdExchange) && c == 0;
 
   for (int s = 0; s < Tg && !stop; ++s) {
 #pragma unroll
@@ -266,8 +271,10 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_fwd_cl_kernel(RecArgs a) {
       for (int i = 0; i < NV; ++i) acc[i] = 0.f;
       if (s > 0) {  // h_{-1} = 0
         const int e = s - 1;
-        ok = mbar_wait_bounded(smem_addr(&mb[2 * h + (e & 1)]), (e >> 1) & 1) && ok;
-        if (t == 0 && e + 2 <= Tg - 2) mbar_arm(smem_addr(&mb[2 * h + (e & 1)]), Gm::kXBytes);
+        ok = mbar_wait_bounded(smem_addr(&mb[2 * h + (e & 1)]), (e >> 1) & 1, cap) && ok;
+        // re-arm only a phase that completed: arriving again on a phase whose
+        // wait ran out would over-arrive on it (its one arrival is spent)
+        if (t == 0 && ok && e + 2 <= Tg - 2) mbar_arm(smem_addr(&mb[2 * h + (e & 1)]), Gm::kXBytes);
         const float *hv = hb + (2 * h + (e & 1)) * BH * HPAD + kb + 4 * kl;
 #pragma unroll
         for (int k4 = 0; k4 < RK / 4; ++k4) {
@@ -350,7 +357,7 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_fwd_cl_kernel(RecArgs a) {
         stop = true;
         break;
       }
-      if (s + 1 < Tg) {  // exchange s of half h: this CTA's slice to every CTA of the cluster
+      if (s + 1 < Tg && !withhold) {  // exchange s of half h: this CTA's slice to every CTA of the cluster
         const uint32_t dst0 = smem_addr(hb + (2 * h + (s & 1)) * BH * HPAD), mbl = smem_addr(&mb[2 * h + (s & 1)]);
         for (int n = t; n < CS * SEND4; n += NTH) {
           const int peer = n / SEND4, rem = n % SEND4, b = rem / (Hc / 4), u4 = rem % (Hc / 4);
@@ -362,6 +369,9 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_fwd_cl_kernel(RecArgs a) {
       }
     }
   }
+  // after an abort, stores a peer issued before it gave up may still be in
+  // flight toward this CTA: give them time to land before the cluster exits
+  if (stop) __nanosleep(20000);
   cluster_barrier_all();  // no CTA leaves while a peer may still address its shared memory
 }
 
@@ -467,6 +477,9 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a) {
     }
   cp_commit_cl();
   bool ok = true, stop = false;
+  const int cap = a.wf.poll_cap > 0 ? a.wf.poll_cap : kClPolls;
+  // failure-detection hook: CTA 0 of the cluster withholds its exchange data
+  const bool withhold = (a.wf.withhold & kWithholdExchange) && c == 0;
 
   for (int it = 0; it < Tg && !stop; ++it) {
     const int s = Tg - 1 - it;
@@ -480,8 +493,10 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a) {
     for (int h = 0; h < NH; ++h) {
       if (it > 0) {
         const int e = it - 1;
-        ok = mbar_wait_bounded(smem_addr(&mb[2 * h + (e & 1)]), (e >> 1) & 1) && ok;
-        if (t == 0 && e + 2 <= Tg - 2) mbar_arm(smem_addr(&mb[2 * h + (e & 1)]), Gm::kXBytes);
+        ok = mbar_wait_bounded(smem_addr(&mb[2 * h + (e & 1)]), (e >> 1) & 1, cap) && ok;
+        // re-arm only a phase that completed: arriving again on a phase whose
+        // wait ran out would over-arrive on it (its one arrival is spent)
+        if (t == 0 && ok && e + 2 <= Tg - 2) mbar_arm(smem_addr(&mb[2 * h + (e & 1)]), Gm::kXBytes);
       }
       float *dzb = dzs + (2 * h + (it & 1)) * DZS;
       // phase B
@@ -528,7 +543,7 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a) {
         stop = true;
         break;
       }
-      if (it + 1 >= Tg) continue;  // dh_{-1} is not needed
+      if (it + 1 >= Tg || withhold) continue;  // dh_{-1} is not needed
       // phase A: partial W_hh^T dz over this thread's 64 rows, columns k0..k0+3
       // (a [batch row][gate row] dz layout made phase B cheaper but this loop
       // slower, a net loss)
@@ -576,6 +591,7 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a) {
     }
   }
   cp_wait_all_cl();
+  if (stop) __nanosleep(20000);  // in-flight peer stores after an abort (see the forward kernel)
   cluster_barrier_all();
 }
 

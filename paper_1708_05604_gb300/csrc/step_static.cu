@@ -29,6 +29,18 @@ extern "C" int bkt_lstm_ctc_step_static(const bkt_model_cfg *cfg, const bkt_batc
     return bkt::report_error(BKT_ECUDA, "cudaGetDevice: %s (%s)", cudaGetErrorName(e), cudaGetErrorString(e));
   if (dev < 0 || dev >= kMaxDevices)
     return bkt::report_error(BKT_EINVAL, "bkt_lstm_ctc_step_static: device %d out of range", dev);
+  if (stream) {
+    // the work goes to the stream's device: it must be the current one,
+    // whose copy of the array is used (checked before anything is enqueued)
+    int sdev = -1;
+    e = cudaStreamGetDevice((cudaStream_t)stream, &sdev);
+    if (e != cudaSuccess)
+      return bkt::report_error(BKT_ECUDA, "cudaStreamGetDevice: %s (%s)", cudaGetErrorName(e), cudaGetErrorString(e));
+    if (sdev != dev)
+      return bkt::report_error(BKT_EINVAL,
+                               "bkt_lstm_ctc_step_static: the stream belongs to device %d but device %d is current",
+                               sdev, dev);
+  }
   DeviceScratch ds;
   {
     // first call on this device (with it current): look up the array's

@@ -1,12 +1,14 @@
-"""Host-side logic of bench.py that needs no GPU: the roofline arithmetic,
-the committed DRAM-traffic record (reported only while the kernel source it
-was taken from is unchanged) and the peak table."""
+"""Host-side logic of bench.py that needs no GPU: the roofline arithmetic
+per bound, the epoch budget rule, the committed DRAM-traffic record
+(reported only while the kernel source it was taken from is unchanged), the
+peak table and the defaults (the full-epoch bimodal sweep)."""
 import hashlib
 import importlib.util
 import json
 import os
 import shutil
 
+import numpy as np
 import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
@@ -20,25 +22,63 @@ def bench():
     return mod
 
 
+def stat(name, launches, ms, flops=0.0, nbytes=0.0, steps=0):
+    return {"name": name, "launches": launches, "total_ms": ms, "flops": flops, "bytes": nbytes,
+            "serial_steps": steps}
+
+
 def test_roofline_alu_arithmetic(bench):
-    work = {"lstm_fwd": ("alu", 4.0e9)}
-    r = bench.roofline_for("lstm_fwd", 10, 20.0, work, {"sm_max_mhz": 2000.0}, "measured",
-                           {"sm_mhz": 1000.0})
-    # 10 launches in 20 ms: 2 ms each; 4 GFLOP / 2 ms = 2 TFLOP/s
+    r = bench.roofline_for(stat("lstm_fwd", 10, 20.0, flops=4.0e10, steps=4000),
+                           {"sm_max_mhz": 2000.0}, "measured", {"sm_mhz": 1000.0}, n_sm=152)
+    # 4e10 flop in 20 ms = 2 TFLOP/s; 20 ms over 4000 serial steps = 5 us per step
     assert r["bound"] == "alu" and r["unit"] == "TFLOP/s"
     assert r["achieved"] == pytest.approx(2.0)
     assert r["peak"] == pytest.approx(152 * 128 * 2 * 1000e6 / 1e12)
     assert r["frac"] == pytest.approx(r["achieved"] / r["peak"])
-    assert bench.roofline_for("other", 1, 1.0, work, {}, "measured", {}) is None
+    assert r["us_per_step"] == pytest.approx(5.0)
+    assert r["algorithmic_flops_per_launch"] == pytest.approx(4.0e9)
+    # no work, no roofline
+    assert bench.roofline_for(stat("lstm_fwd", 1, 1.0), {}, "measured", {}) is None
 
 
 def test_roofline_hbm_arithmetic(bench):
-    work = {"ctc_grad": ("hbm", 6.0e6)}
-    r = bench.roofline_for("ctc_grad", 4, 4.0, work, {"hbm_gbs": 6000.0}, "measured", {})
-    # 1 ms per launch: 6e6 B / 1e-3 s = 6e9 B/s = 6 GB/s
+    r = bench.roofline_for(stat("ctc_grad", 4, 4.0, nbytes=2.4e7), {"hbm_gbs": 6000.0}, "measured", {})
+    # 2.4e7 B in 4 ms = 6 GB/s
     assert r["bound"] == "hbm" and r["unit"] == "GB/s"
     assert r["achieved"] == pytest.approx(6.0)
     assert r["frac"] == pytest.approx(6.0 / 6000.0)
+    assert "us_per_step" not in r
+
+
+def test_roofline_tensor_peaks(bench):
+    peaks = {"bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+    r = bench.roofline_for(stat("gemm_tc", 2, 1.0, flops=1.7e15 * 1e-3 * 0.5), peaks, "measured", {})
+    assert r["bound"] == "tensor" and r["peak"] == pytest.approx(1700.0)
+    assert r["frac"] == pytest.approx(0.5)
+    r3 = bench.roofline_for(stat("gemm_tf32x3", 2, 1.0, flops=1e9), peaks, "measured", {})
+    assert r3["peak"] == pytest.approx(1700.0 * (1.1 / 2.25) / 3.0)
+
+
+def test_budget_count(bench):
+    assert bench.budget_count(5700.0, 3000.0, 1, 10) == 1
+    assert bench.budget_count(20.0, 3000.0, 1, 10) == 10
+    assert bench.budget_count(5700.0, 15000.0, 2, 20) == 3
+    assert bench.budget_count(0.0, 1.0, 2, 5) == 5
+
+
+def test_defaults_are_the_full_epoch_sweep(bench):
+    a = bench.parse([])
+    assert a.workload == "lstm3_bi_h256_bf16_bimodal" and a.buckets == 8
+    qs = sorted({a.buckets} | {int(q) for q in a.compare_buckets.split(",")})
+    assert qs == [1, 2, 4, 8, 16, 32]
+    assert bench.METRIC.startswith("unpadded timesteps/sec")
+
+
+def test_serial_steps(bench):
+    class DS:
+        lengths = np.array([5, 9, 2, 7], np.int32)
+    plan = {"n_batches": 2, "batch_off": np.array([0, 2, 4]), "order": np.array([2, 0, 1, 3])}
+    assert bench.serial_steps(plan, DS) == 5 + 9
 
 
 def test_recorded_traffic_matches_committed_source(bench):

@@ -1,8 +1,9 @@
 """GPU parity: the CUDA training step (through the C ABI) against the fp64
 oracle, element by element per parameter block, on seeded synthetic inputs.
 Sizes let the oracle finish in seconds while spanning several tiles, clusters
-and ragged tails; the last tests use full-size batches of the workloads and
-check sampled per-sequence losses plus properties that hold at any size."""
+and ragged tails; the last tests take whole batches of the workloads' own
+plans at full size, launched as the benchmark launches them, and compare
+every gradient with the oracle (run one sequence per process)."""
 import math
 
 import numpy as np
@@ -11,7 +12,7 @@ import pytest
 import oracle
 from paper_1708_05604_gb300 import binding, synth
 
-from gpu_util import BF16_TOL, FP32_TOL, compare, gpu_step, oracle_step
+from gpu_util import BF16_TOL, FP32_TOL, compare, gpu_step, oracle_step, oracle_step_parallel
 
 pytestmark = pytest.mark.gpu
 
@@ -144,10 +145,17 @@ def test_edge_cases_one_step():
     np.cumsum(U, out=off[1:])
     ds = synth.Dataset(ds.lengths, ds.x, ds.x_off, U.astype(np.int32), labels, off)
     params = synth.draw_params(rng, binding.param_count(cfg))
-    lg, gg = gpu_step(cfg, ds, params)
+    ctx = binding.Ctx(cfg, int(ds.lengths.sum()), ds.n, int(ds.label_lengths.max()))
+    lg, gg = gpu_step(cfg, ds, params, ctx=ctx)
     lo, go = oracle_step(cfg, ds, params)
     assert math.isinf(lo[6]) and math.isinf(lg[6]) and lg[6] > 0
     compare(cfg, lg, gg, lo, go, FP32_TOL)
+    # the sequence without an alignment is counted in the ctx, once
+    assert ctx.infeasible_count() == 1
+    assert ctx.infeasible_count() == 0
+    gpu_step(cfg, ds, params, ctx=ctx)
+    gpu_step(cfg, ds, params, ctx=ctx)
+    assert ctx.infeasible_count() == 2
 
 
 def test_single_sequence_and_permutation_invariance():
@@ -280,27 +288,53 @@ def full_batch(wname, Q, which="longest", seed=0):
     return w, ds, ids
 
 
-@pytest.mark.parametrize("wname,Q", [("lstm1_bi_h128", 4), ("lstm1_bi_h128", 1),
-                                     ("lstm1_uni_h32", 2), ("lstm2_uni_h512", 4),
-                                     ("lstm3_bi_h256_bf16", 16)])
-def test_full_size_batch_sampled(wname, Q):
-    w, ds, ids = full_batch(wname, Q)
+@pytest.mark.parametrize("wname,Q,which", [
+    ("lstm1_uni_h32", 2, "longest"),
+    # the longest batch of the 4-bucket plan: 64 sequences, ~58 k tokens
+    ("lstm1_bi_h128", 4, "longest"),
+    ("lstm1_bi_h128", 1, "first"),
+    # the shortest batches of the 16- and 32-bucket plans: 128 sequences,
+    # split-K weight gradients over several accumulators
+    ("lstm3_bi_h256_bf16", 16, "first"),
+    ("lstm3_bi_h256_bf16_bimodal", 32, "first"),
+])
+def test_full_size_batch_vs_oracle(wname, Q, which):
+    """A whole batch of the benchmark's plan, launched as the benchmark
+    launches it (ctx sized for the workload), against the oracle element by
+    element in every parameter block; the bf16 workloads again with fp32
+    contractions at the fp32 bound."""
+    w, ds, ids = full_batch(wname, Q, which)
     cfg = w.model_cfg()
     params = synth.draw_params(np.random.default_rng(1), binding.param_count(cfg))
     dd = binding.DeviceDataset(ds)
-    lg, gg = gpu_step(cfg, ds, params, seq_ids=ids, dd=dd)
-    assert np.all(np.isfinite(gg))
-    # sampled outputs: the oracle's loss of a few sequences, one at a time
-    # (the shortest ones, so the oracle stays within seconds)
-    order = np.argsort(ds.lengths[ids])
-    n_sample = 1 if cfg["hidden"] >= 512 else 2
-    for pos in order[:n_sample]:
-        lo, _ = oracle_step(cfg, ds, params, seq_ids=[ids[pos]])
-        assert abs(lg[pos] - lo[0]) <= tol_for(cfg) * abs(lo[0]), (pos, lg[pos], lo[0])
-    # linearity over sequences: grad(batch) = grad(first half) + grad(second half)
-    h = ids.size // 2
-    _, ga = gpu_step(cfg, ds, params, seq_ids=ids[:h], dd=dd)
-    _, gb = gpu_step(cfg, ds, params, seq_ids=ids[h:], dd=dd)
+    lo, go = oracle_step_parallel(cfg, ds, params, ids)
+    cfgs = [cfg] + ([dict(cfg, gemm_bf16=False)] if cfg["gemm_bf16"] else [])
+    for c in cfgs:
+        ctx = binding.Ctx(c, int(np.sort(ds.lengths)[-w.batch:].sum()), w.batch, int(ds.label_lengths.max()))
+        lg, gg = gpu_step(c, ds, params, seq_ids=ids, dd=dd, ctx=ctx)
+        assert np.all(np.isfinite(gg))
+        compare(c, lg, gg, lo, go, tol_for(c))
+        ctx.close()
+
+
+def test_full_length_h512_wide_batch_vs_oracle():
+    """Three full-length sequences of the H = 512 workload (two layers, fp32)
+    through a ctx sized for its batch of 32: the 16-CTA cluster kernels run
+    in their full-batch configuration, over ~3,000-4,000 steps."""
+    w = synth.WORKLOADS["lstm2_uni_h512"]
+    ds = synth.make_workload(w, seed=0)
+    order = np.argsort(-ds.lengths, kind="stable")
+    ids = np.array([order[0], order[len(order) // 2], order[-1]])
+    cfg = w.model_cfg()
+    params = synth.draw_params(np.random.default_rng(1), binding.param_count(cfg))
+    dd = binding.DeviceDataset(ds)
+    ctx = binding.Ctx(cfg, int(np.sort(ds.lengths)[-w.batch:].sum()), w.batch, int(ds.label_lengths.max()))
+    lg, gg = gpu_step(cfg, ds, params, seq_ids=ids, dd=dd, ctx=ctx)
+    lo, go = oracle_step_parallel(cfg, ds, params, ids)
+    compare(cfg, lg, gg, lo, go, FP32_TOL)
+    # the batch gradient is the sum of the sequences' gradients
+    _, ga = gpu_step(cfg, ds, params, seq_ids=ids[:1], dd=dd, ctx=ctx)
+    _, gb = gpu_step(cfg, ds, params, seq_ids=ids[1:], dd=dd, ctx=ctx)
     assert np.linalg.norm(ga + gb - gg) <= 1e-4 * np.linalg.norm(gg)
 
 
