@@ -1081,7 +1081,8 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
       return cuda_err("side stream", e2);
     }
   }
-  for (int l = 0; l < lo.L; ++l) c->geom[l] = bkt::plan_recurrent(lo.H, max_batch, lo.dirs, c->sm_count);
+  for (int l = 0; l < lo.L; ++l)
+    c->geom[l] = bkt::plan_recurrent(lo.H, max_batch, lo.dirs, c->sm_count, cfg->gemm_precision == BKT_GEMM_BF16);
   *out = c;
   return BKT_OK;
 }
@@ -1352,7 +1353,7 @@ int bkt::step_on_scratch(const bkt_model_cfg *cfg, const bkt_batch *bt, const fl
   w.part_floats = std::min(w.part_floats, 64 * min_part);
 
   RecGeom geom[kMaxLayers];
-  const RecGeom g0 = plan_recurrent(lo.H, b, lo.dirs, sm_count);
+  const RecGeom g0 = plan_recurrent(lo.H, b, lo.dirs, sm_count, cfg->gemm_precision == BKT_GEMM_BF16);
   for (int l = 0; l < lo.L; ++l) geom[l] = g0;
 
   cudaError_t e = cudaMemsetAsync(w.status, 0, kStatusWords * sizeof(int32_t), s);

@@ -182,6 +182,8 @@ cudaError_t launch_ctc_grad(const DevIdx &ix, float *logp_dlogit, int C, int bla
 // Geometry of the recurrent kernels for one layer.
 //   mode 1: one CTA per bc rows holds all of W_hh (H in {32, 64, 128});
 //   mode 2: register-tiled cluster of cs CTAs per bc rows (H in {256, 512});
+//   mode 3: tensor-core cluster of 8 CTAs per bc rows, W_hh in TMEM
+//           (H = 256 with bf16 contractions);
 //   mode 0: a cluster of cs CTAs per bc rows splits the hidden units (any H).
 struct RecGeom {
   int mode;
@@ -192,7 +194,7 @@ struct RecGeom {
   int w_smem;    // 1: the CTA's W_hh slice lives in shared memory
   size_t smem_fwd, smem_bwd;
 };
-RecGeom plan_recurrent(int H, int b, int dirs, int sm_count);
+RecGeom plan_recurrent(int H, int b, int dirs, int sm_count, bool bf16);
 
 // a6: persistent recurrent forward for both directions of one layer.
 //   Z[d]  [n_tok x 4H] pre-activations in, activated gates (i,f,g,o) out
@@ -219,6 +221,14 @@ cudaError_t launch_lstm_bwd(const RecArgs &a, const RecGeom &g, cudaStream_t s);
 int cl_cluster_size(int H);
 int plan_cl_rows(int H, int b, int dirs);
 cudaError_t launch_lstm_cl(const RecArgs &a, int bc, bool bwd, cudaStream_t s);
+
+// Tensor-core cluster kernels for H = 256 on the bf16 path (k_lstm_tc.cu):
+// whether H is handled there (BKT_REC_TC=0 in the environment turns them
+// off), rows per cluster for a batch of b rows (16 or 32; 0: cannot launch),
+// launch.
+bool tc_rec_supported(int H);
+int plan_tc_rows(int b, int dirs);
+cudaError_t launch_lstm_tc(const RecArgs &a, int rows, bool bwd, cudaStream_t s);
 
 // Single-CTA recurrent kernels (k_lstm_cta.cu).
 bool cta_supported(int H);

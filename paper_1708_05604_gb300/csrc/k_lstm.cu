@@ -327,10 +327,22 @@ bool cluster_fits(K kernel, int cs, int threads, size_t smem) {
 
 }  // namespace
 
-RecGeom plan_recurrent(int H, int b, int dirs, int sm_count) {
+RecGeom plan_recurrent(int H, int b, int dirs, int sm_count, bool bf16) {
   const int Tcap = kTokSmemCap - 1;
   const size_t lim = 220 * 1024;
   RecGeom g{};
+  if (bf16 && tc_rec_supported(H)) {
+    const int rows = plan_tc_rows(b, dirs);
+    if (rows > 0) {
+      g.mode = 3;
+      g.cs = 8;
+      g.bc = rows;
+      g.ks = 1;
+      g.threads = 128;
+      g.w_smem = 0;
+      return g;
+    }
+  }
   if (cta_supported(H)) {
     g.mode = 1;
     g.cs = 1;
@@ -412,6 +424,7 @@ cudaError_t launch_rec(K kernel, const RecArgs &a, const RecGeom &g, bool bwd, c
 }  // namespace
 
 cudaError_t launch_lstm_fwd(const RecArgs &a, const RecGeom &g, cudaStream_t s) {
+  if (g.mode == 3) return launch_lstm_tc(a, g.bc, false, s);
   if (g.mode == 1) return launch_lstm_cta(a, g.bc, false, s);
   if (g.mode == 2) return launch_lstm_cl(a, g.bc, false, s);
   if (a.H % g.cs != 0) return cudaErrorInvalidValue;
@@ -420,6 +433,7 @@ cudaError_t launch_lstm_fwd(const RecArgs &a, const RecGeom &g, cudaStream_t s) 
 }
 
 cudaError_t launch_lstm_bwd(const RecArgs &a, const RecGeom &g, cudaStream_t s) {
+  if (g.mode == 3) return launch_lstm_tc(a, g.bc, true, s);
   if (g.mode == 1) return launch_lstm_cta(a, g.bc, true, s);
   if (g.mode == 2) return launch_lstm_cl(a, g.bc, true, s);
   if (a.H % g.cs != 0) return cudaErrorInvalidValue;

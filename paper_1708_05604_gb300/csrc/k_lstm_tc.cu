@@ -1,0 +1,786 @@
+// k_lstm_tc.cu -- the recurrence of the bf16 configuration at H = 256 on the
+// 5th-generation tensor cores (a6 forward, a11 BPTT).
+//
+// One step of the recurrence is a small dense contraction per batch row:
+// forward z_t = Zx_t + W_hh h_{t-1} ([4H x H] by [H]), BPTT
+// dh_{t-1} = W_hh^T dz_t.  A thread-block cluster of 8 CTAs owns one
+// direction and N = 16 or 32 consecutive rows of the length-sorted batch;
+// CTA c owns the hidden units [32c, 32c + 32), i.e. the 128 gate rows
+// {q H + 32c + u : q = i, f, g, o; u < 32}, and keeps its slice of W_hh for
+// the whole sequence in tensor memory as the A operand of tcgen05.mma, split
+// into two bf16 parts (w = w_hi + w_lo, 16 significant bits).  The other
+// operand (h_{t-1}, or dz_t) is split the same way in shared memory, and each
+// step issues the three products hi*hi + hi*lo + lo*hi with fp32
+// accumulation in TMEM (relative error near 2^-16 per product; the cell
+// state, the gates and every elementwise step stay fp32).  W never leaves
+// the SM: per step only N rows of h (or dz) are read from shared memory.
+//
+// TMEM lane m = 4u + q holds gate row q H + 32c + u of the CTA (forward: A =
+// W slice, K = the 256 units; BPTT: A = W slice transposed in two 128-unit
+// halves, K = the CTA's 128 gate rows in the same 4u + q order).  Operands in
+// shared memory use the K-major layout without swizzle: 8 x 16-byte core
+// matrices, element (n, k) at (k / 8) * 16 N + n * 16 + (k % 8) * 2 bytes, so
+// the 32 units of one CTA are one contiguous 64 N-byte block.
+//
+// Forward step: one thread issues the 48 MMAs (16 k-steps of 16 x 3
+// products) once h_{t-1} has arrived and commits them to an mbarrier; the
+// 128 threads read the accumulator (thread = gate row, N columns), add Zx,
+// apply sigma / tanh, swap gates inside groups of four lanes so that each
+// lane holds the four gates of one unit for N / 4 rows, update the cell
+// state in registers, write gates, c_t and h_t, and stage h_t (bf16 hi and
+// lo) to send it to every CTA of the cluster with st.async (16-byte remote
+// stores completing bytes on the receiver's mbarrier; double-buffered by step
+// parity, so the data dependence orders buffer reuse).
+// BPTT step: dh = dY + the sum of the 8 partials of W_hh^T dz_{t+1} received
+// for this CTA's units, then dc and dz of the four gates (fp32, written to
+// the gate buffer in place and, split, to the B operand); the MMAs form this
+// CTA's partial W_hh^T dz over its 128 gate rows for all 256 units (two
+// 128-lane halves), and each 32-unit block goes to the CTA that owns it.
+//
+// Every wait is bounded (status bit 4 on expiry, as in the other cluster
+// kernels); on an abort the kernel still waits for its last MMA batch before
+// it frees TMEM, sleeps 20 us so peers' in-flight stores land, and meets its
+// peers at a final cluster barrier.  A CTA takes all 512 TMEM columns; its
+// shared-memory request (>= 120 KB) keeps any other CTA off its SM.
+#include <cuda_bf16.h>
+
+#include <cstdint>
+
+#include <algorithm>
+
+#include "bkt_internal.h"
+
+namespace bkt {
+
+namespace {
+
+constexpr int kTH = 256;           // hidden units
+constexpr int kTCS = 8;            // CTAs per cluster
+constexpr int kTHc = kTH / kTCS;   // units per CTA
+constexpr int kTTokCap = 8192;     // time offsets staged in shared memory up to this T
+constexpr int kTPolls = 1 << 22;
+constexpr size_t kTSmemFloor = 120 * 1024;  // one CTA per SM: each CTA holds all of TMEM
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kAccCol = 256;  // first accumulator column (A operands take 0 .. 255)
+
+// kind::f16 instruction descriptor: D fp32, A and B bf16, both K-major,
+// N >> 3 at bit 17, M = 128 (>> 4 at bit 24).
+template <int N>
+__host__ __device__ constexpr uint32_t tc_idesc() {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+}
+
+__device__ __forceinline__ uint32_t sa(const void *p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
+__device__ __forceinline__ uint32_t peer(uint32_t a, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void mb_init(uint32_t mb, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(mb), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mb_arm(uint32_t mb, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(mb), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mb_arrive(uint32_t mb) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(mb) : "memory");
+}
+__device__ __forceinline__ bool mb_wait(uint32_t mb, uint32_t parity, int cap) {
+  for (int i = 0; i < cap; ++i) {
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(mb), "r"(parity)
+        : "memory");
+    if (done) return true;
+  }
+  return false;
+}
+__device__ __forceinline__ void st_async16(uint32_t raddr, uint4 v, uint32_t rmbar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.b32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(raddr),
+               "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "r"(rmbar)
+               : "memory");
+}
+__device__ __forceinline__ void fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+// Shared-memory descriptor of a K-major operand without swizzle: core
+// matrices of 8 rows x 16 bytes, `lbo` bytes apart along K, `sbo` along N.
+__device__ __forceinline__ uint64_t desc_kmajor(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = (uint64_t)((addr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;  // descriptor version
+  return d;                // swizzle mode 0: none
+}
+// D (TMEM) (+)= A (TMEM) * B (shared memory)
+__device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d),
+      "r"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint32_t mbar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(mbar) : "memory");
+}
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&v)[8]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"r"(taddr), "r"(v[0]),
+               "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+               : "memory");
+}
+// C = N / 4 consecutive columns of this thread's lane, added into x (C = 4 or 8).
+template <int C>
+__device__ __forceinline__ void tmem_ld_add(uint32_t taddr, float (&x)[C]) {
+  uint32_t r[C];
+  if constexpr (C == 4) {
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(taddr)
+                 : "memory");
+  } else {
+    static_assert(C == 8, "4 or 8 columns per thread");
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                 : "r"(taddr)
+                 : "memory");
+  }
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int j = 0; j < C; ++j) x[j] += __uint_as_float(r[j]);
+}
+
+// x = hi + lo, both bf16 (hi rounded to nearest, lo the rounded rest).
+__device__ __forceinline__ void split_bf16(float x, __nv_bfloat16 &hi, __nv_bfloat16 &lo) {
+  hi = __float2bfloat16_rn(x);
+  lo = __float2bfloat16_rn(x - __bfloat162float(hi));
+}
+__device__ __forceinline__ uint32_t pack2(__nv_bfloat16 a, __nv_bfloat16 b) {
+  return (uint32_t)__bfloat16_as_ushort(a) | ((uint32_t)__bfloat16_as_ushort(b) << 16);
+}
+// Gate nonlinearities from the exponential intrinsic (as in the other
+// recurrent kernels): sigma(x) = 1 / (1 + e^-x), tanh(x) = 2 sigma(2x) - 1.
+__device__ __forceinline__ float sigm_tc(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
+__device__ __forceinline__ float tanh_tc(float x) { return 1.f - __fdividef(2.f, 1.f + __expf(2.f * x)); }
+__device__ __forceinline__ float sel4(float a, float b, float c, float d, int i) {
+  return i == 0 ? a : i == 1 ? b : i == 2 ? c : d;
+}
+
+// Shared-memory layout (bytes).
+template <int N>
+struct TcFwdLayout {
+  static constexpr uint32_t kB = N * kTH * 2;      // one B operand (hi or lo): N rows x 256 bf16
+  static constexpr uint32_t kSlice = 64 * N;       // this CTA's 32 units of one B operand
+  static constexpr uint32_t kStepBytes = kTCS * 2 * kSlice;  // received per step: 8 CTAs x (hi + lo)
+  static constexpr uint32_t oB = 0;                // [2 parity][2 hi/lo][kB]
+  static constexpr uint32_t oStg = oB + 4 * kB;    // [2 parity][2 hi/lo][kSlice]
+  static constexpr uint32_t oBar = oStg + 4 * kSlice;  // hbar[2], mmabar
+  static constexpr uint32_t oSlot = oBar + 3 * 8;
+  static constexpr uint32_t oLen = oSlot + 16;     // [N] row lengths
+  static constexpr uint32_t oToff = oLen + 4 * N;  // [T+1] when it fits
+};
+template <int N>
+struct TcBwdLayout {
+  static constexpr uint32_t kB = N * 128 * 2;      // one B operand (dz hi or lo): N rows x 128 gate rows
+  static constexpr int kRS = kTHc + 8;             // floats per (source, row) of received partials (32 units + pad)
+  static constexpr uint32_t kRed = kTCS * N * kRS * 4;     // received partials per parity
+  static constexpr uint32_t kStepBytes = kTCS * kTHc * N * 4;
+  static constexpr uint32_t oB = 0;                // [2 hi/lo][kB]
+  static constexpr uint32_t oRed = oB + 2 * kB;    // [2 parity][8 src][N rows][kRS] fp32
+  static constexpr uint32_t oStg = oRed + 2 * kRed;  // [8 owners][N rows][32 units] fp32 partials to send
+  static constexpr uint32_t oBar = oStg + kTCS * N * kTHc * 4;  // rbar[2], mmabar
+  static constexpr uint32_t oSlot = oBar + 3 * 8;
+  static constexpr uint32_t oLen = oSlot + 16;
+  static constexpr uint32_t oToff = oLen + 4 * N;
+};
+
+size_t tc_smem_bytes(size_t base, int T) {
+  const size_t need = base + (T + 1 <= kTTokCap ? (size_t)(T + 1) * 4 : 0);
+  return std::max(need, kTSmemFloor);
+}
+
+}  // namespace
+
+// Thread roles (both kernels; QW warps per TMEM lane quarter, 128 QW threads):
+// warp w reads TMEM lane quarter qt = w % 4 and columns C cs .. C cs + C - 1
+// (cs = w / 4, C = N / QW, a multiple of 4) of each accumulator;
+// lane l of it is TMEM lane m = 32 qt + l.  In the forward kernel lane m is
+// gate row q = m % 4 of unit u = m / 4; after the gate swap the thread holds
+// unit u, gates i, f, g, o, for rows C cs + 4 j + q (j < C / 4).  BPTT's
+// phase B uses the same (u, row) pairs; its accumulator lanes are units.
+template <int N, int QW>
+__global__ void __launch_bounds__(128 * QW, 1) lstm_fwd_tc_kernel(RecArgs a) {
+  using Lay = TcFwdLayout<N>;
+  constexpr int H = kTH, G = 4 * H, C = N / QW, NJ = C / 4, kTThreads = 128 * QW;
+  static_assert(C % 4 == 0, "whole 4-row blocks per warp");
+  constexpr uint32_t idesc = tc_idesc<N>();
+  extern __shared__ __align__(16) uint8_t smem[];
+  uint8_t *Bb = smem + Lay::oB;
+  uint8_t *stg = smem + Lay::oStg;
+  uint64_t *bar = reinterpret_cast<uint64_t *>(smem + Lay::oBar);
+  uint32_t *tslot = reinterpret_cast<uint32_t *>(smem + Lay::oSlot);
+  int *rlen = reinterpret_cast<int *>(smem + Lay::oLen);
+  int *toff_s = reinterpret_cast<int *>(smem + Lay::oToff);
+
+  const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+  const int qt = warp & 3, cs = warp >> 2;
+  const int m = 32 * qt + lane, u = m >> 2, q = m & 3;  // TMEM lane m = gate row q H + 32c + u
+  const int col0 = C * cs;                              // this thread's first column (row of the group)
+  const uint32_t c = cluster_rank();
+  const int gu = (int)c * kTHc + u;
+  const int n_groups = (a.ix.b + N - 1) / N;
+  const int cid = blockIdx.x / kTCS;
+  const int d = cid / n_groups, r0 = (cid % n_groups) * N;
+  const int DH = a.dirs * H, T = a.ix.T;
+  const bool toff_sm = T + 1 <= kTTokCap;
+  const int *toff = toff_sm ? toff_s : a.ix.tok_off;
+  const int cap = a.wf.poll_cap > 0 ? a.wf.poll_cap : kTPolls;
+  const bool withhold = (a.wf.withhold & kWithholdExchange) && c == 0;
+
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(tslot)), "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  // zero the B operands (rows past the batch stay zero), stage the index
+  for (uint32_t i = t; i < 4 * Lay::kB / 16; i += kTThreads) reinterpret_cast<uint4 *>(Bb)[i] = make_uint4(0, 0, 0, 0);
+  if (toff_sm)
+    for (int i = t; i <= T; i += kTThreads) toff_s[i] = a.ix.tok_off[i];
+  if (t < N) rlen[t] = r0 + t < a.ix.b ? a.ix.row_len[r0 + t] : 0;
+  if (t == 0) {
+    mb_init(sa(&bar[0]), 1);
+    mb_init(sa(&bar[1]), 1);
+    mb_init(sa(&bar[2]), 3);  // one commit from each of the three MMA issuers
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  fence_proxy();
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = *tslot;
+  const uint32_t tl = tmem + ((uint32_t)(32 * qt) << 16);  // this warp's TMEM lanes
+  // W_hh slice into TMEM (warps of the first column slice): row q H + gu,
+  // split into bf16 hi (columns 0..127) and lo (128..255), two k per column
+  // (low half = even k)
+  if (cs == 0) {
+    const float *wrow = a.Whh[d] + (size_t)(q * H + gu) * H;
+#pragma unroll 1
+    for (int c0 = 0; c0 < 128; c0 += 8) {
+      uint32_t hi[8], lo[8];
+#pragma unroll
+      for (int j = 0; j < 8; j += 2) {
+        const float4 v = __ldg(reinterpret_cast<const float4 *>(wrow + 2 * (c0 + j)));
+        __nv_bfloat16 h0, l0, h1, l1, h2, l2, h3, l3;
+        split_bf16(v.x, h0, l0);
+        split_bf16(v.y, h1, l1);
+        split_bf16(v.z, h2, l2);
+        split_bf16(v.w, h3, l3);
+        hi[j] = pack2(h0, h1);
+        lo[j] = pack2(l0, l1);
+        hi[j + 1] = pack2(h2, h3);
+        lo[j + 1] = pack2(l2, l3);
+      }
+      tmem_st8(tl + c0, hi);
+      tmem_st8(tl + 128 + c0, lo);
+    }
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+  }
+  fence_before();  // the slice is in TMEM before the issuers' MMAs read it
+  __syncthreads();
+  const int Tg = rlen[0];
+  cluster_sync_all();  // barriers and buffers ready everywhere before any remote store
+  if (t == 0) {
+    if (Tg >= 2) mb_arm(sa(&bar[0]), Lay::kStepBytes);
+    if (Tg >= 3) mb_arm(sa(&bar[1]), Lay::kStepBytes);
+  }
+
+  float *__restrict__ Z = a.Z[d];
+  float *__restrict__ Cs = a.Cst[d];
+  float *__restrict__ Y = a.Y;
+  int len[C], lenq[NJ];  // lengths of this thread's columns; of its rows col0 + 4 j + q
+#pragma unroll
+  for (int k = 0; k < C; ++k) len[k] = rlen[col0 + k];
+#pragma unroll
+  for (int j = 0; j < NJ; ++j) lenq[j] = rlen[col0 + 4 * j + q];
+  auto tok_col = [&](int k, int s) { return toff[d == 0 ? s : len[k] - 1 - s] + r0 + col0 + k; };
+  auto tok_q = [&](int j, int s) { return toff[d == 0 ? s : lenq[j] - 1 - s] + r0 + col0 + 4 * j + q; };
+  float zn[C];
+#pragma unroll
+  for (int k = 0; k < C; ++k) zn[k] = 0 < len[k] ? Z[(size_t)tok_col(k, 0) * G + q * H + gu] : 0.f;
+  float cst[NJ];
+#pragma unroll
+  for (int j = 0; j < NJ; ++j) cst[j] = 0.f;
+  const float scale = q == 2 ? 2.f : 1.f;  // tanh(x) = 2 sigma(2x) - 1 for the g gate
+  // MMA issuers: lane 0 of warps 0, 1, 2 issue the products W_hi h_hi,
+  // W_hi h_lo and W_lo h_hi into their own accumulators (columns kAccCol +
+  // 32 p), which the epilogue adds
+  const int prod = (lane == 0 && warp < 3) ? warp : -1;
+  bool ok = true, stop = false;
+  int mma_issued = 0, mma_seen = 0;
+
+  for (int s = 0; s < Tg && !stop; ++s) {
+    float acc[C];
+#pragma unroll
+    for (int k = 0; k < C; ++k) acc[k] = zn[k];
+    if (s + 1 < Tg) {
+#pragma unroll
+      for (int k = 0; k < C; ++k) zn[k] = s + 1 < len[k] ? Z[(size_t)tok_col(k, s + 1) * G + q * H + gu] : 0.f;
+    }
+    if (s > 0) {
+      const int e = s - 1;
+      ok = mb_wait(sa(&bar[e & 1]), (e >> 1) & 1, cap) && ok;
+      if (t == 0 && ok && e + 2 <= Tg - 2) mb_arm(sa(&bar[e & 1]), Lay::kStepBytes);
+      if (prod >= 0) {
+        if (ok) {
+          fence_proxy();
+          fence_after();
+          const uint32_t bh = sa(Bb + (2 * (e & 1)) * Lay::kB);
+          const uint32_t bsel = bh + (prod == 1 ? Lay::kB : 0u);   // h_lo for W_hi h_lo
+          const uint32_t asel = tmem + (prod == 2 ? 128u : 0u);    // W_lo for W_lo h_hi
+          const uint32_t dcol = tmem + kAccCol + 32u * (uint32_t)prod;
+#pragma unroll
+          for (int j = 0; j < H / 16; ++j)  // k-step j: K columns 16 j .. 16 j + 15 (8 TMEM columns)
+            mma_ts(dcol, asel + 8 * j, desc_kmajor(bsel + (uint32_t)(2 * j) * (16u * N), 16 * N, 128), idesc, j > 0);
+          mma_commit(sa(&bar[2]));
+        } else {
+          mb_arrive(sa(&bar[2]));
+        }
+      }
+      ++mma_issued;
+      const bool got = mb_wait(sa(&bar[2]), (uint32_t)(e & 1), cap);
+      if (got) ++mma_seen;
+      ok = got && ok;
+      fence_after();
+#pragma unroll
+      for (int p = 0; p < 3; ++p) tmem_ld_add<C>(tl + kAccCol + 32 * p + col0, acc);
+    }
+    // this lane's gate for each of its columns, written where the row is still running
+    float act[C];
+#pragma unroll
+    for (int k = 0; k < C; ++k) {
+      const float sg = sigm_tc(scale * acc[k]);
+      act[k] = fmaf(scale, sg, 1.f - scale);
+      if (s < len[k]) Z[(size_t)tok_col(k, s) * G + q * H + gu] = act[k];
+    }
+    // four lanes of a unit swap gates: lane q ends with gates i, f, g, o of
+    // rows col0 + 4 j + q (round r: send the gate value of row 4 j + (q ^ r),
+    // receive gate q ^ r of row 4 j + q from lane q ^ r)
+    const uint32_t par = (uint32_t)(s & 1);
+    uint8_t *sg_hi = stg + (2 * par) * Lay::kSlice, *sg_lo = sg_hi + Lay::kSlice;
+#pragma unroll
+    for (int j = 0; j < NJ; ++j) {
+      float g4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        const int qs = q ^ r;
+        const float send = sel4(act[4 * j], act[4 * j + 1], act[4 * j + 2], act[4 * j + 3], qs);
+        const float recv = r == 0 ? send : __shfl_xor_sync(0xffffffffu, send, r);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) g4[k] = (k == qs) ? recv : g4[k];
+      }
+      const int n = col0 + 4 * j + q;
+      const float cn = fmaf(g4[1], cst[j], g4[0] * g4[2]);
+      float h = g4[3] * tanh_tc(cn);
+      if (s < lenq[j]) {
+        cst[j] = cn;
+        const size_t tk = (size_t)tok_q(j, s);
+        Cs[tk * H + gu] = cn;
+        Y[tk * DH + d * H + gu] = h;
+      } else {
+        h = 0.f;
+      }
+      __nv_bfloat16 hh, hl;
+      split_bf16(h, hh, hl);
+      const uint32_t off = (uint32_t)(u >> 3) * (16u * N) + (uint32_t)n * 16u + (uint32_t)(u & 7) * 2u;
+      *reinterpret_cast<__nv_bfloat16 *>(sg_hi + off) = hh;
+      *reinterpret_cast<__nv_bfloat16 *>(sg_lo + off) = hl;
+    }
+    fence_before();
+    if (__syncthreads_or(!ok)) {
+      if (t == 0) atomicOr(a.status, kErrExchWait);
+      stop = true;
+      break;
+    }
+    if (s + 1 < Tg && !withhold) {
+      // h_t of this CTA's units to every CTA of the cluster (itself included)
+      constexpr int kPieces = 2 * Lay::kSlice / 16;  // per destination
+      const uint32_t dst0 = sa(Bb + (2 * par) * Lay::kB) + c * (uint32_t)Lay::kSlice;
+      const uint32_t mbl = sa(&bar[par]);
+#pragma unroll
+      for (int i = t; i < kTCS * kPieces; i += kTThreads) {
+        const int pr = i / kPieces, rem = i % kPieces, hl = rem / (kPieces / 2), o = (rem % (kPieces / 2)) * 16;
+        const uint4 v = *reinterpret_cast<const uint4 *>(stg + (2 * par + hl) * Lay::kSlice + o);
+        st_async16(peer(dst0 + (uint32_t)hl * Lay::kB + (uint32_t)o, (uint32_t)pr), v, peer(mbl, (uint32_t)pr));
+      }
+    }
+  }
+  // an MMA batch whose completion was not observed may still be running:
+  // wait for it (bounded) before TMEM is released
+  if (mma_seen < mma_issued) mb_wait(sa(&bar[2]), (uint32_t)((mma_issued - 1) & 1), kTPolls);
+  if (stop) __nanosleep(20000);  // peers' in-flight stores after an abort
+  fence_before();
+  cluster_sync_all();
+  fence_after();
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+}
+
+template <int N, int QW>
+__global__ void __launch_bounds__(128 * QW, 1) lstm_bwd_tc_kernel(RecArgs a) {
+  using Lay = TcBwdLayout<N>;
+  constexpr int H = kTH, G = 4 * H, C = N / QW, NJ = C / 4, RS = Lay::kRS, kTThreads = 128 * QW;
+  static_assert(C % 4 == 0, "whole 4-row blocks per warp");
+  constexpr uint32_t idesc = tc_idesc<N>();
+  extern __shared__ __align__(16) uint8_t smem[];
+  uint8_t *Bz = smem + Lay::oB;
+  float *red = reinterpret_cast<float *>(smem + Lay::oRed);
+  float *pst = reinterpret_cast<float *>(smem + Lay::oStg);
+  uint64_t *bar = reinterpret_cast<uint64_t *>(smem + Lay::oBar);
+  uint32_t *tslot = reinterpret_cast<uint32_t *>(smem + Lay::oSlot);
+  int *rlen = reinterpret_cast<int *>(smem + Lay::oLen);
+  int *toff_s = reinterpret_cast<int *>(smem + Lay::oToff);
+
+  const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+  const int qt = warp & 3, cs = warp >> 2;
+  const int m = 32 * qt + lane, u = m >> 2, q = m & 3;  // phase B: unit u, rows col0 + 4 j + q
+  const int col0 = C * cs;
+  const uint32_t c = cluster_rank();
+  const int gu = (int)c * kTHc + u;
+  const int n_groups = (a.ix.b + N - 1) / N;
+  const int cid = blockIdx.x / kTCS;
+  const int d = cid / n_groups, r0 = (cid % n_groups) * N;
+  const int DH = a.dirs * H, T = a.ix.T;
+  const bool toff_sm = T + 1 <= kTTokCap;
+  const int *toff = toff_sm ? toff_s : a.ix.tok_off;
+  const int cap = a.wf.poll_cap > 0 ? a.wf.poll_cap : kTPolls;
+  const bool withhold = (a.wf.withhold & kWithholdExchange) && c == 0;
+
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(tslot)), "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  for (uint32_t i = t; i < 2 * Lay::kB / 16; i += kTThreads) reinterpret_cast<uint4 *>(Bz)[i] = make_uint4(0, 0, 0, 0);
+  if (toff_sm)
+    for (int i = t; i <= T; i += kTThreads) toff_s[i] = a.ix.tok_off[i];
+  if (t < N) rlen[t] = r0 + t < a.ix.b ? a.ix.row_len[r0 + t] : 0;
+  if (t == 0) {
+    mb_init(sa(&bar[0]), 1);
+    mb_init(sa(&bar[1]), 1);
+    mb_init(sa(&bar[2]), 6);  // one commit from each of the six MMA issuers
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = *tslot;
+  const uint32_t tl = tmem + ((uint32_t)(32 * qt) << 16);
+  // W_hh^T into TMEM: half hf = 0, 1 (warps of column slices 0, 1) holds
+  // units 128 hf + m in lane m; K = the CTA's gate rows k = 4 uu + qq (global
+  // row qq H + 32c + uu); hi part in columns 128 hf .. + 63, lo part 64 after
+  if (cs < 2) {
+    const int hf = cs;
+    const float *W = a.Whh[d];
+    const int col = 128 * hf + m;
+#pragma unroll 1
+    for (int k0 = 0; k0 < 128; k0 += 16) {
+      uint32_t hi[8], lo[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int k = k0 + 2 * j;
+        const float w0 = __ldg(W + (size_t)((k & 3) * H + (int)c * kTHc + (k >> 2)) * H + col);
+        const float w1 = __ldg(W + (size_t)(((k + 1) & 3) * H + (int)c * kTHc + ((k + 1) >> 2)) * H + col);
+        __nv_bfloat16 h0, l0, h1, l1;
+        split_bf16(w0, h0, l0);
+        split_bf16(w1, h1, l1);
+        hi[j] = pack2(h0, h1);
+        lo[j] = pack2(l0, l1);
+      }
+      tmem_st8(tl + 128 * hf + k0 / 2, hi);
+      tmem_st8(tl + 128 * hf + 64 + k0 / 2, lo);
+    }
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+  }
+  fence_before();
+  __syncthreads();
+  const int Tg = rlen[0];
+  cluster_sync_all();
+  if (t == 0) {
+    if (Tg >= 2) mb_arm(sa(&bar[0]), Lay::kStepBytes);
+    if (Tg >= 3) mb_arm(sa(&bar[1]), Lay::kStepBytes);
+  }
+
+  float *__restrict__ Z = a.Z[d];
+  const float *__restrict__ Cs = a.Cst[d];
+  const float *__restrict__ dY = a.dY;
+  int len[NJ];  // lengths of this thread's rows col0 + 4 j + q
+#pragma unroll
+  for (int j = 0; j < NJ; ++j) len[j] = rlen[col0 + 4 * j + q];
+  auto tok_at = [&](int j, int s) { return toff[d == 0 ? s : len[j] - 1 - s] + r0 + col0 + 4 * j + q; };
+  // phase B inputs of a step, loaded one step ahead: gates i, f, g, o, c_t,
+  // c_{t-1} (in this direction's order), dY
+  float in[NJ][7], nx[NJ][7];
+  auto load_in = [&](int s, float (&v)[NJ][7]) {
+#pragma unroll
+    for (int j = 0; j < NJ; ++j) {
+      if (s >= 0 && s < len[j]) {
+        const size_t tk = (size_t)tok_at(j, s);
+#pragma unroll
+        for (int g = 0; g < 4; ++g) v[j][g] = Z[tk * G + g * H + gu];
+        v[j][4] = Cs[tk * H + gu];
+        v[j][5] = s > 0 ? Cs[(size_t)tok_at(j, s - 1) * H + gu] : 0.f;
+        v[j][6] = dY[tk * DH + d * H + gu];
+      } else {
+#pragma unroll
+        for (int g = 0; g < 7; ++g) v[j][g] = 0.f;
+      }
+    }
+  };
+  load_in(Tg - 1, nx);
+  float dc[NJ];
+#pragma unroll
+  for (int j = 0; j < NJ; ++j) dc[j] = 0.f;
+  // MMA issuers: lane 0 of warps 0..5, issuer i forms product i % 3 (W_hi dz_hi,
+  // W_hi dz_lo, W_lo dz_hi) of half i / 3 into columns kAccCol + 32 i
+  const int iss = (lane == 0 && warp < 6) ? warp : -1;
+  bool ok = true, stop = false;
+  int mma_issued = 0, mma_seen = 0;
+  const uint32_t bh = sa(Bz);
+
+  for (int it = 0; it < Tg && !stop; ++it) {
+    const int s = Tg - 1 - it;
+#pragma unroll
+    for (int j = 0; j < NJ; ++j)
+#pragma unroll
+      for (int g = 0; g < 7; ++g) in[j][g] = nx[j][g];
+    load_in(s - 1, nx);
+    const float *rp = nullptr;
+    if (it > 0) {
+      const int e = it - 1;
+      ok = mb_wait(sa(&bar[e & 1]), (e >> 1) & 1, cap) && ok;
+      if (t == 0 && ok && e + 2 <= Tg - 2) mb_arm(sa(&bar[e & 1]), Lay::kStepBytes);
+      rp = red + (size_t)(e & 1) * (kTCS * N * RS) + u;
+    }
+    // phase B: dh, dc and dz of unit u for rows col0 + 4 j + q
+#pragma unroll
+    for (int j = 0; j < NJ; ++j) {
+      const int n = col0 + 4 * j + q;
+      float dz4[4] = {0.f, 0.f, 0.f, 0.f};
+      if (s < len[j]) {
+        float dh = in[j][6];
+        if (rp) {
+#pragma unroll
+          for (int src = 0; src < kTCS; ++src) dh += rp[((size_t)src * N + n) * RS];
+        }
+        const float ig = in[j][0], fg = in[j][1], gg = in[j][2], og = in[j][3], ct = in[j][4], cp = in[j][5];
+        const float tch = tanh_tc(ct);
+        const float dcv = fmaf(dh * og, 1.f - tch * tch, dc[j]);
+        dz4[0] = dcv * gg * ig * (1.f - ig);
+        dz4[1] = dcv * cp * fg * (1.f - fg);
+        dz4[2] = dcv * ig * (1.f - gg * gg);
+        dz4[3] = dh * tch * og * (1.f - og);
+        dc[j] = dcv * fg;
+        float *zr = Z + (size_t)tok_at(j, s) * G + gu;
+        zr[0] = dz4[0];
+        zr[H] = dz4[1];
+        zr[2 * H] = dz4[2];
+        zr[3 * H] = dz4[3];
+      } else {
+        dc[j] = 0.f;
+      }
+      // B operand: k = 4u .. 4u + 3 of row n (8 bytes of each part)
+      __nv_bfloat16 h0, l0, h1, l1, h2, l2, h3, l3;
+      split_bf16(dz4[0], h0, l0);
+      split_bf16(dz4[1], h1, l1);
+      split_bf16(dz4[2], h2, l2);
+      split_bf16(dz4[3], h3, l3);
+      const uint32_t off = (uint32_t)(u >> 1) * (16u * N) + (uint32_t)n * 16u + (uint32_t)(u & 1) * 8u;
+      *reinterpret_cast<uint2 *>(Bz + off) = make_uint2(pack2(h0, h1), pack2(h2, h3));
+      *reinterpret_cast<uint2 *>(Bz + Lay::kB + off) = make_uint2(pack2(l0, l1), pack2(l2, l3));
+    }
+    fence_proxy();
+    fence_before();
+    if (__syncthreads_or(!ok)) {
+      if (t == 0) atomicOr(a.status, kErrExchWait);
+      stop = true;
+      break;
+    }
+    fence_after();
+    if (it + 1 >= Tg) continue;  // dh_{-1} is not needed
+    // this CTA's partial W_hh^T dz for all 256 units (two halves of 128 lanes)
+    if (iss >= 0) {
+      const int hf = iss / 3, p = iss % 3;
+      const uint32_t dcol = tmem + kAccCol + 32u * (uint32_t)iss;
+      const uint32_t asel = tmem + 128u * (uint32_t)hf + (p == 2 ? 64u : 0u);
+      const uint32_t bsel = bh + (p == 1 ? Lay::kB : 0u);
+#pragma unroll
+      for (int j = 0; j < 128 / 16; ++j)
+        mma_ts(dcol, asel + 8 * j, desc_kmajor(bsel + (uint32_t)(2 * j) * (16u * N), 16 * N, 128), idesc, j > 0);
+      mma_commit(sa(&bar[2]));
+    }
+    ++mma_issued;
+    const bool got = mb_wait(sa(&bar[2]), (uint32_t)((mma_issued - 1) & 1), cap);
+    if (got) ++mma_seen;
+    ok = got && ok;
+    fence_after();
+    float p0[C], p1[C];
+#pragma unroll
+    for (int k = 0; k < C; ++k) p0[k] = p1[k] = 0.f;
+#pragma unroll
+    for (int p = 0; p < 3; ++p) {
+      tmem_ld_add<C>(tl + kAccCol + 32 * p + col0, p0);
+      tmem_ld_add<C>(tl + kAccCol + 32 * (3 + p) + col0, p1);
+    }
+    // stage the partials by owner (unit 32 qt + lane of half hf belongs to
+    // CTA qt + 4 hf), rows contiguous, so that the sends below are whole
+    // 16-byte pieces of consecutive memory on both sides
+#pragma unroll
+    for (int k = 0; k < C; ++k) {
+      pst[((qt)*N + col0 + k) * kTHc + lane] = p0[k];
+      pst[((qt + 4) * N + col0 + k) * kTHc + lane] = p1[k];
+    }
+    __syncthreads();
+    if (!withhold && got) {
+      const uint32_t par = (uint32_t)(it & 1);
+      const uint32_t mbl = sa(&bar[par]);
+      constexpr int kPer = N * kTHc / 4;  // 16-byte pieces per owner
+#pragma unroll
+      for (int i = t; i < kTCS * kPer; i += kTThreads) {
+        const int owner = i / kPer, rem = i % kPer, n = rem / (kTHc / 4), ch = rem % (kTHc / 4);
+        const uint4 v = *reinterpret_cast<const uint4 *>(pst + (owner * N + n) * kTHc + 4 * ch);
+        const uint32_t dst = sa(red) + (((par * kTCS + c) * N + n) * RS + 4 * ch) * 4u;
+        st_async16(peer(dst, (uint32_t)owner), v, peer(mbl, (uint32_t)owner));
+      }
+    }
+    fence_before();  // the accumulators are read before the next step's MMAs overwrite them
+  }
+  if (mma_seen < mma_issued) mb_wait(sa(&bar[2]), (uint32_t)((mma_issued - 1) & 1), kTPolls);
+  if (stop) __nanosleep(20000);
+  fence_before();
+  cluster_sync_all();
+  fence_after();
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+}
+
+// ---------------------------------------------------------------------------
+namespace {
+
+template <typename K>
+cudaLaunchConfig_t tc_config(int clusters, int threads, size_t smem, cudaStream_t s, cudaLaunchAttribute *attr) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(clusters * kTCS, 1, 1);
+  cfg.blockDim = dim3(threads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  attr->id = cudaLaunchAttributeClusterDimension;
+  attr->val.clusterDim.x = kTCS;
+  attr->val.clusterDim.y = 1;
+  attr->val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cfg;
+}
+
+template <int N>
+size_t tc_smem(bool bwd, int T) {
+  return tc_smem_bytes(bwd ? TcBwdLayout<N>::oToff : TcFwdLayout<N>::oToff, T);
+}
+
+template <int N, int QW>
+cudaError_t launch_tc(const RecArgs &a, bool bwd, cudaStream_t s) {
+  if (a.ix.b <= 0 || a.ix.T <= 0) return cudaSuccess;
+  if (a.H != kTH) return cudaErrorInvalidValue;
+  const size_t smem = tc_smem<N>(bwd, a.ix.T);
+  const int clusters = ((a.ix.b + N - 1) / N) * a.dirs;
+  cudaLaunchAttribute attr;
+  if (bwd) {
+    auto k = lstm_bwd_tc_kernel<N, QW>;
+    cudaError_t e = ensure_smem((const void *)k, smem);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg = tc_config<decltype(k)>(clusters, 128 * QW, smem, s, &attr);
+    return cudaLaunchKernelEx(&cfg, k, a);
+  }
+  auto k = lstm_fwd_tc_kernel<N, QW>;
+  cudaError_t e = ensure_smem((const void *)k, smem);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = tc_config<decltype(k)>(clusters, 128 * QW, smem, s, &attr);
+  return cudaLaunchKernelEx(&cfg, k, a);
+}
+
+// 8-CTA clusters of both kernels that can be resident at once (0: cannot launch).
+template <int N, int QW>
+int tc_resident() {
+  int lo = 1 << 30;
+  for (int bwd = 0; bwd < 2; ++bwd) {
+    const size_t smem = tc_smem<N>(bwd != 0, kTTokCap - 1);
+    cudaLaunchAttribute attr;
+    int n = 0;
+    cudaError_t e;
+    if (bwd) {
+      auto k = lstm_bwd_tc_kernel<N, QW>;
+      e = ensure_smem((const void *)k, smem);
+      cudaLaunchConfig_t cfg = tc_config<decltype(k)>(1, 128 * QW, smem, 0, &attr);
+      if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, k, &cfg);
+    } else {
+      auto k = lstm_fwd_tc_kernel<N, QW>;
+      e = ensure_smem((const void *)k, smem);
+      cudaLaunchConfig_t cfg = tc_config<decltype(k)>(1, 128 * QW, smem, 0, &attr);
+      if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, k, &cfg);
+    }
+    if (e != cudaSuccess) {
+      cudaGetLastError();
+      return 0;
+    }
+    lo = std::min(lo, n);
+  }
+  return lo;
+}
+
+// Warps per TMEM lane quarter at 32 rows per cluster: 4 (512 threads; BKT_TC_QW=8
+// selects 1024 threads, measured no faster: the step is bound by the SM's
+// elementwise and exchange throughput, not by latency within a warp).
+int tc_qw32() {
+  static const int qw = [] {
+    const char *e = getenv("BKT_TC_QW");
+    return (e && atoi(e) == 8) ? 8 : 4;
+  }();
+  return qw;
+}
+
+}  // namespace
+
+bool tc_rec_supported(int H) {
+  static const bool off = [] {
+    const char *e = getenv("BKT_REC_TC");
+    return e && e[0] == '0';
+  }();
+  return H == kTH && !off;
+}
+
+int plan_tc_rows(int b, int dirs) {
+  // 32 rows per cluster: an MMA costs the same at N = 16 and 32 (its issue,
+  // not its columns, bounds it), so fewer, wider clusters leave SMs to the
+  // side stream; 16 when the batch is small enough for its clusters to fit
+  // either way (0: neither can launch)
+  const int r16 = tc_resident<16, 4>(), r32 = tc_qw32() == 8 ? tc_resident<32, 8>() : tc_resident<32, 4>();
+  if (r16 > 0 && ((b + 15) / 16) * dirs <= std::min(r16, 4)) return 16;
+  if (r32 > 0) return 32;
+  return r16 > 0 ? 16 : 0;
+}
+
+cudaError_t launch_lstm_tc(const RecArgs &a, int rows, bool bwd, cudaStream_t s) {
+  if (rows == 16) return launch_tc<16, 4>(a, bwd, s);
+  if (rows == 32) return tc_qw32() == 8 ? launch_tc<32, 8>(a, bwd, s) : launch_tc<32, 4>(a, bwd, s);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace bkt

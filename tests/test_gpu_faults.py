@@ -46,14 +46,17 @@ def expect_timeout_then_recover(cfg, ds, params, ctx, withhold, tol):
     compare(cfg, lg, gg, lo, go, tol)
 
 
-@pytest.mark.parametrize("H,bi", [(256, True), (512, False)])
-def test_cluster_exchange_wait_runs_out(H, bi):
+@pytest.mark.parametrize("H,bi,bf16", [(256, True, False), (512, False, False), (256, True, True)])
+def test_cluster_exchange_wait_runs_out(H, bi, bf16):
     """CTA 0 of every recurrent cluster withholds its h / partial sums: its
     peers' bounded mbarrier waits expire, the kernels leave their loops and
-    report bit 4; the forward kernel and BPTT both take that path."""
-    cfg = {"n_layers": 1, "bidirectional": bi, "in_dim": 4, "hidden": H, "n_classes": 81, "blank": 0}
+    report bit 4; the forward kernel and BPTT both take that path (the
+    register-tiled fp32 kernels at H = 256 and 512, the tensor-core kernels
+    of the bf16 configuration at H = 256)."""
+    cfg = {"n_layers": 1, "bidirectional": bi, "in_dim": 4, "hidden": H, "n_classes": 81, "blank": 0,
+           "gemm_bf16": bf16}
     ds, params, ctx = small_case(cfg, [14, 11, 9, 5, 2], seed=H)
-    expect_timeout_then_recover(cfg, ds, params, ctx, binding.BKT_WITHHOLD_EXCHANGE, FP32_TOL)
+    expect_timeout_then_recover(cfg, ds, params, ctx, binding.BKT_WITHHOLD_EXCHANGE, BF16_TOL if bf16 else FP32_TOL)
     ctx.close()
 
 
