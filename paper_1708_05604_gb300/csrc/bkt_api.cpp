@@ -472,19 +472,21 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
         return bkt::launch_proj_narrow(w.X, NT, lo.D0, params, lo.w_ih[0], lo.stride(0), H, dirs, Zl, s);
       });
     } else if (bf16) {
-      // a5 on the tensor cores: Zx = bf16(Y_{l-1}) bf16(W_ih)^T + b, fp32 accumulation
-      L.run("cast_bf16", pass_w(NT, DH, 4, 2), [&] { return bkt::launch_cast_bf16(w.Y[l - 1], DH, NT, DH, w.Yb, DH, s); });
+      // a5 on the tensor cores: Zx = bf16(Y_{l-1}) bf16(W_ih)^T + b, fp32
+      // accumulation; bf16(Y_{l-1}) was written by layer l-1's recurrent
+      // kernel (or cast after it); bf16(W_ih) is kept for dX
       for (int d = 0; d < dirs; ++d) {
+        void *Wb = w.Wb[l * dirs + d];
         L.run("cast_bf16", pass_w(4.0 * H, DH, 4, 2), [&] {
-          return bkt::launch_cast_bf16(params + lo.w_ih[l * dirs + d], DH, 4 * H, DH, w.Wb, DH, s);
+          return bkt::launch_cast_bf16(params + lo.w_ih[l * dirs + d], DH, 4 * H, DH, Wb, DH, s);
         });
         bkt::TcGemmArgs g{};
         g.M = NT;
         g.N = 4 * H;
         g.K = DH;
-        g.A = w.Yb;
+        g.A = w.Yb[l - 1];
         g.lda = DH;
-        g.B = w.Wb;
+        g.B = Wb;
         g.ldb = DH;
         g.D = Zl[d];
         g.ldd = 4 * H;
@@ -531,7 +533,13 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     ra.Y = w.Y[l];
     ra.status = w.status;
     ra.wf = wf;
+    if (bf16) {  // the bf16 copies the contractions read (written by the kernel when it can)
+      ra.Yb = l + 1 < lo.L ? w.Yb[l] : nullptr;
+      for (int d = 0; d < dirs; ++d) ra.Hs[d] = w.Hs[l * dirs + d];
+    }
     L.run("lstm_fwd", flops_w(8.0 * H * H * (double)NT * dirs, ix.T), [&] { return bkt::launch_lstm_fwd(ra, geom[l], s); });
+    if (bf16 && l + 1 < lo.L && !bkt::rec_writes_bf16(geom[l]))
+      L.run("cast_bf16", pass_w(NT, DH, 4, 2), [&] { return bkt::launch_cast_bf16(w.Y[l], DH, NT, DH, w.Yb[l], DH, s); });
   }
 
   // ---- a7: output layer and log-softmax
@@ -688,7 +696,15 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     ra.status = w.status;
     ra.dY = w.dY;
     ra.wf = wf;
+    const bool fused_bf16 = bkt::rec_writes_bf16(geom[l]);
+    if (bf16)
+      for (int d = 0; d < dirs; ++d) ra.dZb[d] = w.dZb[l * dirs + d];
     L.run("lstm_bwd", flops_w(8.0 * H * H * (double)NT * dirs, ix.T), [&] { return bkt::launch_lstm_bwd(ra, geom[l], s); });
+    if (bf16 && !fused_bf16)
+      for (int d = 0; d < dirs; ++d)
+        L.run("cast_bf16", pass_w(NT, 4.0 * H, 4, 2), [&] {
+          return bkt::launch_cast_bf16(w.Z[l * dirs + d], 4 * H, NT, 4 * H, w.dZb[l * dirs + d], 4 * H, s);
+        });
     if (int rc = fork_to_side()) return rc;
     Launch &X = Ls;  // the weight gradients of layer l
     const int D = lo.D(l);
@@ -705,16 +721,19 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
       });
     };
     if (bf16) {
-      const int NTp = (NT + 7) & ~7;
-      auto tc_reduce = [&](const void *B, int N, float *out) {
+      // token-axis contractions on the tensor cores, reading the token-major
+      // bf16 copies as MN-major tiles (no transposes): A = dz [NT x 4H]
+      auto tc_reduce = [&](const void *A, const void *B, int N, float *out) {
         bkt::TcGemmArgs g{};
         g.M = 4 * H;
         g.N = N;
         g.K = NT;
-        g.A = w.dZT;
-        g.lda = NTp;
+        g.A = A;
+        g.lda = 4 * H;
+        g.a_mn = 1;
         g.B = B;
-        g.ldb = NTp;
+        g.ldb = N;
+        g.b_mn = 1;
         g.P = w.part;
         g.splits = bkt::tc_splits(g.M, g.N, NT, sm_count, w.part_floats);
         g.err = w.status;
@@ -725,20 +744,19 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
       };
       for (int d = 0; d < dirs; ++d) {
         const float *dZ = w.Z[l * dirs + d];
-        // dW_hh = dz^T h_{t-1} on the tensor cores (both operands transposed to bf16)
-        X.run("transpose_bf16", pass_w(NT, 4.0 * H, 4, 2),
-              [&] { return bkt::launch_transpose_bf16(dZ, 4 * H, nullptr, NT, 4 * H, w.dZT, NTp, X.s); });
-        X.run("transpose_bf16", pass_w(NT, H, 4, 2), [&] {
-          return bkt::launch_transpose_bf16(w.Y[l] + d * H, DH, w.prev_tok[d], NT, H, w.BT, NTp, X.s);
-        });
-        tc_reduce(w.BT, H, grads + lo.w_hh(l, d));
+        void *dZb = w.dZb[l * dirs + d], *Hs = w.Hs[l * dirs + d];
+        // dW_hh = dz^T h_{t-1} (bf16 h_{t-1}: from the recurrent kernel, or
+        // gathered here through the previous-token index)
+        if (!fused_bf16)
+          X.run("cast_bf16", pass_w(NT, H, 4, 2), [&] {
+            return bkt::launch_gather_cast_bf16(w.Y[l] + d * H, DH, w.prev_tok[d], NT, H, Hs, H, X.s);
+          });
+        tc_reduce(dZb, Hs, H, grads + lo.w_hh(l, d));
         if (l == 0) {
           // narrow input: [dW_ih | db] = dz^T [X | 1] in fp32
           narrow_on(dZ, grads + lo.w_ih[l * dirs + d], grads + lo.bias(l, d));
         } else {
-          X.run("transpose_bf16", pass_w(NT, D, 4, 2),
-                [&] { return bkt::launch_transpose_bf16(Xl, D, nullptr, NT, D, w.BT, NTp, X.s); });
-          tc_reduce(w.BT, D, grads + lo.w_ih[l * dirs + d]);
+          tc_reduce(dZb, w.Yb[l - 1], D, grads + lo.w_ih[l * dirs + d]);
           bias_sum_on(X, dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
         }
       }
@@ -759,20 +777,17 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     }
     if (l > 0 && bf16) {
       // dX = dz W_ih on the tensor cores, both directions accumulated into dY
+      // (bf16 W_ih as cast for the projection, read MN-major)
       for (int d = 0; d < dirs; ++d) {
-        L.run("cast_bf16", pass_w(NT, 4.0 * H, 4, 2),
-              [&] { return bkt::launch_cast_bf16(w.Z[l * dirs + d], 4 * H, NT, 4 * H, w.dZb, 4 * H, s); });
-        L.run("transpose_bf16", pass_w(4.0 * H, DH, 4, 2), [&] {
-          return bkt::launch_transpose_bf16(params + lo.w_ih[l * dirs + d], DH, nullptr, 4 * H, DH, w.WTb, 4 * H, s);
-        });
         bkt::TcGemmArgs g{};
         g.M = NT;
         g.N = DH;
         g.K = 4 * H;
-        g.A = w.dZb;
+        g.A = w.dZb[l * dirs + d];
         g.lda = 4 * H;
-        g.B = w.WTb;
-        g.ldb = 4 * H;
+        g.B = w.Wb[l * dirs + d];
+        g.ldb = DH;
+        g.b_mn = 1;
         g.D = w.dY;
         g.ldd = DH;
         g.accumulate = d > 0;
@@ -1032,20 +1047,23 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
     BKT_ALLOC(w.part2, w.part2_floats);
   }
   if (cfg->gemm_precision == BKT_GEMM_BF16) {
-    const size_t NTp = (NT + 7) & ~size_t(7);
     uint16_t *p = nullptr;
-    BKT_ALLOC(p, NT * DH);
-    w.Yb = p;
-    BKT_ALLOC(p, NT * 4 * H);
-    w.dZb = p;
-    BKT_ALLOC(p, 4 * H * NTp);
-    w.dZT = p;
-    BKT_ALLOC(p, DH * NTp);
-    w.BT = p;
-    BKT_ALLOC(p, 4 * H * DH);
-    w.Wb = p;
-    BKT_ALLOC(p, DH * 4 * H);
-    w.WTb = p;
+    for (int l = 0; l < lo.L; ++l) {
+      if (l + 1 < lo.L) {
+        BKT_ALLOC(p, NT * DH);
+        w.Yb[l] = p;
+      }
+      for (int d = 0; d < lo.dirs; ++d) {
+        BKT_ALLOC(p, NT * H);
+        w.Hs[l * lo.dirs + d] = p;
+        BKT_ALLOC(p, NT * 4 * H);
+        w.dZb[l * lo.dirs + d] = p;
+        if (l > 0) {
+          BKT_ALLOC(p, 4 * H * DH);
+          w.Wb[l * lo.dirs + d] = p;
+        }
+      }
+    }
   }
   IdxLayout il = idx_layout(max_batch, max_tokens);
   c->idx_bytes = il.bytes;
@@ -1332,13 +1350,14 @@ int bkt::step_on_scratch(const bkt_model_cfg *cfg, const bkt_batch *bt, const fl
     w.WoTl = cv.take<float>((size_t)DH * Cp);
   }
   if (cfg->gemm_precision == BKT_GEMM_BF16) {
-    const size_t NTp = (NT + 7) & ~size_t(7);
-    w.Yb = cv.take<uint16_t>(NT * DH);
-    w.dZb = cv.take<uint16_t>(NT * 4 * H);
-    w.dZT = cv.take<uint16_t>(4 * H * NTp);
-    w.BT = cv.take<uint16_t>(DH * NTp);
-    w.Wb = cv.take<uint16_t>(4 * H * DH);
-    w.WTb = cv.take<uint16_t>(DH * 4 * H);
+    for (int l = 0; l < lo.L; ++l) {
+      if (l + 1 < lo.L) w.Yb[l] = cv.take<uint16_t>(NT * DH);
+      for (int d = 0; d < lo.dirs; ++d) {
+        w.Hs[l * lo.dirs + d] = cv.take<uint16_t>(NT * H);
+        w.dZb[l * lo.dirs + d] = cv.take<uint16_t>(NT * 4 * H);
+        if (l > 0) w.Wb[l * lo.dirs + d] = cv.take<uint16_t>(4 * H * DH);
+      }
+    }
   }
   // split-K partials get the rest: at least one split of the largest block
   const size_t min_part = max_reduce_block(lo);

@@ -106,9 +106,9 @@ cudaError_t launch_splitk_sum(const float *P, int splits, int M, int N, float *o
 
 // Operand preparation for the bf16 GEMMs (k_convert.cu).
 cudaError_t launch_cast_bf16(const float *src, int64_t lds, int R, int C, void *dst, int64_t ldd, cudaStream_t s);
-// dst[c][r] = bf16(src[src_row ? src_row[r] : r][c]), zeros where src_row[r] < 0.
-cudaError_t launch_transpose_bf16(const float *src, int64_t lds, const int32_t *src_row, int R, int C, void *dst,
-                                  int64_t ldd, cudaStream_t s);
+// dst[r][c] = bf16(src[src_row[r]][c]), zeros where src_row[r] < 0.
+cudaError_t launch_gather_cast_bf16(const float *src, int64_t lds, const int32_t *src_row, int R, int C, void *dst,
+                                    int64_t ldd, cudaStream_t s);
 // P[z][m] = sum of A[r][m] over row chunk z of ceil(R / splits) rows (P
 // holds splits * M floats), then launch_splitk_sum finishes the sums;
 // colsum_splits picks about 256 rows per chunk within part_floats.
@@ -123,8 +123,11 @@ cudaError_t launch_split_rows(const float *src, int64_t lds, int R, int C, float
                               cudaStream_t s);
 
 // bf16 tensor-core GEMM (k_gemm_tc.cu):
-//   D[m][n] (+)= sum_k A[m][k] B[n][k] (+ bias[n]); A, B bf16 with K contiguous
-//   (lda, ldb multiples of 8 elements, 16-byte aligned bases); D fp32 row-major.
+//   D[m][n] (+)= sum_k A[m][k] B[n][k] (+ bias[n]); A, B bf16, K-major (A
+//   stored [M x K], B [N x K], K contiguous) or, with a_mn / b_mn, MN-major
+//   (A stored [K x M], B [K x N]: token-major operands read without a
+//   transpose); lda, ldb multiples of 8 elements, 16-byte aligned bases; D
+//   fp32 row-major.
 //   P != null: split the k range over `splits` and write partial tiles
 //   P[z][m][n] instead (D, bias, accumulate unused).  err: device flag word
 //   (bit 1 set if a pipeline wait timed out).
@@ -139,6 +142,7 @@ struct TcGemmArgs {
   int32_t *err;
   int logsoftmax;  // 3xTF32 GEMM only: replace each output row by its log-softmax (N <= 128, no split)
   WaitFaults wf;   // poll cap / withheld first slab (failure-detection tests)
+  int a_mn, b_mn;  // bf16 GEMM only: operand stored MN-major (see above)
 };
 int tc_splits(int M, int N, int K, int sm_count, size_t part_floats);
 cudaError_t launch_gemm_bf16_tc(const TcGemmArgs &g, cudaStream_t s);
@@ -210,8 +214,15 @@ struct RecArgs {
   const float *dY;     // backward: d loss / d Y of this layer [n_tok x dirs*H]
   int32_t *status;     // device error flags (bit 4: a cluster exchange wait timed out)
   WaitFaults wf;       // poll cap / withheld exchange (failure-detection tests)
+  // bf16 copies for the bf16 contractions, written by the kernels that
+  // rec_writes_bf16() names (null: not wanted):
+  void *Yb;            // forward: bf16 Y [n_tok x dirs*H]
+  void *Hs[2];         // forward: bf16 h_{t-1} of every token of direction d [n_tok x H] (zeros at the start)
+  void *dZb[2];        // backward: bf16 dz [n_tok x 4H]
 };
 cudaError_t launch_lstm_fwd(const RecArgs &a, const RecGeom &g, cudaStream_t s);
+// Whether the kernels of geometry g write RecArgs' bf16 copies.
+inline bool rec_writes_bf16(const RecGeom &g) { return g.mode == 3; }
 // a11: BPTT for both directions; Z[d] holds the gates on entry and dz on exit.
 cudaError_t launch_lstm_bwd(const RecArgs &a, const RecGeom &g, cudaStream_t s);
 
@@ -268,13 +279,12 @@ struct StepBufs {
   float *Wh, *Wl;                             // [Cp x dirs*H] W_out split (or its transpose)
   float *Woh, *Wol;                           // [C x DHp] W_out split for the logits (made at the step's start)
   float *WoTh, *WoTl;                         // [dirs*H x Cp] W_out transposed and split for dY
-  // bf16 GEMM path only (null otherwise)
-  void *Yb;                                   // [NT x dirs*H] bf16 layer input of a projection
-  void *dZb;                                  // [NT x 4H] bf16 dz (input-gradient GEMM)
-  void *dZT;                                  // [4H x NTp] bf16 dz transposed (weight gradients)
-  void *BT;                                   // [max(dirs*H, H) x NTp] bf16 transposed X or h_{t-1}
-  void *Wb;                                   // [4H x dirs*H] bf16 W_ih of one layer and direction
-  void *WTb;                                  // [dirs*H x 4H] bf16 W_ih transposed
+  // bf16 GEMM path only (null otherwise); token-major, read by the GEMMs as
+  // K-major (projection, dX) or MN-major (weight gradients) operands
+  void *Yb[kMaxLayers];                       // [NT x dirs*H] bf16 Y of layers 0 .. L-2
+  void *Hs[2 * kMaxLayers];                   // per layer*dirs+dir: [NT x H] bf16 h_{t-1}
+  void *dZb[2 * kMaxLayers];                  // per layer*dirs+dir: [NT x 4H] bf16 dz
+  void *Wb[2 * kMaxLayers];                   // per layer*dirs+dir (layers > 0): [4H x dirs*H] bf16 W_ih
 };
 
 // Records an error message for bkt_last_error() and returns `code`.

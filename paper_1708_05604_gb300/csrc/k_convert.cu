@@ -1,12 +1,13 @@
 // k_convert.cu -- operand preparation for the bf16 tensor-core contractions
 // (all HBM-bound):
-//   cast_bf16:      fp32 [R x C] -> bf16 [R x C] (row-major, own strides)
-//   transpose_bf16: fp32 [R x C] -> bf16 [C x R] (optionally reading row
-//                   src_row[r] instead of r; a negative index gives zeros)
+//   cast_bf16:      fp32 [R x C] -> bf16 [R x C] (row-major, own strides;
+//                   optionally reading row src_row[r] instead of r, a
+//                   negative index giving zeros)
 //   colsum:         P[z][m] = sum over the rows of chunk z of A[r][m]
-// The transposes turn token-major activations into the K-contiguous layout
-// the tensor-core GEMM reads, so every contraction over tokens is a plain
-// "A[M x K] B[N x K]^T" product.
+// The bf16 GEMM reads token-major operands directly (MN-major tiles), so the
+// contractions over tokens need only bf16 copies of dz, h_{t-1} and the layer
+// input, which the tensor-core recurrent kernels write themselves; the casts
+// here serve the other recurrent kernels.
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -15,63 +16,36 @@
 
 namespace bkt {
 
-__global__ void cast_bf16_kernel(const float *__restrict__ src, int64_t lds, int R, int C,
-                                 __nv_bfloat16 *__restrict__ dst, int64_t ldd) {
+__global__ void cast_bf16_kernel(const float *__restrict__ src, int64_t lds, const int32_t *__restrict__ src_row,
+                                 int R, int C, __nv_bfloat16 *__restrict__ dst, int64_t ldd) {
   const int c2 = C / 2;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < (int64_t)R * c2;
        i += (int64_t)gridDim.x * blockDim.x) {
     const int r = (int)(i / c2), c = (int)(i % c2) * 2;
-    const float2 v = *reinterpret_cast<const float2 *>(src + (int64_t)r * lds + c);
+    const int sr = src_row ? src_row[r] : r;
+    const float2 v = sr >= 0 ? *reinterpret_cast<const float2 *>(src + (int64_t)sr * lds + c) : make_float2(0.f, 0.f);
     *reinterpret_cast<__nv_bfloat162 *>(dst + (int64_t)r * ldd + c) = __floats2bfloat162_rn(v.x, v.y);
   }
   if (C & 1)
-    for (int64_t r = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; r < R; r += (int64_t)gridDim.x * blockDim.x)
-      dst[r * ldd + C - 1] = __float2bfloat16_rn(src[r * lds + C - 1]);
+    for (int64_t r = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; r < R; r += (int64_t)gridDim.x * blockDim.x) {
+      const int sr = src_row ? src_row[r] : (int)r;
+      dst[r * ldd + C - 1] = __float2bfloat16_rn(sr >= 0 ? src[(int64_t)sr * lds + C - 1] : 0.f);
+    }
 }
 
-cudaError_t launch_cast_bf16(const float *src, int64_t lds, int R, int C, void *dst, int64_t ldd, cudaStream_t s) {
+cudaError_t launch_gather_cast_bf16(const float *src, int64_t lds, const int32_t *src_row, int R, int C, void *dst,
+                                    int64_t ldd, cudaStream_t s) {
   if (R <= 0 || C <= 0) return cudaSuccess;
   if ((lds & 1) || (ldd & 1) || (reinterpret_cast<uintptr_t>(src) & 7) || (reinterpret_cast<uintptr_t>(dst) & 3))
     return cudaErrorInvalidValue;
   const int64_t work = (int64_t)R * (C / 2 + 1);
   const int blocks = (int)std::min<int64_t>(8192, (work + 255) / 256);
-  cast_bf16_kernel<<<blocks, 256, 0, s>>>(src, lds, R, C, reinterpret_cast<__nv_bfloat16 *>(dst), ldd);
+  cast_bf16_kernel<<<blocks, 256, 0, s>>>(src, lds, src_row, R, C, reinterpret_cast<__nv_bfloat16 *>(dst), ldd);
   return cudaGetLastError();
 }
 
-// 32 x 32 tiles through shared memory; reads coalesced along C, writes
-// coalesced along R.
-__global__ void transpose_bf16_kernel(const float *__restrict__ src, int64_t lds, const int32_t *__restrict__ src_row,
-                                      int R, int C, __nv_bfloat16 *__restrict__ dst, int64_t ldd) {
-  __shared__ float tile[32][33];
-  const int r0 = blockIdx.x * 32, c0 = blockIdx.y * 32;
-  const int tx = threadIdx.x, ty = threadIdx.y;  // 32 x 8
-#pragma unroll
-  for (int i = 0; i < 32; i += 8) {
-    const int r = r0 + ty + i, c = c0 + tx;
-    float v = 0.f;
-    if (r < R && c < C) {
-      const int sr = src_row ? src_row[r] : r;
-      if (sr >= 0) v = src[(int64_t)sr * lds + c];
-    }
-    tile[ty + i][tx] = v;
-  }
-  __syncthreads();
-#pragma unroll
-  for (int i = 0; i < 32; i += 8) {
-    const int c = c0 + ty + i, r = r0 + tx;
-    if (c < C && r < R) dst[(int64_t)c * ldd + r] = __float2bfloat16_rn(tile[tx][ty + i]);
-  }
-}
-
-cudaError_t launch_transpose_bf16(const float *src, int64_t lds, const int32_t *src_row, int R, int C, void *dst,
-                                  int64_t ldd, cudaStream_t s) {
-  if (R <= 0 || C <= 0) return cudaSuccess;
-  dim3 grid((R + 31) / 32, (C + 31) / 32);
-  if (grid.y > 65535u) return cudaErrorInvalidConfiguration;
-  transpose_bf16_kernel<<<grid, dim3(32, 8), 0, s>>>(src, lds, src_row, R, C, reinterpret_cast<__nv_bfloat16 *>(dst),
-                                                     ldd);
-  return cudaGetLastError();
+cudaError_t launch_cast_bf16(const float *src, int64_t lds, int R, int C, void *dst, int64_t ldd, cudaStream_t s) {
+  return launch_gather_cast_bf16(src, lds, nullptr, R, C, dst, ldd, s);
 }
 
 // fp32 [R x C] -> two fp32 [C x R] arrays hi, lo, each a tf32 value (11

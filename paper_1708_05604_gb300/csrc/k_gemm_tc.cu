@@ -42,9 +42,12 @@ constexpr uint32_t kTxBytes = kAStage + kBStage;
 constexpr size_t kTcSmem = 1024 + (size_t)TSTAGES * (kAStage + kBStage) + 256;
 constexpr uint32_t kWaitPolls = 1u << 22;
 // kind::f16 instruction descriptor: D fp32 (bit 4), A and B bf16 (bits 7, 10),
-// both K-major (bits 15, 16 clear), N >> 3 at bit 17, M >> 4 at bit 24.
+// K-major unless bit 15 (A) / bit 16 (B) marks an MN-major operand, N >> 3 at
+// bit 17, M >> 4 at bit 24.
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(TBN >> 3) << 17) |
                             ((uint32_t)(TBM >> 4) << 24);
+constexpr uint32_t kIdescAmn = 1u << 15, kIdescBmn = 1u << 16;
+constexpr uint32_t kMnChunk = 64 * TBK * 2;  // one 64-element MN chunk of a 64-k slab (8 KB)
 
 __device__ __forceinline__ uint32_t su32(const void *p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -96,13 +99,26 @@ __device__ __forceinline__ void tc_mma(uint32_t d, uint64_t a, uint64_t b, uint3
       : "memory");
 }
 // Shared-memory matrix descriptor of a K-major tile written by TMA with the
-// 128-byte swizzle: rows of 128 B, 8-row groups 1024 B apart.
+// 128-byte swizzle: rows of 128 B, 8-row groups 1024 B apart.  (An MN-major
+// tile is 64-element MN chunks of `lbo` bytes, see sw128_desc_mn.)
 __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
   uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
   d |= (uint64_t)1 << 16;            // leading byte offset (not used by swizzled K-major)
   d |= (uint64_t)(1024 >> 4) << 32;  // stride byte offset
   d |= (uint64_t)1 << 46;            // descriptor version
   d |= (uint64_t)2 << 61;            // 128-byte swizzle
+  return d;
+}
+// The same for an MN-major tile (a token-major operand read without a
+// transpose): each 128-byte row holds 64 consecutive M (or N) elements of one
+// k; rows of consecutive k, 8-row groups 1024 B apart; the 64-element chunks
+// along M (N) are `lbo` bytes apart.
+__device__ __forceinline__ uint64_t sw128_desc_mn(uint32_t saddr, uint32_t lbo) {
+  uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;  // leading byte offset: next 64-element MN chunk
+  d |= (uint64_t)(1024 >> 4) << 32;              // stride byte offset: next 8 k
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
   return d;
 }
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
@@ -192,8 +208,21 @@ __global__ void __launch_bounds__(128, 1)
         if (i == 0 && (g.wf.withhold & kWithholdTma)) continue;  // failure-detection hook
         mbar_expect_tx(full0 + 8 * s, kTxBytes);
         const int kx = (kb0 + i) * TBK;
-        tma_load_2d(su32(sA + s * kAStage), &ta, kx, m0, full0 + 8 * s);
-        tma_load_2d(su32(sB + s * kBStage), &tb, kx, n0, full0 + 8 * s);
+        // K-major: one 128-row box; MN-major: 64-element chunks of 64 k rows
+        if (!g.a_mn) {
+          tma_load_2d(su32(sA + s * kAStage), &ta, kx, m0, full0 + 8 * s);
+        } else {
+#pragma unroll
+          for (int ch = 0; ch < TBM / 64; ++ch)
+            tma_load_2d(su32(sA + s * kAStage + ch * kMnChunk), &ta, m0 + 64 * ch, kx, full0 + 8 * s);
+        }
+        if (!g.b_mn) {
+          tma_load_2d(su32(sB + s * kBStage), &tb, kx, n0, full0 + 8 * s);
+        } else {
+#pragma unroll
+          for (int ch = 0; ch < TBN / 64; ++ch)
+            tma_load_2d(su32(sB + s * kBStage + ch * kMnChunk), &tb, n0 + 64 * ch, kx, full0 + 8 * s);
+        }
         last_phase[s] = i / TSTAGES;
       }
       // after an abort, loads issued to stages the MMA warp never consumed
@@ -215,9 +244,14 @@ __global__ void __launch_bounds__(128, 1)
         }
         tc_fence_after();
         const uint32_t a0 = su32(sA + s * kAStage), b0 = su32(sB + s * kBStage);
+        const uint32_t idesc = kIdesc | (g.a_mn ? kIdescAmn : 0u) | (g.b_mn ? kIdescBmn : 0u);
 #pragma unroll
-        for (int kk = 0; kk < TBK / 16; ++kk)
-          tc_mma(tmem, sw128_desc(a0 + kk * 32), sw128_desc(b0 + kk * 32), kIdesc, (i > 0 || kk > 0) ? 1u : 0u);
+        for (int kk = 0; kk < TBK / 16; ++kk) {
+          // k step kk: 32 bytes into each K-major row, or 16 rows (2 KB) of an MN-major tile
+          const uint64_t ad = g.a_mn ? sw128_desc_mn(a0 + kk * 2048, kMnChunk) : sw128_desc(a0 + kk * 32);
+          const uint64_t bd = g.b_mn ? sw128_desc_mn(b0 + kk * 2048, kMnChunk) : sw128_desc(b0 + kk * 32);
+          tc_mma(tmem, ad, bd, idesc, (i > 0 || kk > 0) ? 1u : 0u);
+        }
         tc_commit(empty0 + 8 * s);
         ++issued;
       }
@@ -730,8 +764,12 @@ cudaError_t launch_gemm_bf16_tc(const TcGemmArgs &g, cudaStream_t s) {
       (reinterpret_cast<uintptr_t>(g.B) & 15) || (g.P && g.splits < 1) || (!g.P && !g.D))
     return cudaErrorInvalidValue;
   CUtensorMap ta, tb;
-  if (!make_map(&ta, g.A, (uint64_t)g.K, (uint64_t)g.M, g.lda, TBM)) return cudaErrorInvalidValue;
-  if (!make_map(&tb, g.B, (uint64_t)g.K, (uint64_t)g.N, g.ldb, TBN)) return cudaErrorInvalidValue;
+  // K-major operands are [rows x K]; MN-major ones [K x rows] (rows contiguous)
+  const bool okA = g.a_mn ? make_map(&ta, g.A, (uint64_t)g.M, (uint64_t)g.K, g.lda, TBK)
+                          : make_map(&ta, g.A, (uint64_t)g.K, (uint64_t)g.M, g.lda, TBM);
+  const bool okB = g.b_mn ? make_map(&tb, g.B, (uint64_t)g.N, (uint64_t)g.K, g.ldb, TBK)
+                          : make_map(&tb, g.B, (uint64_t)g.K, (uint64_t)g.N, g.ldb, TBN);
+  if (!okA || !okB) return cudaErrorInvalidValue;
   cudaError_t e = ensure_smem((const void *)gemm_bf16_tc_kernel, kTcSmem);
   if (e != cudaSuccess) return e;
   dim3 grid((g.M + TBM - 1) / TBM, (g.N + TBN - 1) / TBN, g.P ? g.splits : 1);

@@ -307,6 +307,8 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_fwd_tc_kernel(RecArgs a) {
   float *__restrict__ Z = a.Z[d];
   float *__restrict__ Cs = a.Cst[d];
   float *__restrict__ Y = a.Y;
+  __nv_bfloat16 *__restrict__ Yb = reinterpret_cast<__nv_bfloat16 *>(a.Yb);
+  __nv_bfloat16 *__restrict__ Hs = reinterpret_cast<__nv_bfloat16 *>(a.Hs[d]);
   int len[C], lenq[NJ];  // lengths of this thread's columns; of its rows col0 + 4 j + q
 #pragma unroll
   for (int k = 0; k < C; ++k) len[k] = rlen[col0 + k];
@@ -391,16 +393,24 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_fwd_tc_kernel(RecArgs a) {
       const int n = col0 + 4 * j + q;
       const float cn = fmaf(g4[1], cst[j], g4[0] * g4[2]);
       float h = g4[3] * tanh_tc(cn);
+      __nv_bfloat16 hh, hl;
       if (s < lenq[j]) {
         cst[j] = cn;
         const size_t tk = (size_t)tok_q(j, s);
         Cs[tk * H + gu] = cn;
         Y[tk * DH + d * H + gu] = h;
+        split_bf16(h, hh, hl);
+        // bf16 copies for the bf16 contractions: Y, and h as the h_{t-1} of
+        // the row's next token in this direction (zero before its first)
+        if (Yb) Yb[tk * DH + d * H + gu] = hh;
+        if (Hs) {
+          if (s == 0) Hs[tk * H + gu] = __float2bfloat16_rn(0.f);
+          if (s + 1 < lenq[j]) Hs[(size_t)tok_q(j, s + 1) * H + gu] = hh;
+        }
       } else {
         h = 0.f;
+        split_bf16(h, hh, hl);
       }
-      __nv_bfloat16 hh, hl;
-      split_bf16(h, hh, hl);
       const uint32_t off = (uint32_t)(u >> 3) * (16u * N) + (uint32_t)n * 16u + (uint32_t)(u & 7) * 2u;
       *reinterpret_cast<__nv_bfloat16 *>(sg_hi + off) = hh;
       *reinterpret_cast<__nv_bfloat16 *>(sg_lo + off) = hl;
@@ -522,6 +532,7 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_bwd_tc_kernel(RecArgs a) {
   float *__restrict__ Z = a.Z[d];
   const float *__restrict__ Cs = a.Cst[d];
   const float *__restrict__ dY = a.dY;
+  __nv_bfloat16 *__restrict__ dZb = reinterpret_cast<__nv_bfloat16 *>(a.dZb[d]);
   int len[NJ];  // lengths of this thread's rows col0 + 4 j + q
 #pragma unroll
   for (int j = 0; j < NJ; ++j) len[j] = rlen[col0 + 4 * j + q];
@@ -603,6 +614,13 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_bwd_tc_kernel(RecArgs a) {
       split_bf16(dz4[1], h1, l1);
       split_bf16(dz4[2], h2, l2);
       split_bf16(dz4[3], h3, l3);
+      if (dZb && s < len[j]) {  // bf16 dz for the bf16 contractions
+        __nv_bfloat16 *zb = dZb + (size_t)tok_at(j, s) * G + gu;
+        zb[0] = h0;
+        zb[H] = h1;
+        zb[2 * H] = h2;
+        zb[3 * H] = h3;
+      }
       const uint32_t off = (uint32_t)(u >> 1) * (16u * N) + (uint32_t)n * 16u + (uint32_t)(u & 1) * 8u;
       *reinterpret_cast<uint2 *>(Bz + off) = make_uint2(pack2(h0, h1), pack2(h2, h3));
       *reinterpret_cast<uint2 *>(Bz + Lay::kB + off) = make_uint2(pack2(l0, l1), pack2(l2, l3));

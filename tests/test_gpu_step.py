@@ -338,6 +338,22 @@ def test_full_length_h512_wide_batch_vs_oracle():
     assert np.linalg.norm(ga + gb - gg) <= 1e-4 * np.linalg.norm(gg)
 
 
+@pytest.mark.parametrize("layers,bi,H", [(2, True, 128), (2, False, 512), (3, True, 64)])
+def test_bf16_path_with_the_other_recurrent_kernels(layers, bi, H):
+    """The bf16 contractions when the recurrent kernels do not write the bf16
+    copies themselves (single-CTA kernels at H <= 128, register-tiled
+    clusters at H = 512): the step casts them instead.  Parity at the bf16
+    bound."""
+    cfg = {"n_layers": layers, "bidirectional": bi, "in_dim": 4, "hidden": H, "n_classes": 81, "blank": 0,
+           "gemm_bf16": True}
+    rng = np.random.default_rng(H + layers)
+    ds = synth.make_dataset([61, 47, 33, 30, 12, 5, 1], 8, rng)
+    params = synth.draw_params(rng, binding.param_count(cfg))
+    lg, gg = gpu_step(cfg, ds, params)
+    lo, go = oracle_step(cfg, ds, params)
+    compare(cfg, lg, gg, lo, go, BF16_TOL)
+
+
 def test_bf16_workload_runs_on_tensor_cores():
     """The bf16 workloads route their contractions through the tcgen05 GEMM
     (and stay within the bf16 tolerance while differing from fp32 rounding)."""
