@@ -23,9 +23,10 @@ against its roofline comes from the library's per-launch work accounting
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl native|reference]
 
 --impl reference times the fp64 CPU oracle (test infrastructure) on bounded
-samples of the same workload.  Under torchrun each rank runs an independent
-replica of the workload (no collective on the data path) and rank 0 prints
-the whole-job line.
+samples of the same workload.  Under torchrun each rank runs a replica of the workload
+and the replicas' parameters are combined at the end of every epoch by the
+paper's eq. 3 (an NCCL all-reduce, then bkt_average_models: the one
+exchange of the data-parallel method); rank 0 prints the whole-job line.
 """
 from __future__ import annotations
 
@@ -223,12 +224,20 @@ def recorded_traffic(kernel: str, workload: str, buckets: int):
     path = os.path.join(ROOT, "profiles", f"traffic_{workload}.json")
     try:
         rec = json.load(open(path))
-        if rec.get("kernel") != kernel or int(rec.get("buckets", -1)) != buckets:
+        if int(rec.get("buckets", -1)) != buckets:
+            return None, None
+        if "kernels" in rec:  # several kernels of one source file
+            entry = rec["kernels"].get(kernel)
+            if entry is None:
+                return None, None
+        elif rec.get("kernel") == kernel:
+            entry = rec
+        else:
             return None, None
         src = open(os.path.join(ROOT, rec["source"]), "rb").read()
         if hashlib.sha256(src).hexdigest() != rec.get("source_sha256"):
             return None, None
-        return float(rec["dram_bytes_per_launch"]), os.path.relpath(path, ROOT)
+        return float(entry["dram_bytes_per_launch"]), os.path.relpath(path, ROOT)
     except (OSError, ValueError, KeyError):
         return None, None
 
@@ -269,9 +278,13 @@ def run_native(args, world, rank, local):
 
     opt = binding.Adadelta(params) if args.optimizer == "adadelta" else None
 
+    prev = torch.empty_like(params) if world > 1 else None
+
     def epoch(e, Q, dataset=dd, loss_buf=loss):
         plan = binding.plan_buckets(ds.lengths, Q, w.batch, seed=args.seed, epoch=e)
         order, off = plan["order"], plan["batch_off"]
+        if prev is not None:
+            prev.copy_(params)
         for k in range(plan["n_batches"]):
             ids = order[off[k]:off[k + 1]]
             lv = loss_buf[off[k]:off[k + 1]]
@@ -280,6 +293,13 @@ def run_native(args, world, rank, local):
                 binding.sgd_update(params, grads, LR, stream)
             else:
                 opt.step(grads, stream)
+        if prev is not None:
+            # the replicas' models are combined once per epoch (Section III.B
+            # step 5, eq. 3): NCCL all-reduce of the parameters, then
+            # bkt_average_models
+            import torch.distributed as dist
+            dist.all_reduce(params, op=dist.ReduceOp.SUM)
+            binding.average_models(params, prev, world, 1e-6, stream)
         return plan
 
     def timed(Q, steps, warmup, e0=0, with_timer=False, clocks=None):
@@ -410,7 +430,7 @@ def run_native(args, world, rank, local):
                    "buckets": args.buckets, "unpadded_timesteps_per_epoch": unpadded,
                    "step": "one epoch: plan + every batch's fwd/bwd/CTC + SGD, rebucketed and reshuffled",
                    "l2": "flushed between timed steps (256 MiB write, outside the events)",
-                   "parallelism": "replicas" if world > 1 else "1 GPU"},
+                   "parallelism": "replicas, eq.-3 averaging per epoch" if world > 1 else "1 GPU"},
         "padded_efficiency": float(np.mean(pe)),
         "infeasible_sequences_per_epoch": infeasible / max(1, args.steps),
         "epoch_time_vs_buckets": by_q,

@@ -11,6 +11,8 @@
  *     mini-batch, forward + back-propagation through time, on one GPU.
  *   - bkt_adadelta_update: the paper's parameter update rule, ADADELTA
  *     (Section III.B step 4, ref. [21]); bkt_sgd_update: plain SGD.
+ *   - bkt_average_models: the per-epoch model averaging of the paper's
+ *     data-parallel training (Section III.B step 5, eq. 3).
  *
  * Conventions
  *   - Every entry point returns an int status (BKT_OK = 0).  On failure
@@ -231,6 +233,21 @@ int bkt_sgd_update(float *params, const float *grads, int64_t n, float lr,
 int bkt_adadelta_update(float *params, const float *grads, float *eg2,
                         float *edx2, int64_t n, float rho, float eps,
                         float lr, void *stream);
+
+/* Model averaging of the data-parallel training loop (Section III.B step
+ * 5, eq. 3 with alpha = 1): V(t) = V_alpha(t) - beta V(t-1), V_alpha the
+ * mean over the K parallel models of their parameters after the epoch,
+ * V(t-1) the parameters the epoch started from (the paper uses
+ * beta = 1e-6, a decay proportional to the weights).  Given
+ *   v     device fp32 [n]: the element-wise sum of the K models'
+ *         parameters, as an all-reduce with the sum operation leaves it on
+ *         every replica; overwritten with V(t);
+ *   prev  device fp32 [n]: V(t-1);
+ * computes v[i] <- v[i] / K - beta prev[i] (IEEE division, then one fused
+ * multiply-add), enqueued on `stream`.  BKT_EINVAL: n < 0, n_models < 1,
+ * beta < 0 or NaN, or a NULL array with n > 0.                           */
+int bkt_average_models(float *v, const float *prev, int64_t n, int32_t n_models,
+                       float beta, void *stream);
 
 /* Waits for the work this ctx enqueued, then returns BKT_OK or the
  * device-side errors raised since the previous call, and clears them:

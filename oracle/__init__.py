@@ -83,6 +83,8 @@ def _load():
         lib.or_adadelta.argtypes = [f64p, f64p, f64p, f64p, ctypes.c_int64, ctypes.c_double,
                                     ctypes.c_double, ctypes.c_double]
         lib.or_adadelta.restype = None
+        lib.or_average_models.argtypes = [f64p, ctypes.c_int32, f64p, ctypes.c_int64, ctypes.c_double, f64p]
+        lib.or_average_models.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -236,3 +238,20 @@ def adadelta(params, grads, eg2, edx2, rho: float = 0.95, eps: float = 1e-6,
     lib.or_adadelta(_p(p, ctypes.c_double), _p(g, ctypes.c_double), _p(a, ctypes.c_double),
                     _p(b, ctypes.c_double), p.size, rho, eps, lr)
     return p, a, b
+
+
+def average_models(models, prev, beta: float = 1e-6) -> np.ndarray:
+    """Eq. 3 (Section III.B step 5, alpha = 1): the mean of the K models'
+    parameters (rows of `models`) minus beta times the previous epoch's
+    parameters `prev`, in float64."""
+    lib = _load()
+    M = np.ascontiguousarray(np.atleast_2d(np.asarray(models, dtype=np.float64)))
+    p = np.ascontiguousarray(prev, dtype=np.float64)
+    if M.shape[1] != p.size:
+        raise ValueError("models and prev differ in length")
+    out = np.zeros(p.size, dtype=np.float64)
+    rc = lib.or_average_models(_p(M, ctypes.c_double), M.shape[0], _p(p, ctypes.c_double), p.size,
+                               float(beta), _p(out, ctypes.c_double))
+    if rc != 0:
+        raise ValueError(f"or_average_models failed ({rc})")
+    return out

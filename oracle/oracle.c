@@ -36,6 +36,9 @@
  *   or_sgd              theta <- theta - lr * g.
  *   or_adadelta         ADADELTA (Zeiler 2012, the paper's ref. [21], its
  *                       Algorithm 1), the update rule of Section III.B step 4.
+ *   or_average_models   Section III.B step 5, eq. 3 with alpha = 1: the main
+ *                       process averages the parallel models' parameters and
+ *                       subtracts beta times the previous epoch's values.
  *
  * Numerics: all arithmetic is in double; exp/log/tanh are the C library's.
  */
@@ -676,4 +679,21 @@ void or_adadelta(double *x, const double *g, double *eg2, double *edx2,
     edx2[i] = rho * edx2[i] + (1.0 - rho) * dx * dx;
     x[i] += lr * dx;
   }
+}
+
+/* Eq. 3 (Section III.B step 5, alpha = 1): V(t) = V_alpha(t) - beta V(t-1),
+ * V_alpha(t) the mean over the K parallel models of their parameters after
+ * the epoch, V(t-1) the parameters the epoch started from.
+ *   models  [K][n], row k = model k;  prev [n];  out [n].               */
+int or_average_models(const double *models, int32_t K, const double *prev, int64_t n, double beta,
+                      double *out) {
+  int64_t i;
+  int32_t k;
+  if (K < 1 || n < 0) return OR_EINVAL;
+  for (i = 0; i < n; i++) {
+    double s = 0.0;
+    for (k = 0; k < K; k++) s += models[(int64_t)k * n + i];
+    out[i] = s / (double)K - beta * prev[i];
+  }
+  return OR_OK;
 }

@@ -23,7 +23,7 @@ BKT_GEMM_FP32, BKT_GEMM_BF16 = 0, 1
 # Every symbol include/bkt.h declares.
 EXPORTS = ("bkt_plan_buckets", "bkt_plan_buckets_ordered", "bkt_plan_get", "bkt_plan_free", "bkt_param_count",
            "bkt_ctx_create", "bkt_ctx_destroy", "bkt_lstm_ctc_step", "bkt_lstm_ctc_step_static",
-           "bkt_sgd_update", "bkt_adadelta_update",
+           "bkt_sgd_update", "bkt_adadelta_update", "bkt_average_models",
            "bkt_ctx_sync_status", "bkt_ctx_infeasible_count", "bkt_ctx_set_wait_faults",
            "bkt_ctx_set_timing", "bkt_ctx_kernel_times", "bkt_last_error")
 
@@ -96,6 +96,7 @@ def lib() -> ctypes.CDLL:
         L.bkt_lstm_ctc_step_static.argtypes = [ctypes.POINTER(ModelCfg), ctypes.POINTER(Batch), vp,
                                                vp, vp, vp]
         L.bkt_sgd_update.argtypes = [vp, vp, ctypes.c_int64, ctypes.c_float, vp]
+        L.bkt_average_models.argtypes = [vp, vp, ctypes.c_int64, ctypes.c_int32, ctypes.c_float, vp]
         L.bkt_adadelta_update.argtypes = [vp, vp, vp, vp, ctypes.c_int64, ctypes.c_float,
                                           ctypes.c_float, ctypes.c_float, vp]
         L.bkt_ctx_sync_status.argtypes = [vp]
@@ -107,7 +108,7 @@ def lib() -> ctypes.CDLL:
         L.bkt_last_error.restype = ctypes.c_char_p
         for name in ("bkt_plan_buckets", "bkt_plan_buckets_ordered", "bkt_plan_get", "bkt_ctx_create", "bkt_lstm_ctc_step",
                      "bkt_lstm_ctc_step_static",
-                     "bkt_sgd_update", "bkt_adadelta_update", "bkt_ctx_sync_status",
+                     "bkt_sgd_update", "bkt_adadelta_update", "bkt_average_models", "bkt_ctx_sync_status",
                      "bkt_ctx_infeasible_count", "bkt_ctx_set_wait_faults", "bkt_ctx_set_timing",
                      "bkt_ctx_kernel_times"):
             getattr(L, name).restype = ctypes.c_int
@@ -201,6 +202,16 @@ def adadelta_update(params, grads, eg2, edx2, rho: float = 0.95, eps: float = 1e
                                      ctypes.c_void_p(edx2.data_ptr()), n, ctypes.c_float(rho),
                                      ctypes.c_float(eps), ctypes.c_float(lr),
                                      _stream_handle(stream)))
+
+
+def average_models(summed, prev, n_models: int, beta: float = 1e-6, stream=None):
+    """bkt_average_models on two CUDA fp32 tensors: `summed` (the element-wise
+    sum of the n_models replicas' parameters) becomes eq. 3's
+    summed / n_models - beta * prev, in place."""
+    n = summed.numel()
+    assert summed.is_cuda and prev.is_cuda and prev.numel() == n
+    _check(lib().bkt_average_models(ctypes.c_void_p(summed.data_ptr()), ctypes.c_void_p(prev.data_ptr()), n,
+                                    int(n_models), ctypes.c_float(beta), _stream_handle(stream)))
 
 
 class Adadelta:

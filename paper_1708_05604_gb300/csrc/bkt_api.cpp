@@ -1201,6 +1201,16 @@ extern "C" int bkt_adadelta_update(float *params, const float *grads, float *eg2
   return BKT_OK;
 }
 
+extern "C" int bkt_average_models(float *v, const float *prev, int64_t n, int32_t n_models, float beta,
+                                  void *stream) {
+  if (n < 0 || n_models < 1 || (n > 0 && (!v || !prev)) || !(beta >= 0.f))
+    return set_err(BKT_EINVAL, "bkt_average_models: bad arguments");
+  if (n == 0) return BKT_OK;
+  cudaError_t e = bkt::launch_average_models(v, prev, n, n_models, beta, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_err("average kernel launch", e);
+  return BKT_OK;
+}
+
 extern "C" int bkt_sgd_update(float *params, const float *grads, int64_t n, float lr, void *stream) {
   if (n < 0 || (n > 0 && (!params || !grads))) return set_err(BKT_EINVAL, "bkt_sgd_update: bad arguments");
   if (n == 0) return BKT_OK;

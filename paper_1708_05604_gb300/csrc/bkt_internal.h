@@ -248,6 +248,8 @@ cudaError_t launch_lstm_cta(const RecArgs &a, int bc, bool bwd, cudaStream_t s);
 
 // a13
 cudaError_t launch_sgd(float *p, const float *g, int64_t n, float lr, cudaStream_t s);
+// Section III.B step 5, eq. 3: see bkt_average_models in bkt.h
+cudaError_t launch_average_models(float *v, const float *prev, int64_t n, int K, float beta, cudaStream_t s);
 // a13, ADADELTA: see bkt_adadelta_update in bkt.h
 cudaError_t launch_adadelta(float *p, const float *g, float *eg2, float *edx2, int64_t n, float rho, float eps,
                             float lr, cudaStream_t s);

@@ -12,8 +12,17 @@ training loss and the mean validation loss per sequence.
       --buckets 1,2,3,4,6 --epochs 3 [--optimizer adadelta|sgd]
       [--batch-order ascending|descending|shuffle_buckets|shuffle_batches]
 
+Data-parallel training (Section III.B steps 3-5): launched with torchrun on
+N GPUs, every epoch the training sequences are reshuffled into N portions,
+each replica trains its portion from the same starting parameters, and the
+replicas' parameters are combined by eq. 3 (an NCCL all-reduce of the flat
+parameter buffer, then bkt_average_models):
+
+  torchrun --nproc-per-node N -m paper_1708_05604_gb300.train --replicas ...
+
 Every step runs in the library (bkt_plan_buckets_ordered, bkt_lstm_ctc_step,
-bkt_adadelta_update / bkt_sgd_update); this module only sequences the calls.
+bkt_adadelta_update / bkt_sgd_update, bkt_average_models); this module only
+sequences the calls.
 """
 from __future__ import annotations
 
@@ -44,6 +53,28 @@ def epoch_batches(lengths, train_ids, n_buckets: int, batch: int, seed: int, epo
     plan = binding.plan_buckets(lengths[train_ids], n_buckets, batch, seed, epoch, batch_order)
     order, off = plan["order"], plan["batch_off"]
     return [train_ids[order[off[k]:off[k + 1]]] for k in range(plan["n_batches"])], plan
+
+
+def data_portions(train_ids, world: int, seed: int, epoch: int):
+    """Section III.B step 3: every epoch the training sequences are
+    reshuffled (a permutation seeded by (seed, epoch)) and cut into `world`
+    contiguous portions of near-equal size; portion r is replica r's data."""
+    ids = np.asarray(train_ids, dtype=np.int64)
+    perm = np.random.default_rng([int(seed), int(epoch), 0x5EED]).permutation(ids)
+    return [np.sort(p) for p in np.array_split(perm, world)]
+
+
+def data_parallel_epoch(params_start, portion, train_portion, all_reduce_sum, average, world: int):
+    """Section III.B steps 4-5 on one replica: train this replica's portion
+    from params_start (`train_portion(portion)` returns the replica's
+    parameters after the epoch, a new buffer), sum the replicas' parameters
+    in place (`all_reduce_sum`, the one exchange of the loop), then eq. 3:
+    `average(summed, params_start, world)` leaves mean - beta * params_start.
+    Every replica ends the epoch with the same parameters."""
+    local = train_portion(portion)
+    all_reduce_sum(local)
+    average(local, params_start, world)
+    return local
 
 
 def validation_batches(lengths, val_ids, batch: int):
@@ -135,6 +166,62 @@ def train(workload: str, n_buckets: int, epochs: int, optimizer: str = "adadelta
     return record
 
 
+def train_replicas(workload: str, n_buckets: int, epochs: int, seed: int = 0, beta: float = 1e-6,
+                   lr: float | None = None, n_seqs: int | None = None, max_len: int | None = None,
+                   log=None) -> dict:
+    """Data-parallel training on the GPUs of a torchrun launch (one process
+    per GPU, NCCL): per epoch, data portions, a local ADADELTA epoch of the
+    replica's portion (bucketed within the portion), then eq. 3."""
+    import torch
+    import torch.distributed as dist
+
+    from . import binding, build, synth
+
+    world, rank = dist.get_world_size(), dist.get_rank()
+    build.build()
+    w = synth.WORKLOADS[workload]
+    cfg = w.model_cfg()
+    ds = synth.make_workload(w, seed=seed, n_seqs=n_seqs, max_len=max_len)
+    train_ids, _ = split_validation(ds.n, 0.05, seed + 17)
+    P = binding.param_count(cfg)
+    dev = torch.device("cuda", torch.cuda.current_device())
+    params = torch.from_numpy(synth.draw_params(np.random.default_rng(seed + 1), P)).to(dev)
+    dd = binding.DeviceDataset(ds, device=dev)
+    cap = int(np.sort(ds.lengths)[-w.batch:].sum())
+    ctx = binding.Ctx(cfg, cap, w.batch, max(1, int(ds.label_lengths.max())))
+    grads = torch.zeros_like(params)
+    loss = torch.zeros(ds.n, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    record = {"workload": workload, "replicas": world, "n_buckets": n_buckets, "epochs": []}
+    for e in range(epochs):
+        portion = data_portions(train_ids, world, seed, e)[rank]
+
+        def train_portion(ids_portion):
+            local = params.clone()
+            opt = binding.Adadelta(local, lr=1.0 if lr is None else lr)
+            batches, _ = epoch_batches(ds.lengths, ids_portion, n_buckets, w.batch, seed + 1000 * rank, e)
+            pos = 0
+            for ids in batches:
+                ctx.step(dd, ids, local, grads, loss[pos:pos + ids.size], stream)
+                opt.step(grads, stream)
+                pos += ids.size
+            return local
+
+        t0 = time.perf_counter()
+        params = data_parallel_epoch(params, portion, train_portion,
+                                     lambda t: dist.all_reduce(t, op=dist.ReduceOp.SUM),
+                                     lambda v, prev, k: binding.average_models(v, prev, k, beta, stream), world)
+        torch.cuda.synchronize(dev)
+        ctx.sync_status()
+        rec = {"epoch": e, "wall_s": time.perf_counter() - t0, "portion": int(portion.size)}
+        record["epochs"].append(rec)
+        if log and rank == 0:
+            log(rec)
+    record["params"] = params.cpu().numpy()
+    ctx.close()
+    return record
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--workload", default="lstm1_bi_h128")
@@ -145,7 +232,24 @@ def main(argv=None):
                     choices=["ascending", "descending", "shuffle_buckets", "shuffle_batches"])
     ap.add_argument("--lr", type=float, default=None)
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--replicas", action="store_true",
+                    help="data-parallel replicas with eq.-3 averaging (launch with torchrun)")
+    ap.add_argument("--beta", type=float, default=1e-6)
     a = ap.parse_args(argv)
+    if a.replicas:
+        import os
+
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+        dist.init_process_group("nccl")
+        for Q in [int(q) for q in a.buckets.split(",") if q]:
+            r = train_replicas(a.workload, Q, a.epochs, a.seed, a.beta, a.lr)
+            r.pop("params")
+            if dist.get_rank() == 0:
+                print(json.dumps(r), flush=True)
+        dist.destroy_process_group()
+        return 0
     for Q in [int(q) for q in a.buckets.split(",") if q]:
         r = train(a.workload, Q, a.epochs, a.optimizer, a.batch_order, a.seed, lr=a.lr)
         r.pop("params")

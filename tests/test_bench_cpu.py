@@ -119,3 +119,19 @@ def test_measured_peaks_source(bench, tmp_path, monkeypatch):
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
     peaks, src = bench.measured_peaks()
     assert src == "fallback" and peaks["hbm_gbs"] == 6800.0
+
+
+def test_recorded_traffic_per_kernel_record(bench):
+    rec = json.load(open(os.path.join(ROOT, "profiles", "traffic_lstm3_bi_h256_bf16_bimodal.json")))
+    src = open(os.path.join(ROOT, rec["source"]), "rb").read()
+    same = hashlib.sha256(src).hexdigest() == rec["source_sha256"]
+    for k, entry in rec["kernels"].items():
+        tb, where = bench.recorded_traffic(k, rec["workload"], rec["buckets"])
+        if same:
+            assert tb == entry["dram_bytes_per_launch"] and where.endswith(".json")
+            # scaled from the profiled batch by tokens
+            prof = entry["dram_read_bytes_profiled"] + entry["dram_write_bytes_profiled"]
+            assert tb == pytest.approx(prof * rec["mean_tokens_per_launch"] / rec["scaled_from"]["tokens"])
+        else:
+            assert tb is None
+    assert bench.recorded_traffic("gemm_tc", rec["workload"], rec["buckets"]) == (None, None)

@@ -370,3 +370,48 @@ def test_bf16_workload_runs_on_tensor_cores():
     fcfg = dict(cfg, gemm_bf16=False)
     lf, gf = gpu_step(fcfg, ds, params)
     compare(fcfg, lf, gf, lo, go, FP32_TOL)
+
+
+def test_average_models_vs_oracle():
+    """Eq. 3 (Section III.B step 5) on the GPU: from the element-wise sum of K
+    models, v / K - beta prev in fp32 (one IEEE division, one fused
+    multiply-add: within 2 ulp of the exact value's magnitude terms)."""
+    import torch
+    rng = np.random.default_rng(9)
+    for n, K, beta in ((1, 1, 1e-6), (7409, 2, 1e-6), (100003, 6, 0.25), (5003, 3, 0.0)):
+        models = rng.standard_normal((K, n)).astype(np.float32)
+        summed = models.astype(np.float64).sum(axis=0).astype(np.float32)   # what the all-reduce delivers
+        prev = rng.standard_normal(n).astype(np.float32)
+        v = torch.from_numpy(summed).cuda()
+        binding.average_models(v, torch.from_numpy(prev).cuda(), K, beta)
+        torch.cuda.synchronize()
+        exact = oracle.average_models([summed.astype(np.float64) / K], prev.astype(np.float64), float(np.float32(beta)))
+        scale = np.abs(summed.astype(np.float64) / K) + abs(beta) * np.abs(prev.astype(np.float64))
+        assert np.all(np.abs(v.cpu().numpy().astype(np.float64) - exact) <= 2 * 2.0 ** -24 * scale + 1e-38)
+    with pytest.raises(binding.BktError):
+        binding.average_models(torch.zeros(4, device="cuda"), torch.zeros(4, device="cuda"), 0)
+
+
+def test_data_parallel_epoch_on_one_gpu_with_nccl():
+    """The replica loop's GPU data plane with one NCCL rank: the all-reduce is
+    the identity and eq. 3 leaves (start + delta) - beta * start."""
+    import torch
+    import torch.distributed as dist
+
+    from paper_1708_05604_gb300 import train
+    import socket
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        port = s.getsockname()[1]
+    dist.init_process_group("nccl", init_method=f"tcp://127.0.0.1:{port}", rank=0, world_size=1)
+    try:
+        start = torch.randn(10007, device="cuda")
+        delta = torch.randn(10007, device="cuda")
+        out = train.data_parallel_epoch(start, np.arange(5), lambda ids: start + delta,
+                                        lambda t: dist.all_reduce(t, op=dist.ReduceOp.SUM),
+                                        lambda v, prev, k: binding.average_models(v, prev, k, 1e-6), 1)
+        torch.cuda.synchronize()
+        ref = (start.double() + delta.double()) - 1e-6 * start.double()
+        assert torch.allclose(out.double(), ref, rtol=1e-6, atol=1e-6)
+    finally:
+        dist.destroy_process_group()
