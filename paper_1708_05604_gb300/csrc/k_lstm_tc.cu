@@ -178,18 +178,6 @@ __device__ __forceinline__ float sel4(float a, float b, float c, float d, int i)
 
 // Shared-memory layout (bytes).
 template <int N>
-struct TcFwdLayout {
-  static constexpr uint32_t kB = N * kTH * 2;      // one B operand (hi or lo): N rows x 256 bf16
-  static constexpr uint32_t kSlice = 64 * N;       // this CTA's 32 units of one B operand
-  static constexpr uint32_t kStepBytes = kTCS * 2 * kSlice;  // received per step: 8 CTAs x (hi + lo)
-  static constexpr uint32_t oB = 0;                // [2 parity][2 hi/lo][kB]
-  static constexpr uint32_t oStg = oB + 4 * kB;    // [2 parity][2 hi/lo][kSlice]
-  static constexpr uint32_t oBar = oStg + 4 * kSlice;  // hbar[2], mmabar
-  static constexpr uint32_t oSlot = oBar + 3 * 8;
-  static constexpr uint32_t oLen = oSlot + 16;     // [N] row lengths
-  static constexpr uint32_t oToff = oLen + 4 * N;  // [T+1] when it fits
-};
-template <int N>
 struct TcBwdLayout {
   static constexpr uint32_t kB = N * 128 * 2;      // one B operand (dz hi or lo): N rows x 128 gate rows
   static constexpr int kRS = kTHc + 8;             // floats per (source, row) of received partials (32 units + pad)
@@ -211,33 +199,50 @@ size_t tc_smem_bytes(size_t base, int T) {
 
 }  // namespace
 
-// Thread roles (both kernels; QW warps per TMEM lane quarter, 128 QW threads):
-// warp w reads TMEM lane quarter qt = w % 4 and columns C cs .. C cs + C - 1
-// (cs = w / 4, C = N / QW, a multiple of 4) of each accumulator;
-// lane l of it is TMEM lane m = 32 qt + l.  In the forward kernel lane m is
-// gate row q = m % 4 of unit u = m / 4; after the gate swap the thread holds
-// unit u, gates i, f, g, o, for rows C cs + 4 j + q (j < C / 4).  BPTT's
-// phase B uses the same (u, row) pairs; its accumulator lanes are units.
-template <int N, int QW>
-__global__ void __launch_bounds__(128 * QW, 1) lstm_fwd_tc_kernel(RecArgs a) {
+// Thread roles (both kernels, 512 threads): warp w reads TMEM lane quarter
+// w % 4 and columns C (w / 4) .. + C - 1 (C = N / 4) of each accumulator,
+// lane l of it TMEM lane 32 (w % 4) + l; the elementwise phases give thread
+// (w, l) unit l of the CTA's 32 and rows P w .. P w + P - 1 (P = N / 16).
+// Forward kernel.  TMEM lane m = 32 q + u holds gate q of unit u, so warp
+// quarter q holds one gate for 32 consecutive units (coalesced Zx loads and
+// gate stores, a warp-uniform nonlinearity); the four gates of a (unit, row)
+// meet through shared memory, then thread (w, lane) updates the cell of unit
+// `lane` for rows P w .. P w + P - 1 (P = N / 16).  (A lane order 4u + q,
+// with the gates swapped by shuffles inside groups of four lanes, measured
+// 10 % slower per step.)
+template <int N>
+struct TcFwdLayout {
+  static constexpr uint32_t kB = N * kTH * 2;
+  static constexpr uint32_t kSlice = 64 * N;
+  static constexpr uint32_t kStepBytes = kTCS * 2 * kSlice;
+  static constexpr uint32_t oB = 0;                    // [2 parity][2 hi/lo][kB]
+  static constexpr uint32_t oStg = oB + 4 * kB;        // [2 parity][2 hi/lo][kSlice]
+  static constexpr uint32_t oGate = oStg + 4 * kSlice; // [N][4][32] fp32 activated gates
+  static constexpr uint32_t oBar = oGate + N * 4 * kTHc * 4;
+  static constexpr uint32_t oSlot = oBar + 3 * 8;
+  static constexpr uint32_t oLen = oSlot + 16;
+  static constexpr uint32_t oToff = oLen + 4 * N;
+};
+
+template <int N>
+__global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
   using Lay = TcFwdLayout<N>;
-  constexpr int H = kTH, G = 4 * H, C = N / QW, NJ = C / 4, kTThreads = 128 * QW;
-  static_assert(C % 4 == 0, "whole 4-row blocks per warp");
+  constexpr int H = kTH, G = 4 * H, QW = 4, C = N / QW, P = N / 16, kTThreads = 512;
   constexpr uint32_t idesc = tc_idesc<N>();
   extern __shared__ __align__(16) uint8_t smem[];
   uint8_t *Bb = smem + Lay::oB;
   uint8_t *stg = smem + Lay::oStg;
+  float *gate = reinterpret_cast<float *>(smem + Lay::oGate);
   uint64_t *bar = reinterpret_cast<uint64_t *>(smem + Lay::oBar);
   uint32_t *tslot = reinterpret_cast<uint32_t *>(smem + Lay::oSlot);
   int *rlen = reinterpret_cast<int *>(smem + Lay::oLen);
   int *toff_s = reinterpret_cast<int *>(smem + Lay::oToff);
 
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
-  const int qt = warp & 3, cs = warp >> 2;
-  const int m = 32 * qt + lane, u = m >> 2, q = m & 3;  // TMEM lane m = gate row q H + 32c + u
-  const int col0 = C * cs;                              // this thread's first column (row of the group)
+  const int q = warp & 3, cs = warp >> 2;  // TMEM lane quarter = gate; column slice
+  const int col0 = C * cs;
   const uint32_t c = cluster_rank();
-  const int gu = (int)c * kTHc + u;
+  const int gu = (int)c * kTHc + lane;      // the unit of this lane (both phases)
   const int n_groups = (a.ix.b + N - 1) / N;
   const int cid = blockIdx.x / kTCS;
   const int d = cid / n_groups, r0 = (cid % n_groups) * N;
@@ -252,7 +257,6 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_fwd_tc_kernel(RecArgs a) {
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  // zero the B operands (rows past the batch stay zero), stage the index
   for (uint32_t i = t; i < 4 * Lay::kB / 16; i += kTThreads) reinterpret_cast<uint4 *>(Bb)[i] = make_uint4(0, 0, 0, 0);
   if (toff_sm)
     for (int i = t; i <= T; i += kTThreads) toff_s[i] = a.ix.tok_off[i];
@@ -260,7 +264,7 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_fwd_tc_kernel(RecArgs a) {
   if (t == 0) {
     mb_init(sa(&bar[0]), 1);
     mb_init(sa(&bar[1]), 1);
-    mb_init(sa(&bar[2]), 3);  // one commit from each of the three MMA issuers
+    mb_init(sa(&bar[2]), 3);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   fence_proxy();
@@ -268,10 +272,8 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_fwd_tc_kernel(RecArgs a) {
   __syncthreads();
   fence_after();
   const uint32_t tmem = *tslot;
-  const uint32_t tl = tmem + ((uint32_t)(32 * qt) << 16);  // this warp's TMEM lanes
-  // W_hh slice into TMEM (warps of the first column slice): row q H + gu,
-  // split into bf16 hi (columns 0..127) and lo (128..255), two k per column
-  // (low half = even k)
+  const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16);
+  // W_hh slice into TMEM: lane 32 q + u holds row q H + 32c + u
   if (cs == 0) {
     const float *wrow = a.Whh[d] + (size_t)(q * H + gu) * H;
 #pragma unroll 1
@@ -295,10 +297,10 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_fwd_tc_kernel(RecArgs a) {
     }
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
   }
-  fence_before();  // the slice is in TMEM before the issuers' MMAs read it
+  fence_before();
   __syncthreads();
   const int Tg = rlen[0];
-  cluster_sync_all();  // barriers and buffers ready everywhere before any remote store
+  cluster_sync_all();
   if (t == 0) {
     if (Tg >= 2) mb_arm(sa(&bar[0]), Lay::kStepBytes);
     if (Tg >= 3) mb_arm(sa(&bar[1]), Lay::kStepBytes);
@@ -309,23 +311,19 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_fwd_tc_kernel(RecArgs a) {
   float *__restrict__ Y = a.Y;
   __nv_bfloat16 *__restrict__ Yb = reinterpret_cast<__nv_bfloat16 *>(a.Yb);
   __nv_bfloat16 *__restrict__ Hs = reinterpret_cast<__nv_bfloat16 *>(a.Hs[d]);
-  int len[C], lenq[NJ];  // lengths of this thread's columns; of its rows col0 + 4 j + q
+  int len[C], lenp[P];  // lengths of this thread's gate columns and cell rows
 #pragma unroll
   for (int k = 0; k < C; ++k) len[k] = rlen[col0 + k];
 #pragma unroll
-  for (int j = 0; j < NJ; ++j) lenq[j] = rlen[col0 + 4 * j + q];
+  for (int j = 0; j < P; ++j) lenp[j] = rlen[P * warp + j];
   auto tok_col = [&](int k, int s) { return toff[d == 0 ? s : len[k] - 1 - s] + r0 + col0 + k; };
-  auto tok_q = [&](int j, int s) { return toff[d == 0 ? s : lenq[j] - 1 - s] + r0 + col0 + 4 * j + q; };
+  auto tok_row = [&](int j, int s) { return toff[d == 0 ? s : lenp[j] - 1 - s] + r0 + P * warp + j; };
   float zn[C];
 #pragma unroll
   for (int k = 0; k < C; ++k) zn[k] = 0 < len[k] ? Z[(size_t)tok_col(k, 0) * G + q * H + gu] : 0.f;
-  float cst[NJ];
+  float cst[P];
 #pragma unroll
-  for (int j = 0; j < NJ; ++j) cst[j] = 0.f;
-  const float scale = q == 2 ? 2.f : 1.f;  // tanh(x) = 2 sigma(2x) - 1 for the g gate
-  // MMA issuers: lane 0 of warps 0, 1, 2 issue the products W_hi h_hi,
-  // W_hi h_lo and W_lo h_hi into their own accumulators (columns kAccCol +
-  // 32 p), which the epilogue adds
+  for (int j = 0; j < P; ++j) cst[j] = 0.f;
   const int prod = (lane == 0 && warp < 3) ? warp : -1;
   bool ok = true, stop = false;
   int mma_issued = 0, mma_seen = 0;
@@ -347,11 +345,11 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_fwd_tc_kernel(RecArgs a) {
           fence_proxy();
           fence_after();
           const uint32_t bh = sa(Bb + (2 * (e & 1)) * Lay::kB);
-          const uint32_t bsel = bh + (prod == 1 ? Lay::kB : 0u);   // h_lo for W_hi h_lo
-          const uint32_t asel = tmem + (prod == 2 ? 128u : 0u);    // W_lo for W_lo h_hi
+          const uint32_t bsel = bh + (prod == 1 ? Lay::kB : 0u);
+          const uint32_t asel = tmem + (prod == 2 ? 128u : 0u);
           const uint32_t dcol = tmem + kAccCol + 32u * (uint32_t)prod;
 #pragma unroll
-          for (int j = 0; j < H / 16; ++j)  // k-step j: K columns 16 j .. 16 j + 15 (8 TMEM columns)
+          for (int j = 0; j < H / 16; ++j)
             mma_ts(dcol, asel + 8 * j, desc_kmajor(bsel + (uint32_t)(2 * j) * (16u * N), 16 * N, 128), idesc, j > 0);
           mma_commit(sa(&bar[2]));
         } else {
@@ -366,54 +364,12 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_fwd_tc_kernel(RecArgs a) {
 #pragma unroll
       for (int p = 0; p < 3; ++p) tmem_ld_add<C>(tl + kAccCol + 32 * p + col0, acc);
     }
-    // this lane's gate for each of its columns, written where the row is still running
-    float act[C];
+    // gate q of unit `lane` for this thread's columns (uniform per warp)
 #pragma unroll
     for (int k = 0; k < C; ++k) {
-      const float sg = sigm_tc(scale * acc[k]);
-      act[k] = fmaf(scale, sg, 1.f - scale);
-      if (s < len[k]) Z[(size_t)tok_col(k, s) * G + q * H + gu] = act[k];
-    }
-    // four lanes of a unit swap gates: lane q ends with gates i, f, g, o of
-    // rows col0 + 4 j + q (round r: send the gate value of row 4 j + (q ^ r),
-    // receive gate q ^ r of row 4 j + q from lane q ^ r)
-    const uint32_t par = (uint32_t)(s & 1);
-    uint8_t *sg_hi = stg + (2 * par) * Lay::kSlice, *sg_lo = sg_hi + Lay::kSlice;
-#pragma unroll
-    for (int j = 0; j < NJ; ++j) {
-      float g4[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int r = 0; r < 4; ++r) {
-        const int qs = q ^ r;
-        const float send = sel4(act[4 * j], act[4 * j + 1], act[4 * j + 2], act[4 * j + 3], qs);
-        const float recv = r == 0 ? send : __shfl_xor_sync(0xffffffffu, send, r);
-#pragma unroll
-        for (int k = 0; k < 4; ++k) g4[k] = (k == qs) ? recv : g4[k];
-      }
-      const int n = col0 + 4 * j + q;
-      const float cn = fmaf(g4[1], cst[j], g4[0] * g4[2]);
-      float h = g4[3] * tanh_tc(cn);
-      __nv_bfloat16 hh, hl;
-      if (s < lenq[j]) {
-        cst[j] = cn;
-        const size_t tk = (size_t)tok_q(j, s);
-        Cs[tk * H + gu] = cn;
-        Y[tk * DH + d * H + gu] = h;
-        split_bf16(h, hh, hl);
-        // bf16 copies for the bf16 contractions: Y, and h as the h_{t-1} of
-        // the row's next token in this direction (zero before its first)
-        if (Yb) Yb[tk * DH + d * H + gu] = hh;
-        if (Hs) {
-          if (s == 0) Hs[tk * H + gu] = __float2bfloat16_rn(0.f);
-          if (s + 1 < lenq[j]) Hs[(size_t)tok_q(j, s + 1) * H + gu] = hh;
-        }
-      } else {
-        h = 0.f;
-        split_bf16(h, hh, hl);
-      }
-      const uint32_t off = (uint32_t)(u >> 3) * (16u * N) + (uint32_t)n * 16u + (uint32_t)(u & 7) * 2u;
-      *reinterpret_cast<__nv_bfloat16 *>(sg_hi + off) = hh;
-      *reinterpret_cast<__nv_bfloat16 *>(sg_lo + off) = hl;
+      const float g = q == 2 ? tanh_tc(acc[k]) : sigm_tc(acc[k]);
+      if (s < len[k]) Z[(size_t)tok_col(k, s) * G + q * H + gu] = g;
+      gate[((col0 + k) * 4 + q) * kTHc + lane] = g;
     }
     fence_before();
     if (__syncthreads_or(!ok)) {
@@ -421,9 +377,39 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_fwd_tc_kernel(RecArgs a) {
       stop = true;
       break;
     }
+    // cell update of unit `lane`, rows P warp + j
+    const uint32_t par = (uint32_t)(s & 1);
+    uint8_t *sg_hi = stg + (2 * par) * Lay::kSlice, *sg_lo = sg_hi + Lay::kSlice;
+#pragma unroll
+    for (int j = 0; j < P; ++j) {
+      const int n = P * warp + j;
+      const float ig = gate[(n * 4 + 0) * kTHc + lane], fg = gate[(n * 4 + 1) * kTHc + lane];
+      const float gg = gate[(n * 4 + 2) * kTHc + lane], og = gate[(n * 4 + 3) * kTHc + lane];
+      const float cn = fmaf(fg, cst[j], ig * gg);
+      float h = og * tanh_tc(cn);
+      __nv_bfloat16 hh, hl;
+      if (s < lenp[j]) {
+        cst[j] = cn;
+        const size_t tk = (size_t)tok_row(j, s);
+        Cs[tk * H + gu] = cn;
+        Y[tk * DH + d * H + gu] = h;
+        split_bf16(h, hh, hl);
+        if (Yb) Yb[tk * DH + d * H + gu] = hh;
+        if (Hs) {
+          if (s == 0) Hs[tk * H + gu] = __float2bfloat16_rn(0.f);
+          if (s + 1 < lenp[j]) Hs[(size_t)tok_row(j, s + 1) * H + gu] = hh;
+        }
+      } else {
+        h = 0.f;
+        split_bf16(h, hh, hl);
+      }
+      const uint32_t off = (uint32_t)(lane >> 3) * (16u * N) + (uint32_t)n * 16u + (uint32_t)(lane & 7) * 2u;
+      *reinterpret_cast<__nv_bfloat16 *>(sg_hi + off) = hh;
+      *reinterpret_cast<__nv_bfloat16 *>(sg_lo + off) = hl;
+    }
+    __syncthreads();
     if (s + 1 < Tg && !withhold) {
-      // h_t of this CTA's units to every CTA of the cluster (itself included)
-      constexpr int kPieces = 2 * Lay::kSlice / 16;  // per destination
+      constexpr int kPieces = 2 * Lay::kSlice / 16;
       const uint32_t dst0 = sa(Bb + (2 * par) * Lay::kB) + c * (uint32_t)Lay::kSlice;
       const uint32_t mbl = sa(&bar[par]);
 #pragma unroll
@@ -434,21 +420,18 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_fwd_tc_kernel(RecArgs a) {
       }
     }
   }
-  // an MMA batch whose completion was not observed may still be running:
-  // wait for it (bounded) before TMEM is released
   if (mma_seen < mma_issued) mb_wait(sa(&bar[2]), (uint32_t)((mma_issued - 1) & 1), kTPolls);
-  if (stop) __nanosleep(20000);  // peers' in-flight stores after an abort
+  if (stop) __nanosleep(20000);
   fence_before();
   cluster_sync_all();
   fence_after();
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
 }
 
-template <int N, int QW>
-__global__ void __launch_bounds__(128 * QW, 1) lstm_bwd_tc_kernel(RecArgs a) {
+template <int N>
+__global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
   using Lay = TcBwdLayout<N>;
-  constexpr int H = kTH, G = 4 * H, C = N / QW, NJ = C / 4, RS = Lay::kRS, kTThreads = 128 * QW;
-  static_assert(C % 4 == 0, "whole 4-row blocks per warp");
+  constexpr int H = kTH, G = 4 * H, QW = 4, C = N / QW, P = N / 16, RS = Lay::kRS, kTThreads = 512;
   constexpr uint32_t idesc = tc_idesc<N>();
   extern __shared__ __align__(16) uint8_t smem[];
   uint8_t *Bz = smem + Lay::oB;
@@ -461,8 +444,8 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_bwd_tc_kernel(RecArgs a) {
 
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int qt = warp & 3, cs = warp >> 2;
-  const int m = 32 * qt + lane, u = m >> 2, q = m & 3;  // phase B: unit u, rows col0 + 4 j + q
   const int col0 = C * cs;
+  const int u = lane;  // phase B: unit `lane`, rows P warp + j
   const uint32_t c = cluster_rank();
   const int gu = (int)c * kTHc + u;
   const int n_groups = (a.ix.b + N - 1) / N;
@@ -500,7 +483,7 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_bwd_tc_kernel(RecArgs a) {
   if (cs < 2) {
     const int hf = cs;
     const float *W = a.Whh[d];
-    const int col = 128 * hf + m;
+    const int col = 128 * hf + 32 * qt + lane;
 #pragma unroll 1
     for (int k0 = 0; k0 < 128; k0 += 16) {
       uint32_t hi[8], lo[8];
@@ -533,16 +516,16 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_bwd_tc_kernel(RecArgs a) {
   const float *__restrict__ Cs = a.Cst[d];
   const float *__restrict__ dY = a.dY;
   __nv_bfloat16 *__restrict__ dZb = reinterpret_cast<__nv_bfloat16 *>(a.dZb[d]);
-  int len[NJ];  // lengths of this thread's rows col0 + 4 j + q
+  int len[P];  // lengths of this thread's rows P warp + j
 #pragma unroll
-  for (int j = 0; j < NJ; ++j) len[j] = rlen[col0 + 4 * j + q];
-  auto tok_at = [&](int j, int s) { return toff[d == 0 ? s : len[j] - 1 - s] + r0 + col0 + 4 * j + q; };
+  for (int j = 0; j < P; ++j) len[j] = rlen[P * warp + j];
+  auto tok_at = [&](int j, int s) { return toff[d == 0 ? s : len[j] - 1 - s] + r0 + P * warp + j; };
   // phase B inputs of a step, loaded one step ahead: gates i, f, g, o, c_t,
   // c_{t-1} (in this direction's order), dY
-  float in[NJ][7], nx[NJ][7];
-  auto load_in = [&](int s, float (&v)[NJ][7]) {
+  float in[P][7], nx[P][7];
+  auto load_in = [&](int s, float (&v)[P][7]) {
 #pragma unroll
-    for (int j = 0; j < NJ; ++j) {
+    for (int j = 0; j < P; ++j) {
       if (s >= 0 && s < len[j]) {
         const size_t tk = (size_t)tok_at(j, s);
 #pragma unroll
@@ -557,9 +540,9 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_bwd_tc_kernel(RecArgs a) {
     }
   };
   load_in(Tg - 1, nx);
-  float dc[NJ];
+  float dc[P];
 #pragma unroll
-  for (int j = 0; j < NJ; ++j) dc[j] = 0.f;
+  for (int j = 0; j < P; ++j) dc[j] = 0.f;
   // MMA issuers: lane 0 of warps 0..5, issuer i forms product i % 3 (W_hi dz_hi,
   // W_hi dz_lo, W_lo dz_hi) of half i / 3 into columns kAccCol + 32 i
   const int iss = (lane == 0 && warp < 6) ? warp : -1;
@@ -570,7 +553,7 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_bwd_tc_kernel(RecArgs a) {
   for (int it = 0; it < Tg && !stop; ++it) {
     const int s = Tg - 1 - it;
 #pragma unroll
-    for (int j = 0; j < NJ; ++j)
+    for (int j = 0; j < P; ++j)
 #pragma unroll
       for (int g = 0; g < 7; ++g) in[j][g] = nx[j][g];
     load_in(s - 1, nx);
@@ -581,10 +564,10 @@ __global__ void __launch_bounds__(128 * QW, 1) lstm_bwd_tc_kernel(RecArgs a) {
       if (t == 0 && ok && e + 2 <= Tg - 2) mb_arm(sa(&bar[e & 1]), Lay::kStepBytes);
       rp = red + (size_t)(e & 1) * (kTCS * N * RS) + u;
     }
-    // phase B: dh, dc and dz of unit u for rows col0 + 4 j + q
+    // phase B: dh, dc and dz of unit u for rows P warp + j
 #pragma unroll
-    for (int j = 0; j < NJ; ++j) {
-      const int n = col0 + 4 * j + q;
+    for (int j = 0; j < P; ++j) {
+      const int n = P * warp + j;
       float dz4[4] = {0.f, 0.f, 0.f, 0.f};
       if (s < len[j]) {
         float dh = in[j][6];
@@ -713,29 +696,30 @@ size_t tc_smem(bool bwd, int T) {
   return tc_smem_bytes(bwd ? TcBwdLayout<N>::oToff : TcFwdLayout<N>::oToff, T);
 }
 
-template <int N, int QW>
+template <int N>
 cudaError_t launch_tc(const RecArgs &a, bool bwd, cudaStream_t s) {
   if (a.ix.b <= 0 || a.ix.T <= 0) return cudaSuccess;
   if (a.H != kTH) return cudaErrorInvalidValue;
   const size_t smem = tc_smem<N>(bwd, a.ix.T);
   const int clusters = ((a.ix.b + N - 1) / N) * a.dirs;
   cudaLaunchAttribute attr;
+
   if (bwd) {
-    auto k = lstm_bwd_tc_kernel<N, QW>;
+    auto k = lstm_bwd_tc_kernel<N>;
     cudaError_t e = ensure_smem((const void *)k, smem);
     if (e != cudaSuccess) return e;
-    cudaLaunchConfig_t cfg = tc_config<decltype(k)>(clusters, 128 * QW, smem, s, &attr);
+    cudaLaunchConfig_t cfg = tc_config<decltype(k)>(clusters, 512, smem, s, &attr);
     return cudaLaunchKernelEx(&cfg, k, a);
   }
-  auto k = lstm_fwd_tc_kernel<N, QW>;
+  auto k = lstm_fwd_tc_kernel<N>;
   cudaError_t e = ensure_smem((const void *)k, smem);
   if (e != cudaSuccess) return e;
-  cudaLaunchConfig_t cfg = tc_config<decltype(k)>(clusters, 128 * QW, smem, s, &attr);
+  cudaLaunchConfig_t cfg = tc_config<decltype(k)>(clusters, 512, smem, s, &attr);
   return cudaLaunchKernelEx(&cfg, k, a);
 }
 
 // 8-CTA clusters of both kernels that can be resident at once (0: cannot launch).
-template <int N, int QW>
+template <int N>
 int tc_resident() {
   int lo = 1 << 30;
   for (int bwd = 0; bwd < 2; ++bwd) {
@@ -744,14 +728,14 @@ int tc_resident() {
     int n = 0;
     cudaError_t e;
     if (bwd) {
-      auto k = lstm_bwd_tc_kernel<N, QW>;
+      auto k = lstm_bwd_tc_kernel<N>;
       e = ensure_smem((const void *)k, smem);
-      cudaLaunchConfig_t cfg = tc_config<decltype(k)>(1, 128 * QW, smem, 0, &attr);
+      cudaLaunchConfig_t cfg = tc_config<decltype(k)>(1, 512, smem, 0, &attr);
       if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, k, &cfg);
     } else {
-      auto k = lstm_fwd_tc_kernel<N, QW>;
+      auto k = lstm_fwd_tc_kernel<N>;
       e = ensure_smem((const void *)k, smem);
-      cudaLaunchConfig_t cfg = tc_config<decltype(k)>(1, 128 * QW, smem, 0, &attr);
+      cudaLaunchConfig_t cfg = tc_config<decltype(k)>(1, 512, smem, 0, &attr);
       if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, k, &cfg);
     }
     if (e != cudaSuccess) {
@@ -761,17 +745,6 @@ int tc_resident() {
     lo = std::min(lo, n);
   }
   return lo;
-}
-
-// Warps per TMEM lane quarter at 32 rows per cluster: 4 (512 threads; BKT_TC_QW=8
-// selects 1024 threads, measured no faster: the step is bound by the SM's
-// elementwise and exchange throughput, not by latency within a warp).
-int tc_qw32() {
-  static const int qw = [] {
-    const char *e = getenv("BKT_TC_QW");
-    return (e && atoi(e) == 8) ? 8 : 4;
-  }();
-  return qw;
 }
 
 }  // namespace
@@ -789,15 +762,15 @@ int plan_tc_rows(int b, int dirs) {
   // not its columns, bounds it), so fewer, wider clusters leave SMs to the
   // side stream; 16 when the batch is small enough for its clusters to fit
   // either way (0: neither can launch)
-  const int r16 = tc_resident<16, 4>(), r32 = tc_qw32() == 8 ? tc_resident<32, 8>() : tc_resident<32, 4>();
+  const int r16 = tc_resident<16>(), r32 = tc_resident<32>();
   if (r16 > 0 && ((b + 15) / 16) * dirs <= std::min(r16, 4)) return 16;
   if (r32 > 0) return 32;
   return r16 > 0 ? 16 : 0;
 }
 
 cudaError_t launch_lstm_tc(const RecArgs &a, int rows, bool bwd, cudaStream_t s) {
-  if (rows == 16) return launch_tc<16, 4>(a, bwd, s);
-  if (rows == 32) return tc_qw32() == 8 ? launch_tc<32, 8>(a, bwd, s) : launch_tc<32, 4>(a, bwd, s);
+  if (rows == 16) return launch_tc<16>(a, bwd, s);
+  if (rows == 32) return launch_tc<32>(a, bwd, s);
   return cudaErrorInvalidValue;
 }
 
