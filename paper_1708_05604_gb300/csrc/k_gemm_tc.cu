@@ -35,11 +35,14 @@ namespace bkt {
 
 namespace {
 
-constexpr int TBM = 128, TBN = 256, TBK = 64, TSTAGES = 4;
+constexpr int TBM = 128, TBN = 256, TBK = 64;
 constexpr uint32_t kAStage = TBM * TBK * 2;  // 16 KB
 constexpr uint32_t kBStage = TBN * TBK * 2;  // 32 KB
 constexpr uint32_t kTxBytes = kAStage + kBStage;
-constexpr size_t kTcSmem = 1024 + (size_t)TSTAGES * (kAStage + kBStage) + 256;
+// 4 stages for long-K contractions (one CTA per SM); 2 stages (97 KB) for the
+// many short-K tiles of the projections and dX, so that two CTAs share an SM
+// and one's epilogue overlaps the other's loads and MMAs
+constexpr size_t tc_smem_for(int stages) { return 1024 + (size_t)stages * (kAStage + kBStage) + 256; }
 constexpr uint32_t kWaitPolls = 1u << 22;
 // kind::f16 instruction descriptor: D fp32 (bit 4), A and B bf16 (bits 7, 10),
 // K-major unless bit 15 (A) / bit 16 (B) marks an MN-major operand, N >> 3 at
@@ -156,7 +159,8 @@ __device__ __forceinline__ void tc_mma_tf32(uint32_t d, uint64_t a, uint64_t b, 
 
 }  // namespace
 
-__global__ void __launch_bounds__(128, 1)
+template <int TSTAGES>
+__global__ void __launch_bounds__(128, TSTAGES <= 2 ? 2 : 1)
     gemm_bf16_tc_kernel(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb, TcGemmArgs g) {
   extern __shared__ uint8_t tc_smem_raw[];
   uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(tc_smem_raw) + 1023) & ~uintptr_t(1023));
@@ -262,51 +266,76 @@ __global__ void __launch_bounds__(128, 1)
     __syncwarp();
   }
 
-  // epilogue: TMEM -> registers -> global
-  const bool ready = mbar_wait(done, 0, cap);
-  if (!ready) *abort_s = 1;
+  // epilogue: TMEM -> registers -> shared memory -> global.  TMEM lane = tile
+  // row, so a thread holds one row; each 32-column chunk goes through a
+  // per-warp staging block (the idle A stages: every MMA has completed) and
+  // leaves as float4 stores that cover four whole 128-byte row pieces per
+  // instruction (one row per thread would touch 32 rows per instruction)
+  const bool ready_t = mbar_wait(done, 0, cap);
+  if (!ready_t) *abort_s = 1;
+  const bool ready = __all_sync(0xffffffffu, ready_t);  // uniform per warp: the chunk loop below syncs the warp
   tc_fence_after();
-  const int row = warp * 32 + lane;
-  const int m = m0 + row;
   const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
-  const bool write = ready && m < g.M;
-  float *out;
+  float *out_base;
   int64_t ld;
   if (g.P) {
-    out = g.P + (int64_t)blockIdx.z * g.M * g.N + (int64_t)m * g.N;
+    out_base = g.P + (int64_t)blockIdx.z * g.M * g.N;
     ld = g.N;
   } else {
-    out = g.D + (int64_t)m * g.ldd;
+    out_base = g.D;
     ld = g.ldd;
   }
-  const bool vec = ((ld & 3) == 0) && ((reinterpret_cast<uintptr_t>(g.P ? g.P : g.D) & 15) == 0);
+  const bool vec = ((ld & 3) == 0) && ((reinterpret_cast<uintptr_t>(out_base) & 15) == 0);
+  constexpr int kSt = 36;  // staging row stride (floats): 16-byte pieces of 8 consecutive rows hit distinct banks
+  float *stg = reinterpret_cast<float *>(sA) + warp * 32 * kSt;
+  const int cq = lane & 7, rq = lane >> 3;  // write phase: columns 4 cq .. 4 cq + 3 of rows rq + 4 i
 #pragma unroll 1
   for (int c0 = 0; c0 < TBN; c0 += 32) {
     uint32_t v[32];
     __syncwarp();
     tmem_ld32(trow + c0, v);
-    if (!write) continue;
     const int nb = n0 + c0;
-    if (nb >= g.N) continue;
-    float x[32];
+    if (!ready || nb >= g.N) continue;  // uniform across the warp
 #pragma unroll
-    for (int j = 0; j < 32; ++j) x[j] = nk > 0 ? __uint_as_float(v[j]) : 0.f;
-    if (!g.P) {
-      if (g.bias)
-#pragma unroll
-        for (int j = 0; j < 32; ++j) x[j] += (nb + j < g.N) ? g.bias[nb + j] : 0.f;
-      if (g.accumulate)
-#pragma unroll
-        for (int j = 0; j < 32; ++j) x[j] += (nb + j < g.N) ? out[nb + j] : 0.f;
+    for (int j = 0; j < 32; j += 4)
+      *reinterpret_cast<float4 *>(stg + lane * kSt + j) =
+          nk > 0 ? make_float4(__uint_as_float(v[j]), __uint_as_float(v[j + 1]), __uint_as_float(v[j + 2]),
+                               __uint_as_float(v[j + 3]))
+                 : make_float4(0.f, 0.f, 0.f, 0.f);
+    __syncwarp();
+    const int n = nb + 4 * cq;
+    float4 bias4 = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (!g.P && g.bias) {
+      bias4.x = n < g.N ? g.bias[n] : 0.f;
+      bias4.y = n + 1 < g.N ? g.bias[n + 1] : 0.f;
+      bias4.z = n + 2 < g.N ? g.bias[n + 2] : 0.f;
+      bias4.w = n + 3 < g.N ? g.bias[n + 3] : 0.f;
     }
-    if (vec && nb + 32 <= g.N) {
 #pragma unroll
-      for (int j = 0; j < 32; j += 4)
-        *reinterpret_cast<float4 *>(out + nb + j) = make_float4(x[j], x[j + 1], x[j + 2], x[j + 3]);
-    } else {
+    for (int i = 0; i < 8; ++i) {
+      const int r = rq + 4 * i, m = m0 + warp * 32 + r;
+      if (m >= g.M) continue;
+      float4 x = *reinterpret_cast<const float4 *>(stg + r * kSt + 4 * cq);
+      x.x += bias4.x;
+      x.y += bias4.y;
+      x.z += bias4.z;
+      x.w += bias4.w;
+      float *o = out_base + (int64_t)m * ld + n;
+      if (vec && n + 4 <= g.N) {
+        if (!g.P && g.accumulate) {
+          const float4 y = *reinterpret_cast<const float4 *>(o);
+          x.x += y.x;
+          x.y += y.y;
+          x.z += y.z;
+          x.w += y.w;
+        }
+        *reinterpret_cast<float4 *>(o) = x;
+      } else {
+        const float xs[4] = {x.x, x.y, x.z, x.w};
 #pragma unroll
-      for (int j = 0; j < 32; ++j)
-        if (nb + j < g.N) out[nb + j] = x[j];
+        for (int j = 0; j < 4; ++j)
+          if (n + j < g.N) o[j] = xs[j] + ((!g.P && g.accumulate) ? o[j] : 0.f);
+      }
     }
   }
   tc_fence_before();
@@ -770,11 +799,19 @@ cudaError_t launch_gemm_bf16_tc(const TcGemmArgs &g, cudaStream_t s) {
   const bool okB = g.b_mn ? make_map(&tb, g.B, (uint64_t)g.N, (uint64_t)g.K, g.ldb, TBK)
                           : make_map(&tb, g.B, (uint64_t)g.K, (uint64_t)g.N, g.ldb, TBN);
   if (!okA || !okB) return cudaErrorInvalidValue;
-  cudaError_t e = ensure_smem((const void *)gemm_bf16_tc_kernel, kTcSmem);
-  if (e != cudaSuccess) return e;
   dim3 grid((g.M + TBM - 1) / TBM, (g.N + TBN - 1) / TBN, g.P ? g.splits : 1);
   if (grid.y > 65535u || grid.z > 65535u) return cudaErrorInvalidConfiguration;
-  gemm_bf16_tc_kernel<<<grid, 128, kTcSmem, s>>>(ta, tb, g);
+  const int nkb = (g.K + TBK - 1) / TBK;
+  const bool short_k = !g.P && nkb <= 16 && (int64_t)grid.x * grid.y >= 512;
+  if (short_k) {
+    cudaError_t e = ensure_smem((const void *)gemm_bf16_tc_kernel<2>, tc_smem_for(2));
+    if (e != cudaSuccess) return e;
+    gemm_bf16_tc_kernel<2><<<grid, 128, tc_smem_for(2), s>>>(ta, tb, g);
+  } else {
+    cudaError_t e = ensure_smem((const void *)gemm_bf16_tc_kernel<4>, tc_smem_for(4));
+    if (e != cudaSuccess) return e;
+    gemm_bf16_tc_kernel<4><<<grid, 128, tc_smem_for(4), s>>>(ta, tb, g);
+  }
   return cudaGetLastError();
 }
 

@@ -41,7 +41,7 @@
 // kernels); on an abort the kernel still waits for its last MMA batch before
 // it frees TMEM, sleeps 20 us so peers' in-flight stores land, and meets its
 // peers at a final cluster barrier.  A CTA takes all 512 TMEM columns; its
-// shared-memory request (>= 120 KB) keeps any other CTA off its SM.
+// shared-memory request (>= 140 KB) keeps any other TMEM user off its SM.
 #include <cuda_bf16.h>
 
 #include <cstdint>
@@ -59,7 +59,9 @@ constexpr int kTCS = 8;            // CTAs per cluster
 constexpr int kTHc = kTH / kTCS;   // units per CTA
 constexpr int kTTokCap = 8192;     // time offsets staged in shared memory up to this T
 constexpr int kTPolls = 1 << 22;
-constexpr size_t kTSmemFloor = 120 * 1024;  // one CTA per SM: each CTA holds all of TMEM
+// One CTA per SM, and no bf16 GEMM CTA (97 KB at its smallest) beside it:
+// each CTA holds all of TMEM for the whole sequence.
+constexpr size_t kTSmemFloor = 140 * 1024;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAccCol = 256;  // first accumulator column (A operands take 0 .. 255)
 
