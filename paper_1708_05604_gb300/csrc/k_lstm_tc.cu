@@ -320,9 +320,14 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
   for (int j = 0; j < P; ++j) lenp[j] = rlen[P * warp + j];
   auto tok_col = [&](int k, int s) { return toff[d == 0 ? s : len[k] - 1 - s] + r0 + col0 + k; };
   auto tok_row = [&](int j, int s) { return toff[d == 0 ? s : lenp[j] - 1 - s] + r0 + P * warp + j; };
-  float zn[C];
+  // Zx of the next two steps in registers (DRAM latency under the step's own
+  // traffic exceeds one step)
+  float zn[C], zn2[C];
 #pragma unroll
-  for (int k = 0; k < C; ++k) zn[k] = 0 < len[k] ? Z[(size_t)tok_col(k, 0) * G + q * H + gu] : 0.f;
+  for (int k = 0; k < C; ++k) {
+    zn[k] = 0 < len[k] ? Z[(size_t)tok_col(k, 0) * G + q * H + gu] : 0.f;
+    zn2[k] = 1 < len[k] ? Z[(size_t)tok_col(k, 1) * G + q * H + gu] : 0.f;
+  }
   float cst[P];
 #pragma unroll
   for (int j = 0; j < P; ++j) cst[j] = 0.f;
@@ -333,10 +338,13 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
   for (int s = 0; s < Tg && !stop; ++s) {
     float acc[C];
 #pragma unroll
-    for (int k = 0; k < C; ++k) acc[k] = zn[k];
-    if (s + 1 < Tg) {
+    for (int k = 0; k < C; ++k) {
+      acc[k] = zn[k];
+      zn[k] = zn2[k];
+    }
+    if (s + 2 < Tg) {
 #pragma unroll
-      for (int k = 0; k < C; ++k) zn[k] = s + 1 < len[k] ? Z[(size_t)tok_col(k, s + 1) * G + q * H + gu] : 0.f;
+      for (int k = 0; k < C; ++k) zn2[k] = s + 2 < len[k] ? Z[(size_t)tok_col(k, s + 2) * G + q * H + gu] : 0.f;
     }
     if (s > 0) {
       const int e = s - 1;
@@ -522,10 +530,10 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
 #pragma unroll
   for (int j = 0; j < P; ++j) len[j] = rlen[P * warp + j];
   auto tok_at = [&](int j, int s) { return toff[d == 0 ? s : len[j] - 1 - s] + r0 + P * warp + j; };
-  // phase B inputs of a step, loaded one step ahead: gates i, f, g, o, c_t,
-  // c_{t-1} (in this direction's order), dY
-  float in[P][7], nx[P][7];
-  auto load_in = [&](int s, float (&v)[P][7]) {
+  // phase B inputs of a step, loaded two steps ahead: gates i, f, g, o,
+  // c_t, dY (c_{t-1} is the next step's c_t, zero before the first step)
+  float in[P][6], nx[P][6], nx2[P][6];
+  auto load_in = [&](int s, float (&v)[P][6]) {
 #pragma unroll
     for (int j = 0; j < P; ++j) {
       if (s >= 0 && s < len[j]) {
@@ -533,15 +541,15 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
 #pragma unroll
         for (int g = 0; g < 4; ++g) v[j][g] = Z[tk * G + g * H + gu];
         v[j][4] = Cs[tk * H + gu];
-        v[j][5] = s > 0 ? Cs[(size_t)tok_at(j, s - 1) * H + gu] : 0.f;
-        v[j][6] = dY[tk * DH + d * H + gu];
+        v[j][5] = dY[tk * DH + d * H + gu];
       } else {
 #pragma unroll
-        for (int g = 0; g < 7; ++g) v[j][g] = 0.f;
+        for (int g = 0; g < 6; ++g) v[j][g] = 0.f;
       }
     }
   };
   load_in(Tg - 1, nx);
+  load_in(Tg - 2, nx2);
   float dc[P];
 #pragma unroll
   for (int j = 0; j < P; ++j) dc[j] = 0.f;
@@ -557,8 +565,11 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
 #pragma unroll
     for (int j = 0; j < P; ++j)
 #pragma unroll
-      for (int g = 0; g < 7; ++g) in[j][g] = nx[j][g];
-    load_in(s - 1, nx);
+      for (int g = 0; g < 6; ++g) {
+        in[j][g] = nx[j][g];
+        nx[j][g] = nx2[j][g];
+      }
+    load_in(s - 2, nx2);
     const float *rp = nullptr;
     if (it > 0) {
       const int e = it - 1;
@@ -572,12 +583,13 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
       const int n = P * warp + j;
       float dz4[4] = {0.f, 0.f, 0.f, 0.f};
       if (s < len[j]) {
-        float dh = in[j][6];
+        float dh = in[j][5];
         if (rp) {
 #pragma unroll
           for (int src = 0; src < kTCS; ++src) dh += rp[((size_t)src * N + n) * RS];
         }
-        const float ig = in[j][0], fg = in[j][1], gg = in[j][2], og = in[j][3], ct = in[j][4], cp = in[j][5];
+        // c_{t-1}: the c_t of step s - 1 (zero when s is the row's first step)
+        const float ig = in[j][0], fg = in[j][1], gg = in[j][2], og = in[j][3], ct = in[j][4], cp = nx[j][4];
         const float tch = tanh_tc(ct);
         const float dcv = fmaf(dh * og, 1.f - tch * tch, dc[j]);
         dz4[0] = dcv * gg * ig * (1.f - ig);
