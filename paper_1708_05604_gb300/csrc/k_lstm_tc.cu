@@ -15,27 +15,36 @@
 // state, the gates and every elementwise step stay fp32).  W never leaves
 // the SM: per step only N rows of h (or dz) are read from shared memory.
 //
-// TMEM lane m = 4u + q holds gate row q H + 32c + u of the CTA (forward: A =
-// W slice, K = the 256 units; BPTT: A = W slice transposed in two 128-unit
-// halves, K = the CTA's 128 gate rows in the same 4u + q order).  Operands in
+// A cluster's rows form two teams of 16 rows (one team of 16 for batches of
+// at most 64 rows); each team runs its own recurrence on 8 of the CTA's 16
+// warps (its own MMAs, TMEM accumulators, exchange buffers, mbarriers and
+// named barrier), so that one team's MMAs and exchange overlap the other
+// team's elementwise work; the teams share only W in TMEM.
+//
+// Forward: TMEM lane 32 q + u holds gate row q H + 32c + u (A = the W slice,
+// K = the 256 units; hi part in columns 0 .. 127, lo part in 128 .. 255).
+// BPTT: A = the W slice transposed in two 128-unit halves (lane m = unit
+// 128 hf + m), K = the CTA's 128 gate rows in the order 4u + q.  Operands in
 // shared memory use the K-major layout without swizzle: 8 x 16-byte core
 // matrices, element (n, k) at (k / 8) * 16 N + n * 16 + (k % 8) * 2 bytes, so
 // the 32 units of one CTA are one contiguous 64 N-byte block.
 //
-// Forward step: one thread issues the 48 MMAs (16 k-steps of 16 x 3
-// products) once h_{t-1} has arrived and commits them to an mbarrier; the
-// 128 threads read the accumulator (thread = gate row, N columns), add Zx,
-// apply sigma / tanh, swap gates inside groups of four lanes so that each
-// lane holds the four gates of one unit for N / 4 rows, update the cell
-// state in registers, write gates, c_t and h_t, and stage h_t (bf16 hi and
-// lo) to send it to every CTA of the cluster with st.async (16-byte remote
-// stores completing bytes on the receiver's mbarrier; double-buffered by step
-// parity, so the data dependence orders buffer reuse).
+// Forward step: once h_{t-1} has arrived, three issuing threads (one per
+// product) issue 16 MMAs each into their own accumulators and commit them
+// to an mbarrier; each warp then reads one TMEM lane quarter (one gate for
+// the 32 units) for C rows, adds Zx, applies sigma or tanh, writes the
+// gates, and leaves them in shared memory, where thread (w, lane) finds the
+// four gates of unit `lane` for its rows, updates c in registers, writes c,
+// h and the bf16 copies, and stages h_t (bf16 hi and lo) for st.async
+// stores to every CTA of the cluster (16-byte remote stores completing
+// bytes on the receiver's mbarrier; double-buffered by step parity, so the
+// data dependence orders buffer reuse).
 // BPTT step: dh = dY + the sum of the 8 partials of W_hh^T dz_{t+1} received
-// for this CTA's units, then dc and dz of the four gates (fp32, written to
-// the gate buffer in place and, split, to the B operand); the MMAs form this
-// CTA's partial W_hh^T dz over its 128 gate rows for all 256 units (two
-// 128-lane halves), and each 32-unit block goes to the CTA that owns it.
+// for this CTA's units, then dc and dz of the four gates (fp32, written in
+// place of the gates and, split, to the B operand); four issuing threads
+// (six with one team) form this CTA's partial W_hh^T dz over its 128 gate
+// rows for all 256 units (two 128-lane halves), and each warp sends its
+// 16-byte pieces of the 32-unit blocks straight to the CTAs that own them.
 //
 // Every wait is bounded (status bit 4 on expiry, as in the other cluster
 // kernels); on an abort the kernel still waits for its last MMA batch before
@@ -174,11 +183,22 @@ __device__ __forceinline__ uint32_t pack2(__nv_bfloat16 a, __nv_bfloat16 b) {
 // recurrent kernels): sigma(x) = 1 / (1 + e^-x), tanh(x) = 2 sigma(2x) - 1.
 __device__ __forceinline__ float sigm_tc(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
 __device__ __forceinline__ float tanh_tc(float x) { return 1.f - __fdividef(2.f, 1.f + __expf(2.f * x)); }
-__device__ __forceinline__ float sel4(float a, float b, float c, float d, int i) {
-  return i == 0 ? a : i == 1 ? b : i == 2 ? c : d;
+
+// Named barrier of one team (id >= 1; id 0 is __syncthreads) of n threads,
+// and the same barrier returning the OR of a predicate over them.
+__device__ __forceinline__ void team_sync(int id, int n) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory"); }
+__device__ __forceinline__ bool team_sync_or(int id, int n, bool p) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred a, b;\n\tsetp.ne.u32 a, %1, 0;\n\tbar.red.or.pred b, %2, %3, a;\n\tselp.u32 %0, 1, 0, b;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)p), "r"(id), "r"(n)
+      : "memory");
+  return r != 0;
 }
 
-// Shared-memory layout (bytes).
+// Shared-memory layout (bytes): one region of kTeam bytes per team, then the
+// TMEM address slot, the lengths of the cluster's rows and the time offsets.
 template <int N>
 struct TcBwdLayout {
   static constexpr uint32_t kB = N * 128 * 2;      // one B operand (dz hi or lo): N rows x 128 gate rows
@@ -189,9 +209,27 @@ struct TcBwdLayout {
   static constexpr uint32_t oRed = oB + 2 * kB;    // [2 parity][8 src][N rows][kRS] fp32
   static constexpr uint32_t oStg = oRed + 2 * kRed;  // [8 owners][N rows][32 units] fp32 partials to send
   static constexpr uint32_t oBar = oStg + kTCS * N * kTHc * 4;  // rbar[2], mmabar
-  static constexpr uint32_t oSlot = oBar + 3 * 8;
+  static constexpr uint32_t kTeam = oBar + 32;
+};
+
+template <int N>
+struct TcFwdLayout {
+  static constexpr uint32_t kB = N * kTH * 2;
+  static constexpr uint32_t kSlice = 64 * N;
+  static constexpr uint32_t kStepBytes = kTCS * 2 * kSlice;
+  static constexpr uint32_t oB = 0;                    // [2 parity][2 hi/lo][kB]
+  static constexpr uint32_t oStg = oB + 4 * kB;        // [2 parity][2 hi/lo][kSlice]
+  static constexpr uint32_t oGate = oStg + 4 * kSlice; // [N][4][32] fp32 activated gates
+  static constexpr uint32_t oBar = oGate + N * 4 * kTHc * 4;  // xbar[2], mmabar
+  static constexpr uint32_t kTeam = oBar + 32;
+};
+
+template <typename L, int N, int TM>
+struct TcSmem {
+  static constexpr uint32_t oSlot = TM * L::kTeam;
   static constexpr uint32_t oLen = oSlot + 16;
-  static constexpr uint32_t oToff = oLen + 4 * N;
+  static constexpr uint32_t oToff = oLen + 4 * N * TM;
+  static_assert(L::kTeam % 16 == 0, "team regions keep 16-byte operand alignment");
 };
 
 size_t tc_smem_bytes(size_t base, int T) {
@@ -201,72 +239,77 @@ size_t tc_smem_bytes(size_t base, int T) {
 
 }  // namespace
 
-// Thread roles (both kernels, 512 threads): warp w reads TMEM lane quarter
-// w % 4 and columns C (w / 4) .. + C - 1 (C = N / 4) of each accumulator,
-// lane l of it TMEM lane 32 (w % 4) + l; the elementwise phases give thread
-// (w, l) unit l of the CTA's 32 and rows P w .. P w + P - 1 (P = N / 16).
+// Teams.  A CTA's 16 warps form TM teams of TW = 16 / TM warps; team k owns
+// N consecutive rows of the cluster's R = TM N and runs its own recurrence
+// over them: its own MMAs and accumulators, exchange buffers, mbarriers and
+// a named barrier, so that with two teams one team's MMAs and exchange wait
+// overlap the other team's elementwise work (they share W in TMEM only).
+// Thread roles inside a team: warp w of TW reads TMEM lane quarter w % 4
+// and columns C (w / 4) .. + C - 1 (C = 4 N / TW) of each accumulator, lane
+// l of it TMEM lane 32 (w % 4) + l; the elementwise phases give thread (w, l)
+// unit l of the CTA's 32 and rows P w .. P w + P - 1 (P = N / TW).
 // Forward kernel.  TMEM lane m = 32 q + u holds gate q of unit u, so warp
 // quarter q holds one gate for 32 consecutive units (coalesced Zx loads and
 // gate stores, a warp-uniform nonlinearity); the four gates of a (unit, row)
 // meet through shared memory, then thread (w, lane) updates the cell of unit
-// `lane` for rows P w .. P w + P - 1 (P = N / 16).  (A lane order 4u + q,
-// with the gates swapped by shuffles inside groups of four lanes, measured
-// 10 % slower per step.)
-template <int N>
-struct TcFwdLayout {
-  static constexpr uint32_t kB = N * kTH * 2;
-  static constexpr uint32_t kSlice = 64 * N;
-  static constexpr uint32_t kStepBytes = kTCS * 2 * kSlice;
-  static constexpr uint32_t oB = 0;                    // [2 parity][2 hi/lo][kB]
-  static constexpr uint32_t oStg = oB + 4 * kB;        // [2 parity][2 hi/lo][kSlice]
-  static constexpr uint32_t oGate = oStg + 4 * kSlice; // [N][4][32] fp32 activated gates
-  static constexpr uint32_t oBar = oGate + N * 4 * kTHc * 4;
-  static constexpr uint32_t oSlot = oBar + 3 * 8;
-  static constexpr uint32_t oLen = oSlot + 16;
-  static constexpr uint32_t oToff = oLen + 4 * N;
-};
-
-template <int N>
+// `lane` for its P rows.  (A lane order 4u + q, with the gates swapped by
+// shuffles inside groups of four lanes, measured 10 % slower per step.)
+template <int N, int TM>
 __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
   using Lay = TcFwdLayout<N>;
-  constexpr int H = kTH, G = 4 * H, QW = 4, C = N / QW, P = N / 16, kTThreads = 512;
+  using Sm = TcSmem<Lay, N, TM>;
+  constexpr int H = kTH, G = 4 * H, kTThreads = 512, TW = 16 / TM, TT = 32 * TW, QW = TW / 4, C = N / QW,
+                P = N / TW, R = N * TM;
+  static_assert(C == 4 || C == 8, "4 or 8 accumulator columns per thread");
+  static_assert(P * TW == N, "whole rows per warp");
   constexpr uint32_t idesc = tc_idesc<N>();
   extern __shared__ __align__(16) uint8_t smem[];
-  uint8_t *Bb = smem + Lay::oB;
-  uint8_t *stg = smem + Lay::oStg;
-  float *gate = reinterpret_cast<float *>(smem + Lay::oGate);
-  uint64_t *bar = reinterpret_cast<uint64_t *>(smem + Lay::oBar);
-  uint32_t *tslot = reinterpret_cast<uint32_t *>(smem + Lay::oSlot);
-  int *rlen = reinterpret_cast<int *>(smem + Lay::oLen);
-  int *toff_s = reinterpret_cast<int *>(smem + Lay::oToff);
-
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
-  const int q = warp & 3, cs = warp >> 2;  // TMEM lane quarter = gate; column slice
+  const int tm = warp / TW, wt = warp % TW, tt = t % TT;  // team; warp and thread within it
+  uint8_t *team = smem + tm * Lay::kTeam;
+  uint8_t *Bb = team + Lay::oB;
+  uint8_t *stg = team + Lay::oStg;
+  float *gate = reinterpret_cast<float *>(team + Lay::oGate);
+  uint64_t *bar = reinterpret_cast<uint64_t *>(team + Lay::oBar);
+  uint32_t *tslot = reinterpret_cast<uint32_t *>(smem + Sm::oSlot);
+  int *rlen_c = reinterpret_cast<int *>(smem + Sm::oLen);
+  const int *rlen = rlen_c + tm * N;
+  int *toff_s = reinterpret_cast<int *>(smem + Sm::oToff);
+
+  const int q = wt & 3, cs = wt >> 2;  // TMEM lane quarter = gate; column slice
   const int col0 = C * cs;
   const uint32_t c = cluster_rank();
   const int gu = (int)c * kTHc + lane;      // the unit of this lane (both phases)
-  const int n_groups = (a.ix.b + N - 1) / N;
+  const int n_groups = (a.ix.b + R - 1) / R;
   const int cid = blockIdx.x / kTCS;
-  const int d = cid / n_groups, r0 = (cid % n_groups) * N;
+  const int d = cid / n_groups, rc = (cid % n_groups) * R, r0 = rc + tm * N;
   const int DH = a.dirs * H, T = a.ix.T;
   const bool toff_sm = T + 1 <= kTTokCap;
   const int *toff = toff_sm ? toff_s : a.ix.tok_off;
   const int cap = a.wf.poll_cap > 0 ? a.wf.poll_cap : kTPolls;
   const bool withhold = (a.wf.withhold & kWithholdExchange) && c == 0;
+  const int bid = 1 + tm;
 
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(tslot)), "r"(kTmemCols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  for (uint32_t i = t; i < 4 * Lay::kB / 16; i += kTThreads) reinterpret_cast<uint4 *>(Bb)[i] = make_uint4(0, 0, 0, 0);
+#pragma unroll
+  for (int k = 0; k < TM; ++k)
+    for (uint32_t i = t; i < 4 * Lay::kB / 16; i += kTThreads)
+      reinterpret_cast<uint4 *>(smem + k * Lay::kTeam + Lay::oB)[i] = make_uint4(0, 0, 0, 0);
   if (toff_sm)
     for (int i = t; i <= T; i += kTThreads) toff_s[i] = a.ix.tok_off[i];
-  if (t < N) rlen[t] = r0 + t < a.ix.b ? a.ix.row_len[r0 + t] : 0;
+  if (t < R) rlen_c[t] = rc + t < a.ix.b ? a.ix.row_len[rc + t] : 0;
   if (t == 0) {
-    mb_init(sa(&bar[0]), 1);
-    mb_init(sa(&bar[1]), 1);
-    mb_init(sa(&bar[2]), 3);
+#pragma unroll
+    for (int k = 0; k < TM; ++k) {
+      uint64_t *b = reinterpret_cast<uint64_t *>(smem + k * Lay::kTeam + Lay::oBar);
+      mb_init(sa(&b[0]), 1);
+      mb_init(sa(&b[1]), 1);
+      mb_init(sa(&b[2]), 3);
+    }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   fence_proxy();
@@ -275,8 +318,9 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
   fence_after();
   const uint32_t tmem = *tslot;
   const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16);
-  // W_hh slice into TMEM: lane 32 q + u holds row q H + 32c + u
-  if (cs == 0) {
+  // W_hh slice into TMEM (warps 0 .. 3, warp q = lane quarter q): lane
+  // 32 q + u holds row q H + 32c + u
+  if (warp < 4) {
     const float *wrow = a.Whh[d] + (size_t)(q * H + gu) * H;
 #pragma unroll 1
     for (int c0 = 0; c0 < 128; c0 += 8) {
@@ -303,7 +347,7 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
   __syncthreads();
   const int Tg = rlen[0];
   cluster_sync_all();
-  if (t == 0) {
+  if (tt == 0) {
     if (Tg >= 2) mb_arm(sa(&bar[0]), Lay::kStepBytes);
     if (Tg >= 3) mb_arm(sa(&bar[1]), Lay::kStepBytes);
   }
@@ -317,9 +361,9 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
 #pragma unroll
   for (int k = 0; k < C; ++k) len[k] = rlen[col0 + k];
 #pragma unroll
-  for (int j = 0; j < P; ++j) lenp[j] = rlen[P * warp + j];
+  for (int j = 0; j < P; ++j) lenp[j] = rlen[P * wt + j];
   auto tok_col = [&](int k, int s) { return toff[d == 0 ? s : len[k] - 1 - s] + r0 + col0 + k; };
-  auto tok_row = [&](int j, int s) { return toff[d == 0 ? s : lenp[j] - 1 - s] + r0 + P * warp + j; };
+  auto tok_row = [&](int j, int s) { return toff[d == 0 ? s : lenp[j] - 1 - s] + r0 + P * wt + j; };
   // Zx of the next two steps in registers (DRAM latency under the step's own
   // traffic exceeds one step)
   float zn[C], zn2[C];
@@ -331,7 +375,10 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
   float cst[P];
 #pragma unroll
   for (int j = 0; j < P; ++j) cst[j] = 0.f;
-  const int prod = (lane == 0 && warp < 3) ? warp : -1;
+  // MMA issuers: lane 0 of the team's warps 0 .. 2, issuer p forms product p
+  // (W_hi h_hi, W_hi h_lo, W_lo h_hi) into its own accumulator
+  const int prod = (lane == 0 && wt < 3) ? wt : -1;
+  const uint32_t acc0 = kAccCol + 32u * (uint32_t)(3 * tm);  // the team's three accumulators
   bool ok = true, stop = false;
   int mma_issued = 0, mma_seen = 0;
 
@@ -348,16 +395,16 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
     }
     if (s > 0) {
       const int e = s - 1;
-      ok = mb_wait(sa(&bar[e & 1]), (e >> 1) & 1, cap) && ok;
-      if (t == 0 && ok && e + 2 <= Tg - 2) mb_arm(sa(&bar[e & 1]), Lay::kStepBytes);
       if (prod >= 0) {
+        ok = mb_wait(sa(&bar[e & 1]), (e >> 1) & 1, cap) && ok;
+        if (tt == 0 && ok && e + 2 <= Tg - 2) mb_arm(sa(&bar[e & 1]), Lay::kStepBytes);
         if (ok) {
           fence_proxy();
           fence_after();
           const uint32_t bh = sa(Bb + (2 * (e & 1)) * Lay::kB);
           const uint32_t bsel = bh + (prod == 1 ? Lay::kB : 0u);
           const uint32_t asel = tmem + (prod == 2 ? 128u : 0u);
-          const uint32_t dcol = tmem + kAccCol + 32u * (uint32_t)prod;
+          const uint32_t dcol = tmem + acc0 + 32u * (uint32_t)prod;
 #pragma unroll
           for (int j = 0; j < H / 16; ++j)
             mma_ts(dcol, asel + 8 * j, desc_kmajor(bsel + (uint32_t)(2 * j) * (16u * N), 16 * N, 128), idesc, j > 0);
@@ -372,7 +419,7 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
       ok = got && ok;
       fence_after();
 #pragma unroll
-      for (int p = 0; p < 3; ++p) tmem_ld_add<C>(tl + kAccCol + 32 * p + col0, acc);
+      for (int p = 0; p < 3; ++p) tmem_ld_add<C>(tl + acc0 + 32 * p + col0, acc);
     }
     // gate q of unit `lane` for this thread's columns (uniform per warp)
 #pragma unroll
@@ -382,17 +429,18 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
       gate[((col0 + k) * 4 + q) * kTHc + lane] = g;
     }
     fence_before();
-    if (__syncthreads_or(!ok)) {
-      if (t == 0) atomicOr(a.status, kErrExchWait);
+    // an issuer that gave up on the exchange stops the whole team
+    if (team_sync_or(bid, TT, !ok)) {
+      if (tt == 0) atomicOr(a.status, kErrExchWait);
       stop = true;
       break;
     }
-    // cell update of unit `lane`, rows P warp + j
+    // cell update of unit `lane`, rows P wt + j
     const uint32_t par = (uint32_t)(s & 1);
     uint8_t *sg_hi = stg + (2 * par) * Lay::kSlice, *sg_lo = sg_hi + Lay::kSlice;
 #pragma unroll
     for (int j = 0; j < P; ++j) {
-      const int n = P * warp + j;
+      const int n = P * wt + j;
       const float ig = gate[(n * 4 + 0) * kTHc + lane], fg = gate[(n * 4 + 1) * kTHc + lane];
       const float gg = gate[(n * 4 + 2) * kTHc + lane], og = gate[(n * 4 + 3) * kTHc + lane];
       const float cn = fmaf(fg, cst[j], ig * gg);
@@ -417,13 +465,13 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
       *reinterpret_cast<__nv_bfloat16 *>(sg_hi + off) = hh;
       *reinterpret_cast<__nv_bfloat16 *>(sg_lo + off) = hl;
     }
-    __syncthreads();
+    team_sync(bid, TT);
     if (s + 1 < Tg && !withhold) {
       constexpr int kPieces = 2 * Lay::kSlice / 16;
       const uint32_t dst0 = sa(Bb + (2 * par) * Lay::kB) + c * (uint32_t)Lay::kSlice;
       const uint32_t mbl = sa(&bar[par]);
 #pragma unroll
-      for (int i = t; i < kTCS * kPieces; i += kTThreads) {
+      for (int i = tt; i < kTCS * kPieces; i += TT) {
         const int pr = i / kPieces, rem = i % kPieces, hl = rem / (kPieces / 2), o = (rem % (kPieces / 2)) * 16;
         const uint4 v = *reinterpret_cast<const uint4 *>(stg + (2 * par + hl) * Lay::kSlice + o);
         st_async16(peer(dst0 + (uint32_t)hl * Lay::kB + (uint32_t)o, (uint32_t)pr), v, peer(mbl, (uint32_t)pr));
@@ -438,48 +486,68 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
 }
 
-template <int N>
+template <int N, int TM>
 __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
   using Lay = TcBwdLayout<N>;
-  constexpr int H = kTH, G = 4 * H, QW = 4, C = N / QW, P = N / 16, RS = Lay::kRS, kTThreads = 512;
+  using Sm = TcSmem<Lay, N, TM>;
+  constexpr int H = kTH, G = 4 * H, kTThreads = 512, TW = 16 / TM, TT = 32 * TW, QW = TW / 4, C = N / QW,
+                P = N / TW, R = N * TM, RS = Lay::kRS;
+  // Accumulators per 128-unit half: with one team, one per product (three
+  // issuers per half); with two, one per half of the k-steps (two issuers
+  // per half, each forming all three products), so that both teams'
+  // accumulators fit the 256 free TMEM columns at 32-column spacing.
+  constexpr int AH = TM == 1 ? 3 : 2;
+  static_assert(C == 4 || C == 8, "4 or 8 accumulator columns per thread");
+  static_assert(P * TW == N && 2 * AH <= TW, "whole rows per warp; an issuer per warp");
   constexpr uint32_t idesc = tc_idesc<N>();
   extern __shared__ __align__(16) uint8_t smem[];
-  uint8_t *Bz = smem + Lay::oB;
-  float *red = reinterpret_cast<float *>(smem + Lay::oRed);
-  float *pst = reinterpret_cast<float *>(smem + Lay::oStg);
-  uint64_t *bar = reinterpret_cast<uint64_t *>(smem + Lay::oBar);
-  uint32_t *tslot = reinterpret_cast<uint32_t *>(smem + Lay::oSlot);
-  int *rlen = reinterpret_cast<int *>(smem + Lay::oLen);
-  int *toff_s = reinterpret_cast<int *>(smem + Lay::oToff);
-
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
-  const int qt = warp & 3, cs = warp >> 2;
+  const int tm = warp / TW, wt = warp % TW, tt = t % TT;
+  uint8_t *team = smem + tm * Lay::kTeam;
+  uint8_t *Bz = team + Lay::oB;
+  float *red = reinterpret_cast<float *>(team + Lay::oRed);
+  float *pst = reinterpret_cast<float *>(team + Lay::oStg);
+  uint64_t *bar = reinterpret_cast<uint64_t *>(team + Lay::oBar);
+  uint32_t *tslot = reinterpret_cast<uint32_t *>(smem + Sm::oSlot);
+  int *rlen_c = reinterpret_cast<int *>(smem + Sm::oLen);
+  const int *rlen = rlen_c + tm * N;
+  int *toff_s = reinterpret_cast<int *>(smem + Sm::oToff);
+
+  const int qt = wt & 3, cs = wt >> 2;
   const int col0 = C * cs;
-  const int u = lane;  // phase B: unit `lane`, rows P warp + j
+  const int u = lane;  // phase B: unit `lane`, rows P wt + j
   const uint32_t c = cluster_rank();
   const int gu = (int)c * kTHc + u;
-  const int n_groups = (a.ix.b + N - 1) / N;
+  const int n_groups = (a.ix.b + R - 1) / R;
   const int cid = blockIdx.x / kTCS;
-  const int d = cid / n_groups, r0 = (cid % n_groups) * N;
+  const int d = cid / n_groups, rc = (cid % n_groups) * R, r0 = rc + tm * N;
   const int DH = a.dirs * H, T = a.ix.T;
   const bool toff_sm = T + 1 <= kTTokCap;
   const int *toff = toff_sm ? toff_s : a.ix.tok_off;
   const int cap = a.wf.poll_cap > 0 ? a.wf.poll_cap : kTPolls;
   const bool withhold = (a.wf.withhold & kWithholdExchange) && c == 0;
+  const int bid = 1 + tm;
 
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(tslot)), "r"(kTmemCols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  for (uint32_t i = t; i < 2 * Lay::kB / 16; i += kTThreads) reinterpret_cast<uint4 *>(Bz)[i] = make_uint4(0, 0, 0, 0);
+#pragma unroll
+  for (int k = 0; k < TM; ++k)
+    for (uint32_t i = t; i < 2 * Lay::kB / 16; i += kTThreads)
+      reinterpret_cast<uint4 *>(smem + k * Lay::kTeam + Lay::oB)[i] = make_uint4(0, 0, 0, 0);
   if (toff_sm)
     for (int i = t; i <= T; i += kTThreads) toff_s[i] = a.ix.tok_off[i];
-  if (t < N) rlen[t] = r0 + t < a.ix.b ? a.ix.row_len[r0 + t] : 0;
+  if (t < R) rlen_c[t] = rc + t < a.ix.b ? a.ix.row_len[rc + t] : 0;
   if (t == 0) {
-    mb_init(sa(&bar[0]), 1);
-    mb_init(sa(&bar[1]), 1);
-    mb_init(sa(&bar[2]), 6);  // one commit from each of the six MMA issuers
+#pragma unroll
+    for (int k = 0; k < TM; ++k) {
+      uint64_t *b = reinterpret_cast<uint64_t *>(smem + k * Lay::kTeam + Lay::oBar);
+      mb_init(sa(&b[0]), 1);
+      mb_init(sa(&b[1]), 1);
+      mb_init(sa(&b[2]), 2 * AH);  // one commit from each of the team's MMA issuers
+    }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   fence_before();
@@ -487,11 +555,11 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
   fence_after();
   const uint32_t tmem = *tslot;
   const uint32_t tl = tmem + ((uint32_t)(32 * qt) << 16);
-  // W_hh^T into TMEM: half hf = 0, 1 (warps of column slices 0, 1) holds
-  // units 128 hf + m in lane m; K = the CTA's gate rows k = 4 uu + qq (global
-  // row qq H + 32c + uu); hi part in columns 128 hf .. + 63, lo part 64 after
-  if (cs < 2) {
-    const int hf = cs;
+  // W_hh^T into TMEM (warps 0 .. 7): half hf = warp / 4 holds units
+  // 128 hf + m in lane m; K = the CTA's gate rows k = 4 uu + qq (global row
+  // qq H + 32c + uu); hi part in columns 128 hf .. + 63, lo part 64 after
+  if (warp < 8) {
+    const int hf = warp >> 2;
     const float *W = a.Whh[d];
     const int col = 128 * hf + 32 * qt + lane;
 #pragma unroll 1
@@ -517,7 +585,7 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
   __syncthreads();
   const int Tg = rlen[0];
   cluster_sync_all();
-  if (t == 0) {
+  if (tt == 0) {
     if (Tg >= 2) mb_arm(sa(&bar[0]), Lay::kStepBytes);
     if (Tg >= 3) mb_arm(sa(&bar[1]), Lay::kStepBytes);
   }
@@ -526,10 +594,10 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
   const float *__restrict__ Cs = a.Cst[d];
   const float *__restrict__ dY = a.dY;
   __nv_bfloat16 *__restrict__ dZb = reinterpret_cast<__nv_bfloat16 *>(a.dZb[d]);
-  int len[P];  // lengths of this thread's rows P warp + j
+  int len[P];  // lengths of this thread's rows P wt + j
 #pragma unroll
-  for (int j = 0; j < P; ++j) len[j] = rlen[P * warp + j];
-  auto tok_at = [&](int j, int s) { return toff[d == 0 ? s : len[j] - 1 - s] + r0 + P * warp + j; };
+  for (int j = 0; j < P; ++j) len[j] = rlen[P * wt + j];
+  auto tok_at = [&](int j, int s) { return toff[d == 0 ? s : len[j] - 1 - s] + r0 + P * wt + j; };
   // phase B inputs of a step, loaded two steps ahead: gates i, f, g, o,
   // c_t, dY (c_{t-1} is the next step's c_t, zero before the first step)
   float in[P][6], nx[P][6], nx2[P][6];
@@ -553,9 +621,12 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
   float dc[P];
 #pragma unroll
   for (int j = 0; j < P; ++j) dc[j] = 0.f;
-  // MMA issuers: lane 0 of warps 0..5, issuer i forms product i % 3 (W_hi dz_hi,
-  // W_hi dz_lo, W_lo dz_hi) of half i / 3 into columns kAccCol + 32 i
-  const int iss = (lane == 0 && warp < 6) ? warp : -1;
+  // MMA issuers: lane 0 of the team's warps 0 .. 2 AH - 1; issuer i works on
+  // half i / AH into accumulator i of the team (AH = 3: product i % 3 of
+  // W_hi dz_hi, W_hi dz_lo, W_lo dz_hi over all eight k-steps; AH = 2: all
+  // three products over k-steps 4 (i % 2) .. + 3)
+  const int iss = (lane == 0 && wt < 2 * AH) ? wt : -1;
+  const uint32_t acc0 = kAccCol + 32u * (uint32_t)(2 * AH * tm);  // the team's 2 AH accumulators
   bool ok = true, stop = false;
   int mma_issued = 0, mma_seen = 0;
   const uint32_t bh = sa(Bz);
@@ -574,13 +645,13 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
     if (it > 0) {
       const int e = it - 1;
       ok = mb_wait(sa(&bar[e & 1]), (e >> 1) & 1, cap) && ok;
-      if (t == 0 && ok && e + 2 <= Tg - 2) mb_arm(sa(&bar[e & 1]), Lay::kStepBytes);
+      if (tt == 0 && ok && e + 2 <= Tg - 2) mb_arm(sa(&bar[e & 1]), Lay::kStepBytes);
       rp = red + (size_t)(e & 1) * (kTCS * N * RS) + u;
     }
-    // phase B: dh, dc and dz of unit u for rows P warp + j
+    // phase B: dh, dc and dz of unit u for rows P wt + j
 #pragma unroll
     for (int j = 0; j < P; ++j) {
-      const int n = P * warp + j;
+      const int n = P * wt + j;
       float dz4[4] = {0.f, 0.f, 0.f, 0.f};
       if (s < len[j]) {
         float dh = in[j][5];
@@ -624,8 +695,8 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
     }
     fence_proxy();
     fence_before();
-    if (__syncthreads_or(!ok)) {
-      if (t == 0) atomicOr(a.status, kErrExchWait);
+    if (team_sync_or(bid, TT, !ok)) {
+      if (tt == 0) atomicOr(a.status, kErrExchWait);
       stop = true;
       break;
     }
@@ -633,13 +704,23 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
     if (it + 1 >= Tg) continue;  // dh_{-1} is not needed
     // this CTA's partial W_hh^T dz for all 256 units (two halves of 128 lanes)
     if (iss >= 0) {
-      const int hf = iss / 3, p = iss % 3;
-      const uint32_t dcol = tmem + kAccCol + 32u * (uint32_t)iss;
-      const uint32_t asel = tmem + 128u * (uint32_t)hf + (p == 2 ? 64u : 0u);
-      const uint32_t bsel = bh + (p == 1 ? Lay::kB : 0u);
+      const int hf = iss / AH, ia = iss % AH;
+      const uint32_t dcol = tmem + acc0 + 32u * (uint32_t)iss;
+      const uint32_t abase = tmem + 128u * (uint32_t)hf;
+      auto one = [&](int j, int p, bool accum) {
+        const uint32_t asel = abase + (p == 2 ? 64u : 0u);
+        const uint32_t bsel = bh + (p == 1 ? Lay::kB : 0u);
+        mma_ts(dcol, asel + 8 * j, desc_kmajor(bsel + (uint32_t)(2 * j) * (16u * N), 16 * N, 128), idesc, accum);
+      };
+      if constexpr (AH == 3) {
 #pragma unroll
-      for (int j = 0; j < 128 / 16; ++j)
-        mma_ts(dcol, asel + 8 * j, desc_kmajor(bsel + (uint32_t)(2 * j) * (16u * N), 16 * N, 128), idesc, j > 0);
+        for (int j = 0; j < 128 / 16; ++j) one(j, ia, j > 0);
+      } else {
+#pragma unroll
+        for (int jj = 0; jj < 4; ++jj)
+#pragma unroll
+          for (int p = 0; p < 3; ++p) one(4 * ia + jj, p, jj > 0 || p > 0);
+      }
       mma_commit(sa(&bar[2]));
     }
     ++mma_issued;
@@ -651,26 +732,28 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
 #pragma unroll
     for (int k = 0; k < C; ++k) p0[k] = p1[k] = 0.f;
 #pragma unroll
-    for (int p = 0; p < 3; ++p) {
-      tmem_ld_add<C>(tl + kAccCol + 32 * p + col0, p0);
-      tmem_ld_add<C>(tl + kAccCol + 32 * (3 + p) + col0, p1);
+    for (int i = 0; i < AH; ++i) {
+      tmem_ld_add<C>(tl + acc0 + 32 * i + col0, p0);
+      tmem_ld_add<C>(tl + acc0 + 32 * (AH + i) + col0, p1);
     }
     // stage the partials by owner (unit 32 qt + lane of half hf belongs to
-    // CTA qt + 4 hf), rows contiguous, so that the sends below are whole
-    // 16-byte pieces of consecutive memory on both sides
+    // CTA qt + 4 hf), rows contiguous, so that each remote store is a whole
+    // 16-byte piece of consecutive memory on both sides; the warp's pieces
+    // (its C rows for owners qt and qt + 4) are its own, so it sends them
+    // as soon as it has staged them
 #pragma unroll
     for (int k = 0; k < C; ++k) {
       pst[((qt)*N + col0 + k) * kTHc + lane] = p0[k];
       pst[((qt + 4) * N + col0 + k) * kTHc + lane] = p1[k];
     }
-    __syncthreads();
+    __syncwarp();
     if (!withhold && got) {
       const uint32_t par = (uint32_t)(it & 1);
       const uint32_t mbl = sa(&bar[par]);
-      constexpr int kPer = N * kTHc / 4;  // 16-byte pieces per owner
+      constexpr int kWP = C * (kTHc / 4);  // pieces per owner
 #pragma unroll
-      for (int i = t; i < kTCS * kPer; i += kTThreads) {
-        const int owner = i / kPer, rem = i % kPer, n = rem / (kTHc / 4), ch = rem % (kTHc / 4);
+      for (int i = lane; i < 2 * kWP; i += 32) {
+        const int owner = qt + 4 * (i / kWP), rem = i % kWP, n = col0 + rem / (kTHc / 4), ch = rem % (kTHc / 4);
         const uint4 v = *reinterpret_cast<const uint4 *>(pst + (owner * N + n) * kTHc + 4 * ch);
         const uint32_t dst = sa(red) + (((par * kTCS + c) * N + n) * RS + 4 * ch) * 4u;
         st_async16(peer(dst, (uint32_t)owner), v, peer(mbl, (uint32_t)owner));
@@ -705,61 +788,63 @@ cudaLaunchConfig_t tc_config(int clusters, int threads, size_t smem, cudaStream_
   return cfg;
 }
 
-template <int N>
+template <int N, int TM>
 size_t tc_smem(bool bwd, int T) {
-  return tc_smem_bytes(bwd ? TcBwdLayout<N>::oToff : TcFwdLayout<N>::oToff, T);
+  return tc_smem_bytes(bwd ? TcSmem<TcBwdLayout<N>, N, TM>::oToff : TcSmem<TcFwdLayout<N>, N, TM>::oToff, T);
 }
 
-template <int N>
+// N rows per team, TM teams: N TM rows per cluster.
+template <int N, int TM>
 cudaError_t launch_tc(const RecArgs &a, bool bwd, cudaStream_t s) {
   if (a.ix.b <= 0 || a.ix.T <= 0) return cudaSuccess;
   if (a.H != kTH) return cudaErrorInvalidValue;
-  const size_t smem = tc_smem<N>(bwd, a.ix.T);
-  const int clusters = ((a.ix.b + N - 1) / N) * a.dirs;
+  const size_t smem = tc_smem<N, TM>(bwd, a.ix.T);
+  const int clusters = ((a.ix.b + N * TM - 1) / (N * TM)) * a.dirs;
   cudaLaunchAttribute attr;
 
   if (bwd) {
-    auto k = lstm_bwd_tc_kernel<N>;
+    auto k = lstm_bwd_tc_kernel<N, TM>;
     cudaError_t e = ensure_smem((const void *)k, smem);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = tc_config<decltype(k)>(clusters, 512, smem, s, &attr);
     return cudaLaunchKernelEx(&cfg, k, a);
   }
-  auto k = lstm_fwd_tc_kernel<N>;
+  auto k = lstm_fwd_tc_kernel<N, TM>;
   cudaError_t e = ensure_smem((const void *)k, smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = tc_config<decltype(k)>(clusters, 512, smem, s, &attr);
   return cudaLaunchKernelEx(&cfg, k, a);
 }
 
-// 8-CTA clusters of both kernels that can be resident at once (0: cannot launch).
-template <int N>
-int tc_resident() {
-  int lo = 1 << 30;
-  for (int bwd = 0; bwd < 2; ++bwd) {
-    const size_t smem = tc_smem<N>(bwd != 0, kTTokCap - 1);
-    cudaLaunchAttribute attr;
-    int n = 0;
-    cudaError_t e;
-    if (bwd) {
-      auto k = lstm_bwd_tc_kernel<N>;
-      e = ensure_smem((const void *)k, smem);
-      cudaLaunchConfig_t cfg = tc_config<decltype(k)>(1, 512, smem, 0, &attr);
-      if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, k, &cfg);
-    } else {
-      auto k = lstm_fwd_tc_kernel<N>;
-      e = ensure_smem((const void *)k, smem);
-      cudaLaunchConfig_t cfg = tc_config<decltype(k)>(1, 512, smem, 0, &attr);
-      if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, k, &cfg);
-    }
-    if (e != cudaSuccess) {
-      cudaGetLastError();
-      return 0;
-    }
-    lo = std::min(lo, n);
+// 8-CTA clusters of one kernel that can be resident at once (0: cannot launch).
+template <int N, int TM>
+int tc_resident_one(bool bwd) {
+  const size_t smem = tc_smem<N, TM>(bwd, kTTokCap - 1);
+  cudaLaunchAttribute attr;
+  int n = 0;
+  cudaError_t e;
+  if (bwd) {
+    auto k = lstm_bwd_tc_kernel<N, TM>;
+    e = ensure_smem((const void *)k, smem);
+    cudaLaunchConfig_t cfg = tc_config<decltype(k)>(1, 512, smem, 0, &attr);
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, k, &cfg);
+  } else {
+    auto k = lstm_fwd_tc_kernel<N, TM>;
+    e = ensure_smem((const void *)k, smem);
+    cudaLaunchConfig_t cfg = tc_config<decltype(k)>(1, 512, smem, 0, &attr);
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, k, &cfg);
   }
-  return lo;
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
 }
+
+// 32 rows per cluster, as two teams of 16 rows (one team's MMAs and
+// exchange overlap the other's elementwise work).
+int tc_resident32() { return std::min(tc_resident_one<16, 2>(false), tc_resident_one<16, 2>(true)); }
+cudaError_t launch_tc32(const RecArgs &a, bool bwd, cudaStream_t s) { return launch_tc<16, 2>(a, bwd, s); }
 
 }  // namespace
 
@@ -776,15 +861,15 @@ int plan_tc_rows(int b, int dirs) {
   // not its columns, bounds it), so fewer, wider clusters leave SMs to the
   // side stream; 16 when the batch is small enough for its clusters to fit
   // either way (0: neither can launch)
-  const int r16 = tc_resident<16>(), r32 = tc_resident<32>();
+  const int r16 = std::min(tc_resident_one<16, 1>(false), tc_resident_one<16, 1>(true)), r32 = tc_resident32();
   if (r16 > 0 && ((b + 15) / 16) * dirs <= std::min(r16, 4)) return 16;
   if (r32 > 0) return 32;
   return r16 > 0 ? 16 : 0;
 }
 
 cudaError_t launch_lstm_tc(const RecArgs &a, int rows, bool bwd, cudaStream_t s) {
-  if (rows == 16) return launch_tc<16>(a, bwd, s);
-  if (rows == 32) return launch_tc<32>(a, bwd, s);
+  if (rows == 16) return launch_tc<16, 1>(a, bwd, s);
+  if (rows == 32) return launch_tc32(a, bwd, s);
   return cudaErrorInvalidValue;
 }
 
