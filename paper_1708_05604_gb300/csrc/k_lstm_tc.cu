@@ -135,6 +135,17 @@ __device__ __forceinline__ uint64_t desc_kmajor(uint32_t addr, uint32_t lbo, uin
   d |= (uint64_t)1 << 46;  // descriptor version
   return d;                // swizzle mode 0: none
 }
+// The same for a K-major operand in the 128-byte swizzle: rows of 128 B
+// (64 bf16 of K) whose 16-byte chunks are permuted by chunk ^ (row % 8),
+// 8-row groups 1024 B apart (the tile 1024-byte aligned).
+__device__ __forceinline__ uint64_t desc_sw128(uint32_t addr) {
+  uint64_t d = (uint64_t)((addr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1 << 16;            // leading byte offset (unused in this mode)
+  d |= (uint64_t)(1024 >> 4) << 32;  // stride byte offset
+  d |= (uint64_t)1 << 46;            // descriptor version
+  d |= (uint64_t)2 << 61;            // 128-byte swizzle
+  return d;
+}
 // D (TMEM) (+)= A (TMEM) * B (shared memory)
 __device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
   asm volatile(
@@ -201,7 +212,7 @@ __device__ __forceinline__ bool team_sync_or(int id, int n, bool p) {
 // TMEM address slot, the lengths of the cluster's rows and the time offsets.
 template <int N>
 struct TcBwdLayout {
-  static constexpr uint32_t kB = N * 128 * 2;      // one B operand (dz hi or lo): N rows x 128 gate rows
+  static constexpr uint32_t kB = N * 128 * 2;      // one B operand (dz hi or lo): N rows x 128 gate rows, 128-byte swizzle
   static constexpr int kRS = kTHc + 8;             // floats per (source, row) of received partials (32 units + pad)
   static constexpr uint32_t kRed = kTCS * N * kRS * 4;     // received partials per parity
   static constexpr uint32_t kStepBytes = kTCS * kTHc * N * 4;
@@ -209,7 +220,7 @@ struct TcBwdLayout {
   static constexpr uint32_t oRed = oB + 2 * kB;    // [2 parity][8 src][N rows][kRS] fp32
   static constexpr uint32_t oStg = oRed + 2 * kRed;  // [8 owners][N rows][32 units] fp32 partials to send
   static constexpr uint32_t oBar = oStg + kTCS * N * kTHc * 4;  // rbar[2], mmabar
-  static constexpr uint32_t kTeam = oBar + 32;
+  static constexpr uint32_t kTeam = (oBar + 32 + 1023) & ~1023u;  // keeps each team's B operand 1024-byte aligned
 };
 
 template <int N>
@@ -218,8 +229,13 @@ struct TcFwdLayout {
   static constexpr uint32_t kSlice = 64 * N;
   static constexpr uint32_t kStepBytes = kTCS * 2 * kSlice;
   static constexpr uint32_t oB = 0;                    // [2 parity][2 hi/lo][kB]
-  static constexpr uint32_t oStg = oB + 4 * kB;        // [2 parity][2 hi/lo][kSlice]
-  static constexpr uint32_t oGate = oStg + 4 * kSlice; // [N][4][32] fp32 activated gates
+  // staging of h_t: [2 parity][2 hi/lo][4 unit octets][N rows][16 B], the
+  // octets 16 N + 16 bytes apart so that a warp's stores of one row (four
+  // octets) fall in distinct banks
+  static constexpr uint32_t kOct = 16 * N + 16;
+  static constexpr uint32_t kStgS = 4 * kOct;
+  static constexpr uint32_t oStg = oB + 4 * kB;
+  static constexpr uint32_t oGate = oStg + 4 * kStgS;  // [N][4][32] fp32 activated gates
   static constexpr uint32_t oBar = oGate + N * 4 * kTHc * 4;  // xbar[2], mmabar
   static constexpr uint32_t kTeam = oBar + 32;
 };
@@ -437,7 +453,7 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
     }
     // cell update of unit `lane`, rows P wt + j
     const uint32_t par = (uint32_t)(s & 1);
-    uint8_t *sg_hi = stg + (2 * par) * Lay::kSlice, *sg_lo = sg_hi + Lay::kSlice;
+    uint8_t *sg_hi = stg + (2 * par) * Lay::kStgS, *sg_lo = sg_hi + Lay::kStgS;
 #pragma unroll
     for (int j = 0; j < P; ++j) {
       const int n = P * wt + j;
@@ -461,7 +477,7 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
         h = 0.f;
         split_bf16(h, hh, hl);
       }
-      const uint32_t off = (uint32_t)(lane >> 3) * (16u * N) + (uint32_t)n * 16u + (uint32_t)(lane & 7) * 2u;
+      const uint32_t off = (uint32_t)(lane >> 3) * Lay::kOct + (uint32_t)n * 16u + (uint32_t)(lane & 7) * 2u;
       *reinterpret_cast<__nv_bfloat16 *>(sg_hi + off) = hh;
       *reinterpret_cast<__nv_bfloat16 *>(sg_lo + off) = hl;
     }
@@ -472,9 +488,11 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
       const uint32_t mbl = sa(&bar[par]);
 #pragma unroll
       for (int i = tt; i < kTCS * kPieces; i += TT) {
-        const int pr = i / kPieces, rem = i % kPieces, hl = rem / (kPieces / 2), o = (rem % (kPieces / 2)) * 16;
-        const uint4 v = *reinterpret_cast<const uint4 *>(stg + (2 * par + hl) * Lay::kSlice + o);
-        st_async16(peer(dst0 + (uint32_t)hl * Lay::kB + (uint32_t)o, (uint32_t)pr), v, peer(mbl, (uint32_t)pr));
+        // piece pc = (octet, row) of part hl: 16 pc bytes into the K-major slice
+        const int pr = i / kPieces, rem = i % kPieces, hl = rem / (kPieces / 2), pc = rem % (kPieces / 2);
+        const uint32_t o = (uint32_t)pc * 16u, so = (uint32_t)(pc / N) * Lay::kOct + (uint32_t)(pc % N) * 16u;
+        const uint4 v = *reinterpret_cast<const uint4 *>(stg + (2 * par + hl) * Lay::kStgS + so);
+        st_async16(peer(dst0 + (uint32_t)hl * Lay::kB + o, (uint32_t)pr), v, peer(mbl, (uint32_t)pr));
       }
     }
   }
@@ -500,7 +518,8 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
   static_assert(C == 4 || C == 8, "4 or 8 accumulator columns per thread");
   static_assert(P * TW == N && 2 * AH <= TW, "whole rows per warp; an issuer per warp");
   constexpr uint32_t idesc = tc_idesc<N>();
-  extern __shared__ __align__(16) uint8_t smem[];
+  extern __shared__ __align__(16) uint8_t smem_raw[];
+  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int tm = warp / TW, wt = warp % TW, tt = t % TT;
   uint8_t *team = smem + tm * Lay::kTeam;
@@ -676,7 +695,9 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
       } else {
         dc[j] = 0.f;
       }
-      // B operand: k = 4u .. 4u + 3 of row n (8 bytes of each part)
+      // B operand: k = 4u .. 4u + 3 of row n (8 bytes of each part), in
+      // 64-k atom u / 16 at 16-byte chunk (u % 16) / 2 swizzled by n % 8, so
+      // that a warp's 32 stores fill two whole 128-byte rows
       __nv_bfloat16 h0, l0, h1, l1, h2, l2, h3, l3;
       split_bf16(dz4[0], h0, l0);
       split_bf16(dz4[1], h1, l1);
@@ -689,7 +710,8 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
         zb[2 * H] = h2;
         zb[3 * H] = h3;
       }
-      const uint32_t off = (uint32_t)(u >> 1) * (16u * N) + (uint32_t)n * 16u + (uint32_t)(u & 1) * 8u;
+      const uint32_t off = (uint32_t)(u >> 4) * (128u * N) + (uint32_t)n * 128u +
+                           (uint32_t)((((u & 15) >> 1) ^ (n & 7)) * 16) + (uint32_t)(u & 1) * 8u;
       *reinterpret_cast<uint2 *>(Bz + off) = make_uint2(pack2(h0, h1), pack2(h2, h3));
       *reinterpret_cast<uint2 *>(Bz + Lay::kB + off) = make_uint2(pack2(l0, l1), pack2(l2, l3));
     }
@@ -710,7 +732,7 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
       auto one = [&](int j, int p, bool accum) {
         const uint32_t asel = abase + (p == 2 ? 64u : 0u);
         const uint32_t bsel = bh + (p == 1 ? Lay::kB : 0u);
-        mma_ts(dcol, asel + 8 * j, desc_kmajor(bsel + (uint32_t)(2 * j) * (16u * N), 16 * N, 128), idesc, accum);
+        mma_ts(dcol, asel + 8 * j, desc_sw128(bsel + (uint32_t)(j >> 2) * (128u * N) + (uint32_t)(j & 3) * 32u), idesc, accum);
       };
       if constexpr (AH == 3) {
 #pragma unroll
@@ -790,7 +812,8 @@ cudaLaunchConfig_t tc_config(int clusters, int threads, size_t smem, cudaStream_
 
 template <int N, int TM>
 size_t tc_smem(bool bwd, int T) {
-  return tc_smem_bytes(bwd ? TcSmem<TcBwdLayout<N>, N, TM>::oToff : TcSmem<TcFwdLayout<N>, N, TM>::oToff, T);
+  // (BPTT: + 1 KB to align its base to 1024 bytes)
+  return tc_smem_bytes(bwd ? TcSmem<TcBwdLayout<N>, N, TM>::oToff + 1024 : TcSmem<TcFwdLayout<N>, N, TM>::oToff, T);
 }
 
 // N rows per team, TM teams: N TM rows per cluster.
