@@ -8,12 +8,15 @@
 // CTA c owns the hidden units [32c, 32c + 32), i.e. the 128 gate rows
 // {q H + 32c + u : q = i, f, g, o; u < 32}, and keeps its slice of W_hh for
 // the whole sequence in tensor memory as the A operand of tcgen05.mma, split
-// into two bf16 parts (w = w_hi + w_lo, 16 significant bits).  The other
-// operand (h_{t-1}, or dz_t) is split the same way in shared memory, and each
-// step issues the three products hi*hi + hi*lo + lo*hi with fp32
-// accumulation in TMEM (relative error near 2^-16 per product; the cell
-// state, the gates and every elementwise step stay fp32).  W never leaves
-// the SM: per step only N rows of h (or dz) are read from shared memory.
+// into two parts, with fp32 accumulation in TMEM; the cell state, h, the
+// gates and every elementwise step stay fp32.  Forward: w = w_hi + 2^-11 w_lo
+// in fp16 (about 22 significant bits) times h_{t-1} rounded to fp16
+// (relative error 2^-12 in each h, within the bf16 input projection's 2^-9),
+// two products per step.  BPTT: w = w_hi + w_lo in bf16 (16 bits) and dz_t
+// split the same way (bf16 keeps the range that small gradients need), the
+// three products hi*hi + hi*lo + lo*hi (relative error near 2^-16).  W never
+// leaves the SM: per step only N rows of h (or dz) are read from shared
+// memory.
 //
 // A cluster's rows form two teams of 16 rows (one team of 16 for batches of
 // at most 64 rows); each team runs its own recurrence on 8 of the CTA's 16
@@ -22,23 +25,25 @@
 // team's elementwise work; the teams share only W in TMEM.
 //
 // Forward: TMEM lane 32 q + u holds gate row q H + 32c + u (A = the W slice,
-// K = the 256 units; hi part in columns 0 .. 127, lo part in 128 .. 255).
+// K = the 256 units; hi part in columns 0 .. 127, scaled lo part in
+// 128 .. 255).
 // BPTT: A = the W slice transposed in two 128-unit halves (lane m = unit
 // 128 hf + m), K = the CTA's 128 gate rows in the order 4u + q.  Operands in
 // shared memory use the K-major layout without swizzle: 8 x 16-byte core
 // matrices, element (n, k) at (k / 8) * 16 N + n * 16 + (k % 8) * 2 bytes, so
 // the 32 units of one CTA are one contiguous 64 N-byte block.
 //
-// Forward step: once h_{t-1} has arrived, three issuing threads (one per
-// product) issue 16 MMAs each into their own accumulators and commit them
+// Forward step: once h_{t-1} has arrived, four issuing threads (product x
+// half of K) issue 8 MMAs each into their own accumulators and commit them
 // to an mbarrier; each warp then reads one TMEM lane quarter (one gate for
-// the 32 units) for C rows, adds Zx, applies sigma or tanh, writes the
-// gates, and leaves them in shared memory, where thread (w, lane) finds the
-// four gates of unit `lane` for its rows, updates c in registers, writes c,
-// h and the bf16 copies, and stages h_t (bf16 hi and lo) for st.async
-// stores to every CTA of the cluster (16-byte remote stores completing
-// bytes on the receiver's mbarrier; double-buffered by step parity, so the
-// data dependence orders buffer reuse).
+// the 32 units) for C rows, adds Zx and the four accumulators (the lo ones
+// scaled by 2^-11), applies sigma or tanh, writes the gates, and leaves
+// them in shared memory, where thread (w, lane) finds the four gates of
+// unit `lane` for its rows, updates c in registers, writes c, h and the
+// bf16 copies, and stages h_t in fp16 for st.async stores to every CTA of
+// the cluster (16-byte remote stores completing bytes on the receiver's
+// mbarrier; double-buffered by step parity, so the data dependence orders
+// buffer reuse).
 // BPTT step: dh = dY + the sum of the 8 partials of W_hh^T dz_{t+1} received
 // for this CTA's units, then dc and dz of the four gates (fp32, written in
 // place of the gates and, split, to the B operand); four issuing threads
@@ -52,6 +57,7 @@
 // peers at a final cluster barrier.  A CTA takes all 512 TMEM columns; its
 // shared-memory request (>= 140 KB) keeps any other TMEM user off its SM.
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 
 #include <cstdint>
 
@@ -74,11 +80,12 @@ constexpr size_t kTSmemFloor = 140 * 1024;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kAccCol = 256;  // first accumulator column (A operands take 0 .. 255)
 
-// kind::f16 instruction descriptor: D fp32, A and B bf16, both K-major,
-// N >> 3 at bit 17, M = 128 (>> 4 at bit 24).
-template <int N>
+// kind::f16 instruction descriptor: D fp32, A and B bf16 (format 1 at bits
+// 7 and 10) or fp16 (format 0), both K-major, N >> 3 at bit 17, M = 128
+// (>> 4 at bit 24).
+template <int N, bool F16 = false>
 __host__ __device__ constexpr uint32_t tc_idesc() {
-  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+  return (1u << 4) | (F16 ? 0u : (1u << 7) | (1u << 10)) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
 }
 
 __device__ __forceinline__ uint32_t sa(const void *p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
@@ -190,6 +197,33 @@ __device__ __forceinline__ void split_bf16(float x, __nv_bfloat16 &hi, __nv_bflo
 __device__ __forceinline__ uint32_t pack2(__nv_bfloat16 a, __nv_bfloat16 b) {
   return (uint32_t)__bfloat16_as_ushort(a) | ((uint32_t)__bfloat16_as_ushort(b) << 16);
 }
+// x = hi + 2^-11 lo, both fp16: hi rounded to nearest, lo the rounded rest
+// scaled by 2^11 so that it keeps fp16's full precision (the rest alone is
+// often subnormal); hi + 2^-11 lo carries about 22 significant bits
+constexpr float kF16LoScale = 2048.f;
+__device__ __forceinline__ void split_f16(float x, __half &hi, __half &lo) {
+  hi = __float2half_rn(x);
+  lo = __float2half_rn((x - __half2float(hi)) * kF16LoScale);
+}
+__device__ __forceinline__ uint32_t pack2h(__half a, __half b) {
+  return (uint32_t)__half_as_ushort(a) | ((uint32_t)__half_as_ushort(b) << 16);
+}
+// C consecutive columns of this thread's lane, not yet waited for
+template <int C>
+__device__ __forceinline__ void tmem_ld_raw(uint32_t taddr, uint32_t (&r)[C]) {
+  if constexpr (C == 4) {
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(taddr)
+                 : "memory");
+  } else {
+    static_assert(C == 8, "4 or 8 columns per thread");
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                 : "r"(taddr)
+                 : "memory");
+  }
+}
 // Gate nonlinearities from the exponential intrinsic (as in the other
 // recurrent kernels): sigma(x) = 1 / (1 + e^-x), tanh(x) = 2 sigma(2x) - 1.
 __device__ __forceinline__ float sigm_tc(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
@@ -225,17 +259,17 @@ struct TcBwdLayout {
 
 template <int N>
 struct TcFwdLayout {
-  static constexpr uint32_t kB = N * kTH * 2;
-  static constexpr uint32_t kSlice = 64 * N;
-  static constexpr uint32_t kStepBytes = kTCS * 2 * kSlice;
-  static constexpr uint32_t oB = 0;                    // [2 parity][2 hi/lo][kB]
-  // staging of h_t: [2 parity][2 hi/lo][4 unit octets][N rows][16 B], the
-  // octets 16 N + 16 bytes apart so that a warp's stores of one row (four
-  // octets) fall in distinct banks
+  static constexpr uint32_t kB = N * kTH * 2;          // h_{t-1} in fp16: N rows x 256 units
+  static constexpr uint32_t kSlice = 64 * N;           // one CTA's 32 units of it
+  static constexpr uint32_t kStepBytes = kTCS * kSlice;
+  static constexpr uint32_t oB = 0;                    // [2 parity][kB]
+  // staging of h_t: [2 parity][4 unit octets][N rows][16 B], the octets
+  // 16 N + 16 bytes apart so that a warp's stores of one row (four octets)
+  // fall in distinct banks
   static constexpr uint32_t kOct = 16 * N + 16;
   static constexpr uint32_t kStgS = 4 * kOct;
-  static constexpr uint32_t oStg = oB + 4 * kB;
-  static constexpr uint32_t oGate = oStg + 4 * kStgS;  // [N][4][32] fp32 activated gates
+  static constexpr uint32_t oStg = oB + 2 * kB;
+  static constexpr uint32_t oGate = oStg + 2 * kStgS;  // [N][4][32] fp32 activated gates
   static constexpr uint32_t oBar = oGate + N * 4 * kTHc * 4;  // xbar[2], mmabar
   static constexpr uint32_t kTeam = oBar + 32;
 };
@@ -278,7 +312,7 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
                 P = N / TW, R = N * TM;
   static_assert(C == 4 || C == 8, "4 or 8 accumulator columns per thread");
   static_assert(P * TW == N, "whole rows per warp");
-  constexpr uint32_t idesc = tc_idesc<N>();
+  constexpr uint32_t idesc = tc_idesc<N, true>();
   extern __shared__ __align__(16) uint8_t smem[];
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int tm = warp / TW, wt = warp % TW, tt = t % TT;  // team; warp and thread within it
@@ -313,7 +347,7 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
   }
 #pragma unroll
   for (int k = 0; k < TM; ++k)
-    for (uint32_t i = t; i < 4 * Lay::kB / 16; i += kTThreads)
+    for (uint32_t i = t; i < 2 * Lay::kB / 16; i += kTThreads)
       reinterpret_cast<uint4 *>(smem + k * Lay::kTeam + Lay::oB)[i] = make_uint4(0, 0, 0, 0);
   if (toff_sm)
     for (int i = t; i <= T; i += kTThreads) toff_s[i] = a.ix.tok_off[i];
@@ -324,7 +358,7 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
       uint64_t *b = reinterpret_cast<uint64_t *>(smem + k * Lay::kTeam + Lay::oBar);
       mb_init(sa(&b[0]), 1);
       mb_init(sa(&b[1]), 1);
-      mb_init(sa(&b[2]), 3);
+      mb_init(sa(&b[2]), 4);
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -344,15 +378,15 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
 #pragma unroll
       for (int j = 0; j < 8; j += 2) {
         const float4 v = __ldg(reinterpret_cast<const float4 *>(wrow + 2 * (c0 + j)));
-        __nv_bfloat16 h0, l0, h1, l1, h2, l2, h3, l3;
-        split_bf16(v.x, h0, l0);
-        split_bf16(v.y, h1, l1);
-        split_bf16(v.z, h2, l2);
-        split_bf16(v.w, h3, l3);
-        hi[j] = pack2(h0, h1);
-        lo[j] = pack2(l0, l1);
-        hi[j + 1] = pack2(h2, h3);
-        lo[j + 1] = pack2(l2, l3);
+        __half h0, l0, h1, l1, h2, l2, h3, l3;
+        split_f16(v.x, h0, l0);
+        split_f16(v.y, h1, l1);
+        split_f16(v.z, h2, l2);
+        split_f16(v.w, h3, l3);
+        hi[j] = pack2h(h0, h1);
+        lo[j] = pack2h(l0, l1);
+        hi[j + 1] = pack2h(h2, h3);
+        lo[j + 1] = pack2h(l2, l3);
       }
       tmem_st8(tl + c0, hi);
       tmem_st8(tl + 128 + c0, lo);
@@ -391,10 +425,11 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
   float cst[P];
 #pragma unroll
   for (int j = 0; j < P; ++j) cst[j] = 0.f;
-  // MMA issuers: lane 0 of the team's warps 0 .. 2, issuer p forms product p
-  // (W_hi h_hi, W_hi h_lo, W_lo h_hi) into its own accumulator
-  const int prod = (lane == 0 && wt < 3) ? wt : -1;
-  const uint32_t acc0 = kAccCol + 32u * (uint32_t)(3 * tm);  // the team's three accumulators
+  // MMA issuers: lane 0 of the team's warps 0 .. 3; issuer i forms W_hi h
+  // (i < 2) or W_lo h (i >= 2) over k-steps 8 (i % 2) .. + 7 into its own
+  // accumulator
+  const int prod = (lane == 0 && wt < 4) ? wt : -1;
+  const uint32_t acc0 = kAccCol + 32u * (uint32_t)(4 * tm);  // the team's four accumulators
   bool ok = true, stop = false;
   int mma_issued = 0, mma_seen = 0;
 
@@ -417,13 +452,13 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
         if (ok) {
           fence_proxy();
           fence_after();
-          const uint32_t bh = sa(Bb + (2 * (e & 1)) * Lay::kB);
-          const uint32_t bsel = bh + (prod == 1 ? Lay::kB : 0u);
-          const uint32_t asel = tmem + (prod == 2 ? 128u : 0u);
+          const uint32_t bsel = sa(Bb + (e & 1) * Lay::kB);
+          const uint32_t asel = tmem + (prod >= 2 ? 128u : 0u);
           const uint32_t dcol = tmem + acc0 + 32u * (uint32_t)prod;
+          const int j0 = 8 * (prod & 1);
 #pragma unroll
-          for (int j = 0; j < H / 16; ++j)
-            mma_ts(dcol, asel + 8 * j, desc_kmajor(bsel + (uint32_t)(2 * j) * (16u * N), 16 * N, 128), idesc, j > 0);
+          for (int j = j0; j < j0 + 8; ++j)
+            mma_ts(dcol, asel + 8 * j, desc_kmajor(bsel + (uint32_t)(2 * j) * (16u * N), 16 * N, 128), idesc, j > j0);
           mma_commit(sa(&bar[2]));
         } else {
           mb_arrive(sa(&bar[2]));
@@ -434,8 +469,14 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
       if (got) ++mma_seen;
       ok = got && ok;
       fence_after();
+      uint32_t r[4][C];
 #pragma unroll
-      for (int p = 0; p < 3; ++p) tmem_ld_add<C>(tl + acc0 + 32 * p + col0, acc);
+      for (int p = 0; p < 4; ++p) tmem_ld_raw<C>(tl + acc0 + 32 * p + col0, r[p]);
+      asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+      for (int k = 0; k < C; ++k)
+        acc[k] += (__uint_as_float(r[0][k]) + __uint_as_float(r[1][k])) +
+                  (__uint_as_float(r[2][k]) + __uint_as_float(r[3][k])) * (1.f / kF16LoScale);
     }
     // gate q of unit `lane` for this thread's columns (uniform per warp)
 #pragma unroll
@@ -453,7 +494,7 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
     }
     // cell update of unit `lane`, rows P wt + j
     const uint32_t par = (uint32_t)(s & 1);
-    uint8_t *sg_hi = stg + (2 * par) * Lay::kStgS, *sg_lo = sg_hi + Lay::kStgS;
+    uint8_t *sg = stg + par * Lay::kStgS;
 #pragma unroll
     for (int j = 0; j < P; ++j) {
       const int n = P * wt + j;
@@ -461,38 +502,35 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
       const float gg = gate[(n * 4 + 2) * kTHc + lane], og = gate[(n * 4 + 3) * kTHc + lane];
       const float cn = fmaf(fg, cst[j], ig * gg);
       float h = og * tanh_tc(cn);
-      __nv_bfloat16 hh, hl;
       if (s < lenp[j]) {
         cst[j] = cn;
         const size_t tk = (size_t)tok_row(j, s);
         Cs[tk * H + gu] = cn;
         Y[tk * DH + d * H + gu] = h;
-        split_bf16(h, hh, hl);
-        if (Yb) Yb[tk * DH + d * H + gu] = hh;
+        const __nv_bfloat16 hb = __float2bfloat16_rn(h);
+        if (Yb) Yb[tk * DH + d * H + gu] = hb;
         if (Hs) {
           if (s == 0) Hs[tk * H + gu] = __float2bfloat16_rn(0.f);
-          if (s + 1 < lenp[j]) Hs[(size_t)tok_row(j, s + 1) * H + gu] = hh;
+          if (s + 1 < lenp[j]) Hs[(size_t)tok_row(j, s + 1) * H + gu] = hb;
         }
       } else {
         h = 0.f;
-        split_bf16(h, hh, hl);
       }
       const uint32_t off = (uint32_t)(lane >> 3) * Lay::kOct + (uint32_t)n * 16u + (uint32_t)(lane & 7) * 2u;
-      *reinterpret_cast<__nv_bfloat16 *>(sg_hi + off) = hh;
-      *reinterpret_cast<__nv_bfloat16 *>(sg_lo + off) = hl;
+      *reinterpret_cast<__half *>(sg + off) = __float2half_rn(h);
     }
     team_sync(bid, TT);
     if (s + 1 < Tg && !withhold) {
-      constexpr int kPieces = 2 * Lay::kSlice / 16;
-      const uint32_t dst0 = sa(Bb + (2 * par) * Lay::kB) + c * (uint32_t)Lay::kSlice;
+      constexpr int kPieces = Lay::kSlice / 16;
+      const uint32_t dst0 = sa(Bb + par * Lay::kB) + c * (uint32_t)Lay::kSlice;
       const uint32_t mbl = sa(&bar[par]);
 #pragma unroll
       for (int i = tt; i < kTCS * kPieces; i += TT) {
-        // piece pc = (octet, row) of part hl: 16 pc bytes into the K-major slice
-        const int pr = i / kPieces, rem = i % kPieces, hl = rem / (kPieces / 2), pc = rem % (kPieces / 2);
+        // piece pc = (octet, row): 16 pc bytes into the K-major slice
+        const int pr = i / kPieces, pc = i % kPieces;
         const uint32_t o = (uint32_t)pc * 16u, so = (uint32_t)(pc / N) * Lay::kOct + (uint32_t)(pc % N) * 16u;
-        const uint4 v = *reinterpret_cast<const uint4 *>(stg + (2 * par + hl) * Lay::kStgS + so);
-        st_async16(peer(dst0 + (uint32_t)hl * Lay::kB + o, (uint32_t)pr), v, peer(mbl, (uint32_t)pr));
+        const uint4 v = *reinterpret_cast<const uint4 *>(sg + so);
+        st_async16(peer(dst0 + o, (uint32_t)pr), v, peer(mbl, (uint32_t)pr));
       }
     }
   }
