@@ -186,8 +186,9 @@ cudaError_t launch_ctc_grad(const DevIdx &ix, float *logp_dlogit, int C, int bla
 // Geometry of the recurrent kernels for one layer.
 //   mode 1: one CTA per bc rows holds all of W_hh (H in {32, 64, 128});
 //   mode 2: register-tiled cluster of cs CTAs per bc rows (H in {256, 512});
-//   mode 3: tensor-core cluster of 8 CTAs per bc rows, W_hh in TMEM
-//           (H = 256 with bf16 contractions);
+//   mode 3: tensor-core clusters of 8 CTAs, 16 or 32 rows each, W_hh in
+//           TMEM (H = 256 with bf16 contractions); bc = the clusters that
+//           can be resident at once;
 //   mode 0: a cluster of cs CTAs per bc rows splits the hidden units (any H).
 struct RecGeom {
   int mode;
@@ -235,11 +236,12 @@ cudaError_t launch_lstm_cl(const RecArgs &a, int bc, bool bwd, cudaStream_t s);
 
 // Tensor-core cluster kernels for H = 256 on the bf16 path (k_lstm_tc.cu):
 // whether H is handled there (BKT_REC_TC=0 in the environment turns them
-// off), rows per cluster for a batch of b rows (16 or 32; 0: cannot launch),
-// launch.
+// off), how many of their 8-CTA clusters can be resident at once (0: they
+// cannot launch), and the launch, which lays the batch's rows out over at
+// most max_clusters clusters.
 bool tc_rec_supported(int H);
-int plan_tc_rows(int b, int dirs);
-cudaError_t launch_lstm_tc(const RecArgs &a, int rows, bool bwd, cudaStream_t s);
+int tc_clusters_resident();
+cudaError_t launch_lstm_tc(const RecArgs &a, int max_clusters, bool bwd, cudaStream_t s);
 
 // Single-CTA recurrent kernels (k_lstm_cta.cu).
 bool cta_supported(int H);

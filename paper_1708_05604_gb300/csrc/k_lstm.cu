@@ -332,13 +332,13 @@ RecGeom plan_recurrent(int H, int b, int dirs, int sm_count, bool bf16) {
   const size_t lim = 220 * 1024;
   RecGeom g{};
   if (bf16 && tc_rec_supported(H)) {
-    const int rows = plan_tc_rows(b, dirs);
-    if (rows > 0) {
+    const int resident = tc_clusters_resident();
+    if (resident > 0) {
       g.mode = 3;
       g.cs = 8;
-      g.bc = rows;
+      g.bc = resident;
       g.ks = 1;
-      g.threads = 128;
+      g.threads = 512;
       g.w_smem = 0;
       return g;
     }

@@ -304,8 +304,9 @@ size_t tc_smem_bytes(size_t base, int T) {
 // meet through shared memory, then thread (w, lane) updates the cell of unit
 // `lane` for its P rows.  (A lane order 4u + q, with the gates swapped by
 // shuffles inside groups of four lanes, measured 10 % slower per step.)
+// The body of one cluster: direction d, rows rc .. rc + TM N - 1.
 template <int N, int TM>
-__global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
+__device__ __forceinline__ void fwd_tc_body(const RecArgs &a, uint8_t *smem, const int d, const int rc) {
   using Lay = TcFwdLayout<N>;
   using Sm = TcSmem<Lay, N, TM>;
   constexpr int H = kTH, G = 4 * H, kTThreads = 512, TW = 16 / TM, TT = 32 * TW, QW = TW / 4, C = N / QW,
@@ -313,7 +314,6 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
   static_assert(C == 4 || C == 8, "4 or 8 accumulator columns per thread");
   static_assert(P * TW == N, "whole rows per warp");
   constexpr uint32_t idesc = tc_idesc<N, true>();
-  extern __shared__ __align__(16) uint8_t smem[];
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int tm = warp / TW, wt = warp % TW, tt = t % TT;  // team; warp and thread within it
   uint8_t *team = smem + tm * Lay::kTeam;
@@ -330,9 +330,7 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
   const int col0 = C * cs;
   const uint32_t c = cluster_rank();
   const int gu = (int)c * kTHc + lane;      // the unit of this lane (both phases)
-  const int n_groups = (a.ix.b + R - 1) / R;
-  const int cid = blockIdx.x / kTCS;
-  const int d = cid / n_groups, rc = (cid % n_groups) * R, r0 = rc + tm * N;
+  const int r0 = rc + tm * N;
   const int DH = a.dirs * H, T = a.ix.T;
   const bool toff_sm = T + 1 <= kTTokCap;
   const int *toff = toff_sm ? toff_s : a.ix.tok_off;
@@ -542,8 +540,10 @@ __global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a) {
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
 }
 
+// The body of one cluster: direction d, rows rc .. rc + TM N - 1 (smem
+// 1024-byte aligned).
 template <int N, int TM>
-__global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
+__device__ __forceinline__ void bwd_tc_body(const RecArgs &a, uint8_t *smem, const int d, const int rc) {
   using Lay = TcBwdLayout<N>;
   using Sm = TcSmem<Lay, N, TM>;
   constexpr int H = kTH, G = 4 * H, kTThreads = 512, TW = 16 / TM, TT = 32 * TW, QW = TW / 4, C = N / QW,
@@ -556,8 +556,6 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
   static_assert(C == 4 || C == 8, "4 or 8 accumulator columns per thread");
   static_assert(P * TW == N && 2 * AH <= TW, "whole rows per warp; an issuer per warp");
   constexpr uint32_t idesc = tc_idesc<N>();
-  extern __shared__ __align__(16) uint8_t smem_raw[];
-  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int tm = warp / TW, wt = warp % TW, tt = t % TT;
   uint8_t *team = smem + tm * Lay::kTeam;
@@ -575,9 +573,7 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
   const int u = lane;  // phase B: unit `lane`, rows P wt + j
   const uint32_t c = cluster_rank();
   const int gu = (int)c * kTHc + u;
-  const int n_groups = (a.ix.b + R - 1) / R;
-  const int cid = blockIdx.x / kTCS;
-  const int d = cid / n_groups, rc = (cid % n_groups) * R, r0 = rc + tm * N;
+  const int r0 = rc + tm * N;
   const int DH = a.dirs * H, T = a.ix.T;
   const bool toff_sm = T + 1 <= kTTokCap;
   const int *toff = toff_sm ? toff_s : a.ix.tok_off;
@@ -830,13 +826,62 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a) {
 }
 
 // ---------------------------------------------------------------------------
+// Cluster layout of a launch.  A cluster of one team (16 rows on all 16
+// warps) takes a step in about 1.7 us, a cluster of two teams (32 rows, 8
+// warps each) about 2.9 us: the step is latency-bound, and two teams only
+// partly hide each other's waits.  So one-team clusters are used wherever
+// they fit: the longest rows of the length-sorted batch go to n1 one-team
+// clusters per direction, the shortest to n2 two-team clusters, with
+// dirs (n1 + n2) no more than the 8-CTA clusters that can be resident at
+// once (15 on a 152-SM GB300; a cluster beyond them would start only when
+// another ends, after the rows it was meant to run beside).
 namespace {
 
-template <typename K>
-cudaLaunchConfig_t tc_config(int clusters, int threads, size_t smem, cudaStream_t s, cudaLaunchAttribute *attr) {
+constexpr int kTN = 16;  // rows per team: the N of the MMAs
+
+struct TcSplit {
+  int n1, n2;  // clusters per direction of one team (16 rows) and of two teams (32 rows)
+};
+
+}  // namespace
+
+template <int N>
+__global__ void __launch_bounds__(512, 1) lstm_fwd_tc_kernel(RecArgs a, TcSplit sp) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  const int cid = blockIdx.x / kTCS, per = sp.n1 + sp.n2;
+  const int d = cid / per, g = cid % per;
+  if (g < sp.n1)
+    fwd_tc_body<N, 1>(a, smem, d, N * g);
+  else
+    fwd_tc_body<N, 2>(a, smem, d, N * sp.n1 + 2 * N * (g - sp.n1));
+}
+
+template <int N>
+__global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a, TcSplit sp) {
+  extern __shared__ __align__(16) uint8_t smem_raw[];
+  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int cid = blockIdx.x / kTCS, per = sp.n1 + sp.n2;
+  const int d = cid / per, g = cid % per;
+  if (g < sp.n1)
+    bwd_tc_body<N, 1>(a, smem, d, N * g);
+  else
+    bwd_tc_body<N, 2>(a, smem, d, N * sp.n1 + 2 * N * (g - sp.n1));
+}
+
+namespace {
+
+// Dynamic shared memory of a launch: the larger of the two bodies' layouts
+// (BPTT: + 1 KB to align its base to 1024 bytes) and the time offsets.
+size_t tc_smem(bool bwd, int T) {
+  const size_t f = std::max(TcSmem<TcFwdLayout<kTN>, kTN, 1>::oToff, TcSmem<TcFwdLayout<kTN>, kTN, 2>::oToff);
+  const size_t b = std::max(TcSmem<TcBwdLayout<kTN>, kTN, 1>::oToff, TcSmem<TcBwdLayout<kTN>, kTN, 2>::oToff) + 1024;
+  return tc_smem_bytes(bwd ? b : f, T);
+}
+
+cudaLaunchConfig_t tc_config(int clusters, size_t smem, cudaStream_t s, cudaLaunchAttribute *attr) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(clusters * kTCS, 1, 1);
-  cfg.blockDim = dim3(threads, 1, 1);
+  cfg.blockDim = dim3(512, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   attr->id = cudaLaunchAttributeClusterDimension;
@@ -848,53 +893,14 @@ cudaLaunchConfig_t tc_config(int clusters, int threads, size_t smem, cudaStream_
   return cfg;
 }
 
-template <int N, int TM>
-size_t tc_smem(bool bwd, int T) {
-  // (BPTT: + 1 KB to align its base to 1024 bytes)
-  return tc_smem_bytes(bwd ? TcSmem<TcBwdLayout<N>, N, TM>::oToff + 1024 : TcSmem<TcFwdLayout<N>, N, TM>::oToff, T);
-}
-
-// N rows per team, TM teams: N TM rows per cluster.
-template <int N, int TM>
-cudaError_t launch_tc(const RecArgs &a, bool bwd, cudaStream_t s) {
-  if (a.ix.b <= 0 || a.ix.T <= 0) return cudaSuccess;
-  if (a.H != kTH) return cudaErrorInvalidValue;
-  const size_t smem = tc_smem<N, TM>(bwd, a.ix.T);
-  const int clusters = ((a.ix.b + N * TM - 1) / (N * TM)) * a.dirs;
-  cudaLaunchAttribute attr;
-
-  if (bwd) {
-    auto k = lstm_bwd_tc_kernel<N, TM>;
-    cudaError_t e = ensure_smem((const void *)k, smem);
-    if (e != cudaSuccess) return e;
-    cudaLaunchConfig_t cfg = tc_config<decltype(k)>(clusters, 512, smem, s, &attr);
-    return cudaLaunchKernelEx(&cfg, k, a);
-  }
-  auto k = lstm_fwd_tc_kernel<N, TM>;
-  cudaError_t e = ensure_smem((const void *)k, smem);
-  if (e != cudaSuccess) return e;
-  cudaLaunchConfig_t cfg = tc_config<decltype(k)>(clusters, 512, smem, s, &attr);
-  return cudaLaunchKernelEx(&cfg, k, a);
-}
-
 // 8-CTA clusters of one kernel that can be resident at once (0: cannot launch).
-template <int N, int TM>
-int tc_resident_one(bool bwd) {
-  const size_t smem = tc_smem<N, TM>(bwd, kTTokCap - 1);
+template <typename K>
+int tc_resident_one(K k, size_t smem) {
   cudaLaunchAttribute attr;
   int n = 0;
-  cudaError_t e;
-  if (bwd) {
-    auto k = lstm_bwd_tc_kernel<N, TM>;
-    e = ensure_smem((const void *)k, smem);
-    cudaLaunchConfig_t cfg = tc_config<decltype(k)>(1, 512, smem, 0, &attr);
-    if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, k, &cfg);
-  } else {
-    auto k = lstm_fwd_tc_kernel<N, TM>;
-    e = ensure_smem((const void *)k, smem);
-    cudaLaunchConfig_t cfg = tc_config<decltype(k)>(1, 512, smem, 0, &attr);
-    if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, k, &cfg);
-  }
+  cudaError_t e = ensure_smem((const void *)k, smem);
+  cudaLaunchConfig_t cfg = tc_config(1, smem, 0, &attr);
+  if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, k, &cfg);
   if (e != cudaSuccess) {
     cudaGetLastError();
     return 0;
@@ -902,10 +908,22 @@ int tc_resident_one(bool bwd) {
   return n;
 }
 
-// 32 rows per cluster, as two teams of 16 rows (one team's MMAs and
-// exchange overlap the other's elementwise work).
-int tc_resident32() { return std::min(tc_resident_one<16, 2>(false), tc_resident_one<16, 2>(true)); }
-cudaError_t launch_tc32(const RecArgs &a, bool bwd, cudaStream_t s) { return launch_tc<16, 2>(a, bwd, s); }
+TcSplit tc_split(int b, int dirs, int max_clusters) {
+  const int groups = (b + kTN - 1) / kTN;                // 16-row groups per direction
+  const int per = std::max(1, max_clusters / dirs);      // clusters per direction resident at once
+  TcSplit sp;
+  if (groups <= per) {
+    sp.n1 = groups;
+    sp.n2 = 0;
+  } else if (groups - per >= (groups + 1) / 2) {
+    sp.n1 = 0;  // two teams everywhere (clusters beyond the resident ones wait)
+    sp.n2 = (groups + 1) / 2;
+  } else {
+    sp.n2 = groups - per;  // each two-team cluster saves one cluster
+    sp.n1 = groups - 2 * sp.n2;
+  }
+  return sp;
+}
 
 }  // namespace
 
@@ -917,21 +935,30 @@ bool tc_rec_supported(int H) {
   return H == kTH && !off;
 }
 
-int plan_tc_rows(int b, int dirs) {
-  // 32 rows per cluster: an MMA costs the same at N = 16 and 32 (its issue,
-  // not its columns, bounds it), so fewer, wider clusters leave SMs to the
-  // side stream; 16 when the batch is small enough for its clusters to fit
-  // either way (0: neither can launch)
-  const int r16 = std::min(tc_resident_one<16, 1>(false), tc_resident_one<16, 1>(true)), r32 = tc_resident32();
-  if (r16 > 0 && ((b + 15) / 16) * dirs <= std::min(r16, 4)) return 16;
-  if (r32 > 0) return 32;
-  return r16 > 0 ? 16 : 0;
+int tc_clusters_resident() {
+  const int f = tc_resident_one(lstm_fwd_tc_kernel<kTN>, tc_smem(false, kTTokCap - 1));
+  const int b = tc_resident_one(lstm_bwd_tc_kernel<kTN>, tc_smem(true, kTTokCap - 1));
+  return std::min(f, b);
 }
 
-cudaError_t launch_lstm_tc(const RecArgs &a, int rows, bool bwd, cudaStream_t s) {
-  if (rows == 16) return launch_tc<16, 1>(a, bwd, s);
-  if (rows == 32) return launch_tc32(a, bwd, s);
-  return cudaErrorInvalidValue;
+cudaError_t launch_lstm_tc(const RecArgs &a, int max_clusters, bool bwd, cudaStream_t s) {
+  if (a.ix.b <= 0 || a.ix.T <= 0) return cudaSuccess;
+  if (a.H != kTH || max_clusters <= 0 || a.dirs < 1 || a.dirs > 2) return cudaErrorInvalidValue;
+  const TcSplit sp = tc_split(a.ix.b, a.dirs, max_clusters);
+  const size_t smem = tc_smem(bwd, a.ix.T);
+  const int clusters = (sp.n1 + sp.n2) * a.dirs;
+  cudaLaunchAttribute attr;
+  cudaLaunchConfig_t cfg = tc_config(clusters, smem, s, &attr);
+  if (bwd) {
+    auto k = lstm_bwd_tc_kernel<kTN>;
+    cudaError_t e = ensure_smem((const void *)k, smem);
+    if (e != cudaSuccess) return e;
+    return cudaLaunchKernelEx(&cfg, k, a, sp);
+  }
+  auto k = lstm_fwd_tc_kernel<kTN>;
+  cudaError_t e = ensure_smem((const void *)k, smem);
+  if (e != cudaSuccess) return e;
+  return cudaLaunchKernelEx(&cfg, k, a, sp);
 }
 
 }  // namespace bkt

@@ -2,10 +2,11 @@
 per-kernel CUDA-event times (per launch and per recurrent time step).
 
   python -m paper_1708_05604_gb300.profile_step [--workload NAME] [--buckets Q]
-         [--batch K] [--repeat R]
+         [--batch K] [--rows M] [--repeat R]
 
-The batch is batch K of the epoch-0 plan with Q buckets; the step runs R times
-on it (the first run includes one-time set-up).  Useful on its own and as the
+The batch is batch K of the epoch-0 plan with Q buckets (its first M
+sequences with --rows); the step runs R times on it (the first run includes
+one-time set-up).  Useful on its own and as the
 target of an ncu capture of a single kernel.
 """
 from __future__ import annotations
@@ -22,6 +23,7 @@ def main(argv=None):
     ap.add_argument("--workload", default="lstm1_bi_h128")
     ap.add_argument("--buckets", type=int, default=4)
     ap.add_argument("--batch", type=int, default=8)
+    ap.add_argument("--rows", type=int, default=0, help="keep the batch's first M sequences")
     ap.add_argument("--repeat", type=int, default=3)
     ap.add_argument("--seed", type=int, default=0)
     a = ap.parse_args(argv)
@@ -36,6 +38,8 @@ def main(argv=None):
     plan = binding.plan_buckets(ds.lengths, a.buckets, w.batch, a.seed, 0)
     k = min(a.batch, plan["n_batches"] - 1)
     ids = plan["order"][plan["batch_off"][k]:plan["batch_off"][k + 1]]
+    if a.rows > 0:
+        ids = ids[:a.rows]
     cfg = w.model_cfg()
     dd = binding.DeviceDataset(ds)
     ctx = binding.Ctx(cfg, int(ds.lengths[ids].sum()), len(ids), int(ds.label_lengths.max()))

@@ -354,6 +354,26 @@ def test_bf16_path_with_the_other_recurrent_kernels(layers, bi, H):
     compare(cfg, lg, gg, lo, go, BF16_TOL)
 
 
+@pytest.mark.parametrize("b", [100, 120, 232])
+def test_tensor_core_recurrence_cluster_layouts(b):
+    """The H = 256 tensor-core recurrence spreads a batch over one-team
+    (16-row) and two-team (32-row) clusters, no more of them than can be
+    resident at once (15 on a GB300): 100 rows run on one-team clusters
+    only, 120 on six one-team clusters and one two-team cluster per
+    direction (its second team partly filled), 232 on two-team clusters only
+    (one team empty; more clusters than fit at once).  Rows end at every
+    step; one bidirectional layer with bf16 contractions, at the bf16
+    bound."""
+    cfg = {"n_layers": 1, "bidirectional": True, "in_dim": 4, "hidden": 256, "n_classes": 81, "blank": 0,
+           "gemm_bf16": True}
+    rng = np.random.default_rng(b)
+    ds = synth.make_dataset(rng.integers(1, 15, size=b), 4, rng)
+    params = synth.draw_params(rng, binding.param_count(cfg))
+    lg, gg = gpu_step(cfg, ds, params)
+    lo, go = oracle_step_parallel(cfg, ds, params, np.arange(ds.n))
+    compare(cfg, lg, gg, lo, go, BF16_TOL)
+
+
 def test_bf16_workload_runs_on_tensor_cores():
     """The bf16 workloads route their contractions through the tcgen05 GEMM
     (and stay within the bf16 tolerance while differing from fp32 rounding)."""
