@@ -536,6 +536,9 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     if (bf16) {  // the bf16 copies the contractions read (written by the kernel when it can)
       ra.Yb = l + 1 < lo.L ? w.Yb[l] : nullptr;
       for (int d = 0; d < dirs; ++d) ra.Hs[d] = w.Hs[l * dirs + d];
+      // below the top layer only the bf16 copies are read when the kernel
+      // writes them (projection, dW_ih and dW_hh): no fp32 h
+      if (l + 1 < lo.L && bkt::rec_writes_bf16(geom[l])) ra.Y = nullptr;
     }
     L.run("lstm_fwd", flops_w(8.0 * H * H * (double)NT * dirs, ix.T), [&] { return bkt::launch_lstm_fwd(ra, geom[l], s); });
     if (bf16 && l + 1 < lo.L && !bkt::rec_writes_bf16(geom[l]))

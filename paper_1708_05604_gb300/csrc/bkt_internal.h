@@ -211,7 +211,7 @@ struct RecArgs {
   float *Z[2];
   float *Cst[2];
   const float *Whh[2];
-  float *Y;            // forward output / backward: h source for nothing
+  float *Y;            // forward: fp32 h [n_tok x dirs*H] (the tensor-core kernels take null: no fp32 copy)
   const float *dY;     // backward: d loss / d Y of this layer [n_tok x dirs*H]
   int32_t *status;     // device error flags (bit 4: a cluster exchange wait timed out)
   WaitFaults wf;       // poll cap / withheld exchange (failure-detection tests)

@@ -208,6 +208,18 @@ __device__ __forceinline__ void split_f16(float x, __half &hi, __half &lo) {
 __device__ __forceinline__ uint32_t pack2h(__half a, __half b) {
   return (uint32_t)__half_as_ushort(a) | ((uint32_t)__half_as_ushort(b) << 16);
 }
+__device__ __forceinline__ uint32_t pack2bf(float a, float b) {
+  return pack2(__float2bfloat16_rn(a), __float2bfloat16_rn(b));
+}
+// 16-byte asynchronous copy global -> shared; `bytes` = 0 fills zeros.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, uint32_t bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void cp_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int K>
+__device__ __forceinline__ void cp_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(K) : "memory");
+}
 // C consecutive columns of this thread's lane, not yet waited for
 template <int C>
 __device__ __forceinline__ void tmem_ld_raw(uint32_t taddr, uint32_t (&r)[C]) {
@@ -269,9 +281,13 @@ struct TcFwdLayout {
   static constexpr uint32_t kOct = 16 * N + 16;
   static constexpr uint32_t kStgS = 4 * kOct;
   static constexpr uint32_t oStg = oB + 2 * kB;
-  static constexpr uint32_t oGate = oStg + 2 * kStgS;  // [N][4][32] fp32 activated gates
-  static constexpr uint32_t oBar = oGate + N * 4 * kTHc * 4;  // xbar[2], mmabar
+  static constexpr uint32_t kRowF = 4 * kTHc;                    // floats of one row: [4 gates][32 units]
+  static constexpr uint32_t oGate = oStg + 2 * kStgS;            // [2 parity][N][4][32] fp32 activated gates
+  static constexpr uint32_t oCell = oGate + 2 * N * kRowF * 4;   // [2 parity][c, h][N][32] fp32
+  static constexpr uint32_t oZx = oCell + 2 * 2 * N * kTHc * 4;  // [3 stages][N][4][32] fp32 Zx
+  static constexpr uint32_t oBar = oZx + 3 * N * kRowF * 4;      // xbar[2], mmabar
   static constexpr uint32_t kTeam = oBar + 32;
+  static_assert(oGate % 16 == 0 && oCell % 16 == 0 && oZx % 16 == 0, "16-byte staging rows");
 };
 
 template <typename L, int N, int TM>
@@ -282,8 +298,25 @@ struct TcSmem {
   static_assert(L::kTeam % 16 == 0, "team regions keep 16-byte operand alignment");
 };
 
-size_t tc_smem_bytes(size_t base, int T) {
-  const size_t need = base + (T + 1 <= kTTokCap ? (size_t)(T + 1) * 4 : 0);
+// Dynamic shared memory of a launch: the larger of the one- and two-team
+// layouts (BPTT: + 1 KB to align its base to 1024 bytes), then the time
+// offsets when they fit under the per-block limit (else they are read from
+// global memory; only the warps that move data read them).
+constexpr uint32_t kSmemMax = 232448;
+__host__ __device__ constexpr uint32_t umax(uint32_t x, uint32_t y) { return x > y ? x : y; }
+template <int N>
+__host__ __device__ constexpr uint32_t tc_base(bool bwd) {
+  return bwd ? umax(TcSmem<TcBwdLayout<N>, N, 1>::oToff, TcSmem<TcBwdLayout<N>, N, 2>::oToff) + 1024
+             : umax(TcSmem<TcFwdLayout<N>, N, 1>::oToff, TcSmem<TcFwdLayout<N>, N, 2>::oToff);
+}
+template <int N>
+__host__ __device__ constexpr int tc_tok_cap(bool bwd) {
+  return (int)((kSmemMax - tc_base<N>(bwd)) / 4) < kTTokCap ? (int)((kSmemMax - tc_base<N>(bwd)) / 4) : kTTokCap;
+}
+
+template <int N>
+size_t tc_smem_bytes(bool bwd, int T) {
+  const size_t need = tc_base<N>(bwd) + (T + 1 <= tc_tok_cap<N>(bwd) ? (size_t)(T + 1) * 4 : 0);
   return std::max(need, kTSmemFloor);
 }
 
@@ -305,14 +338,25 @@ size_t tc_smem_bytes(size_t base, int T) {
 // `lane` for its P rows.  (A lane order 4u + q, with the gates swapped by
 // shuffles inside groups of four lanes, measured 10 % slower per step.)
 // The body of one cluster: direction d, rows rc .. rc + TM N - 1.
+//
+// A step's chain (exchange, MMAs, gates, cell update, exchange) touches
+// only shared memory and TMEM.  The step's outputs go to a staging area
+// (gates and c, h in fp32, double-buffered by step parity), and during the
+// next step's exchange wait and MMAs the team's warps that issue no MMAs
+// (warps 4 .. TW - 1) write them to global memory as 16-byte pieces and
+// bring Zx of two steps ahead into a three-stage ring with asynchronous
+// copies.  (A step's stores, ~14 KB per CTA, take ~450 cycles at the SM's
+// ~32 bytes per clock to L2, measured; inside the gate and cell phases, or
+// issued by every warp after the send, they lengthened the step.)
 template <int N, int TM>
 __device__ __forceinline__ void fwd_tc_body(const RecArgs &a, uint8_t *smem, const int d, const int rc) {
   using Lay = TcFwdLayout<N>;
   using Sm = TcSmem<Lay, N, TM>;
   constexpr int H = kTH, G = 4 * H, kTThreads = 512, TW = 16 / TM, TT = 32 * TW, QW = TW / 4, C = N / QW,
-                P = N / TW, R = N * TM;
+                P = N / TW, R = N * TM, RF = Lay::kRowF, NWK = TT - 128;
   static_assert(C == 4 || C == 8, "4 or 8 accumulator columns per thread");
   static_assert(P * TW == N, "whole rows per warp");
+  static_assert(NWK > 0, "warps 4 .. TW - 1 of a team move the step's data");
   constexpr uint32_t idesc = tc_idesc<N, true>();
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int tm = warp / TW, wt = warp % TW, tt = t % TT;  // team; warp and thread within it
@@ -320,6 +364,8 @@ __device__ __forceinline__ void fwd_tc_body(const RecArgs &a, uint8_t *smem, con
   uint8_t *Bb = team + Lay::oB;
   uint8_t *stg = team + Lay::oStg;
   float *gate = reinterpret_cast<float *>(team + Lay::oGate);
+  float *cell = reinterpret_cast<float *>(team + Lay::oCell);
+  float *zx = reinterpret_cast<float *>(team + Lay::oZx);
   uint64_t *bar = reinterpret_cast<uint64_t *>(team + Lay::oBar);
   uint32_t *tslot = reinterpret_cast<uint32_t *>(smem + Sm::oSlot);
   int *rlen_c = reinterpret_cast<int *>(smem + Sm::oLen);
@@ -332,11 +378,64 @@ __device__ __forceinline__ void fwd_tc_body(const RecArgs &a, uint8_t *smem, con
   const int gu = (int)c * kTHc + lane;      // the unit of this lane (both phases)
   const int r0 = rc + tm * N;
   const int DH = a.dirs * H, T = a.ix.T;
-  const bool toff_sm = T + 1 <= kTTokCap;
+  const bool toff_sm = T + 1 <= tc_tok_cap<N>(false);
   const int *toff = toff_sm ? toff_s : a.ix.tok_off;
   const int cap = a.wf.poll_cap > 0 ? a.wf.poll_cap : kTPolls;
   const bool withhold = (a.wf.withhold & kWithholdExchange) && c == 0;
   const int bid = 1 + tm;
+  float *__restrict__ Z = a.Z[d];
+  float *__restrict__ Cs = a.Cst[d];
+  float *__restrict__ Y = a.Y;
+  __nv_bfloat16 *__restrict__ Yb = reinterpret_cast<__nv_bfloat16 *>(a.Yb);
+  __nv_bfloat16 *__restrict__ Hs = reinterpret_cast<__nv_bfloat16 *>(a.Hs[d]);
+  // token of row n (of the team) at step s of its direction
+  auto tok_of = [&](int n, int L, int s) { return (size_t)(toff[d == 0 ? s : L - 1 - s] + r0 + n); };
+  // Zx of step sl into ring stage sl % 3 (zeros for rows that have ended),
+  // pieces w0, w0 + nw, ... of the team's 32 N 16-byte pieces
+  auto load_zx = [&](int sl, int w0, int nw) {
+    const uint32_t zs = sa(zx + (sl % 3) * N * RF);
+    for (int i = w0; i < N * 32; i += nw) {
+      const int n = i >> 5, qq = (i >> 3) & 3, ch = i & 7, L = rlen[n];
+      const bool act = sl < L;
+      const float *src = Z + (act ? tok_of(n, L, sl) * G : 0) + qq * H + c * kTHc + 4 * ch;
+      cp_async16(zs + (uint32_t)((n * 4 + qq) * kTHc + 4 * ch) * 4u, src, act ? 16u : 0u);
+    }
+  };
+  // the staged outputs of step sp: gates in place of Zx; c, h; the bf16 h
+  // as Y's copy and as h_{t-1} of the row's next token
+  auto store_step = [&](int sp, int w0, int nw) {
+    const float *gs = gate + (sp & 1) * N * RF;
+    const float *cl = cell + (sp & 1) * 2 * N * kTHc;
+    for (int i = w0; i < N * 32; i += nw) {
+      const int n = i >> 5, qq = (i >> 3) & 3, ch = i & 7, L = rlen[n];
+      if (sp < L)
+        *reinterpret_cast<float4 *>(Z + tok_of(n, L, sp) * G + qq * H + c * kTHc + 4 * ch) =
+            *reinterpret_cast<const float4 *>(gs + (n * 4 + qq) * kTHc + 4 * ch);
+    }
+    for (int i = w0; i < N * 8; i += nw) {
+      const int n = i >> 3, ch = i & 7, L = rlen[n];
+      if (sp < L) {
+        const size_t tk = tok_of(n, L, sp);
+        *reinterpret_cast<float4 *>(Cs + tk * H + c * kTHc + 4 * ch) =
+            *reinterpret_cast<const float4 *>(cl + n * kTHc + 4 * ch);
+        if (Y)
+          *reinterpret_cast<float4 *>(Y + tk * DH + d * H + c * kTHc + 4 * ch) =
+              *reinterpret_cast<const float4 *>(cl + (N + n) * kTHc + 4 * ch);
+      }
+    }
+    if (Yb || Hs) {
+      for (int i = w0; i < N * 4; i += nw) {
+        const int n = i >> 2, ch = i & 3, L = rlen[n];
+        if (sp < L) {
+          const float4 h0 = *reinterpret_cast<const float4 *>(cl + (N + n) * kTHc + 8 * ch);
+          const float4 h1 = *reinterpret_cast<const float4 *>(cl + (N + n) * kTHc + 8 * ch + 4);
+          const uint4 v = make_uint4(pack2bf(h0.x, h0.y), pack2bf(h0.z, h0.w), pack2bf(h1.x, h1.y), pack2bf(h1.z, h1.w));
+          if (Yb) *reinterpret_cast<uint4 *>(Yb + tok_of(n, L, sp) * DH + d * H + c * kTHc + 8 * ch) = v;
+          if (Hs && sp + 1 < L) *reinterpret_cast<uint4 *>(Hs + tok_of(n, L, sp + 1) * H + c * kTHc + 8 * ch) = v;
+        }
+      }
+    }
+  };
 
   if (warp == 0) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(sa(tslot)), "r"(kTmemCols)
@@ -366,6 +465,15 @@ __device__ __forceinline__ void fwd_tc_body(const RecArgs &a, uint8_t *smem, con
   fence_after();
   const uint32_t tmem = *tslot;
   const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16);
+  // Zx of the first two steps; the rows' first h_{t-1} (zero)
+  load_zx(0, tt, TT);
+  load_zx(1, tt, TT);
+  cp_commit();
+  if (Hs)
+    for (int i = tt; i < N * 4; i += TT) {
+      const int n = i >> 2, ch = i & 3, L = rlen[n];
+      if (L > 0) *reinterpret_cast<uint4 *>(Hs + tok_of(n, L, 0) * H + c * kTHc + 8 * ch) = make_uint4(0, 0, 0, 0);
+    }
   // W_hh slice into TMEM (warps 0 .. 3, warp q = lane quarter q): lane
   // 32 q + u holds row q H + 32c + u
   if (warp < 4) {
@@ -391,6 +499,7 @@ __device__ __forceinline__ void fwd_tc_body(const RecArgs &a, uint8_t *smem, con
     }
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
   }
+  cp_wait<0>();
   fence_before();
   __syncthreads();
   const int Tg = rlen[0];
@@ -400,26 +509,9 @@ __device__ __forceinline__ void fwd_tc_body(const RecArgs &a, uint8_t *smem, con
     if (Tg >= 3) mb_arm(sa(&bar[1]), Lay::kStepBytes);
   }
 
-  float *__restrict__ Z = a.Z[d];
-  float *__restrict__ Cs = a.Cst[d];
-  float *__restrict__ Y = a.Y;
-  __nv_bfloat16 *__restrict__ Yb = reinterpret_cast<__nv_bfloat16 *>(a.Yb);
-  __nv_bfloat16 *__restrict__ Hs = reinterpret_cast<__nv_bfloat16 *>(a.Hs[d]);
-  int len[C], lenp[P];  // lengths of this thread's gate columns and cell rows
-#pragma unroll
-  for (int k = 0; k < C; ++k) len[k] = rlen[col0 + k];
+  int lenp[P];  // lengths of this thread's cell rows
 #pragma unroll
   for (int j = 0; j < P; ++j) lenp[j] = rlen[P * wt + j];
-  auto tok_col = [&](int k, int s) { return toff[d == 0 ? s : len[k] - 1 - s] + r0 + col0 + k; };
-  auto tok_row = [&](int j, int s) { return toff[d == 0 ? s : lenp[j] - 1 - s] + r0 + P * wt + j; };
-  // Zx of the next two steps in registers (DRAM latency under the step's own
-  // traffic exceeds one step)
-  float zn[C], zn2[C];
-#pragma unroll
-  for (int k = 0; k < C; ++k) {
-    zn[k] = 0 < len[k] ? Z[(size_t)tok_col(k, 0) * G + q * H + gu] : 0.f;
-    zn2[k] = 1 < len[k] ? Z[(size_t)tok_col(k, 1) * G + q * H + gu] : 0.f;
-  }
   float cst[P];
 #pragma unroll
   for (int j = 0; j < P; ++j) cst[j] = 0.f;
@@ -432,36 +524,37 @@ __device__ __forceinline__ void fwd_tc_body(const RecArgs &a, uint8_t *smem, con
   int mma_issued = 0, mma_seen = 0;
 
   for (int s = 0; s < Tg && !stop; ++s) {
+    const int e = s - 1;
+    if (s > 0 && prod >= 0) {
+      ok = mb_wait(sa(&bar[e & 1]), (e >> 1) & 1, cap) && ok;
+      if (tt == 0 && ok && e + 2 <= Tg - 2) mb_arm(sa(&bar[e & 1]), Lay::kStepBytes);
+      if (ok) {
+        fence_proxy();
+        fence_after();
+        const uint32_t bsel = sa(Bb + (e & 1) * Lay::kB);
+        const uint32_t asel = tmem + (prod >= 2 ? 128u : 0u);
+        const uint32_t dcol = tmem + acc0 + 32u * (uint32_t)prod;
+        const int j0 = 8 * (prod & 1);
+#pragma unroll
+        for (int j = j0; j < j0 + 8; ++j)
+          mma_ts(dcol, asel + 8 * j, desc_kmajor(bsel + (uint32_t)(2 * j) * (16u * N), 16 * N, 128), idesc, j > j0);
+        mma_commit(sa(&bar[2]));
+      } else {
+        mb_arrive(sa(&bar[2]));
+      }
+    }
+    // the movers: step s - 1's outputs out, Zx of step s + 2 in (one
+    // asynchronous-copy group per step)
+    if (wt >= 4) {
+      if (s > 0) store_step(s - 1, tt - 128, NWK);
+      if (s + 2 < Tg) load_zx(s + 2, tt - 128, NWK);
+      cp_commit();
+    }
+    const float *zs = zx + (s % 3) * N * RF;
     float acc[C];
 #pragma unroll
-    for (int k = 0; k < C; ++k) {
-      acc[k] = zn[k];
-      zn[k] = zn2[k];
-    }
-    if (s + 2 < Tg) {
-#pragma unroll
-      for (int k = 0; k < C; ++k) zn2[k] = s + 2 < len[k] ? Z[(size_t)tok_col(k, s + 2) * G + q * H + gu] : 0.f;
-    }
+    for (int k = 0; k < C; ++k) acc[k] = zs[((col0 + k) * 4 + q) * kTHc + lane];
     if (s > 0) {
-      const int e = s - 1;
-      if (prod >= 0) {
-        ok = mb_wait(sa(&bar[e & 1]), (e >> 1) & 1, cap) && ok;
-        if (tt == 0 && ok && e + 2 <= Tg - 2) mb_arm(sa(&bar[e & 1]), Lay::kStepBytes);
-        if (ok) {
-          fence_proxy();
-          fence_after();
-          const uint32_t bsel = sa(Bb + (e & 1) * Lay::kB);
-          const uint32_t asel = tmem + (prod >= 2 ? 128u : 0u);
-          const uint32_t dcol = tmem + acc0 + 32u * (uint32_t)prod;
-          const int j0 = 8 * (prod & 1);
-#pragma unroll
-          for (int j = j0; j < j0 + 8; ++j)
-            mma_ts(dcol, asel + 8 * j, desc_kmajor(bsel + (uint32_t)(2 * j) * (16u * N), 16 * N, 128), idesc, j > j0);
-          mma_commit(sa(&bar[2]));
-        } else {
-          mb_arrive(sa(&bar[2]));
-        }
-      }
       ++mma_issued;
       const bool got = mb_wait(sa(&bar[2]), (uint32_t)(e & 1), cap);
       if (got) ++mma_seen;
@@ -477,12 +570,10 @@ __device__ __forceinline__ void fwd_tc_body(const RecArgs &a, uint8_t *smem, con
                   (__uint_as_float(r[2][k]) + __uint_as_float(r[3][k])) * (1.f / kF16LoScale);
     }
     // gate q of unit `lane` for this thread's columns (uniform per warp)
+    const uint32_t par = (uint32_t)(s & 1);
+    float *gs = gate + par * N * RF;
 #pragma unroll
-    for (int k = 0; k < C; ++k) {
-      const float g = q == 2 ? tanh_tc(acc[k]) : sigm_tc(acc[k]);
-      if (s < len[k]) Z[(size_t)tok_col(k, s) * G + q * H + gu] = g;
-      gate[((col0 + k) * 4 + q) * kTHc + lane] = g;
-    }
+    for (int k = 0; k < C; ++k) gs[((col0 + k) * 4 + q) * kTHc + lane] = q == 2 ? tanh_tc(acc[k]) : sigm_tc(acc[k]);
     fence_before();
     // an issuer that gave up on the exchange stops the whole team
     if (team_sync_or(bid, TT, !ok)) {
@@ -491,32 +582,25 @@ __device__ __forceinline__ void fwd_tc_body(const RecArgs &a, uint8_t *smem, con
       break;
     }
     // cell update of unit `lane`, rows P wt + j
-    const uint32_t par = (uint32_t)(s & 1);
     uint8_t *sg = stg + par * Lay::kStgS;
+    float *cl = cell + par * 2 * N * kTHc;
 #pragma unroll
     for (int j = 0; j < P; ++j) {
       const int n = P * wt + j;
-      const float ig = gate[(n * 4 + 0) * kTHc + lane], fg = gate[(n * 4 + 1) * kTHc + lane];
-      const float gg = gate[(n * 4 + 2) * kTHc + lane], og = gate[(n * 4 + 3) * kTHc + lane];
+      const float ig = gs[(n * 4 + 0) * kTHc + lane], fg = gs[(n * 4 + 1) * kTHc + lane];
+      const float gg = gs[(n * 4 + 2) * kTHc + lane], og = gs[(n * 4 + 3) * kTHc + lane];
       const float cn = fmaf(fg, cst[j], ig * gg);
       float h = og * tanh_tc(cn);
-      if (s < lenp[j]) {
+      if (s < lenp[j])
         cst[j] = cn;
-        const size_t tk = (size_t)tok_row(j, s);
-        Cs[tk * H + gu] = cn;
-        Y[tk * DH + d * H + gu] = h;
-        const __nv_bfloat16 hb = __float2bfloat16_rn(h);
-        if (Yb) Yb[tk * DH + d * H + gu] = hb;
-        if (Hs) {
-          if (s == 0) Hs[tk * H + gu] = __float2bfloat16_rn(0.f);
-          if (s + 1 < lenp[j]) Hs[(size_t)tok_row(j, s + 1) * H + gu] = hb;
-        }
-      } else {
+      else
         h = 0.f;
-      }
+      cl[n * kTHc + lane] = cn;
+      cl[(N + n) * kTHc + lane] = h;
       const uint32_t off = (uint32_t)(lane >> 3) * Lay::kOct + (uint32_t)n * 16u + (uint32_t)(lane & 7) * 2u;
       *reinterpret_cast<__half *>(sg + off) = __float2half_rn(h);
     }
+    if (wt >= 4) cp_wait<1>();  // Zx of step s + 1 has landed (seen by all after the barrier)
     team_sync(bid, TT);
     if (s + 1 < Tg && !withhold) {
       constexpr int kPieces = Lay::kSlice / 16;
@@ -532,6 +616,8 @@ __device__ __forceinline__ void fwd_tc_body(const RecArgs &a, uint8_t *smem, con
       }
     }
   }
+  if (!stop && Tg > 0) store_step(Tg - 1, tt, TT);  // the last step's outputs
+  cp_wait<0>();
   if (mma_seen < mma_issued) mb_wait(sa(&bar[2]), (uint32_t)((mma_issued - 1) & 1), kTPolls);
   if (stop) __nanosleep(20000);
   fence_before();
@@ -575,7 +661,7 @@ __device__ __forceinline__ void bwd_tc_body(const RecArgs &a, uint8_t *smem, con
   const int gu = (int)c * kTHc + u;
   const int r0 = rc + tm * N;
   const int DH = a.dirs * H, T = a.ix.T;
-  const bool toff_sm = T + 1 <= kTTokCap;
+  const bool toff_sm = T + 1 <= tc_tok_cap<N>(true);
   const int *toff = toff_sm ? toff_s : a.ix.tok_off;
   const int cap = a.wf.poll_cap > 0 ? a.wf.poll_cap : kTPolls;
   const bool withhold = (a.wf.withhold & kWithholdExchange) && c == 0;
@@ -870,13 +956,8 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a, TcSplit 
 
 namespace {
 
-// Dynamic shared memory of a launch: the larger of the two bodies' layouts
-// (BPTT: + 1 KB to align its base to 1024 bytes) and the time offsets.
-size_t tc_smem(bool bwd, int T) {
-  const size_t f = std::max(TcSmem<TcFwdLayout<kTN>, kTN, 1>::oToff, TcSmem<TcFwdLayout<kTN>, kTN, 2>::oToff);
-  const size_t b = std::max(TcSmem<TcBwdLayout<kTN>, kTN, 1>::oToff, TcSmem<TcBwdLayout<kTN>, kTN, 2>::oToff) + 1024;
-  return tc_smem_bytes(bwd ? b : f, T);
-}
+size_t tc_smem(bool bwd, int T) { return tc_smem_bytes<kTN>(bwd, T); }
+static_assert(tc_base<kTN>(false) <= kSmemMax && tc_base<kTN>(true) <= kSmemMax, "team layouts fit a CTA");
 
 cudaLaunchConfig_t tc_config(int clusters, size_t smem, cudaStream_t s, cudaLaunchAttribute *attr) {
   cudaLaunchConfig_t cfg = {};
