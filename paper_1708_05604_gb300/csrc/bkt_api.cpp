@@ -702,6 +702,13 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     const bool fused_bf16 = bkt::rec_writes_bf16(geom[l]);
     if (bf16)
       for (int d = 0; d < dirs; ++d) ra.dZb[d] = w.dZb[l * dirs + d];
+    // tensor-core BPTT above layer 1: db as per-cluster partials, and dz only
+    // in bf16 (nothing else reads the fp32 dz there)
+    const bool tc_db = bf16 && l > 0 && geom[l].mode == 3 && w.dbp[l];
+    if (tc_db) {
+      ra.dbp = w.dbp[l];
+      ra.no_dz32 = 1;
+    }
     L.run("lstm_bwd", flops_w(8.0 * H * H * (double)NT * dirs, ix.T), [&] { return bkt::launch_lstm_bwd(ra, geom[l], s); });
     if (bf16 && !fused_bf16)
       for (int d = 0; d < dirs; ++d)
@@ -760,7 +767,14 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
           narrow_on(dZ, grads + lo.w_ih[l * dirs + d], grads + lo.bias(l, d));
         } else {
           tc_reduce(dZb, w.Yb[l - 1], D, grads + lo.w_ih[l * dirs + d]);
-          bias_sum_on(X, dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
+          if (tc_db) {
+            const int ncl = bkt::tc_clusters_per_dir(ix.b, dirs, geom[l].bc);
+            X.run("splitk_sum", pass_w(1, 4 * H, 4.0 * ncl, 4), [&] {
+              return bkt::launch_splitk_sum(w.dbp[l] + (size_t)d * ncl * 4 * H, ncl, 1, 4 * H, grads + lo.bias(l, d), X.s);
+            });
+          } else {
+            bias_sum_on(X, dZ, 4 * H, 4 * H, grads + lo.bias(l, d));
+          }
         }
       }
     } else {
@@ -1066,6 +1080,7 @@ extern "C" int bkt_ctx_create(const bkt_model_cfg *cfg, int64_t max_tokens, int3
           w.Wb[l * lo.dirs + d] = p;
         }
       }
+      if (l > 0) BKT_ALLOC(w.dbp[l], (size_t)lo.dirs * ((max_batch + 15) / 16) * 4 * H);
     }
   }
   IdxLayout il = idx_layout(max_batch, max_tokens);
@@ -1368,6 +1383,7 @@ int bkt::step_on_scratch(const bkt_model_cfg *cfg, const bkt_batch *bt, const fl
       for (int d = 0; d < lo.dirs; ++d) {
         w.Hs[l * lo.dirs + d] = cv.take<uint16_t>(NT * H);
         w.dZb[l * lo.dirs + d] = cv.take<uint16_t>(NT * 4 * H);
+        if (l > 0 && d == 0) w.dbp[l] = cv.take<float>((size_t)lo.dirs * ((b + 15) / 16) * 4 * H);
         if (l > 0) w.Wb[l * lo.dirs + d] = cv.take<uint16_t>(4 * H * DH);
       }
     }

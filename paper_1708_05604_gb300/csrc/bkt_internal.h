@@ -220,6 +220,9 @@ struct RecArgs {
   void *Yb;            // forward: bf16 Y [n_tok x dirs*H]
   void *Hs[2];         // forward: bf16 h_{t-1} of every token of direction d [n_tok x H] (zeros at the start)
   void *dZb[2];        // backward: bf16 dz [n_tok x 4H]
+  // backward, tensor-core kernels only:
+  float *dbp;          // db as one partial sum per cluster, [dirs][clusters per direction][4H] (null: not formed)
+  int no_dz32;         // 1: dz only as the bf16 copy, not over the gates in fp32
 };
 cudaError_t launch_lstm_fwd(const RecArgs &a, const RecGeom &g, cudaStream_t s);
 // Whether the kernels of geometry g write RecArgs' bf16 copies.
@@ -242,6 +245,8 @@ cudaError_t launch_lstm_cl(const RecArgs &a, int bc, bool bwd, cudaStream_t s);
 bool tc_rec_supported(int H);
 int tc_clusters_resident();
 cudaError_t launch_lstm_tc(const RecArgs &a, int max_clusters, bool bwd, cudaStream_t s);
+// clusters per direction that a launch of b rows uses (their db partials)
+int tc_clusters_per_dir(int b, int dirs, int max_clusters);
 
 // Single-CTA recurrent kernels (k_lstm_cta.cu).
 bool cta_supported(int H);
@@ -288,6 +293,7 @@ struct StepBufs {
   void *Yb[kMaxLayers];                       // [NT x dirs*H] bf16 Y of layers 0 .. L-2
   void *Hs[2 * kMaxLayers];                   // per layer*dirs+dir: [NT x H] bf16 h_{t-1}
   void *dZb[2 * kMaxLayers];                  // per layer*dirs+dir: [NT x 4H] bf16 dz
+  float *dbp[kMaxLayers];                     // layers > 0: db partials of the tensor-core BPTT [dirs x ceil(b/16) x 4H]
   void *Wb[2 * kMaxLayers];                   // per layer*dirs+dir (layers > 0): [4H x dirs*H] bf16 W_ih
 };
 

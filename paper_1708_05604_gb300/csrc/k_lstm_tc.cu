@@ -629,7 +629,8 @@ __device__ __forceinline__ void fwd_tc_body(const RecArgs &a, uint8_t *smem, con
 // The body of one cluster: direction d, rows rc .. rc + TM N - 1 (smem
 // 1024-byte aligned).
 template <int N, int TM>
-__device__ __forceinline__ void bwd_tc_body(const RecArgs &a, uint8_t *smem, const int d, const int rc) {
+__device__ __forceinline__ void bwd_tc_body(const RecArgs &a, uint8_t *smem, const int d, const int rc, const int gcl,
+                                            const int ncl) {
   using Lay = TcBwdLayout<N>;
   using Sm = TcSmem<Lay, N, TM>;
   constexpr int H = kTH, G = 4 * H, kTThreads = 512, TW = 16 / TM, TT = 32 * TW, QW = TW / 4, C = N / QW,
@@ -760,6 +761,9 @@ __device__ __forceinline__ void bwd_tc_body(const RecArgs &a, uint8_t *smem, con
   float dc[P];
 #pragma unroll
   for (int j = 0; j < P; ++j) dc[j] = 0.f;
+  // db of unit u, per gate, over this thread's rows and steps (fp32)
+  float dbs[4] = {0.f, 0.f, 0.f, 0.f};
+  const bool dz32 = !a.no_dz32;
   // MMA issuers: lane 0 of the team's warps 0 .. 2 AH - 1; issuer i works on
   // half i / AH into accumulator i of the team (AH = 3: product i % 3 of
   // W_hi dz_hi, W_hi dz_lo, W_lo dz_hi over all eight k-steps; AH = 2: all
@@ -807,11 +811,15 @@ __device__ __forceinline__ void bwd_tc_body(const RecArgs &a, uint8_t *smem, con
         dz4[2] = dcv * ig * (1.f - gg * gg);
         dz4[3] = dh * tch * og * (1.f - og);
         dc[j] = dcv * fg;
-        float *zr = Z + (size_t)tok_at(j, s) * G + gu;
-        zr[0] = dz4[0];
-        zr[H] = dz4[1];
-        zr[2 * H] = dz4[2];
-        zr[3 * H] = dz4[3];
+        if (dz32) {
+          float *zr = Z + (size_t)tok_at(j, s) * G + gu;
+          zr[0] = dz4[0];
+          zr[H] = dz4[1];
+          zr[2 * H] = dz4[2];
+          zr[3 * H] = dz4[3];
+        }
+#pragma unroll
+        for (int g = 0; g < 4; ++g) dbs[g] += dz4[g];
       } else {
         dc[j] = 0.f;
       }
@@ -904,6 +912,22 @@ __device__ __forceinline__ void bwd_tc_body(const RecArgs &a, uint8_t *smem, con
     fence_before();  // the accumulators are read before the next step's MMAs overwrite them
   }
   if (mma_seen < mma_issued) mb_wait(sa(&bar[2]), (uint32_t)((mma_issued - 1) & 1), kTPolls);
+  if (a.dbp) {
+    // db: the 16 warps' sums (both teams) meet in the first team's send
+    // staging, then one thread per (gate, unit) adds them in warp order
+    // and writes the cluster's partial (deterministic)
+    float *red4 = reinterpret_cast<float *>(smem + Lay::oStg);  // [16 warps][4][32]
+    __syncthreads();
+#pragma unroll
+    for (int g = 0; g < 4; ++g) red4[(warp * 4 + g) * kTHc + lane] = dbs[g];
+    __syncthreads();
+    if (t < 4 * kTHc) {
+      const int g = t >> 5;
+      float v = 0.f;
+      for (int w = 0; w < kTThreads / 32; ++w) v += red4[(w * 4 + g) * kTHc + lane];
+      a.dbp[((size_t)d * ncl + gcl) * G + g * H + (int)c * kTHc + lane] = v;
+    }
+  }
   if (stop) __nanosleep(20000);
   fence_before();
   cluster_sync_all();
@@ -949,9 +973,9 @@ __global__ void __launch_bounds__(512, 1) lstm_bwd_tc_kernel(RecArgs a, TcSplit 
   const int cid = blockIdx.x / kTCS, per = sp.n1 + sp.n2;
   const int d = cid / per, g = cid % per;
   if (g < sp.n1)
-    bwd_tc_body<N, 1>(a, smem, d, N * g);
+    bwd_tc_body<N, 1>(a, smem, d, N * g, g, per);
   else
-    bwd_tc_body<N, 2>(a, smem, d, N * sp.n1 + 2 * N * (g - sp.n1));
+    bwd_tc_body<N, 2>(a, smem, d, N * sp.n1 + 2 * N * (g - sp.n1), g, per);
 }
 
 namespace {
@@ -1014,6 +1038,11 @@ bool tc_rec_supported(int H) {
     return e && e[0] == '0';
   }();
   return H == kTH && !off;
+}
+
+int tc_clusters_per_dir(int b, int dirs, int max_clusters) {
+  const TcSplit sp = tc_split(b, dirs, max_clusters);
+  return sp.n1 + sp.n2;
 }
 
 int tc_clusters_resident() {
