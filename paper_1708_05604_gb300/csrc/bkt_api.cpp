@@ -793,25 +793,28 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
       }
     }
     if (l > 0 && bf16) {
-      // dX = dz W_ih on the tensor cores, both directions accumulated into dY
-      // (bf16 W_ih as cast for the projection, read MN-major)
-      for (int d = 0; d < dirs; ++d) {
-        bkt::TcGemmArgs g{};
-        g.M = NT;
-        g.N = DH;
-        g.K = 4 * H;
-        g.A = w.dZb[l * dirs + d];
-        g.lda = 4 * H;
-        g.B = w.Wb[l * dirs + d];
-        g.ldb = DH;
-        g.b_mn = 1;
-        g.D = w.dY;
-        g.ldd = DH;
-        g.accumulate = d > 0;
-        g.err = w.status;
-        g.wf = wf;
-        L.run("gemm_tc", gemm_w(g.M, g.N, g.K), [&] { return bkt::launch_gemm_bf16_tc(g, s); });
+      // dX = sum_d dz_d W_ih,d on the tensor cores as one contraction over
+      // both directions' 4H (bf16 W_ih as cast for the projection, read
+      // MN-major): no second pass over dY
+      bkt::TcGemmArgs g{};
+      g.M = NT;
+      g.N = DH;
+      g.K = 4 * H;
+      g.A = w.dZb[l * dirs];
+      g.lda = 4 * H;
+      g.B = w.Wb[l * dirs];
+      g.ldb = DH;
+      g.b_mn = 1;
+      if (dirs == 2) {
+        g.A2 = w.dZb[l * dirs + 1];
+        g.B2 = w.Wb[l * dirs + 1];
+        g.K2 = 4 * H;
       }
+      g.D = w.dY;
+      g.ldd = DH;
+      g.err = w.status;
+      g.wf = wf;
+      L.run("gemm_tc", gemm_w(g.M, g.N, (double)g.K + g.K2), [&] { return bkt::launch_gemm_bf16_tc(g, s); });
     } else if (l > 0) {
       // dX = dz W_ih in fp32 on the tensor cores (3xTF32): dz rows are
       // K-contiguous already, W_ih is transposed while it is split

@@ -143,6 +143,10 @@ struct TcGemmArgs {
   int logsoftmax;  // 3xTF32 GEMM only: replace each output row by its log-softmax (N <= 128, no split)
   WaitFaults wf;   // poll cap / withheld first slab (failure-detection tests)
   int a_mn, b_mn;  // bf16 GEMM only: operand stored MN-major (see above)
+  // bf16 GEMM without a split only: a second pair summed into the same
+  // tile, D = A B^T + A2 B2^T (A2 [M x K2], B2 like B; same strides and
+  // layouts), e.g. both directions' dX in one contraction (null: none)
+  const void *A2, *B2; int K2;
 };
 int tc_splits(int M, int N, int K, int sm_count, size_t part_floats);
 cudaError_t launch_gemm_bf16_tc(const TcGemmArgs &g, cudaStream_t s);

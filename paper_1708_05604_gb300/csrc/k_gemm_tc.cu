@@ -344,6 +344,226 @@ __global__ void __launch_bounds__(128, TSTAGES <= 2 ? 2 : 1)
   if (threadIdx.x == 0 && *abort_s && g.err) atomicOr(g.err, kErrTcWait);
 }
 
+// Persistent variant for contractions without a split (the projections and
+// dX): one CTA per SM walks the tiles n-fastest (m0 = (t / tiles_n) * 128),
+// t = blockIdx.x, blockIdx.x + gridDim.x, ...  Warp 0 (one lane) streams
+// the k slabs of every tile through a 4-stage TMA ring; warp 1 (one lane)
+// issues each tile's MMAs into one of two 256-column TMEM accumulators in
+// turn and commits it to that accumulator's `full` barrier; warps 2 .. 5
+// (TMEM lane quarters 2, 3, 0, 1) drain the other accumulator to global
+// memory through their own staging blocks and release it on its `empty`
+// barrier, so a tile's epilogue overlaps the next tile's loads and MMAs.
+constexpr int kPStages = 4, kPThreads = 192, kPSt = 36;
+constexpr size_t kPStgBytes = 4 * 32 * kPSt * 4;
+constexpr size_t kPSmem = 1024 + (size_t)kPStages * (kAStage + kBStage) + kPStgBytes + 256;
+
+__global__ void __launch_bounds__(kPThreads, 1)
+    gemm_bf16_tc_persistent_kernel(const __grid_constant__ CUtensorMap ta, const __grid_constant__ CUtensorMap tb,
+                                   const __grid_constant__ CUtensorMap ta2, const __grid_constant__ CUtensorMap tb2,
+                                   TcGemmArgs g) {
+  extern __shared__ uint8_t tc_smem_raw[];
+  uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(tc_smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t *sA = base;
+  uint8_t *sB = base + kPStages * kAStage;
+  float *stg_all = reinterpret_cast<float *>(sB + kPStages * kBStage);
+  uint64_t *bars = reinterpret_cast<uint64_t *>(reinterpret_cast<uint8_t *>(stg_all) + kPStgBytes);
+  // full[S], empty[S], acc_full[2], acc_empty[2], done
+  uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 2 * kPStages + 5);
+  int *abort_s = reinterpret_cast<int *>(tslot + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int tiles_m = (g.M + TBM - 1) / TBM, tiles_n = (g.N + TBN - 1) / TBN, total = tiles_m * tiles_n;
+  // k slabs of the first pair, then of the second (if any)
+  const int nkb1 = (g.K + TBK - 1) / TBK, nkb = nkb1 + (g.A2 ? (g.K2 + TBK - 1) / TBK : 0);
+  const uint32_t full0 = su32(bars), empty0 = su32(bars + kPStages), afull0 = su32(bars + 2 * kPStages),
+                 aempty0 = su32(bars + 2 * kPStages + 2), done = su32(bars + 2 * kPStages + 4);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kPStages; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(afull0 + 8 * b, 1);
+      mbar_init(aempty0 + 8 * b, 4);  // one arrival per epilogue warp
+    }
+    mbar_init(done, 1);
+    *abort_s = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(tslot)), "r"(2 * TBN)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tslot;
+  const uint32_t cap = wait_cap(g.wf);
+
+  if (warp == 0) {
+    if (lane == 0) {  // TMA producer
+      int last_phase[kPStages];  // phase of each stage's last armed load (-1: none)
+#pragma unroll
+      for (int s = 0; s < kPStages; ++s) last_phase[s] = -1;
+      int it = 0;
+      bool stop = false;
+      for (int t = blockIdx.x; t < total && !stop; t += gridDim.x) {
+        const int m0 = (t / tiles_n) * TBM, n0 = (t % tiles_n) * TBN;
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const int s = it % kPStages;
+          if (it >= kPStages && !mbar_wait(empty0 + 8 * s, ((it / kPStages) - 1) & 1, cap)) {
+            *abort_s = 1;
+            stop = true;
+            break;
+          }
+          if (it == 0 && (g.wf.withhold & kWithholdTma)) continue;  // failure-detection hook
+          mbar_expect_tx(full0 + 8 * s, kTxBytes);
+          const bool second = kb >= nkb1;
+          const int kx = (second ? kb - nkb1 : kb) * TBK;
+          const CUtensorMap *ma = second ? &ta2 : &ta, *mb = second ? &tb2 : &tb;
+          if (!g.a_mn) {
+            tma_load_2d(su32(sA + s * kAStage), ma, kx, m0, full0 + 8 * s);
+          } else {
+#pragma unroll
+            for (int ch = 0; ch < TBM / 64; ++ch)
+              tma_load_2d(su32(sA + s * kAStage + ch * kMnChunk), ma, m0 + 64 * ch, kx, full0 + 8 * s);
+          }
+          if (!g.b_mn) {
+            tma_load_2d(su32(sB + s * kBStage), mb, kx, n0, full0 + 8 * s);
+          } else {
+#pragma unroll
+            for (int ch = 0; ch < TBN / 64; ++ch)
+              tma_load_2d(su32(sB + s * kBStage + ch * kMnChunk), mb, n0 + 64 * ch, kx, full0 + 8 * s);
+          }
+          last_phase[s] = it / kPStages;
+        }
+      }
+      // loads issued to stages that no MMA consumed may still be in flight
+      // after an abort: wait (bounded) until every armed stage has landed
+#pragma unroll
+      for (int s = 0; s < kPStages; ++s)
+        if (last_phase[s] >= 0 && !mbar_wait(full0 + 8 * s, last_phase[s] & 1, cap)) *abort_s = 1;
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {  // MMA issuer
+      int it = 0, lt = 0, issued = 0;
+      bool stop = false;
+      const uint32_t idesc = kIdesc | (g.a_mn ? kIdescAmn : 0u) | (g.b_mn ? kIdescBmn : 0u);
+      for (int t = blockIdx.x; t < total && !stop; t += gridDim.x, ++lt) {
+        const int ab = lt & 1;
+        if (lt >= 2 && !mbar_wait(aempty0 + 8 * ab, ((lt >> 1) - 1) & 1, cap)) {
+          *abort_s = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem + (uint32_t)(ab * TBN);
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const int s = it % kPStages;
+          if (!mbar_wait(full0 + 8 * s, (it / kPStages) & 1, cap)) {
+            *abort_s = 1;
+            stop = true;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = su32(sA + s * kAStage), b0 = su32(sB + s * kBStage);
+#pragma unroll
+          for (int kk = 0; kk < TBK / 16; ++kk) {
+            const uint64_t ad = g.a_mn ? sw128_desc_mn(a0 + kk * 2048, kMnChunk) : sw128_desc(a0 + kk * 32);
+            const uint64_t bd = g.b_mn ? sw128_desc_mn(b0 + kk * 2048, kMnChunk) : sw128_desc(b0 + kk * 32);
+            tc_mma(d, ad, bd, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+          }
+          tc_commit(empty0 + 8 * s);
+          ++issued;
+        }
+        if (!stop) tc_commit(afull0 + 8 * ab);
+      }
+      // the final commit tracks every MMA issued above
+      if (issued > 0) tc_commit(done);
+      else mbar_arrive(done);
+    }
+    __syncwarp();
+  } else {
+    // epilogue: warp w owns TMEM lane quarter w % 4 (tile rows 32 (w % 4) ..);
+    // each 32-column chunk goes through the warp's staging block and leaves
+    // as float4 stores covering four whole 128-byte row pieces
+    const int q = warp & 3;
+    float *stg = stg_all + (warp - 2) * 32 * kPSt;
+    const int cq = lane & 7, rq = lane >> 3;  // write phase: columns 4 cq .. + 3 of rows rq + 4 i
+    int lt = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x, ++lt) {
+      const int ab = lt & 1;
+      const bool ready_t = mbar_wait(afull0 + 8 * ab, (lt >> 1) & 1, cap);
+      if (!ready_t) *abort_s = 1;
+      if (!__all_sync(0xffffffffu, ready_t)) break;  // uniform per warp
+      tc_fence_after();
+      const int m0 = (t / tiles_n) * TBM, n0 = (t % tiles_n) * TBN;
+      const uint32_t trow = tmem + (uint32_t)(ab * TBN) + ((uint32_t)(q * 32) << 16);
+#pragma unroll 1
+      for (int c0 = 0; c0 < TBN; c0 += 32) {
+        uint32_t v[32];
+        __syncwarp();
+        tmem_ld32(trow + c0, v);
+        const int nb = n0 + c0;
+        if (nb >= g.N) continue;  // uniform across the warp
+#pragma unroll
+        for (int j = 0; j < 32; j += 4)
+          *reinterpret_cast<float4 *>(stg + lane * kPSt + j) = make_float4(
+              __uint_as_float(v[j]), __uint_as_float(v[j + 1]), __uint_as_float(v[j + 2]), __uint_as_float(v[j + 3]));
+        __syncwarp();
+        const int n = nb + 4 * cq;
+        float4 bias4 = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (g.bias) {
+          bias4.x = n < g.N ? g.bias[n] : 0.f;
+          bias4.y = n + 1 < g.N ? g.bias[n + 1] : 0.f;
+          bias4.z = n + 2 < g.N ? g.bias[n + 2] : 0.f;
+          bias4.w = n + 3 < g.N ? g.bias[n + 3] : 0.f;
+        }
+        const bool vec = ((g.ldd & 3) == 0) && ((reinterpret_cast<uintptr_t>(g.D) & 15) == 0);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int r = rq + 4 * i, m = m0 + q * 32 + r;
+          if (m >= g.M) continue;
+          float4 x = *reinterpret_cast<const float4 *>(stg + r * kPSt + 4 * cq);
+          x.x += bias4.x;
+          x.y += bias4.y;
+          x.z += bias4.z;
+          x.w += bias4.w;
+          float *o = g.D + (int64_t)m * g.ldd + n;
+          if (vec && n + 4 <= g.N) {
+            if (g.accumulate) {
+              const float4 y = *reinterpret_cast<const float4 *>(o);
+              x.x += y.x;
+              x.y += y.y;
+              x.z += y.z;
+              x.w += y.w;
+            }
+            *reinterpret_cast<float4 *>(o) = x;
+          } else {
+            const float xs[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              if (n + j < g.N) o[j] = xs[j] + (g.accumulate ? o[j] : 0.f);
+          }
+        }
+      }
+      // every tcgen05.ld of this accumulator has completed (each waited):
+      // hand it back to the issuer
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(aempty0 + 8 * ab);
+    }
+  }
+  // no MMA may be in flight when TMEM is freed
+  if (!mbar_wait(done, 0, cap)) *abort_s = 1;
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(2 * TBN) : "memory");
+  if (threadIdx.x == 0 && *abort_s && g.err) atomicOr(g.err, kErrTcWait);
+}
+
+
 __global__ void __launch_bounds__(128, 1)
     gemm_tf32x3_tc_kernel(const __grid_constant__ CUtensorMap tah, const __grid_constant__ CUtensorMap tal,
                           const __grid_constant__ CUtensorMap tbh, const __grid_constant__ CUtensorMap tbl,
@@ -792,21 +1012,45 @@ cudaError_t launch_gemm_bf16_tc(const TcGemmArgs &g, cudaStream_t s) {
   if (g.K <= 0 || (g.lda & 7) || (g.ldb & 7) || (reinterpret_cast<uintptr_t>(g.A) & 15) ||
       (reinterpret_cast<uintptr_t>(g.B) & 15) || (g.P && g.splits < 1) || (!g.P && !g.D))
     return cudaErrorInvalidValue;
-  CUtensorMap ta, tb;
+  if (g.A2 && (g.P || !g.B2 || g.K2 <= 0 || ((reinterpret_cast<uintptr_t>(g.A2) | reinterpret_cast<uintptr_t>(g.B2)) & 15)))
+    return cudaErrorInvalidValue;
+  CUtensorMap ta, tb, ta2, tb2;
   // K-major operands are [rows x K]; MN-major ones [K x rows] (rows contiguous)
   const bool okA = g.a_mn ? make_map(&ta, g.A, (uint64_t)g.M, (uint64_t)g.K, g.lda, TBK)
                           : make_map(&ta, g.A, (uint64_t)g.K, (uint64_t)g.M, g.lda, TBM);
   const bool okB = g.b_mn ? make_map(&tb, g.B, (uint64_t)g.N, (uint64_t)g.K, g.ldb, TBK)
                           : make_map(&tb, g.B, (uint64_t)g.K, (uint64_t)g.N, g.ldb, TBN);
   if (!okA || !okB) return cudaErrorInvalidValue;
+  if (g.A2) {
+    const bool okA2 = g.a_mn ? make_map(&ta2, g.A2, (uint64_t)g.M, (uint64_t)g.K2, g.lda, TBK)
+                             : make_map(&ta2, g.A2, (uint64_t)g.K2, (uint64_t)g.M, g.lda, TBM);
+    const bool okB2 = g.b_mn ? make_map(&tb2, g.B2, (uint64_t)g.N, (uint64_t)g.K2, g.ldb, TBK)
+                             : make_map(&tb2, g.B2, (uint64_t)g.K2, (uint64_t)g.N, g.ldb, TBN);
+    if (!okA2 || !okB2) return cudaErrorInvalidValue;
+  } else {
+    ta2 = ta;
+    tb2 = tb;
+  }
   dim3 grid((g.M + TBM - 1) / TBM, (g.N + TBN - 1) / TBN, g.P ? g.splits : 1);
   if (grid.y > 65535u || grid.z > 65535u) return cudaErrorInvalidConfiguration;
-  const int nkb = (g.K + TBK - 1) / TBK;
-  const bool short_k = !g.P && nkb <= 16 && (int64_t)grid.x * grid.y >= 512;
-  if (short_k) {
-    cudaError_t e = ensure_smem((const void *)gemm_bf16_tc_kernel<2>, tc_smem_for(2));
+  if (!g.P) {
+    // persistent: one CTA per SM over the tiles
+    static int sms[64] = {0};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    gemm_bf16_tc_kernel<2><<<grid, 128, tc_smem_for(2), s>>>(ta, tb, g);
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    if (sms[dev] == 0) {
+      int n = 0;
+      e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+      if (e != cudaSuccess) return e;
+      sms[dev] = n;
+    }
+    e = ensure_smem((const void *)gemm_bf16_tc_persistent_kernel, kPSmem);
+    if (e != cudaSuccess) return e;
+    const int64_t tiles = (int64_t)grid.x * grid.y;
+    const unsigned blocks = (unsigned)std::min<int64_t>(tiles, sms[dev]);
+    gemm_bf16_tc_persistent_kernel<<<blocks, kPThreads, kPSmem, s>>>(ta, tb, ta2, tb2, g);
   } else {
     cudaError_t e = ensure_smem((const void *)gemm_bf16_tc_kernel<4>, tc_smem_for(4));
     if (e != cudaSuccess) return e;
