@@ -197,6 +197,7 @@ __device__ __forceinline__ void split_bf16(float x, __nv_bfloat16 &hi, __nv_bflo
 __device__ __forceinline__ uint32_t pack2(__nv_bfloat16 a, __nv_bfloat16 b) {
   return (uint32_t)__bfloat16_as_ushort(a) | ((uint32_t)__bfloat16_as_ushort(b) << 16);
 }
+__device__ __forceinline__ uint32_t bf2u(__nv_bfloat162 v) { return pack2(v.x, v.y); }
 // x = hi + 2^-11 lo, both fp16: hi rounded to nearest, lo the rounded rest
 // scaled by 2^11 so that it keeps fp16's full precision (the rest alone is
 // often subnormal); hi + 2^-11 lo carries about 22 significant bits
@@ -826,22 +827,22 @@ __device__ __forceinline__ void bwd_tc_body(const RecArgs &a, uint8_t *smem, con
       // B operand: k = 4u .. 4u + 3 of row n (8 bytes of each part), in
       // 64-k atom u / 16 at 16-byte chunk (u % 16) / 2 swizzled by n % 8, so
       // that a warp's 32 stores fill two whole 128-byte rows
-      __nv_bfloat16 h0, l0, h1, l1, h2, l2, h3, l3;
-      split_bf16(dz4[0], h0, l0);
-      split_bf16(dz4[1], h1, l1);
-      split_bf16(dz4[2], h2, l2);
-      split_bf16(dz4[3], h3, l3);
+      // (hi rounded to nearest, lo the rounded rest, two values per conversion)
+      const __nv_bfloat162 h01 = __floats2bfloat162_rn(dz4[0], dz4[1]), h23 = __floats2bfloat162_rn(dz4[2], dz4[3]);
+      const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+      const __nv_bfloat162 l01 = __floats2bfloat162_rn(dz4[0] - f01.x, dz4[1] - f01.y);
+      const __nv_bfloat162 l23 = __floats2bfloat162_rn(dz4[2] - f23.x, dz4[3] - f23.y);
       if (dZb && s < len[j]) {  // bf16 dz for the bf16 contractions
         __nv_bfloat16 *zb = dZb + (size_t)tok_at(j, s) * G + gu;
-        zb[0] = h0;
-        zb[H] = h1;
-        zb[2 * H] = h2;
-        zb[3 * H] = h3;
+        zb[0] = h01.x;
+        zb[H] = h01.y;
+        zb[2 * H] = h23.x;
+        zb[3 * H] = h23.y;
       }
       const uint32_t off = (uint32_t)(u >> 4) * (128u * N) + (uint32_t)n * 128u +
                            (uint32_t)((((u & 15) >> 1) ^ (n & 7)) * 16) + (uint32_t)(u & 1) * 8u;
-      *reinterpret_cast<uint2 *>(Bz + off) = make_uint2(pack2(h0, h1), pack2(h2, h3));
-      *reinterpret_cast<uint2 *>(Bz + Lay::kB + off) = make_uint2(pack2(l0, l1), pack2(l2, l3));
+      *reinterpret_cast<uint2 *>(Bz + off) = make_uint2(bf2u(h01), bf2u(h23));
+      *reinterpret_cast<uint2 *>(Bz + Lay::kB + off) = make_uint2(bf2u(l01), bf2u(l23));
     }
     fence_proxy();
     fence_before();
