@@ -189,7 +189,8 @@ cudaError_t launch_ctc_grad(const DevIdx &ix, float *logp_dlogit, int C, int bla
 
 // Geometry of the recurrent kernels for one layer.
 //   mode 1: one CTA per bc rows holds all of W_hh (H in {32, 64, 128});
-//   mode 2: register-tiled cluster of cs CTAs per bc rows (H in {256, 512});
+//   mode 2: register-tiled clusters of cs CTAs, 4 or 8 rows each (H in
+//           {256, 512}); bc = the clusters that can be resident at once;
 //   mode 3: tensor-core clusters of 8 CTAs, 16 or 32 rows each, W_hh in
 //           TMEM (H = 256 with bf16 contractions); bc = the clusters that
 //           can be resident at once;
@@ -235,11 +236,13 @@ inline bool rec_writes_bf16(const RecGeom &g) { return g.mode == 3; }
 cudaError_t launch_lstm_bwd(const RecArgs &a, const RecGeom &g, cudaStream_t s);
 
 // Register-tiled cluster kernels for H = 256 and 512 (k_lstm_cl.cu):
-// CTAs per cluster for H (0: not handled there), batch rows per cluster for a
-// batch of b rows (0: the configuration cannot launch), launch.
+// CTAs per cluster for H (0: not handled there), how many of their clusters
+// can be resident at once (0: they cannot launch), and the launch, which
+// lays the batch's rows out over 4- and 8-row clusters, at most
+// max_clusters of them.
 int cl_cluster_size(int H);
 int plan_cl_rows(int H, int b, int dirs);
-cudaError_t launch_lstm_cl(const RecArgs &a, int bc, bool bwd, cudaStream_t s);
+cudaError_t launch_lstm_cl(const RecArgs &a, int max_clusters, bool bwd, cudaStream_t s);
 
 // Tensor-core cluster kernels for H = 256 on the bf16 path (k_lstm_tc.cu):
 // whether H is handled there (BKT_REC_TC=0 in the environment turns them

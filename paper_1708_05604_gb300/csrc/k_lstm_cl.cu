@@ -162,15 +162,15 @@ size_t cl_tail_bytes(int NH, int T) { return 16 * NH + (T + 1 <= kClTokCap ? (si
 // Rows of a cluster are processed as NH halves of BH rows, one after the
 // other within a step, each with its own receive buffers and mbarriers, so
 // the exchange of one half overlaps the arithmetic of the other.
+// The body of one cluster: direction d, rows r0 .. r0 + BC - 1.
 template <int H, int CS, int BC, int NH>
-__global__ void __launch_bounds__(kClThreads, 1) lstm_fwd_cl_kernel(RecArgs a) {
+__device__ __forceinline__ void fwd_cl_body(const RecArgs &a, float *sm, const int d, const int r0) {
   using Gm = ClGeom<H, CS, BC, NH>;
   constexpr int Hc = Gm::Hc, KS = Gm::KS, HPAD = Gm::HPAD, BH = Gm::BH, G = 4 * H, NTH = kClThreads;
   constexpr int NV = 4 * BH, NPL = NV / KS;  // partial sums per thread, per lane after the reduction
   static_assert(NPL == 2 || NPL % 4 == 0, "a lane finishes whole units or one gate pair");
   constexpr int RPL = NPL >= 4 ? NPL / 4 : 1;  // rows of a half finished per lane
   constexpr int SEND4 = BH * Hc / 4;           // float4 sent to each CTA per half and step
-  extern __shared__ __align__(16) float sm[];
   constexpr int RK = Gm::RKF, SK4 = (64 - RK) / 4;  // register columns, shared float4 columns
   float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [SK4][4][NTH] columns RK..63 of each slice
   float *hb = sm + SK4 * 4 * NTH * 4;            // [NH][2][BH][HPAD] received h
@@ -185,9 +185,6 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_fwd_cl_kernel(RecArgs a) {
   const int kl = t % KS, u = t / KS;
   const uint32_t c = cta_rank_in_cluster();
   const int gu = (int)c * Hc + u, kb = kl * 64;
-  const int n_groups = (a.ix.b + BC - 1) / BC;
-  const int cid = blockIdx.x / CS;
-  const int d = cid / n_groups, grp = cid % n_groups, r0 = grp * BC;
   const int DH = a.dirs * H;
   const float *__restrict__ Whh = a.Whh[d];
 
@@ -375,14 +372,14 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_fwd_cl_kernel(RecArgs a) {
   cluster_barrier_all();  // no CTA leaves while a peer may still address its shared memory
 }
 
+// The body of one cluster: direction d, rows r0 .. r0 + BC - 1.
 template <int H, int CS, int BC, int NH>
-__global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a) {
+__device__ __forceinline__ void bwd_cl_body(const RecArgs &a, float *sm, const int d, const int r0) {
   using Gm = ClGeom<H, CS, BC, NH>;
   constexpr int Hc = Gm::Hc, RSL = Gm::RSL, BH = Gm::BH, G = 4 * H, NTH = kClThreads, DZS = Gm::DZS;
   constexpr int NV = 4 * BH, NPL = NV / RSL;  // partials per thread, per lane after the reduction
   static_assert(NPL % 4 == 0, "a lane finishes whole float4 column groups");
   constexpr int PAIRS = Hc * BH, PPT = Gm::PPT;  // (unit, row) pairs of a half
-  extern __shared__ __align__(16) float sm[];
   float4 *Wb4 = reinterpret_cast<float4 *>(sm);  // [32][NTH] rows 32..63 of each row slice
   float *dzs = sm + 32 * NTH * 4;                // [NH][2][DZS] dz of this CTA's gate rows
   float *red = dzs + 2 * NH * DZS;               // [NH][2][CS][BH][Hc] received partials of W_hh^T dz
@@ -396,9 +393,6 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a) {
   const int t = threadIdx.x, lane = t & 31;
   const int rs = t % RSL, cgp = t / RSL, k0 = 4 * cgp;
   const uint32_t c = cta_rank_in_cluster();
-  const int n_groups = (a.ix.b + BC - 1) / BC;
-  const int cid = blockIdx.x / CS;
-  const int d = cid / n_groups, grp = cid % n_groups, r0 = grp * BC;
   const int DH = a.dirs * H;
   const float *__restrict__ Whh = a.Whh[d];
   auto dz_at = [&](int r, int b) { return r * BH + (r >> 6) * 4 + b; };
@@ -596,21 +590,56 @@ __global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a) {
 }
 
 // ---------------------------------------------------------------------------
+// Cluster layout of a launch.  Clusters of 4 rows step faster than
+// clusters of 8 (at H = 512, 16-CTA clusters, half the FMAs per CTA and
+// step), but at most 7 such 16-CTA clusters fit on the GPU at once.  As in
+// the tensor-core kernels, the longest rows of the length-sorted batch go to
+// n4 four-row clusters per direction and the shortest to n8 eight-row
+// clusters, with dirs (n4 + n8) no more than the resident clusters.
 namespace {
 
-template <int H, int CS, int BC, int NH>
+struct ClSplit {
+  int n4, n8;  // clusters per direction of 4 and of 8 rows
+};
+
+}  // namespace
+
+template <int H, int CS>
+__global__ void __launch_bounds__(kClThreads, 1) lstm_fwd_cl_kernel(RecArgs a, ClSplit sp) {
+  extern __shared__ __align__(16) float sm[];
+  const int cid = blockIdx.x / CS, per = sp.n4 + sp.n8;
+  const int d = cid / per, g = cid % per;
+  if (g < sp.n4)
+    fwd_cl_body<H, CS, 4, 1>(a, sm, d, 4 * g);
+  else
+    fwd_cl_body<H, CS, 8, 1>(a, sm, d, 4 * sp.n4 + 8 * (g - sp.n4));
+}
+
+template <int H, int CS>
+__global__ void __launch_bounds__(kClThreads, 1) lstm_bwd_cl_kernel(RecArgs a, ClSplit sp) {
+  extern __shared__ __align__(16) float sm[];
+  const int cid = blockIdx.x / CS, per = sp.n4 + sp.n8;
+  const int d = cid / per, g = cid % per;
+  if (g < sp.n4)
+    bwd_cl_body<H, CS, 4, 1>(a, sm, d, 4 * g);
+  else
+    bwd_cl_body<H, CS, 8, 1>(a, sm, d, 4 * sp.n4 + 8 * (g - sp.n4));
+}
+
+namespace {
+
+template <int H, int CS, int BC>
+size_t cl_smem_one(bool bwd, int T) {
+  using Gm = ClGeom<H, CS, BC, 1>;
+  return (bwd ? Gm::bwd_floats() : Gm::fwd_floats()) * 4 + cl_tail_bytes(1, T);
+}
+// dynamic shared memory of a launch: the larger of the two bodies' layouts
+template <int H, int CS>
 size_t cl_smem(bool bwd, int T) {
-  using Gm = ClGeom<H, CS, BC, NH>;
-  return (bwd ? Gm::bwd_floats() : Gm::fwd_floats()) * 4 + cl_tail_bytes(NH, T);
+  return std::max(cl_smem_one<H, CS, 4>(bwd, T), cl_smem_one<H, CS, 8>(bwd, T));
 }
 
-template <typename K>
-cudaError_t cl_prepare(K kernel, int cs, size_t smem) {
-  return ensure_smem((const void *)kernel, smem, cs > 8);
-}
-
-template <typename K>
-cudaLaunchConfig_t cl_config(K, int cs, int clusters, size_t smem, cudaStream_t s, cudaLaunchAttribute *attr) {
+cudaLaunchConfig_t cl_config(int cs, int clusters, size_t smem, cudaStream_t s, cudaLaunchAttribute *attr) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(clusters * cs, 1, 1);
   cfg.blockDim = dim3(kClThreads, 1, 1);
@@ -625,45 +654,62 @@ cudaLaunchConfig_t cl_config(K, int cs, int clusters, size_t smem, cudaStream_t 
   return cfg;
 }
 
-template <int H, int CS, int BC, int NH>
-cudaError_t launch_cl(const RecArgs &a, bool bwd, cudaStream_t s) {
-  if (a.ix.b <= 0 || a.ix.T <= 0) return cudaSuccess;
-  const size_t smem = cl_smem<H, CS, BC, NH>(bwd, a.ix.T);
-  const int clusters = ((a.ix.b + BC - 1) / BC) * a.dirs;
-  cudaLaunchAttribute attr;
-  if (bwd) {
-    auto k = lstm_bwd_cl_kernel<H, CS, BC, NH>;
-    cudaError_t e = cl_prepare(k, CS, smem);
-    if (e != cudaSuccess) return e;
-    cudaLaunchConfig_t cfg = cl_config(k, CS, clusters, smem, s, &attr);
-    return cudaLaunchKernelEx(&cfg, k, a);
+ClSplit cl_split(int b, int dirs, int max_clusters) {
+  const int groups = (b + 3) / 4;                    // 4-row groups per direction
+  const int per = std::max(1, max_clusters / dirs);  // clusters per direction resident at once
+  ClSplit sp;
+  if (groups <= per) {
+    sp.n4 = groups;
+    sp.n8 = 0;
+  } else if (groups - per >= (groups + 1) / 2) {
+    sp.n4 = 0;  // eight rows everywhere (clusters beyond the resident ones wait)
+    sp.n8 = (groups + 1) / 2;
+  } else {
+    sp.n8 = groups - per;  // each eight-row cluster saves one cluster
+    sp.n4 = groups - 2 * sp.n8;
   }
-  auto k = lstm_fwd_cl_kernel<H, CS, BC, NH>;
-  cudaError_t e = cl_prepare(k, CS, smem);
+  return sp;
+}
+
+template <int H, int CS>
+cudaError_t launch_cl(const RecArgs &a, int max_clusters, bool bwd, cudaStream_t s) {
+  if (a.ix.b <= 0 || a.ix.T <= 0) return cudaSuccess;
+  if (max_clusters <= 0 || a.dirs < 1 || a.dirs > 2) return cudaErrorInvalidValue;
+  const ClSplit sp = cl_split(a.ix.b, a.dirs, max_clusters);
+  const size_t smem = cl_smem<H, CS>(bwd, a.ix.T);
+  const int clusters = (sp.n4 + sp.n8) * a.dirs;
+  cudaLaunchAttribute attr;
+  cudaLaunchConfig_t cfg = cl_config(CS, clusters, smem, s, &attr);
+  if (bwd) {
+    auto k = lstm_bwd_cl_kernel<H, CS>;
+    cudaError_t e = ensure_smem((const void *)k, smem, CS > 8);
+    if (e != cudaSuccess) return e;
+    return cudaLaunchKernelEx(&cfg, k, a, sp);
+  }
+  auto k = lstm_fwd_cl_kernel<H, CS>;
+  cudaError_t e = ensure_smem((const void *)k, smem, CS > 8);
   if (e != cudaSuccess) return e;
-  cudaLaunchConfig_t cfg = cl_config(k, CS, clusters, smem, s, &attr);
-  return cudaLaunchKernelEx(&cfg, k, a);
+  return cudaLaunchKernelEx(&cfg, k, a, sp);
 }
 
 // Clusters of the forward and the BPTT kernel that can be resident at once
 // (0: the configuration cannot launch on this device).
-template <int H, int CS, int BC, int NH>
+template <int H, int CS>
 int cl_resident(int T) {
   int lo = 1 << 30;
   for (int bwd = 0; bwd < 2; ++bwd) {
-    const size_t smem = cl_smem<H, CS, BC, NH>(bwd != 0, T);
+    const size_t smem = cl_smem<H, CS>(bwd != 0, T);
     cudaLaunchAttribute attr;
     int n = 0;
     cudaError_t e;
+    cudaLaunchConfig_t cfg = cl_config(CS, 1, smem, 0, &attr);
     if (bwd) {
-      auto k = lstm_bwd_cl_kernel<H, CS, BC, NH>;
-      e = cl_prepare(k, CS, smem);
-      cudaLaunchConfig_t cfg = cl_config(k, CS, 1, smem, 0, &attr);
+      auto k = lstm_bwd_cl_kernel<H, CS>;
+      e = ensure_smem((const void *)k, smem, CS > 8);
       if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, k, &cfg);
     } else {
-      auto k = lstm_fwd_cl_kernel<H, CS, BC, NH>;
-      e = cl_prepare(k, CS, smem);
-      cudaLaunchConfig_t cfg = cl_config(k, CS, 1, smem, 0, &attr);
+      auto k = lstm_fwd_cl_kernel<H, CS>;
+      e = ensure_smem((const void *)k, smem, CS > 8);
       if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, k, &cfg);
     }
     if (e != cudaSuccess) {
@@ -680,25 +726,17 @@ int cl_resident(int T) {
 int cl_cluster_size(int H) { return H == 256 ? 4 : H == 512 ? 16 : 0; }
 
 int plan_cl_rows(int H, int b, int dirs) {
-  // the smallest rows-per-cluster whose clusters are all resident at once;
-  // otherwise the larger one (fewer, longer clusters)
+  (void)b;
+  (void)dirs;
   const int T = kClTokCap - 1;
-  int r4 = 0, r8 = 0;
-  if (H == 256) {
-    r4 = cl_resident<256, 4, 4, 1>(T);
-    r8 = cl_resident<256, 4, 8, 1>(T);
-  } else if (H == 512) {
-    r4 = cl_resident<512, 16, 4, 1>(T);
-    r8 = cl_resident<512, 16, 8, 1>(T);
-  }
-  if (r4 > 0 && ((b + 3) / 4) * dirs <= r4) return 4;
-  if (r8 > 0) return 8;
-  return r4 > 0 ? 4 : 0;
+  if (H == 256) return cl_resident<256, 4>(T);
+  if (H == 512) return cl_resident<512, 16>(T);
+  return 0;
 }
 
-cudaError_t launch_lstm_cl(const RecArgs &a, int bc, bool bwd, cudaStream_t s) {
-  if (a.H == 256) return bc == 4 ? launch_cl<256, 4, 4, 1>(a, bwd, s) : launch_cl<256, 4, 8, 1>(a, bwd, s);
-  if (a.H == 512) return bc == 4 ? launch_cl<512, 16, 4, 1>(a, bwd, s) : launch_cl<512, 16, 8, 1>(a, bwd, s);
+cudaError_t launch_lstm_cl(const RecArgs &a, int max_clusters, bool bwd, cudaStream_t s) {
+  if (a.H == 256) return launch_cl<256, 4>(a, max_clusters, bwd, s);
+  if (a.H == 512) return launch_cl<512, 16>(a, max_clusters, bwd, s);
   return cudaErrorInvalidValue;
 }
 

@@ -374,6 +374,23 @@ def test_tensor_core_recurrence_cluster_layouts(b):
     compare(cfg, lg, gg, lo, go, BF16_TOL)
 
 
+@pytest.mark.parametrize("H,bi,b", [(512, False, 24), (512, False, 32), (512, False, 60), (256, True, 100)])
+def test_register_tiled_cluster_layouts(H, bi, b):
+    """The fp32 cluster kernels (H = 256 and 512) spread a batch over 4-row
+    and 8-row clusters, no more of them than can be resident at once (7
+    sixteen-CTA clusters at H = 512): 24 rows run on 4-row clusters only,
+    32 on six 4-row clusters and one 8-row cluster, 60 on 8-row clusters
+    only (more than fit at once); at H = 256, 100 rows per direction mix
+    both.  Rows end at every step; fp32 contractions, at the fp32 bound."""
+    cfg = {"n_layers": 1, "bidirectional": bi, "in_dim": 4, "hidden": H, "n_classes": 81, "blank": 0}
+    rng = np.random.default_rng(H + b)
+    ds = synth.make_dataset(rng.integers(1, 13, size=b), 4, rng)
+    params = synth.draw_params(rng, binding.param_count(cfg))
+    lg, gg = gpu_step(cfg, ds, params)
+    lo, go = oracle_step_parallel(cfg, ds, params, np.arange(ds.n))
+    compare(cfg, lg, gg, lo, go, FP32_TOL)
+
+
 def test_bf16_workload_runs_on_tensor_cores():
     """The bf16 workloads route their contractions through the tcgen05 GEMM
     (and stay within the bf16 tolerance while differing from fp32 rounding)."""
