@@ -238,9 +238,25 @@ __device__ __forceinline__ void tmem_ld_raw(uint32_t taddr, uint32_t (&r)[C]) {
   }
 }
 // Gate nonlinearities from the exponential intrinsic (as in the other
-// recurrent kernels): sigma(x) = 1 / (1 + e^-x), tanh(x) = 2 sigma(2x) - 1.
-__device__ __forceinline__ float sigm_tc(float x) { return __fdividef(1.f, 1.f + __expf(-x)); }
+// recurrent kernels): sigma(x) = 1 / (1 + e^-x), tanh(x) = 1 - 2 / (1 + e^2x).
 __device__ __forceinline__ float tanh_tc(float x) { return 1.f - __fdividef(2.f, 1.f + __expf(2.f * x)); }
+// Four values of one nonlinearity with one reciprocal: with d_k = 1 + e^{a_k}
+// (a_k = -x for sigma, 2x for tanh, clamped at 20 so that the product of the
+// four stays finite), 1 / d_k = (prod_{j != k} d_j) / (prod_j d_j).  The
+// clamp changes sigma(x) only for x < -20 and tanh(x) only for x > 10, by
+// less than 5e-9.
+template <bool TANH>
+__device__ __forceinline__ void act4(float (&x)[4]) {
+  float dd[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) dd[k] = 1.f + __expf(fminf(TANH ? 2.f * x[k] : -x[k], 20.f));
+  const float d01 = dd[0] * dd[1], d23 = dd[2] * dd[3];
+  const float r = __fdividef(1.f, d01 * d23);
+  const float r23 = r * d23, r01 = r * d01;
+  const float inv[4] = {dd[1] * r23, dd[0] * r23, dd[3] * r01, dd[2] * r01};
+#pragma unroll
+  for (int k = 0; k < 4; ++k) x[k] = TANH ? 1.f - 2.f * inv[k] : inv[k];
+}
 
 // Named barrier of one team (id >= 1; id 0 is __syncthreads) of n threads,
 // and the same barrier returning the OR of a predicate over them.
@@ -574,7 +590,15 @@ __device__ __forceinline__ void fwd_tc_body(const RecArgs &a, uint8_t *smem, con
     const uint32_t par = (uint32_t)(s & 1);
     float *gs = gate + par * N * RF;
 #pragma unroll
-    for (int k = 0; k < C; ++k) gs[((col0 + k) * 4 + q) * kTHc + lane] = q == 2 ? tanh_tc(acc[k]) : sigm_tc(acc[k]);
+    for (int k0 = 0; k0 < C; k0 += 4) {
+      float v[4] = {acc[k0], acc[k0 + 1], acc[k0 + 2], acc[k0 + 3]};
+      if (q == 2)
+        act4<true>(v);
+      else
+        act4<false>(v);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) gs[((col0 + k0 + k) * 4 + q) * kTHc + lane] = v[k];
+    }
     fence_before();
     // an issuer that gave up on the exchange stops the whole team
     if (team_sync_or(bid, TT, !ok)) {
