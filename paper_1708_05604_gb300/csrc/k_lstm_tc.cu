@@ -18,11 +18,13 @@
 // leaves the SM: per step only N rows of h (or dz) are read from shared
 // memory.
 //
-// A cluster's rows form two teams of 16 rows (one team of 16 for batches of
-// at most 64 rows); each team runs its own recurrence on 8 of the CTA's 16
-// warps (its own MMAs, TMEM accumulators, exchange buffers, mbarriers and
-// named barrier), so that one team's MMAs and exchange overlap the other
-// team's elementwise work; the teams share only W in TMEM.
+// A team is 16 rows of the batch with its own MMAs, TMEM accumulators,
+// exchange buffers, mbarriers and named barrier.  A one-team cluster runs its
+// team on all 16 warps; a two-team cluster runs two teams of 8 warps that
+// share only W in TMEM (one team's MMAs and exchange wait overlap the other's
+// elementwise work).  A launch gives the longest rows to one-team clusters,
+// which step faster, and the rest to two-team clusters, within the clusters
+// that fit on the GPU at once (see the launch code at the end).
 //
 // Forward: TMEM lane 32 q + u holds gate row q H + 32c + u (A = the W slice,
 // K = the 256 units; hi part in columns 0 .. 127, scaled lo part in
@@ -37,19 +39,21 @@
 // half of K) issue 8 MMAs each into their own accumulators and commit them
 // to an mbarrier; each warp then reads one TMEM lane quarter (one gate for
 // the 32 units) for C rows, adds Zx and the four accumulators (the lo ones
-// scaled by 2^-11), applies sigma or tanh, writes the gates, and leaves
-// them in shared memory, where thread (w, lane) finds the four gates of
-// unit `lane` for its rows, updates c in registers, writes c, h and the
-// bf16 copies, and stages h_t in fp16 for st.async stores to every CTA of
-// the cluster (16-byte remote stores completing bytes on the receiver's
-// mbarrier; double-buffered by step parity, so the data dependence orders
-// buffer reuse).
+// scaled by 2^-11), applies sigma or tanh and leaves the gates in shared
+// memory, where thread (w, lane) finds the four gates of unit `lane` for
+// its rows, updates c in registers, stages c and h, and stages h_t in fp16
+// for st.async stores to every CTA of the cluster (16-byte remote stores
+// completing bytes on the receiver's mbarrier; double-buffered by step
+// parity, so the data dependence orders buffer reuse).  The warps that
+// issue no MMAs write the staged outputs to global memory and bring in Zx
+// during the next step's exchange wait and MMAs.
 // BPTT step: dh = dY + the sum of the 8 partials of W_hh^T dz_{t+1} received
-// for this CTA's units, then dc and dz of the four gates (fp32, written in
-// place of the gates and, split, to the B operand); four issuing threads
-// (six with one team) form this CTA's partial W_hh^T dz over its 128 gate
-// rows for all 256 units (two 128-lane halves), and each warp sends its
-// 16-byte pieces of the 32-unit blocks straight to the CTAs that own them.
+// for this CTA's units, then dc and dz of the four gates (bf16, and fp32 in
+// place of the gates for layer 1, and split to the B operand); four issuing
+// threads (six with one team) form this CTA's partial W_hh^T dz over its 128
+// gate rows for all 256 units (two 128-lane halves), and each warp sends
+// its 16-byte pieces of the 32-unit blocks straight to the CTAs that own
+// them.  Above layer 1 the bias gradient is summed in the kernel.
 //
 // Every wait is bounded (status bit 4 on expiry, as in the other cluster
 // kernels); on an abort the kernel still waits for its last MMA batch before
