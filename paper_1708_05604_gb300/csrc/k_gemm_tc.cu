@@ -1,7 +1,11 @@
 // k_gemm_tc.cu -- GEMMs on the 5th-generation tensor cores (tcgen05, TMEM
 // accumulators):
-//   gemm_bf16_tc_kernel    bf16 operands fed by TMA: the bf16 path's input
-//                          projections, weight gradients and input gradients;
+//   gemm_bf16_tc_kernel    bf16 operands fed by TMA, one tile per CTA: the
+//                          bf16 path's split-K weight gradients;
+//   gemm_bf16_tc_persistent_kernel
+//                          the same contraction, persistent with two TMEM
+//                          accumulators: the bf16 path's input projections
+//                          and input gradients (no split);
 //   gemm_tf32x3_tc_kernel  fp32 split into tf32 hi + lo (3 MMAs per product),
 //                          operands fed by TMA: the fp32 path's logits (with
 //                          a log-softmax epilogue), dY, projections and dX,
@@ -39,9 +43,8 @@ constexpr int TBM = 128, TBN = 256, TBK = 64;
 constexpr uint32_t kAStage = TBM * TBK * 2;  // 16 KB
 constexpr uint32_t kBStage = TBN * TBK * 2;  // 32 KB
 constexpr uint32_t kTxBytes = kAStage + kBStage;
-// 4 stages for long-K contractions (one CTA per SM); 2 stages (97 KB) for the
-// many short-K tiles of the projections and dX, so that two CTAs share an SM
-// and one's epilogue overlaps the other's loads and MMAs
+// shared memory of the one-tile-per-CTA kernel with `stages` ring stages (4:
+// the split-K weight gradients, one CTA per SM)
 constexpr size_t tc_smem_for(int stages) { return 1024 + (size_t)stages * (kAStage + kBStage) + 256; }
 constexpr uint32_t kWaitPolls = 1u << 22;
 // kind::f16 instruction descriptor: D fp32 (bit 4), A and B bf16 (bits 7, 10),
