@@ -11,11 +11,20 @@
 // units u0..u0+3 (u0 = 4 rg), ordered [i, f, g, o] per unit; k slice ks is the
 // KPT = H/8 columns ks*KPT .. ks*KPT+KPT-1.  Each thread keeps its 16 x KPT
 // tile of W_hh for the whole sequence: RKK columns in registers (192 weights
-// at H = 128) and the rest in shared memory.  A thread reads only the KPT
-// values of h (forward) or the 16 values of dz (backward) that its tile
-// needs, so the shared-memory bytes per step stay small; a shared-memory
-// broadcast of all of h to every thread would cost 1 KB of load bandwidth
-// per thread per step.
+// at H = 128); the other SKK = KPT - RKK columns sit in tensor memory (TMEM)
+// in the forward kernel, one 16-weight column per tcgen05.ld, and in shared
+// memory in BPTT.  The forward matvec interleaves its two parts: the load of
+// TMEM column j + 1 is in flight while the thread runs the register FMAs of
+// block j + 1, so the TMEM reads (64 KB per step at H = 128) overlap the FMA
+// pipe instead of following it, as shared-memory operands did (0.94 -> 0.72
+// us per step).  BPTT's column sums over the 16 rows of a tile run as short
+// chains per column; with TMEM columns between register blocks they lost
+// their overlap and the step got slower (0.89 -> 1.0 us), so BPTT streams
+// its SKK columns from shared memory.  A
+// thread reads only the KPT values of h (forward) or the 16 values of dz
+// (backward) that its tile needs, so the shared-memory bytes per step stay
+// small; a shared-memory broadcast of all of h to every thread would cost
+// 1 KB of load bandwidth per thread per step.
 //
 // Forward step: 16 partial dot products per thread over its k slice; an
 // 8-lane shuffle reduce-scatter leaves lane ks with rows 2ks, 2ks+1 of the
@@ -67,6 +76,91 @@ __device__ __forceinline__ void cp_wait_pending() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
+// TMEM part of the W_hh tile.  Thread t of warp w owns TMEM lane
+// 32 (w % 4) + t % 32 (the lanes a warp may access) and, within it, the SKK
+// x 16 columns from (w / 4) SKK 16: column 16 kk + ri holds weight
+// (ri, RKK + kk) of its tile.  Columns per lane: SKK 16 for each warp that
+// shares the lane quadrant.
+template <int NTH, int SKK>
+__host__ __device__ constexpr int tm_cols() {
+  return SKK == 0 ? 0 : (NTH > 128 ? 2 : 1) * SKK * 16;
+}
+__device__ __forceinline__ void tm_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tm_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+// Allocated by warp 0; every thread returns the base address (a CTA-wide
+// barrier inside).  The allocation waits while another CTA on the SM holds
+// the columns; none of the recurrent kernels waits on another CTA.
+template <int NCOL>
+__device__ __forceinline__ uint32_t tm_alloc(uint32_t *slot, int warp) {
+  static_assert(NCOL >= 32 && NCOL <= 512 && (NCOL & (NCOL - 1)) == 0, "TMEM allocations are powers of 2 in 32..512");
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     static_cast<uint32_t>(__cvta_generic_to_shared(slot))),
+                 "r"(NCOL)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tm_fence_before();
+  __syncthreads();
+  tm_fence_after();
+  return *slot;
+}
+template <int NCOL>
+__device__ __forceinline__ void tm_free(uint32_t base, int warp) {
+  tm_fence_before();
+  __syncthreads();
+  tm_fence_after();
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(base), "r"(NCOL) : "memory");
+}
+__device__ __forceinline__ void tm_st16(uint32_t taddr, const uint32_t (&v)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16};" ::"r"(taddr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]),
+      "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+      : "memory");
+}
+__device__ __forceinline__ void tm_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, "
+      "[%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr)
+      : "memory");
+}
+// Completes this thread's tcgen05.ld; the loaded registers pass through the
+// wait, so no use of them is scheduled ahead of it.
+__device__ __forceinline__ void tm_wait16(uint32_t (&r)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15])
+               :
+               : "memory");
+}
+// The tile of the thread: RKK columns into w, the other SKK into TMEM at tw.
+template <int H, int RKK, int SKK>
+__device__ __forceinline__ void load_tile(const float *__restrict__ Whh, int u0, int kb, uint32_t tw,
+                                          float (&w)[16][RKK > 0 ? RKK : 1]) {
+#pragma unroll
+  for (int ri = 0; ri < 16; ++ri) {
+    const float *row = Whh + (size_t)((ri & 3) * H + u0 + (ri >> 2)) * H + kb;
+#pragma unroll
+    for (int kk = 0; kk < RKK; ++kk) w[ri][kk] = __ldg(row + kk);
+  }
+  if constexpr (SKK > 0) {
+#pragma unroll 1
+    for (int kk = 0; kk < SKK; ++kk) {
+      uint32_t v[16];
+#pragma unroll
+      for (int ri = 0; ri < 16; ++ri)
+        v[ri] = __float_as_uint(__ldg(Whh + (size_t)((ri & 3) * H + u0 + (ri >> 2)) * H + kb + RKK + kk));
+      tm_st16(tw + 16 * kk, v);
+    }
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+  }
+}
+
 // Reduce-scatter over the 8 lanes of a k-slice group (lane bits 0..2): on
 // return, lane l holds the group sums of positions 2(l%8) and 2(l%8)+1.
 __device__ __forceinline__ void reduce_scatter8(const float (&v)[16], int lane, float &o0, float &o1) {
@@ -113,10 +207,11 @@ __device__ __forceinline__ void reduce_groups(const float (&v)[KPT], int lane, f
 template <int H, int RKK, int BC>
 __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
   constexpr int G = 4 * H, NTH = 2 * H, KPT = H / 8, SKK = KPT - RKK, HS = KPT + 4;
+  constexpr int NCOL = tm_cols<NTH, SKK>();
   static_assert(SKK % 4 == 0 && RKK % 4 == 0, "k split in float4 steps");
   extern __shared__ __align__(16) float sm[];
-  float4 *Ws4 = reinterpret_cast<float4 *>(sm);  // [SKK/4][16][NTH]
-  float *hs = sm + SKK * 16 * NTH;               // [2][BC][8 slices][HS]
+  __shared__ uint32_t tslot;
+  float *hs = sm;                                // [2][BC][8 slices][HS]
   float *zr = hs + 2 * BC * 8 * HS;              // [BC][kRing][4H] Zx rows of upcoming steps
   const int T = a.ix.T;
   const bool toff_sm = T + 1 <= kTokCap;
@@ -133,18 +228,13 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
   const int DH = a.dirs * H;
   const float *__restrict__ Whh = a.Whh[d];
 
-  float w[16][RKK > 0 ? RKK : 1];
-#pragma unroll
-  for (int ri = 0; ri < 16; ++ri) {
-    const float *row = Whh + (size_t)((ri & 3) * H + u0 + (ri >> 2)) * H + kb;
-#pragma unroll
-    for (int kk = 0; kk < RKK; ++kk) w[ri][kk] = __ldg(row + kk);
-#pragma unroll
-    for (int k4 = 0; k4 < SKK / 4; ++k4) {
-      const float *p = row + RKK + 4 * k4;
-      Ws4[(k4 * 16 + ri) * NTH + t] = make_float4(__ldg(p), __ldg(p + 1), __ldg(p + 2), __ldg(p + 3));
-    }
+  uint32_t tbase = 0, tw = 0;
+  if constexpr (NCOL > 0) {
+    tbase = tm_alloc<NCOL>(&tslot, t >> 5);
+    tw = tbase + ((32u * ((t >> 5) & 3)) << 16) + (uint32_t)((t >> 7) * SKK * 16);
   }
+  float w[16][RKK > 0 ? RKK : 1];
+  load_tile<H, RKK, SKK>(Whh, u0, kb, tw, w);
   for (int i = t; i < 2 * BC * 8 * HS; i += NTH) hs[i] = 0.f;
   if (toff_sm)
     for (int i = t; i <= T; i += NTH) toff_s[i] = a.ix.tok_off[i];
@@ -206,27 +296,29 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
       float acc[16];
 #pragma unroll
       for (int ri = 0; ri < 16; ++ri) acc[ri] = 0.f;
+      // register block j (columns 4j .. 4j + 3), then TMEM column RKK + j,
+      // whose load was issued before block j
+      constexpr int NR = RKK / 4, NJ = NR > SKK ? NR : SKK;
+      uint32_t wt[16];
+      if constexpr (SKK > 0) tm_ld16(tw, wt);
 #pragma unroll
-      for (int k4 = 0; k4 < RKK / 4; ++k4) {
-        const float4 h4 = *reinterpret_cast<const float4 *>(hv + 4 * k4);
+      for (int j = 0; j < NJ; ++j) {
+        if (j < NR) {
+          const float4 h4 = *reinterpret_cast<const float4 *>(hv + 4 * j);
 #pragma unroll
-        for (int ri = 0; ri < 16; ++ri) {
-          float x = fmaf(w[ri][4 * k4], h4.x, acc[ri]);
-          x = fmaf(w[ri][4 * k4 + 1], h4.y, x);
-          x = fmaf(w[ri][4 * k4 + 2], h4.z, x);
-          acc[ri] = fmaf(w[ri][4 * k4 + 3], h4.w, x);
+          for (int ri = 0; ri < 16; ++ri) {
+            float x = fmaf(w[ri][4 * j], h4.x, acc[ri]);
+            x = fmaf(w[ri][4 * j + 1], h4.y, x);
+            x = fmaf(w[ri][4 * j + 2], h4.z, x);
+            acc[ri] = fmaf(w[ri][4 * j + 3], h4.w, x);
+          }
         }
-      }
+        if (j < SKK) {
+          tm_wait16(wt);
+          const float hk = hv[RKK + j];
 #pragma unroll
-      for (int k4 = 0; k4 < SKK / 4; ++k4) {
-        const float4 h4 = *reinterpret_cast<const float4 *>(hv + RKK + 4 * k4);
-#pragma unroll
-        for (int ri = 0; ri < 16; ++ri) {
-          const float4 wv = Ws4[(k4 * 16 + ri) * NTH + t];
-          float x = fmaf(wv.x, h4.x, acc[ri]);
-          x = fmaf(wv.y, h4.y, x);
-          x = fmaf(wv.z, h4.z, x);
-          acc[ri] = fmaf(wv.w, h4.w, x);
+          for (int ri = 0; ri < 16; ++ri) acc[ri] = fmaf(__uint_as_float(wt[ri]), hk, acc[ri]);
+          if (j + 1 < SKK) tm_ld16(tw + 16 * (j + 1), wt);
         }
       }
       float v0, v1;
@@ -251,6 +343,7 @@ __global__ void __launch_bounds__(2 * H, 1) lstm_fwd_cta_kernel(RecArgs a) {
     __syncthreads();
   }
   asm volatile("cp.async.wait_all;" ::: "memory");
+  if constexpr (NCOL > 0) tm_free<NCOL>(tbase, t >> 5);
 }
 
 template <int H, int RKK, int BC>
@@ -439,9 +532,9 @@ namespace {
 
 size_t cta_smem_bytes(bool bwd, int H, int RKK, int BC, int T) {
   const int KPT = H / 8, SKK = KPT - RKK, NTH = 2 * H;
-  const size_t wf = (size_t)SKK * 16 * NTH;
+  const size_t wf = (size_t)SKK * 16 * NTH;  // BPTT's shared-memory weights (the forward's are in TMEM)
   const size_t f = bwd ? wf + (size_t)BC * 4 * H + (size_t)BC * (NTH / 32) * H + (size_t)BC * kRing * 7 * H
-                       : wf + (size_t)2 * BC * 8 * (KPT + 4) + (size_t)BC * kRing * 4 * H;
+                       : (size_t)2 * BC * 8 * (KPT + 4) + (size_t)BC * kRing * 4 * H;
   const size_t i = (T + 1 <= kTokCap) ? (size_t)(T + 1) : 0;
   return (f + i) * 4 + 16;
 }

@@ -84,20 +84,25 @@ def test_serial_steps(bench):
 def test_recorded_traffic_matches_committed_source(bench):
     rec = json.load(open(os.path.join(ROOT, "profiles", "traffic_lstm1_bi_h128.json")))
     src = open(os.path.join(ROOT, rec["source"]), "rb").read()
-    tb, where = bench.recorded_traffic(rec["kernel"], rec["workload"], rec["buckets"])
-    if hashlib.sha256(src).hexdigest() == rec["source_sha256"]:
-        assert tb == rec["dram_bytes_per_launch"] and where.endswith("traffic_lstm1_bi_h128.json")
-    else:   # the kernel changed since the counters were taken: nothing is reported
-        assert tb is None and where is None
-    # other workloads or bucket counts have no record
-    assert bench.recorded_traffic(rec["kernel"], rec["workload"], rec["buckets"] + 1) == (None, None)
-    assert bench.recorded_traffic(rec["kernel"], "lstm2_uni_h512", rec["buckets"]) == (None, None)
+    same = hashlib.sha256(src).hexdigest() == rec["source_sha256"]
+    assert set(rec["kernels"]) == {"lstm_fwd", "lstm_bwd"}
+    for k, entry in rec["kernels"].items():
+        tb, where = bench.recorded_traffic(k, rec["workload"], rec["buckets"])
+        if same:
+            assert tb == entry["dram_bytes_per_launch"] and where.endswith("traffic_lstm1_bi_h128.json")
+            assert entry["dram_bytes_per_launch"] == pytest.approx(
+                entry["dram_read_bytes_per_launch"] + entry["dram_write_bytes_per_launch"], abs=1)
+        else:   # the kernels changed since the counters were taken: nothing is reported
+            assert tb is None and where is None
+        # other workloads or bucket counts have no record
+        assert bench.recorded_traffic(k, rec["workload"], rec["buckets"] + 1) == (None, None)
+        assert bench.recorded_traffic(k, "lstm2_uni_h512", rec["buckets"]) == (None, None)
+    assert bench.recorded_traffic("ctc_tables", rec["workload"], rec["buckets"]) == (None, None)
 
 
 def test_recorded_traffic_ignored_after_a_source_change(bench, tmp_path, monkeypatch):
     rec = json.load(open(os.path.join(ROOT, "profiles", "traffic_lstm1_bi_h128.json")))
     (tmp_path / "profiles").mkdir()
-    shutil.copy(os.path.join(ROOT, "profiles", "traffic_lstm1_bi_h128.json"), tmp_path / "profiles")
     dst = tmp_path / rec["source"]
     dst.parent.mkdir(parents=True)
     src = open(os.path.join(ROOT, rec["source"]), "rb").read()
@@ -106,10 +111,11 @@ def test_recorded_traffic_ignored_after_a_source_change(bench, tmp_path, monkeyp
     rec["source_sha256"] = hashlib.sha256(src).hexdigest()
     json.dump(rec, open(tmp_path / "profiles" / "traffic_lstm1_bi_h128.json", "w"))
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
-    assert bench.recorded_traffic(rec["kernel"], rec["workload"], rec["buckets"])[0] == \
-        rec["dram_bytes_per_launch"]
+    for k, entry in rec["kernels"].items():
+        assert bench.recorded_traffic(k, rec["workload"], rec["buckets"])[0] == entry["dram_bytes_per_launch"]
     dst.write_bytes(src + b"\n// changed\n")
-    assert bench.recorded_traffic(rec["kernel"], rec["workload"], rec["buckets"]) == (None, None)
+    for k in rec["kernels"]:
+        assert bench.recorded_traffic(k, rec["workload"], rec["buckets"]) == (None, None)
 
 
 def test_measured_peaks_source(bench, tmp_path, monkeypatch):
