@@ -11,6 +11,14 @@ training loss and the mean validation loss per sequence.
   python -m paper_1708_05604_gb300.train --workload lstm1_bi_h128 \\
       --buckets 1,2,3,4,6 --epochs 3 [--optimizer adadelta|sgd]
       [--batch-order ascending|descending|shuffle_buckets|shuffle_batches]
+      [--checkpoint PATH] [--resume PATH] [--log-jsonl FILE] [--kernel-times]
+
+With --checkpoint the parameters and the optimizer state are stored after
+every epoch (`checkpoint.py`); --resume continues such a run from the epoch
+after its checkpoint with the same mini-batches an uninterrupted run would
+draw.  --log-jsonl appends each epoch's record to a JSON-lines file;
+--kernel-times adds the library's per-kernel CUDA-event times to it (the
+per-launch events add a little to the epoch they time).
 
 Data-parallel training (Section III.B steps 3-5): launched with torchrun on
 N GPUs, every epoch the training sequences are reshuffled into N portions,
@@ -84,14 +92,42 @@ def validation_batches(lengths, val_ids, batch: int):
     return [o[i:i + batch] for i in range(0, o.size, batch)]
 
 
+def run_identity(workload: str, n_buckets: int, optimizer: str, batch_order: str, seed: int,
+                 val_frac: float, lr, n_seqs, max_len, n_params: int) -> dict:
+    """What a checkpoint must agree on for a run to resume from it: the data,
+    the plan's inputs, the update rule and the parameter count."""
+    return {"workload": workload, "n_buckets": int(n_buckets), "optimizer": optimizer,
+            "batch_order": batch_order, "seed": int(seed), "val_frac": float(val_frac),
+            "lr": None if lr is None else float(lr), "n_seqs": n_seqs, "max_len": max_len,
+            "n_params": int(n_params)}
+
+
+def resume_point(meta: dict, identity: dict, epochs: int):
+    """(first epoch to run, per-epoch records so far, wall seconds so far,
+    initial validation loss) of a run resumed from a checkpoint's meta;
+    ValueError when the checkpoint is of another run or already past
+    `epochs`."""
+    from . import checkpoint
+    checkpoint.check_compatible(meta, identity)
+    start = int(meta["epoch_next"])
+    if start > epochs:
+        raise ValueError(f"checkpoint is after epoch {start - 1}; asked for {epochs} epochs in all")
+    return start, list(meta["epochs"]), float(meta["wall_s"]), meta["val_loss_initial"]
+
+
 def train(workload: str, n_buckets: int, epochs: int, optimizer: str = "adadelta",
           batch_order: str = "ascending", seed: int = 0, val_frac: float = 0.05,
           lr: float | None = None, n_seqs: int | None = None, max_len: int | None = None,
-          params0=None, device: str = "cuda", log=None) -> dict:
-    """Trains `epochs` epochs; returns the per-epoch record and final params."""
+          params0=None, device: str = "cuda", log=None, checkpoint_path: str | None = None,
+          resume: str | None = None, kernel_times: bool = False) -> dict:
+    """Trains up to epoch `epochs` (counting from 0, so `epochs` epochs in
+    all, fewer when resumed); returns the per-epoch record and final params.
+    checkpoint_path: store parameters and optimizer state after every epoch;
+    resume: continue the run stored there (same workload, Q, seed, order,
+    update rule); kernel_times: per-kernel CUDA-event ms in each record."""
     import torch
 
-    from . import binding, build, synth
+    from . import binding, build, checkpoint, synth
 
     build.build()
     w = synth.WORKLOADS[workload]
@@ -99,7 +135,14 @@ def train(workload: str, n_buckets: int, epochs: int, optimizer: str = "adadelta
     ds = synth.make_workload(w, seed=seed, n_seqs=n_seqs, max_len=max_len)
     train_ids, val_ids = split_validation(ds.n, val_frac, seed + 17)
     P = binding.param_count(cfg)
-    if params0 is None:
+    ident = run_identity(workload, n_buckets, optimizer, batch_order, seed, val_frac, lr,
+                         n_seqs, max_len, P)
+    start, saved = 0, None
+    if resume:
+        meta, saved = checkpoint.load(resume)
+        start, done, wall0, v_init = resume_point(meta, ident, epochs)
+        params0 = saved["params"]
+    elif params0 is None:
         params0 = synth.draw_params(np.random.default_rng(seed + 1), P)
     dev = torch.device(device)
     params = torch.from_numpy(np.ascontiguousarray(params0, np.float32)).to(dev)
@@ -111,6 +154,9 @@ def train(workload: str, n_buckets: int, epochs: int, optimizer: str = "adadelta
     if optimizer == "adadelta":
         opt = binding.Adadelta(params, lr=1.0 if lr is None else lr)
         update = opt.step
+        if saved is not None:
+            opt.eg2.copy_(torch.from_numpy(saved["eg2"]))
+            opt.edx2.copy_(torch.from_numpy(saved["edx2"]))
     elif optimizer == "sgd":
         step_lr = 1e-3 if lr is None else lr
         update = lambda g, stream=None: binding.sgd_update(params, g, step_lr, stream)
@@ -127,19 +173,33 @@ def train(workload: str, n_buckets: int, epochs: int, optimizer: str = "adadelta
             total += float(lv.double().sum())
         return total / max(1, val_ids.size)
 
+    def store(e_next):
+        arrays = {"params": params.cpu().numpy()}
+        if optimizer == "adadelta":
+            arrays["eg2"], arrays["edx2"] = opt.eg2.cpu().numpy(), opt.edx2.cpu().numpy()
+        checkpoint.save(checkpoint_path, arrays,
+                        {**ident, "epoch_next": e_next, "epochs": record["epochs"], "wall_s": wall,
+                         "val_loss_initial": record["val_loss_initial"]})
+
     record = {"workload": workload, "n_buckets": n_buckets, "optimizer": optimizer,
               "batch_order": batch_order, "n_train": int(train_ids.size),
               "n_val": int(val_ids.size), "epochs": []}
-    wall = 0.0
-    v0 = validate()
-    ctx.sync_status()
-    record["val_loss_initial"] = v0
-    for e in range(epochs):
+    if resume:
+        record["epochs"], wall, record["val_loss_initial"] = done, wall0, v_init
+        record["resumed_at_epoch"] = start
+    else:
+        wall = 0.0
+        v0 = validate()
+        ctx.sync_status()
+        record["val_loss_initial"] = v0
+    for e in range(start, epochs):
         batches, plan = epoch_batches(ds.lengths, train_ids, n_buckets, w.batch, seed, e,
                                       batch_order)
         torch.cuda.synchronize(dev)
         t0 = time.perf_counter()
         ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        if kernel_times:
+            ctx.set_timing(True)
         ev0.record(stream)
         pos = 0
         for ids in batches:
@@ -151,6 +211,10 @@ def train(workload: str, n_buckets: int, epochs: int, optimizer: str = "adadelta
         torch.cuda.synchronize(dev)
         host_s = time.perf_counter() - t0
         ms = ev0.elapsed_time(ev1)
+        kms = None
+        if kernel_times:
+            kms = {k["name"]: round(k["total_ms"], 4) for k in ctx.kernel_stats()}
+            ctx.set_timing(False)
         ctx.sync_status()
         wall += host_s
         tl = float(loss[:pos].double().sum()) / max(1, pos)
@@ -158,8 +222,13 @@ def train(workload: str, n_buckets: int, epochs: int, optimizer: str = "adadelta
         rec = {"epoch": e, "epoch_ms": ms, "host_s": host_s, "wall_s": wall,
                "train_loss": tl, "val_loss": vl, "n_batches": plan["n_batches"],
                "padded_efficiency": plan["unpadded_timesteps"] / plan["padded_timesteps"],
-               "timesteps": int(plan["unpadded_timesteps"])}
+               "timesteps": int(plan["unpadded_timesteps"]),
+               "timesteps_per_s": plan["unpadded_timesteps"] / (ms / 1e3) if ms > 0 else None}
+        if kms is not None:
+            rec["kernel_ms"] = kms
         record["epochs"].append(rec)
+        if checkpoint_path:
+            store(e + 1)
         if log:
             log(rec)
     record["params"] = params.cpu().numpy()
@@ -235,6 +304,12 @@ def main(argv=None):
     ap.add_argument("--replicas", action="store_true",
                     help="data-parallel replicas with eq.-3 averaging (launch with torchrun)")
     ap.add_argument("--beta", type=float, default=1e-6)
+    ap.add_argument("--checkpoint", default=None,
+                    help="store parameters and optimizer state after every epoch (PATH.bin, PATH.json; "
+                         "with several bucket counts, PATH.qQ)")
+    ap.add_argument("--resume", default=None, help="continue the run stored at this checkpoint path")
+    ap.add_argument("--log-jsonl", default=None, help="append every epoch's record to this file")
+    ap.add_argument("--kernel-times", action="store_true", help="per-kernel CUDA-event ms in each record")
     a = ap.parse_args(argv)
     if a.replicas:
         import os
@@ -250,8 +325,18 @@ def main(argv=None):
                 print(json.dumps(r), flush=True)
         dist.destroy_process_group()
         return 0
-    for Q in [int(q) for q in a.buckets.split(",") if q]:
-        r = train(a.workload, Q, a.epochs, a.optimizer, a.batch_order, a.seed, lr=a.lr)
+    from .checkpoint import JsonlLog
+    qs = [int(q) for q in a.buckets.split(",") if q]
+    if a.resume and len(qs) != 1:
+        ap.error("--resume continues one run: give one bucket count")
+
+    def ck(path, Q):
+        return None if path is None else (path if len(qs) == 1 else f"{path}.q{Q}")
+
+    for Q in qs:
+        log = JsonlLog(a.log_jsonl, workload=a.workload, n_buckets=Q) if a.log_jsonl else None
+        r = train(a.workload, Q, a.epochs, a.optimizer, a.batch_order, a.seed, lr=a.lr, log=log,
+                  checkpoint_path=ck(a.checkpoint, Q), resume=a.resume, kernel_times=a.kernel_times)
         r.pop("params")
         print(json.dumps(r), flush=True)
     return 0
