@@ -23,6 +23,9 @@ std::mutex g_devs_mu;
 
 extern "C" int bkt_lstm_ctc_step_static(const bkt_model_cfg *cfg, const bkt_batch *batch, const float *params,
                                         float *grads, float *loss, void *stream) {
+  // NULL arguments are refused before any CUDA call, as by bkt_lstm_ctc_step
+  if (!cfg || !batch || !params || !grads || !loss)
+    return bkt::report_error(BKT_EINVAL, "bkt_lstm_ctc_step_static: NULL argument");
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess)
