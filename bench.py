@@ -67,6 +67,8 @@ def parse(argv=None):
     ap.add_argument("--cpu-baseline-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--reference-seconds", type=float, default=150.0,
+                    help="--impl reference: oracle seconds over all warm-up and timed steps")
     return ap.parse_args(argv)
 
 
@@ -508,7 +510,7 @@ def run_reference(args, world, rank):
                            cfg["n_classes"])
     params0 = synth.draw_params(np.random.default_rng(args.seed + 1), P)
     plan = oracle.plan(ds.lengths, args.buckets, w.batch, seed=args.seed, epoch=0)
-    per_step = max(1.0, 150.0 / (args.steps + args.warmup))
+    per_step = max(0.05, args.reference_seconds / max(1, args.steps + args.warmup))
     pos = 0
     for _ in range(args.warmup):
         _, _, _, pos = oracle_sample(w, ds, params0, plan, per_step, pos)
