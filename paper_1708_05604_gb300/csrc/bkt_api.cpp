@@ -14,6 +14,7 @@
 #include <vector>
 
 #include "bkt_internal.h"
+#include "nvtx_range.h"
 
 namespace {
 
@@ -61,6 +62,7 @@ struct bkt_plan {
 
 extern "C" int bkt_plan_buckets_ordered(const int32_t *lengths, int64_t n, int32_t Q, int32_t batch,
                                         uint64_t seed, uint64_t epoch, int32_t batch_order, bkt_plan **out) {
+  bkt::NvtxRange range("bkt_plan_buckets");
   if (!out) return set_err(BKT_EINVAL, "bkt_plan_buckets: out is NULL");
   if (batch_order < BKT_ORDER_ASCENDING || batch_order > BKT_ORDER_SHUFFLE_BATCHES)
     return set_err(BKT_EINVAL, "bkt_plan_buckets: unknown batch order %d", batch_order);
@@ -389,6 +391,7 @@ struct Launch {
   template <typename F>
   bool run(const char *name, const bkt::Work &wk, F &&f) {
     if (failed) return false;
+    bkt::NvtxRange range(name);
     if (timer) timer->begin(name, wk, s);
     cudaError_t e = f();
     if (timer) timer->end(s);
@@ -465,6 +468,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
 
   // ---- forward, layer by layer
   for (int l = 0; l < lo.L; ++l) {
+    bkt::NvtxRange layer_range("forward layer");
     float *Zl[2] = {w.Z[l * dirs], dirs > 1 ? w.Z[l * dirs + 1] : nullptr};
     if (l == 0) {
       // a5, narrow input: both directions in one launch
@@ -546,6 +550,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
   }
 
   // ---- a7: output layer and log-softmax
+  bkt::NvtxRange output_range("output layer and CTC");
   // logits = Y W_out^T + b_out on the tensor cores (3xTF32; both operands are
   // already K-contiguous, so they are split without transposing); the
   // GEMM's epilogue holds whole rows (C <= 128 columns in one tile) and
@@ -675,6 +680,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     L.run("gemm_tf32x3", gemm_w(g.M, g.N, g.K), [&] { return bkt::launch_gemm_tf32x3_tc(g, w.Ll, w.WoTl, s); });
   }
 
+  output_range.end();
   // ---- a11, a12: BPTT and weight gradients, top layer first.  With a side
   // stream, a layer's weight gradients run there (after its BPTT) while the
   // main stream goes on with dX and the BPTT of the layer below; the side
@@ -686,6 +692,7 @@ int enqueue_kernels(const bkt_model_cfg &cfg, const Layout &lo, const bkt::StepB
     return e == cudaSuccess ? BKT_OK : cuda_err("fork to the side stream", e);
   };
   for (int l = lo.L - 1; l >= 0; --l) {
+    bkt::NvtxRange layer_range("BPTT layer");
     bkt::RecArgs ra{};
     ra.ix = ix;
     ra.H = H;
@@ -1244,6 +1251,7 @@ extern "C" int bkt_sgd_update(float *params, const float *grads, int64_t n, floa
 // The step through a ctx.
 extern "C" int bkt_lstm_ctc_step(bkt_ctx *c, const bkt_batch *bt, const float *params, float *grads, float *loss,
                                  void *stream) {
+  bkt::NvtxRange range("bkt_lstm_ctc_step");
   if (!c || !bt || !params || !grads || !loss) return set_err(BKT_EINVAL, "bkt_lstm_ctc_step: NULL argument");
   int64_t n_tok = 0, cells = 0;
   int32_t S_max = 1;
@@ -1317,6 +1325,7 @@ struct Carve {
 
 int bkt::step_on_scratch(const bkt_model_cfg *cfg, const bkt_batch *bt, const float *params, float *grads,
                          float *loss, cudaStream_t s, void *scratch, size_t scratch_bytes, int sm_count) {
+  bkt::NvtxRange range("bkt_lstm_ctc_step_static");
   if (!cfg_ok(cfg)) return set_err(BKT_EINVAL, "bkt_lstm_ctc_step_static: invalid model cfg");
   if (!bt || !params || !grads || !loss) return set_err(BKT_EINVAL, "bkt_lstm_ctc_step_static: NULL argument");
   int64_t n_tok = 0, cells = 0;
