@@ -195,8 +195,10 @@ int bkt_lstm_ctc_step(bkt_ctx *ctx, const bkt_batch *batch,
  *     fits the array (about (26 H + C + 2 S + 8) * 4 bytes per token for one
  *     bidirectional layer, S = 2U + 1: some 4,500 tokens at H = 128).  A batch beyond them returns
  *     BKT_EINVAL with the needed and available bytes in bkt_last_error().
- *   - The first call on a device looks up the array's address on that
- *     device, so make that first call before any stream capture.
+ *   - It cannot be captured into a CUDA graph: on a stream that is being
+ *     captured it returns BKT_EINVAL before anything is enqueued (the
+ *     index block goes up from one shared pageable buffer, which a replay
+ *     would read as it is then).
  *   - The array used is the current device's; a stream of another device
  *     returns BKT_EINVAL before anything is enqueued.
  *   - All calls share the one array, and it keeps the previous call's

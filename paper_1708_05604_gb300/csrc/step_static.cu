@@ -44,6 +44,18 @@ extern "C" int bkt_lstm_ctc_step_static(const bkt_model_cfg *cfg, const bkt_batc
                                "bkt_lstm_ctc_step_static: the stream belongs to device %d but device %d is current",
                                sdev, dev);
   }
+  {
+    // the index block goes up from one shared pageable buffer: a captured
+    // copy would read whatever that buffer holds when the graph is replayed
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    e = cudaStreamIsCapturing((cudaStream_t)stream, &cs);
+    if (e != cudaSuccess)
+      return bkt::report_error(BKT_ECUDA, "cudaStreamIsCapturing: %s (%s)", cudaGetErrorName(e), cudaGetErrorString(e));
+    if (cs != cudaStreamCaptureStatusNone)
+      return bkt::report_error(BKT_EINVAL,
+                               "bkt_lstm_ctc_step_static: the stream is being captured; this entry point cannot be "
+                               "part of a CUDA graph");
+  }
   DeviceScratch ds;
   {
     // first call on this device (with it current): look up the array's
