@@ -69,10 +69,13 @@ def small_cfg(layers, bi, H, C=7):
             "n_classes": C, "blank": 0}
 
 
-@pytest.mark.parametrize("layers,bi,H", [(1, False, 5), (1, True, 4), (2, True, 3),
-                                         (3, False, 4), (2, False, 6)])
-def test_step_matches_torch(layers, bi, H):
-    cfg = small_cfg(layers, bi, H)
+@pytest.mark.parametrize("layers,bi,H,C", [(1, False, 5, 7), (1, True, 4, 7), (2, True, 3, 7),
+                                           (3, False, 4, 7), (2, False, 6, 7),
+                                           # the benchmarked architecture (3 bidirectional
+                                           # layers, 81 classes) at a tiny H
+                                           (3, True, 4, 81)])
+def test_step_matches_torch(layers, bi, H, C):
+    cfg = small_cfg(layers, bi, H, C)
     rng = np.random.default_rng(layers * 10 + H + bi)
     ds = synth.make_dataset([9, 4, 13, 7, 1], 3, rng, n_classes=cfg["n_classes"])
     P = oracle.param_count(layers, bi, 4, H, cfg["n_classes"])
